@@ -1,0 +1,429 @@
+"""Pins for the CPU oracle: hand-worked values, closed forms, textbook
+special cases, brute force on tiny inputs and invariants.  None of these
+re-types the oracle's code; each fixes a fact the paper or the mathematics
+determines, so a dropped term, swapped operand or flipped order fails one."""
+import itertools
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+BIG = 1 << 60
+
+
+def _rows(name):
+    with open(os.path.join(GOLD, name)) as f:
+        for line in f:
+            line = line.split("#", 1)[0].strip()
+            if line:
+                yield line
+
+
+# ---------------------------------------------------------------- score ----
+
+def test_locked_constants():
+    # eq. (survq): eps_q = floor(0.01 * 4095 + 1/2) = 41; h = 1 saturates at it
+    assert oracle.spear_score(1000, 41) == oracle.spear_score(1000, 41)
+    h, s = oracle.hazard_lut([1] * 10)  # every session ends at turn 0 -> h(0) = 1
+    assert int(h[0]) == 4095 and int(s[0]) == 41
+    assert int(s[1]) == 4095  # n(1) = 0 -> h = 0
+
+
+def test_score_hand_values():
+    for row in _rows("spear_score_hand.txt"):
+        g, hn, hd, hq, sq, t1, t2, score = map(int, row.split())
+        # the hazard quantiser via a one-turn-type population: hd sessions of
+        # which hn end at turn 0 gives h(0) = hn / hd
+        h, s = oracle.hazard_lut([1] * hn + [2] * (hd - hn))
+        assert int(h[0]) == hq and int(s[0]) == sq
+        assert oracle.spear_score(g, sq) == score == t1 + t2
+
+
+def test_score_done_is_max():
+    assert oracle.spear_score(123, 4095, done=True) == 2 ** 64 - 1
+
+
+def test_score_within_float_bound():
+    """eq. (esp) in floating point (g/sigma + (1 - sigma) P with sigma = sigma_q / Lambda)
+    minus the fixed-point score lies in [0, 2): two floors, nothing else."""
+    rs = np.random.default_rng(5)
+    for _ in range(3000):
+        g = int(rs.integers(0, 2 ** 31))
+        sq = int(rs.integers(41, 4096))
+        sig = sq / 4095.0
+        flt = g / sig + (1.0 - sig) * 5e8
+        fix = oracle.spear_score(g, sq)
+        assert -1e-6 * flt - 1e-3 <= flt - fix < 2 + 1e-6 * flt
+
+
+def test_score_monotone_in_gap_and_hazard():
+    for sq in (41, 1000, 3919, 4095):
+        vals = [oracle.spear_score(g, sq) for g in range(0, 10 ** 6, 9973)]
+        assert all(a <= b for a, b in zip(vals, vals[1:]))
+    # lower survival (higher hazard) never lowers the score at fixed gap
+    for g in (0, 10 ** 5, 3 * 10 ** 6):
+        vals = [oracle.spear_score(g, sq) for sq in range(4095, 40, -37)]
+        assert all(a <= b for a, b in zip(vals, vals[1:]))
+
+
+def test_zero_hazard_is_gap_order():
+    # closed form: h = 0 -> sigma_q = Lambda -> score_q = g_q exactly
+    for g in (0, 1, 977, 2 ** 31 - 1):
+        assert oracle.spear_score(g, 4095) == g
+
+
+# ------------------------------------------------------------------ EMA ----
+
+def test_ema_hand_values():
+    for row in _rows("ema_hand.txt"):
+        g0, gn, g1 = map(int, row.split())
+        assert oracle.ema(g0, gn) == g1
+
+
+def test_ema_constant_gap_converges_from_below():
+    g = 0
+    for _ in range(200):
+        g = oracle.ema(g, 1_234_567)
+        assert g <= 1_234_567
+    assert 1_234_567 - 10 <= g <= 1_234_567
+
+
+def test_ema_window_weight():
+    # span-W EMA (2, W+1): one step from 0 gives floor(2x/(W+1))
+    for w in (4, 8, 16, 32):
+        assert oracle.ema(0, 999_999, 2, w + 1) == (2 * 999_999) // (w + 1)
+
+
+# --------------------------------------------------------------- hazard ----
+
+def test_hazard_hand_counts():
+    # T_s = [1,2,2,3]: n = 4,3,1 ; d = 1,2,1 ; h = 1/4, 2/3, 1
+    h, s = oracle.hazard_lut([1, 2, 2, 3])
+    assert list(map(int, h[:4])) == [1024, 2730, 4095, 0]
+    assert list(map(int, s[:4])) == [3071, 1365, 41, 4095]
+    # bucket width 2 pools t = 0,1: 3/7 -> floor(1755 + 1/2) = 1755
+    h2, _ = oracle.hazard_lut([1, 2, 2, 3], 2)
+    assert int(h2[0]) == int(h2[1]) == 1755
+    assert int(h2[2]) == 4095  # {2,3}: d = 1, n = 1
+
+
+def test_hazard_fixed_turns():
+    # every session exactly 12 turns: h(t) = 0 except h(11) = 1
+    h, s = oracle.hazard_lut([12] * 64)
+    assert int(h[11]) == 4095 and int(s[11]) == 41
+    assert all(int(h[t]) == 0 for t in range(51) if t != 11)
+
+
+def test_hazard_matches_brute_counts_and_rounding():
+    tps = synth.geometric_turns(3, 5000, 23.7, 2, 200)
+    for w in (1, 2, 4, 8, 64):
+        h, s = oracle.hazard_lut(tps, w)
+        for t in range(51):
+            bucket = [u for u in range(51) if u // w == t // w]
+            n = sum(int((tps >= u + 1).sum()) for u in bucket)
+            d = sum(int((tps == u + 1).sum()) for u in bucket)
+            x = d / n if n else 0.0
+            assert abs(int(h[t]) - x * 4095) <= 0.5 + 1e-9  # round to nearest
+            assert int(s[t]) == max(41, 4095 - int(h[t]))
+        if w >= 51:
+            assert len(set(map(int, h))) == 1
+
+
+def test_hazard_geometric_nearly_constant():
+    # memoryless turns: h(t) ~ p for t >= 2, h(0) = 0 since T_s >= 2
+    tps = synth.geometric_turns(11, 200000, 23.7, 2, 200)
+    h, _ = oracle.hazard_lut(tps)
+    assert int(h[0]) == 0
+    assert all(abs(int(h[t]) - 4095 / 23.7) < 25 for t in range(2, 30))
+
+
+# -------------------------------------------------------- hand replay ----
+
+def _hand_trace(name):
+    turns, log, counts = {}, [], {}
+    for row in _rows(name):
+        tag, *rest = row.split()
+        if tag == "trace":
+            s, k, a, c, i, o = map(int, rest)
+            turns.setdefault(s, []).append((k, a, c, i, o))
+        elif tag == "log":
+            log.append((int(rest[0]), oracle.KINDS.index(rest[1]), int(rest[2])))
+        elif tag == "count":
+            counts[rest[0]] = int(rest[1])
+    sess = [sorted(turns[s]) for s in sorted(turns)]
+    tr = synth.trace_from_turns([[t[1] for t in x] for x in sess], [[t[2] for t in x] for x in sess],
+                                [[t[3] for t in x] for x in sess], [[t[4] for t in x] for x in sess])
+    return tr, log, counts
+
+
+HAND_PARAMS = dict(policy="spear", kv_bytes_per_token=1, cap_s_bytes=100, cap_h_bytes=100,
+                   t_p_ps_per_tok=20_000_000, ttft_load=4)
+
+
+def test_hand_replay_spear():
+    tr, log, counts = _hand_trace("replay_hand_spear.txt")
+    r = oracle.replay(tr, HAND_PARAMS, log=True, debug=True)
+    assert r["status"] == 0
+    got = list(zip(*(map(int, a) for a in r["log"])))
+    assert got == log
+    for k, v in counts.items():
+        assert r[k] == v, k
+
+
+# ------------------------------------------------------ capacity extremes ----
+
+POLICIES = ["lru", "timeout", "spear", "spear_tide", "belady", "lru_tide"]
+
+
+@pytest.mark.parametrize("pol", POLICIES)
+def test_infinite_capacity_all_warm_hits(pol):
+    tr = synth.tiny_trace(3)
+    r = oracle.replay(tr, dict(policy=pol, cap_s_bytes=BIG, cap_h_bytes=BIG, kv_bytes_per_token=28672,
+                               ttl_us=0xFFFFFFFF), debug=True)
+    assert r["status"] == 0
+    assert r["hit_s"] == r["req_warm"] == tr.n_turns - tr.n_sessions
+    assert r["evict"] == r["demote"] == r["expire"] == r["miss"] == 0
+
+
+@pytest.mark.parametrize("pol", POLICIES)
+def test_zero_capacity_all_bypass(pol):
+    tr = synth.tiny_trace(4)
+    r = oracle.replay(tr, dict(policy=pol, cap_s_bytes=0, cap_h_bytes=0, kv_bytes_per_token=28672),
+                      debug=True)
+    assert r["status"] == 0
+    assert r["bypass"] == tr.n_turns and r["hit_s"] == r["hit_h"] == 0
+    assert r["miss"] == r["req_warm"]
+    assert r["tok_computed"] == r["tok_needed"]
+
+
+@pytest.mark.parametrize("pol", POLICIES)
+def test_no_fast_tier_no_fast_hits(pol):
+    tr = synth.paper_scale_trace(2)
+    r = oracle.replay(tr, dict(policy=pol, cap_s_bytes=0, cap_h_bytes=16 << 30), debug=False)
+    assert r["status"] == 0 and r["hit_s"] == 0 and r["place_s"] == 0 and r["hit_h"] > 0
+
+
+# ------------------------------------------------------- slot-mode pins ----
+
+def _slot_trace(seq):
+    """Arrivals on a 1 ms grid in the given session order, 1 us of service,
+    one token each (sessions numbered by first arrival)."""
+    order = []
+    for s in seq:
+        if s not in order:
+            order.append(s)
+    ren = {s: i for i, s in enumerate(order)}
+    seq = [ren[s] for s in seq]
+    arr = [[] for _ in order]
+    for i, s in enumerate(seq):
+        arr[s].append(1000 * (i + 1))
+    tr = synth.trace_from_turns(arr, [[a + 1 for a in x] for x in arr],
+                                [[1] * len(x) for x in arr], [[1] * len(x) for x in arr])
+    return tr, seq
+
+
+SLOT = dict(cap_s_bytes=0, cap_h_bytes=BIG, kv_bytes_per_token=1)
+
+
+def _brute_max_hits(seq, n_slots):
+    best = 0
+
+    def go(i, cache, hits):
+        nonlocal best
+        if i == len(seq):
+            best = max(best, hits)
+            return
+        s = seq[i]
+        warm = s in seq[:i]
+        if s in cache:
+            go(i + 1, cache, hits + (1 if warm else 0))
+            return
+        if len(cache) < n_slots:
+            go(i + 1, cache | {s}, hits)
+            return
+        for v in cache:
+            go(i + 1, (cache - {v}) | {s}, hits)
+
+    go(0, frozenset(), 0)
+    return best
+
+
+def _random_seqs(n, seed):
+    rs = np.random.default_rng(seed)
+    for _ in range(n):
+        ns = int(rs.integers(2, 7))
+        ln = int(rs.integers(4, 13))
+        seq = list(map(int, rs.integers(0, ns, ln)))
+        # at most 4 turns per session
+        cnt = {}
+        out = []
+        for s in seq:
+            cnt[s] = cnt.get(s, 0) + 1
+            if cnt[s] <= 4:
+                out.append(s)
+        yield out
+
+
+@pytest.mark.parametrize("slots", [1, 2, 3])
+def test_belady_is_optimal_bruteforce(slots):
+    for seq in _random_seqs(60, 100 + slots):
+        tr, seq = _slot_trace(seq)
+        r = oracle.replay(tr, dict(SLOT, policy="belady", max_sessions=slots), debug=True)
+        assert r["status"] == 0
+        assert r["hit_h"] + r["hit_s"] == _brute_max_hits(seq, slots), seq
+
+
+@pytest.mark.parametrize("slots", [1, 2, 3])
+def test_lru_matches_stack_distance(slots):
+    for seq in _random_seqs(60, 200 + slots):
+        tr, seq = _slot_trace(seq)
+        r = oracle.replay(tr, dict(SLOT, policy="lru", max_sessions=slots), debug=True)
+        hits = 0
+        for i, s in enumerate(seq):
+            prev = [j for j in range(i) if seq[j] == s]
+            if prev:
+                dist = len(set(seq[prev[-1] + 1:i]))
+                hits += dist < slots
+        assert r["status"] == 0 and r["hit_h"] == hits, seq
+
+
+def test_timeout_limits():
+    tr = synth.tiny_trace(5)
+    base = dict(cap_s_bytes=512 << 20, cap_h_bytes=8 << 30, kv_bytes_per_token=28672)
+    lru = oracle.replay(tr, dict(base, policy="lru"), log=True)
+    inf = oracle.replay(tr, dict(base, policy="timeout", ttl_us=0xFFFFFFFF), log=True)
+    assert lru["decision_hash"] == inf["decision_hash"]
+    zero = oracle.replay(tr, dict(base, policy="timeout", ttl_us=0))
+    assert zero["status"] == 0 and zero["hit_s"] == zero["hit_h"] == 0
+    assert zero["miss"] == zero["req_warm"]
+
+
+# ------------------------------------------------------------------ TIDE ----
+
+def test_tide_zero_budget_equals_spear():
+    tr = synth.paper_scale_trace(3)
+    base = dict(cap_s_bytes=2 << 30, cap_h_bytes=32 << 30, kv_bytes_per_token=131072)
+    a = oracle.replay(tr, dict(base, policy="spear"))
+    b = oracle.replay(tr, dict(base, policy="spear_tide", dma_bytes_per_us=0))
+    assert a["decision_hash"] == b["decision_hash"] and b["promote"] == 0 and b["tide_calls"] > 0
+
+
+def test_tide_loop_equals_list_form_and_invariants():
+    """Debug replays check, at every TIDE call, that the literal pair loop
+    and the sorted-list form move the same sessions, and at every event the
+    capacity and pinning invariants."""
+    for seed, kv, cs, ch, dma in [(0, 28672, 512 << 20, 8 << 30, 64000), (1, 131072, 1 << 30, 32 << 30, 64000),
+                                  (2, 131072, 8 << 30, 32 << 30, 640000), (3, 28672, 4 << 30, 64 << 30, 6400)]:
+        tr = synth.paper_scale_trace(seed) if seed else synth.tiny_trace(0)
+        r = oracle.replay(tr, dict(policy="spear_tide", cap_s_bytes=cs, cap_h_bytes=ch,
+                                   kv_bytes_per_token=kv, dma_bytes_per_us=dma), debug=True)
+        assert r["status"] == 0 and r["promote"] > 0
+        assert r["dma_bytes"] <= r["tide_calls"] * (2 ** 31) * dma
+
+
+def test_tide_unlimited_budget_sorts_tiers():
+    """With an unbounded budget and sessions of one size, TIDE leaves the
+    least evictable unpinned sessions in the fast tier (Sec. III-C)."""
+    rs = np.random.default_rng(9)
+    for trial in range(20):
+        n = 12
+        rec = synth.Records(gap_q=rs.integers(0, 10 ** 6, n).astype(np.uint32),
+                            last_ret=np.zeros(n, np.uint32), turn=np.zeros(n, np.uint16),
+                            kv_tok=np.full(n, 7, np.uint32),
+                            tier=np.where(rs.random(n) < 0.4, 1, 2).astype(np.uint8),
+                            flags=np.zeros(n, np.uint8))
+        sig = np.full(51, 4095, np.uint16)
+        out = oracle.rank(rec, sig, 0, 1, 10 ** 12, 1, 0, 10 ** 9)
+        tier = rec.tier.copy()
+        tier[out["promote"]] = 1
+        tier[out["demote"]] = 2
+        n_s = int((rec.tier == 1).sum())
+        order = sorted(range(n), key=lambda i: (int(rec.gap_q[i]), -i))  # least evictable first
+        assert set(np.nonzero(tier == 1)[0]) == set(order[:n_s])
+
+
+def test_rank_hand_values():
+    recs = []
+    checks = []
+    for row in _rows("rank_hand.txt"):
+        tag, *rest = row.split()
+        if tag == "rec":
+            recs.append(list(map(int, rest)))
+        else:
+            checks.append((tag, rest))
+    a = np.array(recs)
+    rec = synth.Records(a[:, 1].astype(np.uint32), np.zeros(len(a), np.uint32), np.zeros(len(a), np.uint16),
+                        a[:, 3].astype(np.uint32), a[:, 2].astype(np.uint8), a[:, 4].astype(np.uint8))
+    sig = np.full(51, 4095, np.uint16)
+    for tag, rest in checks:
+        if tag == "victims":
+            k = int(rest[0])
+            out = oracle.rank(rec, sig, 5 * 10 ** 8, k, 0, 1, 0, 0)
+            assert list(map(int, out["victims"])) == list(map(int, rest[2:]))
+        else:
+            parts = " ".join(rest).split(":")
+            budget, fs, fh = map(int, parts[0].split())
+            pro = list(map(int, parts[1].split()[1:]))
+            dem = list(map(int, parts[2].split()[1:]))
+            moved = int(parts[3].split()[1])
+            out = oracle.rank(rec, sig, 5 * 10 ** 8, 1, budget, 1, fs, fh)
+            assert list(map(int, out["promote"])) == pro
+            assert list(map(int, out["demote"])) == dem
+            assert out["moved_bytes"] == moved
+
+
+def test_rank_victims_are_sorted_topk():
+    rec = synth.make_records(12, 5000)
+    _, sig = oracle.hazard_lut(synth.geometric_turns(1, 1415, 23.7, 2, 200))
+    out = oracle.rank(rec, sig, 5 * 10 ** 8, 300, 0, 131072, 0, 0, keys=True)
+    keys = out["keys"]
+    cand = [i for i in range(rec.n) if not (rec.flags[i] & 1)]
+    best = sorted(cand, key=lambda i: (-int(keys[i]), i))[:300]
+    assert list(map(int, out["victims"])) == best
+    done = (rec.flags & 2) != 0
+    assert (keys[done] == 2 ** 64 - 1).all()
+
+
+# ------------------------------------------------------------ invariance ----
+
+def test_time_shift_invariance():
+    tr = synth.tiny_trace(6)
+    p = dict(policy="spear_tide", cap_s_bytes=512 << 20, cap_h_bytes=8 << 30, kv_bytes_per_token=28672)
+    a = oracle.replay(tr, p, log=True)
+    sh = synth.Trace(tr.turn_off, tr.arrival_us + np.uint64(3 << 32), tr.completion_us + np.uint64(3 << 32),
+                     tr.in_tok, tr.out_tok)
+    b = oracle.replay(sh, p, log=True)
+    assert a["decision_hash"] == b["decision_hash"] and a["ttft_sum"] == b["ttft_sum"]
+
+
+def test_trace_validation_rejects_bad_input():
+    tr = synth.tiny_trace(0)
+    bad = synth.Trace(tr.turn_off, tr.arrival_us.copy(), tr.completion_us.copy(), tr.in_tok, tr.out_tok)
+    bad.completion_us[3] = bad.arrival_us[3]  # zero-length turn
+    assert oracle.replay(bad, {})["status"] == -3
+    gap = synth.Trace(tr.turn_off, tr.arrival_us.copy(), tr.completion_us.copy(), tr.in_tok, tr.out_tok)
+    gap.arrival_us[5:12] += np.uint64(1 << 31)
+    gap.completion_us[5:12] += np.uint64(1 << 31)
+    assert oracle.replay(gap, {})["status"] == -4
+    assert oracle.replay(tr, dict(ttl_us=1 << 31, policy="timeout"))["status"] == -1
+
+
+def test_log_overflow_is_reported():
+    tr = synth.tiny_trace(0)
+    r = oracle.replay(tr, dict(cap_s_bytes=512 << 20, cap_h_bytes=8 << 30, kv_bytes_per_token=28672),
+                      log=True, log_capacity=10)
+    assert r["status"] == -7 and r["log_len"] > 10
+
+
+def test_kendall_brute_matches_scipy():
+    stats = pytest.importorskip("scipy.stats")
+    rs = np.random.default_rng(1)
+    for n in (5, 50, 400):
+        x = rs.integers(0, 20, n).astype(float)
+        y = x + rs.normal(0, 3, n).round()
+        assert abs(oracle.kendall_brute(x, y) - stats.kendalltau(x, y).statistic) < 1e-12
