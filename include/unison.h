@@ -1,0 +1,303 @@
+/*
+ * unison.h -- C ABI of the GB300 implementation of UNISON's shared live
+ * ranking (SPEAR score + TIDE fill) and its batched trace replay.
+ *
+ * Method: UNISON (arXiv 2609.09643).  Sec. III-A (problem statement:
+ * sessions, turns, gaps, tiers, capacities, eqs. gap, reuse, cap), Sec. III-B
+ * (SPEAR score, eqs. ema, hazard, surv, esp), Sec. III-C (TIDE, eqs. budget,
+ * promote, demote), Sec. III-D (Algorithm 1, the joint event loop), Sec. IV-C
+ * (the integer contract, eqs. uq, hq, survq, gapq, t1, t2, scoreq, ema-int,
+ * lock) and Sec. V-A (metrics, eqs. hr-amat, prered, br).
+ *
+ * Conventions for every entry point:
+ *  - Every function returns an int status: UNISON_OK (0) or a negative
+ *    UNISON_ERR_* code.  Nothing aborts, traps or throws; a device-side
+ *    problem is reported through the per-replay / per-set status word.
+ *  - "host" pointers are ordinary CPU memory read during the call only;
+ *    "device" pointers are CUDA global memory owned by the caller and must
+ *    stay valid until the work queued on the stream has finished.
+ *  - cuda_stream is a cudaStream_t (NULL = the legacy default stream).  Work
+ *    is queued asynchronously on it, except where a host output is
+ *    requested, in which case the call synchronises that stream.
+ *  - Handles (unison_trace) are thread-compatible, not thread-safe.
+ *  - Times are microseconds.  On the device they are 32-bit and wrap modulo
+ *    2^32; every duration is a wrapping difference, which is exact because a
+ *    loaded trace never has two consecutive events, a turn or a gap 2^31 us
+ *    or more apart.
+ */
+#ifndef UNISON_H
+#define UNISON_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---------------------------------------------------------------- status */
+enum {
+  UNISON_OK = 0,
+  UNISON_ERR_ARG = -1,      /* null pointer, bad enum, inconsistent sizes      */
+  UNISON_ERR_IO = -2,       /* file could not be opened or read                */
+  UNISON_ERR_FORMAT = -3,   /* trace breaks its ordering rules                 */
+  UNISON_ERR_RANGE = -4,    /* value beyond a documented limit (2^31 us gaps,  */
+                            /* 2^24 sessions, 2^32 penalty, ...)               */
+  UNISON_ERR_CUDA = -5,     /* a CUDA runtime call failed                      */
+  UNISON_ERR_OOM = -6,      /* host or device allocation failed                */
+  UNISON_ERR_LOG_FULL = -7, /* decision log capacity exceeded (replay goes on, */
+                            /* counters and hash stay exact)                   */
+  UNISON_ERR_TIMEOUT = -8,  /* a bounded device wait gave up                   */
+  UNISON_ERR_CAPACITY = -9  /* internal resident-list bound exceeded           */
+};
+
+/* Human-readable text for a status code (static storage, never NULL). */
+const char *unison_strerror(int code);
+
+/* ABI version: major * 10000 + minor * 100 + patch. */
+int unison_version(void);
+
+/* ================================================================ traces */
+/*
+ * A trace is a set of agent sessions (Sec. III-A): session s has T_s turns;
+ * turn k arrives at a_{s,k}, completes at c_{s,k}, needs in_tok tokens of
+ * KV (l^in) and leaves out_tok resident (l^out, the prefix the next turn
+ * reuses).  The tool gap before turn k is g_{s,k} = a_{s,k} - c_{s,k-1}
+ * (eq. gap).
+ *
+ * Layout of unison_turns (host, caller-owned, read during the call):
+ *   turn_off[n_sessions+1]  session s owns turns [turn_off[s], turn_off[s+1])
+ *   arrival_us, completion_us [n_turns]  absolute times, u64 microseconds
+ *   in_tok, out_tok [n_turns]
+ * Rules (UNISON_ERR_FORMAT / _RANGE otherwise): 1 <= T_s < 65536;
+ * n_sessions < 2^24 - 1; n_turns < 2^31; sessions are numbered in order of
+ * first arrival; within a session a_k < c_k < a_{k+1}; c_k - a_k, gaps and
+ * the spacing of consecutive events (in event order) are below 2^31 us;
+ * 0 < in_tok_k <= out_tok_k and in_tok_k >= out_tok_{k-1}.
+ *
+ * Event order (a reading; the paper does not fix ties): by time, then
+ * completions before arrivals, then session id.  A completion of a
+ * non-final turn is a gap_start, an arrival of turn k >= 1 a gap_end
+ * (Algorithm 1).
+ */
+typedef struct {
+  uint32_t n_sessions;
+  uint32_t reserved;
+  uint64_t n_turns;
+  const uint64_t *turn_off;
+  const uint64_t *arrival_us;
+  const uint64_t *completion_us;
+  const uint32_t *in_tok;
+  const uint32_t *out_tok;
+} unison_turns;
+
+typedef struct unison_trace unison_trace; /* opaque, library-owned */
+
+/* Validate and order a trace on the host (events, per-turn event indices,
+ * next-arrival indices).  *out receives a new handle; free it with
+ * unison_trace_free.  No device memory is touched. */
+int unison_trace_create(const unison_turns *turns, unison_trace **out);
+
+/* Read a .utr file (little endian: "UTR1", u32 n_sessions, u64 n_turns,
+ * u64 turn_off[S+1], u64 arrival[T], u64 completion[T], u32 in[T],
+ * u32 out[T]) and create a trace from it. */
+int unison_trace_load(const char *path, unison_trace **out);
+
+/* Copy the trace's event arrays to device memory owned by the handle
+ * (allocated on first upload, reused afterwards), asynchronously on
+ * cuda_stream from page-locked host staging.  Must precede replay. */
+int unison_trace_upload(unison_trace *tr, void *cuda_stream);
+
+/* Release host and device memory of a trace (synchronises the device
+ * memory's last stream).  NULL is ignored. */
+void unison_trace_free(unison_trace *tr);
+
+/* Sizes of a trace; any output pointer may be NULL. */
+int unison_trace_info(const unison_trace *tr, uint32_t *n_sessions, uint64_t *n_turns,
+                      uint64_t *n_events);
+
+/* Bytes the last upload copied host-to-device for this trace. */
+uint64_t unison_trace_device_bytes(const unison_trace *tr);
+
+/* ================================================================ replay */
+typedef enum {
+  UNISON_LRU = 0,        /* recency (Tab. main baseline)                       */
+  UNISON_TIMEOUT = 1,    /* recency plus expiry of sessions idle >= ttl_us     */
+  UNISON_SPEAR = 2,      /* SPEAR eviction only (Sec. III-B)                   */
+  UNISON_SPEAR_TIDE = 3, /* UNISON: SPEAR + TIDE (Algorithm 1)                 */
+  UNISON_BELADY = 4,     /* offline oracle: farthest next arrival (Sec. III-A) */
+  UNISON_LRU_TIDE = 5    /* recency keys with TIDE migration (ablation)        */
+} unison_policy;
+
+/* Per-replay parameters (host array in unison_replay_batch). */
+typedef struct {
+  uint32_t policy;             /* unison_policy                                   */
+  uint32_t trace_idx;          /* index into the traces[] argument                */
+  uint64_t cap_fast_bytes;     /* C_S of eq. (cap), bytes                         */
+  uint64_t cap_hbm_bytes;      /* C_H of eq. (cap), bytes                         */
+  uint32_t kv_bytes_per_token; /* 1 .. 2^24; capacities count whole tokens        */
+  uint32_t max_sessions;       /* N_sess of eq. (cap); 0 = no slot limit          */
+  uint32_t ema_num, ema_den;   /* gap-average weight, eq. (ema-int): (3,10);      */
+                               /* a window W reads as (2, W+1)                    */
+  uint32_t hazard_bucket;      /* turns pooled per hazard entry; 1 = eq. (hazard) */
+  uint32_t ttl_us;             /* Timeout idle limit < 2^31; 0xFFFFFFFF = none    */
+  uint64_t penalty_q;          /* P_Z of eq. (t2), < 2^32; 5e8 = eq. (lock)       */
+  uint64_t dma_bytes_per_us;   /* TIDE budget rate B (eq. budget) in bytes/us,    */
+                               /* < 2^32                                          */
+  uint64_t t_s_ps_per_tok;     /* AMAT per-token costs (eq. hr-amat), picoseconds */
+  uint64_t t_h_ps_per_tok;
+  uint64_t t_p_ps_per_tok;     /* prefill cost; TTFT uses t_p / 1000 ns per token */
+  uint32_t ttft_load;          /* arrival compression factor of the TTFT queue    */
+  uint32_t reserved;
+} unison_replay_params;
+
+/* Per-replay counters (written by the device). */
+typedef struct {
+  uint64_t events, req_warm, cold, hit_s, hit_h, miss, bypass, place_s, place_h;
+  uint64_t evict, demote, promote, tide_demote, expire;
+  uint64_t tok_hit_s, tok_hit_h, tok_miss; /* sums of l_i = l^out_{k-1} per class */
+  uint64_t tok_computed, tok_needed;       /* prefill tokens vs tokens needed (warm) */
+  uint64_t dma_bytes, tide_calls, promoted_then_hit_s;
+  uint64_t ttft_sum_lo, ttft_sum_hi;       /* 128-bit sum of TTFT, ns              */
+  uint64_t ttft_p50_ns, ttft_n;            /* lower median over all requests       */
+  uint64_t decision_hash;                  /* see UNISON_KIND_* below              */
+  uint64_t log_len;                        /* decisions made (logged or not)       */
+  int32_t status;
+  uint32_t reserved;
+} unison_replay_result;
+
+/* Decision kinds.  Each decision is logged as {event index, kind << 24 |
+ * session}; decision_hash folds the stream in order, starting from
+ * 0xCBF29CE484222325 and applying h = (h ^ w) * 0x100000001B3 (mod 2^64)
+ * with w = event << 32 | kind << 24 | session.  Within one event the order
+ * is: expiries (ascending session), the request class, then placement
+ * decisions in the order they are taken, or the TIDE moves. */
+enum {
+  UNISON_KIND_COLD = 0, UNISON_KIND_HIT_S = 1, UNISON_KIND_HIT_H = 2, UNISON_KIND_MISS = 3,
+  UNISON_KIND_PLACE_S = 4, UNISON_KIND_PLACE_H = 5, UNISON_KIND_BYPASS = 6,
+  UNISON_KIND_DEMOTE = 7, UNISON_KIND_EVICT = 8, UNISON_KIND_PROMOTE = 9,
+  UNISON_KIND_TIDE_DEMOTE = 10, UNISON_KIND_EXPIRE = 11
+};
+typedef struct {
+  uint32_t event;
+  uint32_t kind_session;
+} unison_decision;
+
+/*
+ * Replay n_replays independent (trace, policy, parameters) combinations,
+ * each one a literal run of Algorithm 1 over its trace's events:
+ *  - gap_end: EMA update of the session's gap average (eq. ema-int);
+ *  - every decision ranks the live sessions by one total order: larger key
+ *    is more evictable, ties go to the smaller session id.  SPEAR keys are
+ *    score_q (eq. scoreq; a completed session has the maximal key) from the
+ *    offline hazard table fitted on the trace (Sec. V-E);
+ *  - placement when a request arrives: the session leaves its tier and is
+ *    placed in the fast tier if its l^out fits beside the pinned sessions,
+ *    demoting the most evictable unpinned fast-tier sessions into HBM
+ *    (where each displaces the most evictable unpinned HBM session, or is
+ *    dropped itself if it is the most evictable); else in HBM, evicting the
+ *    most evictable unpinned HBM sessions; else it is served and not kept.
+ *    With max_sessions > 0, the global most evictable resident is evicted
+ *    while the slot limit is exceeded.  A session is pinned from its
+ *    arrival to its completion and never moved while pinned;
+ *  - gap_start with TIDE and the DMA free: budget = g_q * dma_bytes_per_us
+ *    (eq. budget); first the least evictable HBM sessions are promoted into
+ *    free fast-tier space, then pairs (argmin over HBM, argmax over the
+ *    fast tier; eqs. promote, demote) are swapped while the demoted one is
+ *    strictly more evictable, the pair fits the remaining budget and both
+ *    tiers stay within capacity.  The DMA is then busy for
+ *    ceil(moved / dma_bytes_per_us) us.
+ *
+ * traces[n_traces]: uploaded handles (host array of pointers).
+ * params[n_replays]: host array.
+ * results_dev: device array [n_replays] written by the device (may be NULL
+ *   if results_host is given).
+ * results_host: host array [n_replays]; if non-NULL the call copies the
+ *   results back and synchronises cuda_stream.
+ * log_dev: device array [n_replays * log_capacity_per_replay] or NULL; replay
+ *   r writes its decisions at log_dev + r * log_capacity_per_replay and sets
+ *   status UNISON_ERR_LOG_FULL if it makes more.
+ * Scratch (key streams, TTFT values, descriptors) is allocated
+ * stream-ordered on cuda_stream and released before the call returns its
+ * work to the stream.
+ */
+int unison_replay_batch(const unison_trace *const *traces, int n_traces,
+                        const unison_replay_params *params, int n_replays,
+                        unison_replay_result *results_dev, unison_replay_result *results_host,
+                        unison_decision *log_dev, uint64_t log_capacity_per_replay,
+                        void *cuda_stream);
+
+/* Host-side summary of one replay (Sec. V-A): hit rate HR = (H_S + H_H)/R,
+ * AMAT = (t_s sum_S + t_h sum_H + t_p sum_M)/R in ps (eq. hr-amat), prefill
+ * reduction 1 - computed/needed (eq. prered), prefetch accuracy = promoted
+ * sessions whose next request hit the fast tier / promotions, TTFT mean and
+ * p50 in ns.  Ratios with an empty denominator are 0. */
+typedef struct {
+  double hit_rate, amat_ps, prered, prefetch_acc, ttft_mean_ns, ttft_p50_ns;
+} unison_stats_t;
+int unison_stats(const unison_replay_result *r, const unison_replay_params *p, unison_stats_t *out);
+
+/* ============================================================ hazard LUT */
+/* The survival table of eqs. (hazard), (hq), (survq) built on the device
+ * from turns-per-session counts: n(t) = #{T_s >= t+1}, d(t) = #{T_s = t+1}
+ * for t = 0..50, pooled over buckets of `bucket` consecutive turns,
+ * h_q = round-half-up(4095 d / n) (0 where n = 0), sigma_q = max(41,
+ * 4095 - h_q).  turns_dev: device u32[n_sessions]; sigma_q_dev: device
+ * u16[51] output (h_q_dev, device u16[51], may be NULL). */
+int unison_hazard_lut(const uint32_t *turns_dev, uint64_t n_sessions, uint32_t bucket,
+                      uint16_t *sigma_q_dev, uint16_t *h_q_dev, void *cuda_stream);
+
+/* ================================================================ ranking */
+/* A live set of n session records, structure of arrays, device memory
+ * (caller-owned).  gap_q: gap average in us (eq. gapq, < 2^31); last_ret:
+ * last completion time (carried, not read by the score); turn: register turn
+ * t; kv_tok: resident tokens; tier: 1 fast, 2 HBM, other = not resident;
+ * flags: bit0 pinned (mid-turn), bit1 done (completed session).  n < 2^31. */
+typedef struct {
+  const uint32_t *gap_q;
+  const uint32_t *last_ret;
+  const uint16_t *turn;
+  const uint32_t *kv_tok;
+  const uint8_t *tier;
+  const uint8_t *flags;
+  uint64_t n;
+} unison_records;
+
+typedef struct {
+  uint16_t sigma_q[51];        /* survival table (unison_hazard_lut), host copy  */
+  uint16_t reserved0;
+  uint32_t k;                  /* victims wanted, 0 .. 4096                      */
+  uint64_t penalty_q;          /* P_Z, < 2^32                                    */
+  uint64_t budget_bytes;       /* TIDE budget for this set                       */
+  uint32_t kv_bytes_per_token; /* 1 .. 2^24                                      */
+  uint32_t max_moves;          /* capacity of promote[] and demote[]             */
+  uint64_t free_fast_tok;      /* free fast-tier capacity, tokens                */
+  uint64_t free_hbm_tok;       /* free HBM capacity, tokens                      */
+} unison_rank_params;
+
+/* Device outputs of one set (caller-owned). */
+typedef struct {
+  uint32_t *victims;     /* [k]: most evictable unpinned resident records first */
+  uint32_t *promote;     /* [max_moves]: HBM -> fast, in move order             */
+  uint32_t *demote;      /* [max_moves]: fast -> HBM, paired with promotions    */
+                         /* after the free-space promotions                     */
+  uint32_t *counts;      /* [4]: n_victims, n_promote, n_demote, status         */
+  uint64_t *moved_bytes; /* [1]                                                 */
+  uint64_t *keys;        /* [n] score_q of every record, or NULL                */
+} unison_rank_out;
+
+/*
+ * Rank n_sets live sets in one pass over their records (the scan of
+ * eq. pipe/scan with the victim argmax generalised to a top-k, and one TIDE
+ * fill per set with the selections of eqs. promote/demote).  Keys are
+ * score_q (eq. scoreq); order as in replay (larger key, then smaller index,
+ * is more evictable).  Results are exact: candidate thresholds come from a
+ * sample, and a set whose candidates fall short is re-selected exactly on
+ * the device.  sets, params, outs: host arrays [n_sets].  Asynchronous.
+ */
+int unison_rank_batch(const unison_records *sets, const unison_rank_params *params,
+                      const unison_rank_out *outs, int n_sets, void *cuda_stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* UNISON_H */

@@ -1,0 +1,279 @@
+"""Thin ctypes binding of include/unison.h (argument marshalling only).
+
+Every computation runs in libunison.so's CUDA kernels; this module turns
+numpy/torch objects into the C structs and pointers the ABI takes.  If the
+library is missing the calls raise; there is no CPU path.
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+import threading
+from typing import Iterable, List, Sequence
+
+import numpy as np
+
+from .native import LIB
+
+POLICY = {"lru": 0, "timeout": 1, "spear": 2, "spear_tide": 3, "belady": 4, "lru_tide": 5}
+KIND = ["COLD", "HIT_S", "HIT_H", "MISS", "PLACE_S", "PLACE_H", "BYPASS", "DEMOTE", "EVICT",
+        "PROMOTE", "TIDE_DEMOTE", "EXPIRE"]
+OK, ERR_ARG, ERR_IO, ERR_FORMAT, ERR_RANGE, ERR_CUDA, ERR_OOM, ERR_LOG_FULL, ERR_TIMEOUT, ERR_CAPACITY = \
+    0, -1, -2, -3, -4, -5, -6, -7, -8, -9
+
+DEFAULT_PARAMS = dict(
+    policy="spear_tide", cap_fast_bytes=4 << 30, cap_hbm_bytes=64 << 30, kv_bytes_per_token=131072,
+    max_sessions=0, ema_num=3, ema_den=10, hazard_bucket=1, ttl_us=10_000_000,
+    penalty_q=500_000_000, dma_bytes_per_us=64_000, t_s_ps_per_tok=8192, t_h_ps_per_tok=32768,
+    t_p_ps_per_tok=20_000_000, ttft_load=4,
+)
+
+
+class UnisonError(RuntimeError):
+    def __init__(self, where: str, code: int):
+        super().__init__(f"{where}: {strerror(code)} ({code})")
+        self.code = code
+
+
+class Turns(C.Structure):
+    _fields_ = [("n_sessions", C.c_uint32), ("reserved", C.c_uint32), ("n_turns", C.c_uint64),
+                ("turn_off", C.c_void_p), ("arrival_us", C.c_void_p), ("completion_us", C.c_void_p),
+                ("in_tok", C.c_void_p), ("out_tok", C.c_void_p)]
+
+
+class ReplayParams(C.Structure):
+    _fields_ = [("policy", C.c_uint32), ("trace_idx", C.c_uint32), ("cap_fast_bytes", C.c_uint64),
+                ("cap_hbm_bytes", C.c_uint64), ("kv_bytes_per_token", C.c_uint32),
+                ("max_sessions", C.c_uint32), ("ema_num", C.c_uint32), ("ema_den", C.c_uint32),
+                ("hazard_bucket", C.c_uint32), ("ttl_us", C.c_uint32), ("penalty_q", C.c_uint64),
+                ("dma_bytes_per_us", C.c_uint64), ("t_s_ps_per_tok", C.c_uint64),
+                ("t_h_ps_per_tok", C.c_uint64), ("t_p_ps_per_tok", C.c_uint64),
+                ("ttft_load", C.c_uint32), ("reserved", C.c_uint32)]
+
+
+RESULT_FIELDS = ["events", "req_warm", "cold", "hit_s", "hit_h", "miss", "bypass", "place_s", "place_h",
+                 "evict", "demote", "promote", "tide_demote", "expire", "tok_hit_s", "tok_hit_h",
+                 "tok_miss", "tok_computed", "tok_needed", "dma_bytes", "tide_calls",
+                 "promoted_then_hit_s", "ttft_sum_lo", "ttft_sum_hi", "ttft_p50_ns", "ttft_n",
+                 "decision_hash", "log_len"]
+
+
+class ReplayResult(C.Structure):
+    _fields_ = [(f, C.c_uint64) for f in RESULT_FIELDS] + [("status", C.c_int32), ("reserved", C.c_uint32)]
+
+
+class Stats(C.Structure):
+    _fields_ = [(f, C.c_double) for f in ("hit_rate", "amat_ps", "prered", "prefetch_acc", "ttft_mean_ns",
+                                          "ttft_p50_ns")]
+
+
+class Records(C.Structure):
+    _fields_ = [("gap_q", C.c_void_p), ("last_ret", C.c_void_p), ("turn", C.c_void_p), ("kv_tok", C.c_void_p),
+                ("tier", C.c_void_p), ("flags", C.c_void_p), ("n", C.c_uint64)]
+
+
+class RankParams(C.Structure):
+    _fields_ = [("sigma_q", C.c_uint16 * 51), ("reserved0", C.c_uint16), ("k", C.c_uint32),
+                ("penalty_q", C.c_uint64), ("budget_bytes", C.c_uint64), ("kv_bytes_per_token", C.c_uint32),
+                ("max_moves", C.c_uint32), ("free_fast_tok", C.c_uint64), ("free_hbm_tok", C.c_uint64)]
+
+
+class RankOut(C.Structure):
+    _fields_ = [("victims", C.c_void_p), ("promote", C.c_void_p), ("demote", C.c_void_p),
+                ("counts", C.c_void_p), ("moved_bytes", C.c_void_p), ("keys", C.c_void_p)]
+
+
+_lock = threading.Lock()
+_lib = None
+
+# Every symbol include/unison.h declares (checked by the ABI tests).
+EXPORTS = ["unison_strerror", "unison_version", "unison_trace_create", "unison_trace_load",
+           "unison_trace_upload", "unison_trace_free", "unison_trace_info", "unison_trace_device_bytes",
+           "unison_replay_batch", "unison_stats", "unison_hazard_lut", "unison_rank_batch"]
+
+
+def lib_path() -> str:
+    return LIB
+
+
+def lib():
+    """Load libunison.so (built by paper_2609_09643_gb300.native.build())."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB):
+                raise RuntimeError(f"{LIB} is missing: run __graft_entry__.build() first")
+            L = C.CDLL(LIB)
+            L.unison_strerror.restype = C.c_char_p
+            L.unison_strerror.argtypes = [C.c_int]
+            L.unison_version.restype = C.c_int
+            L.unison_trace_create.argtypes = [C.POINTER(Turns), C.POINTER(C.c_void_p)]
+            L.unison_trace_load.argtypes = [C.c_char_p, C.POINTER(C.c_void_p)]
+            L.unison_trace_upload.argtypes = [C.c_void_p, C.c_void_p]
+            L.unison_trace_free.argtypes = [C.c_void_p]
+            L.unison_trace_free.restype = None
+            L.unison_trace_info.argtypes = [C.c_void_p, C.POINTER(C.c_uint32), C.POINTER(C.c_uint64),
+                                            C.POINTER(C.c_uint64)]
+            L.unison_trace_device_bytes.argtypes = [C.c_void_p]
+            L.unison_trace_device_bytes.restype = C.c_uint64
+            L.unison_replay_batch.argtypes = [C.POINTER(C.c_void_p), C.c_int, C.POINTER(ReplayParams), C.c_int,
+                                              C.c_void_p, C.POINTER(ReplayResult), C.c_void_p, C.c_uint64,
+                                              C.c_void_p]
+            L.unison_stats.argtypes = [C.POINTER(ReplayResult), C.POINTER(ReplayParams), C.POINTER(Stats)]
+            L.unison_hazard_lut.argtypes = [C.c_void_p, C.c_uint64, C.c_uint32, C.c_void_p, C.c_void_p,
+                                            C.c_void_p]
+            L.unison_rank_batch.argtypes = [C.POINTER(Records), C.POINTER(RankParams), C.POINTER(RankOut), C.c_int,
+                                            C.c_void_p]
+            _lib = L
+    return _lib
+
+
+def strerror(code: int) -> str:
+    try:
+        return lib().unison_strerror(code).decode()
+    except RuntimeError:
+        return f"status {code}"
+
+
+def _check(where: str, rc: int, allow=(OK,)):
+    if rc not in allow:
+        raise UnisonError(where, rc)
+    return rc
+
+
+def _stream_handle(stream) -> int | None:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    return getattr(stream, "cuda_stream", stream)
+
+
+# ------------------------------------------------------------------ traces --
+class Trace:
+    """Owner of a unison_trace handle built from host turn arrays (any object
+    with turn_off, arrival_us, completion_us, in_tok, out_tok)."""
+
+    def __init__(self, turns=None, path: str | None = None):
+        h = C.c_void_p()
+        if path is not None:
+            _check("unison_trace_load", lib().unison_trace_load(path.encode(), C.byref(h)))
+        else:
+            arrs = (np.ascontiguousarray(turns.turn_off, np.uint64), np.ascontiguousarray(turns.arrival_us, np.uint64),
+                    np.ascontiguousarray(turns.completion_us, np.uint64), np.ascontiguousarray(turns.in_tok, np.uint32),
+                    np.ascontiguousarray(turns.out_tok, np.uint32))
+            t = Turns(arrs[0].shape[0] - 1, 0, arrs[1].shape[0], *(a.ctypes.data for a in arrs))
+            _check("unison_trace_create", lib().unison_trace_create(C.byref(t), C.byref(h)))
+        self.handle = h
+        self.uploaded = False
+
+    def upload(self, stream=None) -> "Trace":
+        _check("unison_trace_upload", lib().unison_trace_upload(self.handle, _stream_handle(stream)))
+        self.uploaded = True
+        return self
+
+    def info(self):
+        s, t, e = C.c_uint32(), C.c_uint64(), C.c_uint64()
+        _check("unison_trace_info", lib().unison_trace_info(self.handle, C.byref(s), C.byref(t), C.byref(e)))
+        return int(s.value), int(t.value), int(e.value)
+
+    @property
+    def device_bytes(self) -> int:
+        return int(lib().unison_trace_device_bytes(self.handle))
+
+    def close(self):
+        if self.handle:
+            lib().unison_trace_free(self.handle)
+            self.handle = C.c_void_p()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def make_params(p: dict, trace_idx: int = 0) -> ReplayParams:
+    q = dict(DEFAULT_PARAMS)
+    q.update(p)
+    pol = q["policy"]
+    pol = POLICY[pol] if isinstance(pol, str) else int(pol)
+    return ReplayParams(pol, q.get("trace_idx", trace_idx), q["cap_fast_bytes"], q["cap_hbm_bytes"],
+                        q["kv_bytes_per_token"], q["max_sessions"], q["ema_num"], q["ema_den"],
+                        q["hazard_bucket"], q["ttl_us"], q["penalty_q"], q["dma_bytes_per_us"],
+                        q["t_s_ps_per_tok"], q["t_h_ps_per_tok"], q["t_p_ps_per_tok"], q["ttft_load"], 0)
+
+
+def result_dict(r: ReplayResult) -> dict:
+    d = {f: int(getattr(r, f)) for f in RESULT_FIELDS}
+    d["status"] = int(r.status)
+    d["ttft_sum"] = d["ttft_sum_lo"] + (d["ttft_sum_hi"] << 64)
+    return d
+
+
+def replay_batch(traces: Sequence[Trace], params: Sequence[dict], log_capacity: int = 0, stream=None,
+                 results_dev=None, allow_status=(OK, ERR_LOG_FULL)):
+    """Run unison_replay_batch.  Returns (list of result dicts, log) where log
+    is a torch uint32 tensor [n_replays, log_capacity, 2] on the GPU or None."""
+    import torch
+    n = len(params)
+    arr_t = (C.c_void_p * len(traces))(*(t.handle.value for t in traces))
+    arr_p = (ReplayParams * n)(*(make_params(p) for p in params))
+    out = (ReplayResult * n)()
+    log = None
+    if log_capacity:
+        log = torch.zeros((n, log_capacity, 2), dtype=torch.int32, device="cuda")
+    rc = lib().unison_replay_batch(arr_t, len(traces), arr_p, n,
+                                   None if results_dev is None else results_dev.data_ptr(), out,
+                                   None if log is None else log.data_ptr(), log_capacity, _stream_handle(stream))
+    _check("unison_replay_batch", rc)
+    res = [result_dict(out[i]) for i in range(n)]
+    for i, r in enumerate(res):
+        if r["status"] not in allow_status:
+            raise UnisonError(f"replay {i}", r["status"])
+    return res, log
+
+
+def replay_batch_async(traces: Sequence[Trace], params: Sequence[dict], results_dev, stream=None, log=None,
+                       log_capacity: int = 0):
+    """Queue unison_replay_batch with device results only (no host sync)."""
+    n = len(params)
+    arr_t = (C.c_void_p * len(traces))(*(t.handle.value for t in traces))
+    arr_p = (ReplayParams * n)(*(make_params(p) for p in params))
+    rc = lib().unison_replay_batch(arr_t, len(traces), arr_p, n, results_dev.data_ptr(), None,
+                                   None if log is None else log.data_ptr(), log_capacity, _stream_handle(stream))
+    _check("unison_replay_batch", rc)
+
+
+def results_from_tensor(t) -> List[dict]:
+    """Decode a device/host uint8/int64 tensor holding unison_replay_result[n]."""
+    b = t.detach().cpu().contiguous().view(-1).numpy().tobytes()
+    sz = C.sizeof(ReplayResult)
+    return [result_dict(ReplayResult.from_buffer_copy(b[i * sz:(i + 1) * sz])) for i in range(len(b) // sz)]
+
+
+def result_nbytes(n: int) -> int:
+    return n * C.sizeof(ReplayResult)
+
+
+def decode_log(log_row, n: int):
+    """(event, kind, session) numpy arrays of the first n decisions of one replay."""
+    a = log_row[:n].cpu().numpy().astype(np.uint32)
+    return a[:, 0].copy(), (a[:, 1] >> 24).astype(np.uint8), a[:, 1] & 0xFFFFFF
+
+
+def stats(result: dict, params: dict) -> dict:
+    r = ReplayResult(*[result[f] for f in RESULT_FIELDS], result.get("status", 0), 0)
+    p = make_params(params)
+    s = Stats()
+    _check("unison_stats", lib().unison_stats(C.byref(r), C.byref(p), C.byref(s)))
+    return {f: getattr(s, f) for f, _ in Stats._fields_}
+
+
+def hazard_lut(turns_dev, bucket: int = 1, stream=None):
+    """sigma_q[51] and h_q[51] (torch uint16-as-int16 tensors on the device)."""
+    import torch
+    sig = torch.zeros(51, dtype=torch.int16, device=turns_dev.device)
+    hq = torch.zeros(51, dtype=torch.int16, device=turns_dev.device)
+    _check("unison_hazard_lut", lib().unison_hazard_lut(turns_dev.data_ptr(), turns_dev.numel(), bucket,
+                                                        sig.data_ptr(), hq.data_ptr(), _stream_handle(stream)))
+    return sig, hq

@@ -1,0 +1,232 @@
+"""GPU parity of the batched replay against the CPU oracle.
+
+Bar: bit-exact on every decision (the full decision log where it is
+recorded, the decision hash otherwise) and on every counter, including the
+TTFT sum and median (integers here, so exact rather than 1e-6)."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from cases import GIB, MIB, base, to_lib, to_oracle, tiny_case, paper_scale_case, sweep_case, large_pool_params
+
+pytestmark = pytest.mark.gpu
+
+FIELDS = ["events", "req_warm", "cold", "hit_s", "hit_h", "miss", "bypass", "place_s", "place_h", "evict",
+          "demote", "promote", "tide_demote", "expire", "tok_hit_s", "tok_hit_h", "tok_miss", "tok_computed",
+          "tok_needed", "dma_bytes", "tide_calls", "promoted_then_hit_s", "ttft_sum", "ttft_p50_ns", "ttft_n",
+          "decision_hash", "log_len", "status"]
+
+
+@pytest.fixture(scope="module")
+def B():
+    from paper_2609_09643_gb300 import native
+    native.build()
+    from paper_2609_09643_gb300 import binding
+    return binding
+
+
+def run_gpu(B, traces, reps, log_capacity=0):
+    handles = [B.Trace(t).upload() for t in traces]
+    res, log = B.replay_batch(handles, [to_lib(p, ti) for ti, p in reps], log_capacity=log_capacity)
+    return res, log, handles
+
+
+def assert_same(g, o, what=""):
+    for f in FIELDS:
+        assert g[f] == o[f], (what, f, g[f], o[f])
+
+
+def assert_same_log(B, log_row, g, o, what=""):
+    n = min(g["log_len"], log_row.shape[0])
+    ge, gk, gs = B.decode_log(log_row, n)
+    oe, ok, os_ = o["log"]
+    assert n == len(oe), (what, n, len(oe))
+    bad = np.nonzero((ge != oe) | (gk != ok) | (gs != os_))[0]
+    assert bad.size == 0, (what, int(bad[0]), (ge[bad[0]], gk[bad[0]], gs[bad[0]]), (oe[bad[0]], ok[bad[0]], os_[bad[0]]))
+
+
+def test_tiny_all_policies_full_logs(B):
+    tr, _ = tiny_case()
+    pols = ["lru", "timeout", "spear", "spear_tide", "belady", "lru_tide"]
+    reps = [(0, base(p, 512 * MIB, 8 * GIB, 28672)) for p in pols]
+    cap = 8 * tr.n_events
+    res, log, _ = run_gpu(B, [tr], reps, log_capacity=cap)
+    for i, (ti, p) in enumerate(reps):
+        o = oracle.replay(tr, to_oracle(p), log=True, log_capacity=cap)
+        assert_same(res[i], o, p["policy"])
+        assert_same_log(B, log[i], res[i], o, p["policy"])
+
+
+def test_hand_trace_on_device(B):
+    from test_oracle_pins import _hand_trace
+    tr, log, counts = _hand_trace("replay_hand_spear.txt")
+    p = base("spear", 100, 100, 1, t_p=20_000_000)
+    res, lg, _ = run_gpu(B, [tr], [(0, p)], log_capacity=64)
+    r = res[0]
+    got = list(zip(*(map(int, a) for a in B.decode_log(lg[0], r["log_len"]))))
+    assert got == log
+    for k, v in counts.items():
+        assert r[k] == v, k
+
+
+def test_paper_scale_30_replays(B):
+    trs, reps = paper_scale_case()
+    cap = 4 * trs[0].n_events
+    res, log, _ = run_gpu(B, trs, reps, log_capacity=cap)
+    for i, (ti, p) in enumerate(reps):
+        o = oracle.replay(trs[ti], to_oracle(p), log=(i % 6 == 0), log_capacity=cap)
+        assert_same(res[i], o, (ti, p["policy"], p["kvb"]))
+        if i % 6 == 0:
+            assert_same_log(B, log[i], res[i], o, (ti, p["policy"], p["kvb"]))
+
+
+def test_sweep_1024_replays_sampled(B):
+    """The benchmark's launch configuration: one call over all 1,024 replays;
+    a spread of replays is checked against the oracle one by one."""
+    trs, reps = sweep_case()
+    res, _, _ = run_gpu(B, trs, reps)
+    assert len(res) == 1024
+    assert all(r["status"] == 0 for r in res)
+    for i in list(range(0, 1024, 67)) + [1023]:
+        ti, p = reps[i]
+        assert_same(res[i], oracle.replay(trs[ti], to_oracle(p)), i)
+
+
+@pytest.mark.parametrize("seed", [100, 101])
+def test_large_pool_replay(B, seed):
+    tr = synth.large_pool_trace(seed)
+    p = large_pool_params()
+    res, _, _ = run_gpu(B, [tr], [(0, p)])
+    assert_same(res[0], oracle.replay(tr, to_oracle(p)), seed)
+
+
+POLS = ["lru", "timeout", "spear", "spear_tide", "belady", "lru_tide"]
+
+
+@pytest.mark.parametrize("caps", [(1 << 60, 1 << 60), (0, 0), (0, 16 * GIB), (2 * GIB, 0), (300 * MIB, 2 * GIB)])
+def test_capacity_edges(B, caps):
+    tr = synth.paper_scale_trace(5)
+    reps = [(0, base(p, caps[0], caps[1], 131072, ttl=0xFFFFFFFF if p == "timeout" else 10_000_000)) for p in POLS]
+    res, _, _ = run_gpu(B, [tr], reps)
+    for i, (_, p) in enumerate(reps):
+        assert_same(res[i], oracle.replay(tr, to_oracle(p)), (caps, p["policy"]))
+
+
+def test_slot_mode_small_traces(B):
+    from test_oracle_pins import _random_seqs, _slot_trace
+    trs, reps = [], []
+    for k, seq in enumerate(_random_seqs(40, 7)):
+        tr, _ = _slot_trace(seq)
+        trs.append(tr)
+        for slots in (1, 2, 3):
+            for pol in ("belady", "lru", "spear"):
+                reps.append((k, base(pol, 0, 1 << 60, 1, max_sessions=slots)))
+    res, _, _ = run_gpu(B, trs, reps)
+    for i, (ti, p) in enumerate(reps):
+        assert_same(res[i], oracle.replay(trs[ti], to_oracle(p)), (ti, p["policy"], p["max_sessions"]))
+
+
+@pytest.mark.parametrize("ttl", [0, 1, 2_000_000, 10_000_000, (1 << 31) - 1, 0xFFFFFFFF])
+def test_timeout_ttl(B, ttl):
+    tr = synth.paper_scale_trace(6)
+    p = base("timeout", 2 * GIB, 32 * GIB, 131072, ttl=ttl)
+    res, _, _ = run_gpu(B, [tr], [(0, p)])
+    assert_same(res[0], oracle.replay(tr, to_oracle(p)), ttl)
+
+
+@pytest.mark.parametrize("dma", [0, 1, 6400, 64000, (1 << 32) - 1])
+def test_tide_dma_rates(B, dma):
+    tr = synth.paper_scale_trace(7)
+    reps = [(0, base(pol, 2 * GIB, 32 * GIB, 131072, dma=dma)) for pol in ("spear_tide", "lru_tide")]
+    res, _, _ = run_gpu(B, [tr], reps)
+    for i, (_, p) in enumerate(reps):
+        assert_same(res[i], oracle.replay(tr, to_oracle(p)), (dma, p["policy"]))
+
+
+@pytest.mark.parametrize("bucket", [1, 3, 8, 64])
+def test_bimodal_hazard(B, bucket):
+    tr = synth.bimodal_trace(7)
+    reps = [(0, base(pol, 1 * GIB, 8 * GIB, 131072, bucket=bucket, ema_num=2, ema_den=9))
+            for pol in ("spear", "spear_tide")]
+    res, _, _ = run_gpu(B, [tr], reps)
+    for i, (_, p) in enumerate(reps):
+        assert_same(res[i], oracle.replay(tr, to_oracle(p)), (bucket, p["policy"]))
+
+
+def test_time_wrap(B):
+    """Times near 2^32 us wrap the device's 32-bit clock mid-trace."""
+    tr = synth.paper_scale_trace(8)
+    shift = np.uint64((1 << 32) - int(tr.arrival_us[len(tr.arrival_us) // 3]))
+    sh = synth.Trace(tr.turn_off, tr.arrival_us + shift, tr.completion_us + shift, tr.in_tok, tr.out_tok)
+    reps = [(0, base(pol, 2 * GIB, 32 * GIB, 131072, ttl=3_000_000)) for pol in POLS]
+    res, _, _ = run_gpu(B, [sh], reps)
+    for i, (_, p) in enumerate(reps):
+        o = oracle.replay(sh, to_oracle(p))
+        assert_same(res[i], o, p["policy"])
+        assert o["decision_hash"] == oracle.replay(tr, to_oracle(p))["decision_hash"]
+
+
+def test_global_list_path(B):
+    """Resident lists too large for shared memory live in global memory."""
+    tr = synth.make_trace(3, np.full(6000, 4), 0.01, synth.GAP_MIX_CODING)
+    reps = [(0, base(pol, 1 << 60, 1 << 60, 1024)) for pol in ("spear_tide", "lru")]
+    reps.append((0, base("spear_tide", 400 * MIB, 4 * GIB, 1024)))
+    res, _, _ = run_gpu(B, [tr], reps)
+    for i, (_, p) in enumerate(reps):
+        assert_same(res[i], oracle.replay(tr, to_oracle(p)), i)
+
+
+def test_many_sessions_search_path(B):
+    """More sessions than the shared-memory session map holds: residents are
+    found by a warp-wide search."""
+    tr = synth.make_trace(4, np.full(20000, 3), 0.005, synth.GAP_MIX_GENERAL)
+    reps = [(0, base(pol, 2 * GIB, 16 * GIB, 16384)) for pol in ("spear_tide", "belady", "timeout")]
+    res, _, _ = run_gpu(B, [tr], reps)
+    for i, (_, p) in enumerate(reps):
+        assert_same(res[i], oracle.replay(tr, to_oracle(p)), p["policy"])
+
+
+def test_log_overflow_reported(B):
+    tr, _ = tiny_case()
+    p = base("spear_tide", 512 * MIB, 8 * GIB, 28672)
+    res, _, _ = run_gpu(B, [tr], [(0, p)], log_capacity=10)
+    o = oracle.replay(tr, to_oracle(p), log=True, log_capacity=10)
+    assert res[0]["status"] == B.ERR_LOG_FULL == o["status"]
+    assert_same(res[0], o)
+
+
+def test_bad_params_rejected(B):
+    tr, _ = tiny_case()
+    h = [B.Trace(tr).upload()]
+    for bad in (dict(kv_bytes_per_token=0), dict(ema_num=11), dict(penalty_q=1 << 32), dict(ttl_us=1 << 31),
+                dict(policy=9), dict(trace_idx=3), dict(hazard_bucket=0)):
+        q = to_lib(base("spear", 1 * GIB, 8 * GIB, 28672))
+        q.update(bad)
+        with pytest.raises(B.UnisonError):
+            B.replay_batch(h, [q])
+
+
+def test_results_on_device_async(B):
+    import torch
+    trs, reps = paper_scale_case()
+    handles = [B.Trace(t).upload() for t in trs]
+    out = torch.zeros(B.result_nbytes(len(reps)), dtype=torch.uint8, device="cuda")
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        B.replay_batch_async(handles, [to_lib(p, ti) for ti, p in reps], out, stream=s)
+    s.synchronize()
+    got = B.results_from_tensor(out)
+    ref, _ = B.replay_batch(handles, [to_lib(p, ti) for ti, p in reps])
+    assert got == ref
+
+
+def test_hazard_lut_kernel(B):
+    import torch
+    for tps in (np.full(64, 12), synth.geometric_turns(3, 5000, 23.7, 2, 200), np.array([1, 2, 2, 3])):
+        t = torch.tensor(np.asarray(tps, dtype=np.int32), device="cuda")
+        for w in (1, 2, 8, 64):
+            sig, hq = B.hazard_lut(t, w)
+            oh, osig = oracle.hazard_lut(tps, w)
+            assert (sig.cpu().numpy().astype(np.uint16) == osig).all()
+            assert (hq.cpu().numpy().astype(np.uint16) == oh).all()
