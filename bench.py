@@ -1,0 +1,275 @@
+#!/usr/bin/env python3
+"""Benchmark of the UNISON hot path on GB300.
+
+One step = one batched replay of the parameter sweep (1,024 independent
+SPEAR+TIDE replays: 8 trace seeds x 8 tier-capacity pairs x 16 gap-window /
+hazard-bucket settings over the paper-scale coding trace, 131,072 B/token)
+plus one ranking pass over a 2^24-record live set (top-1024 victims and the
+TIDE fill).  Inputs are synthetic (see the synth package) and resident in HBM
+before the timed region; an L2 flush (a 256 MiB write) precedes each step.
+
+Prints one JSON line (rank 0).  --impl reference times the CPU oracle on a
+bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+sys.path.insert(0, os.path.join(ROOT, "tests"))
+
+METRIC = "replay events/s (SPEAR+TIDE batched)"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+# ---------------------------------------------------------------- clocks ----
+CLK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+class ClockSampler:
+    def __init__(self, device: int):
+        self.path = tempfile.mktemp(suffix=".csv")
+        self.proc = None
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(device), f"--query-gpu={CLK_FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for row in csv.reader(f):
+                if len(row) < 9:
+                    continue
+                try:
+                    sm.append(float(row[1]))
+                    mx = max(mx, float(row[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, row[5:9]):
+                    if v.strip().lower() == "active":
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------- workloads ----
+def sweep_workload(rank: int):
+    from cases import sweep_case, to_lib
+    trs, reps = sweep_case()
+    if rank:  # weak scaling: each rank replays its own seeds
+        import synth
+        trs = [synth.paper_scale_trace(8 * rank + i, "coding") for i in range(len(trs))]
+    return trs, reps, [to_lib(p, ti) for ti, p in reps]
+
+
+def cpu_baseline_replay(trs, reps, budget_s: float = 12.0):
+    """The oracle as it stands, single-threaded, on a bounded sample of the
+    sweep's replays (spread over the batch) until budget_s of CPU work."""
+    import oracle
+    from cases import to_oracle
+    order = list(range(0, len(reps), 37)) + list(range(1, len(reps), 37))
+    ev, n, t0 = 0, 0, time.perf_counter()
+    for i in order:
+        ti, p = reps[i]
+        ev += oracle.replay(trs[ti], to_oracle(p))["events"]
+        n += 1
+        if time.perf_counter() - t0 > budget_s and n >= 4:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": ev / dt, "unit": "events/s", "cores": 1, "kind": "oracle",
+            "sample": f"{n} of the 1,024 sweep replays ({ev} events), single thread, {dt:.1f} s"}
+
+
+def run_reference(args):
+    world, rank, _ = dist_env()
+    if rank != 0:
+        return
+    import oracle
+    from cases import to_oracle
+    trs, reps, _ = sweep_workload(0)
+    per_step = 8
+    order = list(range(0, len(reps), 127))
+    times, evs = [], []
+    for step in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        ev = 0
+        for j in range(per_step):
+            ti, p = reps[order[(step * per_step + j) % len(order)]]
+            ev += oracle.replay(trs[ti], to_oracle(p))["events"]
+        dt = time.perf_counter() - t0
+        if step >= args.warmup:
+            times.append(dt)
+            evs.append(ev)
+    v = sum(evs) / sum(times)
+    line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "events/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * sum(times) / len(times),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+            "data": "synthetic",
+            "config": {"workload": "sweep-1024 (8 seeds x 8 capacity pairs x 16 window/bucket settings, "
+                                   "paper-scale coding trace, 131072 B/token, SPEAR+TIDE)",
+                       "sample_per_step": f"{per_step} replays", "l2": "n/a (CPU)"},
+            "cpu_baseline": {"kind": "oracle", "cores": 1, "value": v, "unit": "events/s",
+                             "sample": f"{per_step} sweep replays per step, single-threaded C oracle"},
+            "e2e": {"value": v, "unit": "events/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    import torch
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.cuda.current_device()
+    from paper_2609_09643_gb300 import native
+    native.build()
+    from paper_2609_09643_gb300 import binding as B
+
+    trs, reps, lib_params = sweep_workload(rank)
+    stream = torch.cuda.current_stream()
+    handles = [B.Trace(t).upload(stream) for t in trs]
+    n_rep = len(lib_params)
+    events_per_step = sum(2 * trs[ti].n_turns for ti, _ in reps)
+    res_dev = torch.zeros(B.result_nbytes(n_rep), dtype=torch.uint8, device="cuda")
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+
+    def step():
+        flush.zero_()
+        B.replay_batch_async(handles, lib_params, res_dev, stream=stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    res = B.results_from_tensor(res_dev)
+    assert all(r["status"] == 0 for r in res), "replay status"
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    barrier()
+    torch.cuda.synchronize()
+    clk = ClockSampler(dev)
+    B.profile_enable(True)
+    B.profile_read("replay", reset=True)
+    launches0 = B.launch_count()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    ms = e0.elapsed_time(e1)
+    launches = B.launch_count() - launches0
+    rep_ms, rep_n = B.profile_read("replay", reset=True)
+    ks_ms, ks_n = B.profile_read("key_stream", reset=True)
+    md_ms, md_n = B.profile_read("ttft_median", reset=True)
+    B.profile_enable(False)
+    clocks = clk.stop()
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    value = world * events_per_step * args.steps / (ms / 1e3)
+
+    # end to end through the public API: host trace staging -> device, replay,
+    # results back to the host, every step
+    e2e = None
+    if not args.no_e2e:
+        h2d = sum(h.device_bytes for h in handles)
+        d2h = B.result_nbytes(n_rep)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            for h in handles:
+                h.upload(stream)
+            B.replay_batch(handles, lib_params, stream=stream)
+        torch.cuda.synchronize()
+        dt = time.perf_counter() - t0
+        e2e = {"value": world * events_per_step * args.steps / dt, "unit": "events/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    avg_rep_ms = rep_ms / max(rep_n, 1)
+    alg_bytes = events_per_step * 32  # 16 B event + 4 B prev size + 8 B key + 4 B gap average
+    replay_roof = {"bound": "latency", "kernel": "replay_kernel", "avg_ms": avg_rep_ms,
+                   "ns_per_event_per_replay": 1e6 * avg_rep_ms / (events_per_step / n_rep),
+                   "hbm_gbs": alg_bytes / (avg_rep_ms / 1e3) / 1e9, "launches_timed": rep_n,
+                   "share_of_step": avg_rep_ms * args.steps / ms if ms else None,
+                   "key_stream_avg_ms": ks_ms / max(ks_n, 1), "ttft_median_avg_ms": md_ms / max(md_n, 1)}
+    if rank != 0:
+        return
+    cpu = None if (args.no_cpu_baseline or world > 1) else cpu_baseline_replay(trs, reps)
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        pass
+    line = {"metric": METRIC, "value": value, "unit": "events/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "config": {"workload": "sweep-1024 (8 seeds x 8 capacity pairs x 16 window/bucket settings, "
+                                   "paper-scale coding trace, 131072 B/token, SPEAR+TIDE)",
+                       "replays": n_rep, "events_per_step": events_per_step,
+                       "l2": "flushed before every step (256 MiB write, inside the timed region)"},
+            "roofline": None, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": launches, "clocks": clocks,
+            "peaks": {"hbm_gbs": peaks.get("hbm_gbs"), "source": "MEASURED_PEAKS.json"}}
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -297,6 +297,21 @@ typedef struct {
 int unison_rank_batch(const unison_records *sets, const unison_rank_params *params,
                       const unison_rank_out *outs, int n_sets, void *cuda_stream);
 
+/* ============================================================ measurement */
+/* While enabled (on != 0), every replay and ranking call records a pair of
+ * CUDA events on its own stream around each launch of its main kernels
+ * ("replay" = the event loop, "key_stream", "ttft_median", "rank_sample",
+ * "rank_filter", "rank_finish").  Not thread-safe; meant for benchmarks. */
+int unison_profile_enable(int on);
+
+/* Synchronise the recorded events of one kernel name and return the summed
+ * device time (ms) and the number of timed launches since the last reset;
+ * reset != 0 then discards that kernel's records.  Unknown names give 0. */
+int unison_profile_read(const char *kernel, double *total_ms, uint64_t *launches, int reset);
+
+/* Number of kernels this library has launched since it was loaded. */
+uint64_t unison_launch_count(void);
+
 #ifdef __cplusplus
 }
 #endif

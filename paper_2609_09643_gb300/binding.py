@@ -89,7 +89,8 @@ _lib = None
 # Every symbol include/unison.h declares (checked by the ABI tests).
 EXPORTS = ["unison_strerror", "unison_version", "unison_trace_create", "unison_trace_load",
            "unison_trace_upload", "unison_trace_free", "unison_trace_info", "unison_trace_device_bytes",
-           "unison_replay_batch", "unison_stats", "unison_hazard_lut", "unison_rank_batch"]
+           "unison_replay_batch", "unison_stats", "unison_hazard_lut", "unison_rank_batch",
+           "unison_profile_enable", "unison_profile_read", "unison_launch_count"]
 
 
 def lib_path() -> str:
@@ -124,6 +125,9 @@ def lib():
                                             C.c_void_p]
             L.unison_rank_batch.argtypes = [C.POINTER(Records), C.POINTER(RankParams), C.POINTER(RankOut), C.c_int,
                                             C.c_void_p]
+            L.unison_profile_enable.argtypes = [C.c_int]
+            L.unison_profile_read.argtypes = [C.c_char_p, C.POINTER(C.c_double), C.POINTER(C.c_uint64), C.c_int]
+            L.unison_launch_count.restype = C.c_uint64
             _lib = L
     return _lib
 
@@ -277,3 +281,20 @@ def hazard_lut(turns_dev, bucket: int = 1, stream=None):
     _check("unison_hazard_lut", lib().unison_hazard_lut(turns_dev.data_ptr(), turns_dev.numel(), bucket,
                                                         sig.data_ptr(), hq.data_ptr(), _stream_handle(stream)))
     return sig, hq
+
+
+# ------------------------------------------------------------ measurement --
+def profile_enable(on: bool = True) -> None:
+    _check("unison_profile_enable", lib().unison_profile_enable(1 if on else 0))
+
+
+def profile_read(kernel: str, reset: bool = True):
+    """(summed device ms, timed launches) of one kernel since the last reset."""
+    ms, n = C.c_double(), C.c_uint64()
+    _check("unison_profile_read", lib().unison_profile_read(kernel.encode(), C.byref(ms), C.byref(n),
+                                                            1 if reset else 0))
+    return float(ms.value), int(n.value)
+
+
+def launch_count() -> int:
+    return int(lib().unison_launch_count())

@@ -24,6 +24,7 @@
 #include <vector>
 
 #include "common.cuh"
+#include "profile.cuh"
 
 using namespace unison;
 
@@ -802,6 +803,7 @@ extern "C" int unison_hazard_lut(const uint32_t *turns_dev, uint64_t n_sessions,
   if (!turns_dev || !sigma_q_dev || bucket == 0 || n_sessions >= (1ull << 32)) return UNISON_ERR_ARG;
   hazard_lut_single_kernel<<<1, 256, 0, static_cast<cudaStream_t>(cuda_stream)>>>(
       turns_dev, (uint32_t)n_sessions, bucket, sigma_q_dev, h_q_dev);
+  count_launches(1);
   return cudaGetLastError() == cudaSuccess ? UNISON_OK : UNISON_ERR_CUDA;
 }
 
@@ -973,19 +975,32 @@ extern "C" int unison_replay_batch(const unison_trace *const *traces, int n_trac
     uint32_t max_s = 0;
     for (auto &c : hc) max_s = std::max(max_s, c.n_sessions);
     dim3 g((max_s + 127) / 128, (unsigned)combos.size());
-    key_stream_kernel<<<g, 128, 0, stream>>>(d_combo);
+    {
+      ProfSpan span("key_stream", stream);
+      key_stream_kernel<<<g, 128, 0, stream>>>(d_combo);
+    }
+    count_launches(2);
     ck(cudaGetLastError());
   }
-  if (!in_smem.empty()) {
-    ck(cudaFuncSetAttribute(replay_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)max_smem));
-    replay_kernel<false><<<(unsigned)in_smem.size(), 32, max_smem, stream>>>(d_desc, d_order);
-    ck(cudaGetLastError());
+  {
+    ProfSpan span("replay", stream);
+    if (!in_smem.empty()) {
+      ck(cudaFuncSetAttribute(replay_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)max_smem));
+      replay_kernel<false><<<(unsigned)in_smem.size(), 32, max_smem, stream>>>(d_desc, d_order);
+      count_launches(1);
+      ck(cudaGetLastError());
+    }
+    if (!in_global.empty()) {
+      replay_kernel<true><<<(unsigned)in_global.size(), 32, 0, stream>>>(d_desc, d_order + in_smem.size());
+      count_launches(1);
+      ck(cudaGetLastError());
+    }
   }
-  if (!in_global.empty()) {
-    replay_kernel<true><<<(unsigned)in_global.size(), 32, 0, stream>>>(d_desc, d_order + in_smem.size());
-    ck(cudaGetLastError());
+  {
+    ProfSpan span("ttft_median", stream);
+    ttft_median_kernel<<<(unsigned)n_replays, 256, 0, stream>>>(d_desc, (uint32_t)n_replays);
   }
-  ttft_median_kernel<<<(unsigned)n_replays, 256, 0, stream>>>(d_desc, (uint32_t)n_replays);
+  count_launches(1);
   ck(cudaGetLastError());
   if (results_host)
     ck(cudaMemcpyAsync(results_host, res, sizeof(unison_replay_result) * n_replays, cudaMemcpyDeviceToHost, stream));

@@ -11,7 +11,7 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(PKG, "csrc")
 OUT = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT, "libunison.so")
-SOURCES = ["trace.cu", "replay.cu", "rank.cu"]
+SOURCES = ["trace.cu", "replay.cu", "rank.cu", "profile.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2"]
 
@@ -26,7 +26,8 @@ def nvcc() -> str:
 def _stale(obj: str, src: str) -> bool:
     if not os.path.exists(obj):
         return True
-    deps = [src, os.path.join(CSRC, "common.cuh"), os.path.join(PKG, "..", "include", "unison.h")]
+    deps = [src, os.path.join(CSRC, "common.cuh"), os.path.join(CSRC, "profile.cuh"),
+            os.path.join(PKG, "..", "include", "unison.h")]
     return any(os.path.getmtime(d) > os.path.getmtime(obj) for d in deps if os.path.exists(d))
 
 
