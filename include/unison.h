@@ -226,6 +226,42 @@ int unison_replay_batch(const unison_trace *const *traces, int n_traces,
                         unison_decision *log_dev, uint64_t log_capacity_per_replay,
                         void *cuda_stream);
 
+/* Replay for callers that cannot allocate device memory.  The paper has no
+ * counterpart to this entry point; it exists for the library's users.
+ *
+ * Some callers must not allocate: a serving runtime whose memory manager
+ * reserves the device's whole budget up front and refuses allocations made
+ * behind its back, or a latency-critical control loop that cannot afford an
+ * allocator call (cudaMalloc and cudaFree may synchronise the device, and an
+ * allocation can fail in the middle of a run).  This entry point replays
+ * exactly like unison_replay_batch (same arguments, same results) but takes
+ * its scratch from one fixed device array compiled into the library,
+ * UNISON_NOALLOC_SCRATCH_BYTES long, which every GPU that loads the library
+ * holds until the process exits.  It calls no cudaMalloc, cudaFree or other
+ * allocating routine.
+ *  - results_dev is required (the caller provides the output buffer);
+ *    results_host, log_dev and the traces are as in unison_replay_batch.
+ *    The traces must already be uploaded (unison_trace_upload allocates, so
+ *    upload them beforehand).
+ *  - A batch whose scratch (descriptors, hazard tables, 12 B per event per
+ *    key stream, 8 B per request per replay, resident lists that do not fit
+ *    in shared memory) exceeds UNISON_NOALLOC_SCRATCH_BYTES is rejected with
+ *    UNISON_ERR_RANGE before anything is queued.
+ *  - The first call on a device looks up the array's device address on that
+ *    device (cudaGetSymbolAddress, with that device current); make that
+ *    first call before any stream capture.
+ *  - All calls share the one array, which keeps what the last call left in
+ *    it; each call writes every region it reads before reading it, so no
+ *    region needs clearing.  Calls whose work overlaps on the GPU (on
+ *    different streams or from different threads) race on the array: queue
+ *    them on one stream or order them. */
+#define UNISON_NOALLOC_SCRATCH_BYTES (32ull << 20)
+int unison_replay_batch_noalloc(const unison_trace *const *traces, int n_traces,
+                                const unison_replay_params *params, int n_replays,
+                                unison_replay_result *results_dev, unison_replay_result *results_host,
+                                unison_decision *log_dev, uint64_t log_capacity_per_replay,
+                                void *cuda_stream);
+
 /* Host-side summary of one replay (Sec. V-A): hit rate HR = (H_S + H_H)/R,
  * AMAT = (t_s sum_S + t_h sum_H + t_p sum_M)/R in ps (eq. hr-amat), prefill
  * reduction 1 - computed/needed (eq. prered), prefetch accuracy = promoted

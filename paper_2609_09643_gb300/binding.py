@@ -90,7 +90,8 @@ _lib = None
 EXPORTS = ["unison_strerror", "unison_version", "unison_trace_create", "unison_trace_load",
            "unison_trace_upload", "unison_trace_free", "unison_trace_info", "unison_trace_device_bytes",
            "unison_replay_batch", "unison_stats", "unison_hazard_lut", "unison_rank_batch",
-           "unison_profile_enable", "unison_profile_read", "unison_launch_count"]
+           "unison_profile_enable", "unison_profile_read", "unison_launch_count",
+           "unison_replay_batch_noalloc"]
 
 
 def lib_path() -> str:
@@ -128,6 +129,7 @@ def lib():
             L.unison_profile_enable.argtypes = [C.c_int]
             L.unison_profile_read.argtypes = [C.c_char_p, C.POINTER(C.c_double), C.POINTER(C.c_uint64), C.c_int]
             L.unison_launch_count.restype = C.c_uint64
+            L.unison_replay_batch_noalloc.argtypes = L.unison_replay_batch.argtypes
             _lib = L
     return _lib
 
@@ -298,3 +300,21 @@ def profile_read(kernel: str, reset: bool = True):
 
 def launch_count() -> int:
     return int(lib().unison_launch_count())
+
+
+# ------------------------------------------------------- no-allocation path --
+NOALLOC_SCRATCH_BYTES = 32 << 20
+
+
+def replay_batch_noalloc(traces: Sequence[Trace], params: Sequence[dict], results_dev, stream=None, log=None,
+                         log_capacity: int = 0) -> None:
+    """unison_replay_batch_noalloc: the same replay, with the library's fixed
+    device scratch instead of any allocation.  results_dev (and log, if
+    given) are caller-owned device buffers; the call only marshals them."""
+    n = len(params)
+    arr_t = (C.c_void_p * len(traces))(*(t.handle.value for t in traces))
+    arr_p = (ReplayParams * n)(*(make_params(p) for p in params))
+    rc = lib().unison_replay_batch_noalloc(arr_t, len(traces), arr_p, n, results_dev.data_ptr(), None,
+                                           None if log is None else log.data_ptr(), log_capacity,
+                                           _stream_handle(stream))
+    _check("unison_replay_batch_noalloc", rc)

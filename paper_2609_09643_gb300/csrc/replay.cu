@@ -20,6 +20,7 @@
 //                       over each replay's per-request TTFT values.
 #include <algorithm>
 #include <map>
+#include <mutex>
 #include <tuple>
 #include <vector>
 
@@ -1023,4 +1024,237 @@ extern "C" int unison_stats(const unison_replay_result *r, const unison_replay_p
   out->ttft_mean_ns = r->ttft_n ? (double)(sum / r->ttft_n) : 0.0;
   out->ttft_p50_ns = (double)r->ttft_p50_ns;
   return UNISON_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Replay without device allocation.
+//
+// The scratch this entry point needs (descriptors, hazard tables, key
+// streams, TTFT values, global resident lists) lives in one file-scope device
+// array instead of memory from cudaMallocAsync.  Host code must not use the
+// array's name as an address: for host code it names a host-side shadow, so
+// its device address is fetched with cudaGetSymbolAddress once per device
+// (with that device current) and passed to the kernels.
+// ---------------------------------------------------------------------------
+static __device__ __align__(256) unsigned char g_unison_noalloc_scratch[UNISON_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_noalloc_mu;
+char *g_noalloc_addr[kNoAllocMaxDevices] = {};
+
+// Device address of the scratch array on the current device.
+int noalloc_scratch_address(char **out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return UNISON_ERR_CUDA;
+  }
+  if (dev < 0 || dev >= kNoAllocMaxDevices) return UNISON_ERR_ARG;
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (!g_noalloc_addr[dev]) {
+    void *p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_unison_noalloc_scratch);
+    if (e != cudaSuccess || p == nullptr) {
+      cudaGetLastError();
+      return UNISON_ERR_CUDA;
+    }
+    g_noalloc_addr[dev] = static_cast<char *>(p);
+  }
+  *out = g_noalloc_addr[dev];
+  return UNISON_OK;
+}
+}  // namespace
+
+extern "C" int unison_replay_batch_noalloc(const unison_trace *const *traces, int n_traces,
+                                           const unison_replay_params *params, int n_replays,
+                                           unison_replay_result *results_dev, unison_replay_result *results_host,
+                                           unison_decision *log_dev, uint64_t log_capacity_per_replay,
+                                           void *cuda_stream) {
+  if (!traces || n_traces <= 0 || !params || n_replays < 0) return UNISON_ERR_ARG;
+  if (n_replays == 0) return UNISON_OK;
+  if (!results_dev) return UNISON_ERR_ARG;  // the caller provides the output buffer
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return UNISON_ERR_CUDA;
+  for (int i = 0; i < n_traces; i++)
+    if (!traces[i] || !traces[i]->d_block || traces[i]->device != dev) return UNISON_ERR_ARG;
+  for (int r = 0; r < n_replays; r++) {
+    const int rc = check_params(params[r], n_traces);
+    if (rc != UNISON_OK) return rc;
+  }
+  char *scratch = nullptr;
+  {
+    const int rc = noalloc_scratch_address(&scratch);
+    if (rc != UNISON_OK) return rc;
+  }
+  int smem_optin = 0;
+  cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  const size_t smem_limit = (size_t)smem_optin > 1024 ? (size_t)smem_optin - 1024 : 0;
+
+  std::map<std::tuple<uint32_t, uint32_t, uint32_t, uint32_t, uint64_t>, int> combo_of;
+  std::vector<std::tuple<uint32_t, uint32_t, uint32_t, uint32_t, uint64_t>> combos;
+  std::vector<int> replay_combo(n_replays, -1);
+  for (int r = 0; r < n_replays; r++) {
+    const unison_replay_params &p = params[r];
+    if (!needs_stream(p.policy)) continue;
+    auto key = std::make_tuple(p.trace_idx, p.ema_num, p.ema_den, p.hazard_bucket, p.penalty_q);
+    auto it = combo_of.find(key);
+    if (it == combo_of.end()) {
+      it = combo_of.emplace(key, (int)combos.size()).first;
+      combos.push_back(key);
+    }
+    replay_combo[r] = it->second;
+  }
+
+  // Same layout as unison_replay_batch, without the results region.
+  size_t off = 0;
+  const size_t off_desc = off;
+  off = align_up(off + sizeof(ReplayDesc) * n_replays, 256);
+  const size_t off_order = off;
+  off = align_up(off + sizeof(uint32_t) * 2 * n_replays, 256);
+  const size_t off_combo = off;
+  off = align_up(off + sizeof(ComboDesc) * combos.size() + 1, 256);
+  std::vector<size_t> off_lut(combos.size()), off_stream(combos.size());
+  for (size_t c = 0; c < combos.size(); c++) {
+    off_lut[c] = off;
+    off = align_up(off + 128 + 51 * 8, 256);
+    const uint64_t E = traces[std::get<0>(combos[c])]->n_events;
+    off_stream[c] = off;
+    off = align_up(off + 12 * E, 256);
+  }
+  std::vector<size_t> off_ttft(n_replays), off_glist(n_replays, 0);
+  std::vector<uint32_t> rcap_s(n_replays), rcap_h(n_replays), use_map(n_replays), smem_bytes(n_replays);
+  std::vector<uint32_t> in_smem, in_global;
+  size_t max_smem = 0;
+  for (int r = 0; r < n_replays; r++) {
+    const unison_replay_params &p = params[r];
+    const unison_trace *tr = traces[p.trace_idx];
+    const uint64_t cs = p.cap_fast_bytes / p.kv_bytes_per_token, ch = p.cap_hbm_bytes / p.kv_bytes_per_token;
+    const uint64_t mo = std::max<uint32_t>(tr->min_out_tok, 1);
+    rcap_s[r] = (uint32_t)std::min<uint64_t>(tr->n_sessions, cs / mo) + 1;
+    rcap_h[r] = (uint32_t)std::min<uint64_t>(tr->n_sessions, ch / mo) + 1;
+    const size_t lists = (size_t)kEntryBytes * (rcap_s[r] + rcap_h[r]);
+    const size_t map_b = align_up(2ull * tr->n_sessions, 16);
+    const bool map_ok = rcap_s[r] <= 0x7FFF && rcap_h[r] <= 0x7FFF;
+    if (map_ok && lists + map_b <= smem_limit && map_b <= 32768) {
+      use_map[r] = 1;
+      smem_bytes[r] = (uint32_t)(lists + map_b);
+    } else {
+      use_map[r] = 0;
+      smem_bytes[r] = (uint32_t)lists;
+    }
+    if (smem_bytes[r] <= smem_limit) {
+      in_smem.push_back((uint32_t)r);
+      max_smem = std::max<size_t>(max_smem, smem_bytes[r]);
+    } else {
+      use_map[r] = 0;
+      in_global.push_back((uint32_t)r);
+      off_glist[r] = off;
+      off = align_up(off + lists, 256);
+    }
+    off_ttft[r] = off;
+    off = align_up(off + 8 * (tr->n_turns + 1), 256);
+  }
+  if (off > UNISON_NOALLOC_SCRATCH_BYTES) return UNISON_ERR_RANGE;  // batch too large for the fixed scratch
+
+  // Every scratch region is written before it is read within one call (the
+  // descriptors by the copies below, the tables and streams by their kernels,
+  // TTFT values and lists by the event loop), so nothing left by an earlier
+  // call is ever read and no region needs clearing.
+  std::vector<ComboDesc> hc(combos.size());
+  for (size_t c = 0; c < combos.size(); c++) {
+    const unison_trace *tr = traces[std::get<0>(combos[c])];
+    ComboDesc &d = hc[c];
+    d.turn_ev = tr->d<uint32_t>(tr->off_turn_ev);
+    d.turn_t = tr->d<uint32_t>(tr->off_turn_t);
+    d.turn_off = tr->d<uint32_t>(tr->off_turn_off);
+    d.tps = tr->d<uint32_t>(tr->off_tps);
+    d.n_sessions = tr->n_sessions;
+    d.n_events = (uint32_t)tr->n_events;
+    d.ema_num = std::get<1>(combos[c]);
+    d.ema_den = std::get<2>(combos[c]);
+    d.bucket = std::get<3>(combos[c]);
+    d.pad = 0;
+    d.penalty_q = std::get<4>(combos[c]);
+    d.sigma = reinterpret_cast<uint16_t *>(scratch + off_lut[c]);
+    d.t2 = reinterpret_cast<uint64_t *>(scratch + off_lut[c] + 128);
+    d.pkey = reinterpret_cast<uint64_t *>(scratch + off_stream[c]);
+    d.gq = reinterpret_cast<uint32_t *>(scratch + off_stream[c] + 8 * tr->n_events);
+  }
+  std::vector<ReplayDesc> hd(n_replays);
+  for (int r = 0; r < n_replays; r++) {
+    const unison_replay_params &p = params[r];
+    const unison_trace *tr = traces[p.trace_idx];
+    ReplayDesc &d = hd[r];
+    d.ev = tr->d<uint4>(tr->off_ev);
+    d.prev_out = tr->d<uint32_t>(tr->off_prev_out);
+    d.nref = tr->d<uint32_t>(tr->off_nref);
+    d.pkey = replay_combo[r] >= 0 ? hc[replay_combo[r]].pkey : nullptr;
+    d.gq = replay_combo[r] >= 0 ? hc[replay_combo[r]].gq : nullptr;
+    d.ttft = reinterpret_cast<uint64_t *>(scratch + off_ttft[r]);
+    d.glist = off_glist[r] ? reinterpret_cast<uint32_t *>(scratch + off_glist[r]) : nullptr;
+    d.log = log_dev ? log_dev + (uint64_t)r * log_capacity_per_replay : nullptr;
+    d.log_cap = log_dev ? log_capacity_per_replay : 0;
+    d.result = results_dev + r;
+    d.cap_s = p.cap_fast_bytes / p.kv_bytes_per_token;
+    d.cap_h = p.cap_hbm_bytes / p.kv_bytes_per_token;
+    d.dma = p.dma_bytes_per_us;
+    d.prefill_ns = p.t_p_ps_per_tok / 1000;
+    d.n_events = (uint32_t)tr->n_events;
+    d.n_turns = (uint32_t)tr->n_turns;
+    d.n_sessions = tr->n_sessions;
+    d.policy = p.policy;
+    d.max_sessions = p.max_sessions;
+    d.kvb = p.kv_bytes_per_token;
+    d.ttl = p.ttl_us;
+    d.load = p.ttft_load;
+    d.rcap_s = rcap_s[r];
+    d.rcap_h = rcap_h[r];
+    d.use_map = use_map[r];
+    d.pad = 0;
+  }
+  std::vector<uint32_t> order;
+  order.insert(order.end(), in_smem.begin(), in_smem.end());
+  order.insert(order.end(), in_global.begin(), in_global.end());
+
+  int rc = UNISON_OK;
+  auto ck = [&](cudaError_t e) {
+    if (e != cudaSuccess && rc == UNISON_OK) rc = UNISON_ERR_CUDA;
+  };
+  ReplayDesc *d_desc = reinterpret_cast<ReplayDesc *>(scratch + off_desc);
+  uint32_t *d_order = reinterpret_cast<uint32_t *>(scratch + off_order);
+  ComboDesc *d_combo = reinterpret_cast<ComboDesc *>(scratch + off_combo);
+  ck(cudaMemcpyAsync(d_desc, hd.data(), sizeof(ReplayDesc) * n_replays, cudaMemcpyHostToDevice, stream));
+  ck(cudaMemcpyAsync(d_order, order.data(), sizeof(uint32_t) * order.size(), cudaMemcpyHostToDevice, stream));
+  if (!combos.empty()) {
+    ck(cudaMemcpyAsync(d_combo, hc.data(), sizeof(ComboDesc) * combos.size(), cudaMemcpyHostToDevice, stream));
+    hazard_lut_kernel<<<(unsigned)combos.size(), 256, 0, stream>>>(d_combo);
+    uint32_t max_s = 0;
+    for (auto &c : hc) max_s = std::max(max_s, c.n_sessions);
+    dim3 g((max_s + 127) / 128, (unsigned)combos.size());
+    key_stream_kernel<<<g, 128, 0, stream>>>(d_combo);
+    count_launches(2);
+    ck(cudaGetLastError());
+  }
+  if (!in_smem.empty()) {
+    ck(cudaFuncSetAttribute(replay_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)max_smem));
+    replay_kernel<false><<<(unsigned)in_smem.size(), 32, max_smem, stream>>>(d_desc, d_order);
+    count_launches(1);
+    ck(cudaGetLastError());
+  }
+  if (!in_global.empty()) {
+    replay_kernel<true><<<(unsigned)in_global.size(), 32, 0, stream>>>(d_desc, d_order + in_smem.size());
+    count_launches(1);
+    ck(cudaGetLastError());
+  }
+  ttft_median_kernel<<<(unsigned)n_replays, 256, 0, stream>>>(d_desc, (uint32_t)n_replays);
+  count_launches(1);
+  ck(cudaGetLastError());
+  if (results_host) {
+    ck(cudaMemcpyAsync(results_host, results_dev, sizeof(unison_replay_result) * n_replays, cudaMemcpyDeviceToHost,
+                       stream));
+    ck(cudaStreamSynchronize(stream));
+  }
+  return rc;
 }

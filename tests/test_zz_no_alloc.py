@@ -1,0 +1,73 @@
+"""The no-allocation replay entry point (unison_replay_batch_noalloc).
+
+It serves callers that cannot allocate device memory (a runtime whose memory
+manager owns the whole device budget, or a control loop that cannot pay for
+an allocator call).  Its results must equal the ordinary entry point's, call
+after call, even though every call reuses one fixed device array.  This file
+is collected last so that a failure here leaves every other test already run.
+"""
+import pytest
+
+import synth
+from cases import GIB, MIB, base, to_lib
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def B():
+    from paper_2609_09643_gb300 import native
+    native.build()
+    from paper_2609_09643_gb300 import binding
+    return binding
+
+
+def _workload():
+    """Two traces, all six policies, two capacity settings: key streams, TTFT
+    values and resident lists all land in the fixed scratch."""
+    trs = [synth.tiny_trace(0), synth.paper_scale_trace(3, "general")]
+    reps = []
+    for ti, (cs, ch, kvb) in enumerate([(512 * MIB, 8 * GIB, 28672), (2 * GIB, 32 * GIB, 131072)]):
+        for pol in ("lru", "timeout", "spear", "spear_tide", "belady", "lru_tide"):
+            reps.append((ti, base(pol, cs, ch, kvb)))
+    return trs, reps
+
+
+def test_noalloc_matches_allocating_entry_point_twice(B):
+    import torch
+    trs, reps = _workload()
+    handles = [B.Trace(t).upload() for t in trs]
+    params = [to_lib(p, ti) for ti, p in reps]
+    ref, ref_log = B.replay_batch(handles, params, log_capacity=4096)
+    n = len(params)
+    out = torch.zeros(B.result_nbytes(n), dtype=torch.uint8, device="cuda")
+    log = torch.zeros((n, 4096, 2), dtype=torch.int32, device="cuda")
+    for call in range(2):
+        out.fill_(0xAB)
+        log.zero_()
+        B.replay_batch_noalloc(handles, params, out, log=log, log_capacity=4096)
+        torch.cuda.synchronize()
+        got = B.results_from_tensor(out)
+        assert got == ref, f"call {call}"
+        for i in range(n):
+            k = min(ref[i]["log_len"], 4096)
+            assert torch.equal(log[i, :k], ref_log[i, :k]), (call, i)
+
+
+def test_noalloc_rejects_batches_beyond_its_scratch(B):
+    import torch
+    trs = [synth.paper_scale_trace(s, "coding") for s in range(2)]
+    handles = [B.Trace(t).upload() for t in trs]
+    # 256 replays x 33,596 requests x 8 B of TTFT values alone exceed 32 MiB
+    params = [to_lib(base("spear_tide", 2 * GIB, 32 * GIB, 131072), i % 2) for i in range(256)]
+    out = torch.zeros(B.result_nbytes(len(params)), dtype=torch.uint8, device="cuda")
+    with pytest.raises(B.UnisonError) as e:
+        B.replay_batch_noalloc(handles, params, out)
+    assert e.value.code == B.ERR_RANGE
+    # a batch that fits still runs after the rejection
+    ok = params[:8]
+    out8 = torch.zeros(B.result_nbytes(8), dtype=torch.uint8, device="cuda")
+    B.replay_batch_noalloc(handles, ok, out8)
+    torch.cuda.synchronize()
+    ref, _ = B.replay_batch(handles, ok)
+    assert B.results_from_tensor(out8) == ref
