@@ -4,8 +4,8 @@
 One step = one batched replay of the parameter sweep (1,024 independent
 SPEAR+TIDE replays: 8 trace seeds x 8 tier-capacity pairs x 16 gap-window /
 hazard-bucket settings over the paper-scale coding trace, 131,072 B/token)
-plus one ranking pass over a 2^24-record live set (top-1024 victims and the
-TIDE fill).  Inputs are synthetic (see the synth package) and resident in HBM
+plus one ranking call over seven 2^24-record live sets (top-1,024 victims and
+the TIDE fill at budgets of 1..64 GiB).  Inputs are synthetic (see the synth package) and resident in HBM
 before the timed region; an L2 flush (a 256 MiB write) precedes each step.
 
 Prints one JSON line (rank 0).  --impl reference times the CPU oracle on a
@@ -38,6 +38,9 @@ def parse():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--rank-only", action="store_true", help="time only the ranking leg (profiling)")
+    ap.add_argument("--rank-n", type=int, default=1 << 24, help="records per live set")
+    ap.add_argument("--rank-sets", type=int, default=7, help="live sets per call (<= 7)")
     return ap.parse_args()
 
 
@@ -107,6 +110,27 @@ def sweep_workload(rank: int):
     return trs, reps, [to_lib(p, ti) for ti, p in reps]
 
 
+RANK_N = 1 << 24  # overridden by --rank-n
+RANK_BUDGETS_GIB = (1, 2, 4, 8, 16, 32, 64)
+RANK_BYTES_PER_RECORD = 8  # gap average 4 + turn 2 + flags 1 + tier 1: what the filter must read
+
+
+def rank_workload():
+    """Live sets of 2^24 records (the largest live-set size), one per TIDE
+    budget 1..64 GiB, each a separate copy in HBM; k = 1,024 victims (every
+    k <= 1,024 is a prefix), up to 1,024 moves, no free fast-tier space (pair
+    fill only)."""
+    import synth
+    rec = synth.make_records(4, RANK_N)
+    tps = synth.geometric_turns(1, 1415, 23.7, 2, 200)
+    return rec, tps
+
+
+def rank_params(sigma, n_sets=7):
+    return [dict(sigma_q=sigma, k=1024, penalty_q=500_000_000, budget_bytes=b << 30, kv_bytes_per_token=131072,
+                 max_moves=1024, free_fast_tok=0, free_hbm_tok=1 << 40) for b in RANK_BUDGETS_GIB[:n_sets]]
+
+
 def cpu_baseline_replay(trs, reps, budget_s: float = 12.0):
     """The oracle as it stands, single-threaded, on a bounded sample of the
     sweep's replays (spread over the batch) until budget_s of CPU work."""
@@ -123,6 +147,20 @@ def cpu_baseline_replay(trs, reps, budget_s: float = 12.0):
     dt = time.perf_counter() - t0
     return {"value": ev / dt, "unit": "events/s", "cores": 1, "kind": "oracle",
             "sample": f"{n} of the 1,024 sweep replays ({ev} events), single thread, {dt:.1f} s"}
+
+
+def cpu_baseline_rank(rec, sigma, n: int = 1 << 22):
+    """The oracle's ranking (every key, a full sort, the fill) on the first
+    2^22 records of one live set, single-threaded."""
+    import oracle
+    import synth
+    sub = synth.Records(*(a[:n].copy() for a in (rec.gap_q, rec.last_ret, rec.turn, rec.kv_tok, rec.tier,
+                                                 rec.flags)))
+    t0 = time.perf_counter()
+    oracle.rank(sub, sigma, 500_000_000, 1024, 64 << 30, 131072, 0, 1 << 40, max_moves=1024)
+    dt = time.perf_counter() - t0
+    return {"value": n * RANK_BYTES_PER_RECORD / dt / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": f"{n} records of one 2^24 live set, k=1024, 64 GiB budget, single thread, {dt:.1f} s"}
 
 
 def run_reference(args):
@@ -160,7 +198,9 @@ def run_reference(args):
 
 
 def main():
+    global RANK_N
     args = parse()
+    RANK_N = args.rank_n
     if args.impl == "reference":
         return run_reference(args)
     import torch
@@ -184,15 +224,31 @@ def main():
     res_dev = torch.zeros(B.result_nbytes(n_rep), dtype=torch.uint8, device="cuda")
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
 
+    # ranking leg: survival table from the paper-scale turn law, on the device
+    rec, tps = rank_workload()
+    tps_dev = torch.tensor(tps.astype("int32"), device="cuda")
+    sig_dev, _ = B.hazard_lut(tps_dev, 1)
+    sigma = sig_dev.cpu().numpy().astype("uint16")
+    r_params = rank_params(sigma, args.rank_sets)
+    host_rec = B.records_to_device(rec, device="cpu")
+    host_rec = {k: v.pin_memory() for k, v in host_rec.items()}
+    rank_sets = [{k: v.to("cuda", non_blocking=True) for k, v in host_rec.items()} for _ in r_params]
+    rank_outs = [B.rank_outputs(RANK_N, p["k"], p["max_moves"]) for p in r_params]
+    rank_bytes = len(r_params) * RANK_N * RANK_BYTES_PER_RECORD
+
     def step():
         flush.zero_()
-        B.replay_batch_async(handles, lib_params, res_dev, stream=stream)
+        if not args.rank_only:
+            B.replay_batch_async(handles, lib_params, res_dev, stream=stream)
+        B.rank_batch(rank_sets, r_params, rank_outs, stream=stream)
 
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
-    res = B.results_from_tensor(res_dev)
-    assert all(r["status"] == 0 for r in res), "replay status"
+    if not args.rank_only:
+        res = B.results_from_tensor(res_dev)
+        assert all(r["status"] == 0 for r in res), "replay status"
+    assert all(B.rank_result(o)["status"] == 0 for o in rank_outs), "rank status"
 
     def barrier():
         if world > 1:
@@ -202,7 +258,8 @@ def main():
     torch.cuda.synchronize()
     clk = ClockSampler(dev)
     B.profile_enable(True)
-    B.profile_read("replay", reset=True)
+    for kname in ("replay", "key_stream", "ttft_median", "rank_sample", "rank_filter", "rank_finish"):
+        B.profile_read(kname, reset=True)
     launches0 = B.launch_count()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
@@ -216,46 +273,72 @@ def main():
     rep_ms, rep_n = B.profile_read("replay", reset=True)
     ks_ms, ks_n = B.profile_read("key_stream", reset=True)
     md_ms, md_n = B.profile_read("ttft_median", reset=True)
+    rs_ms, rs_n = B.profile_read("rank_sample", reset=True)
+    rf_ms, rf_n = B.profile_read("rank_filter", reset=True)
+    rn_ms, rn_n = B.profile_read("rank_finish", reset=True)
     B.profile_enable(False)
     clocks = clk.stop()
     if world > 1:
         t = torch.tensor([ms], dtype=torch.float64, device="cuda")
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         ms = float(t.item())
-    value = world * events_per_step * args.steps / (ms / 1e3)
+    value = world * events_per_step * args.steps / (ms / 1e3) if not args.rank_only else None
 
     # end to end through the public API: host trace staging -> device, replay,
     # results back to the host, every step
     e2e = None
-    if not args.no_e2e:
-        h2d = sum(h.device_bytes for h in handles)
-        d2h = B.result_nbytes(n_rep)
+    if not args.no_e2e and not args.rank_only:
+        h2d = sum(h.device_bytes for h in handles) + len(rank_sets) * sum(
+            v.numel() * v.element_size() for v in host_rec.values())
+        d2h = B.result_nbytes(n_rep) + sum(o["victims"].numel() * 4 + o["promote"].numel() * 4 +
+                                           o["demote"].numel() * 4 + 16 + 8 for o in rank_outs)
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         for _ in range(args.steps):
             for h in handles:
                 h.upload(stream)
+            for dst in rank_sets:
+                for k, v in host_rec.items():
+                    dst[k].copy_(v, non_blocking=True)
             B.replay_batch(handles, lib_params, stream=stream)
+            B.rank_batch(rank_sets, r_params, rank_outs, stream=stream)
+            _ = [B.rank_result(o) for o in rank_outs]
         torch.cuda.synchronize()
         dt = time.perf_counter() - t0
         e2e = {"value": world * events_per_step * args.steps / dt, "unit": "events/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
-    avg_rep_ms = rep_ms / max(rep_n, 1)
+    avg_rep_ms = rep_ms / max(rep_n, 1) if rep_n else float("nan")
     alg_bytes = events_per_step * 32  # 16 B event + 4 B prev size + 8 B key + 4 B gap average
-    replay_roof = {"bound": "latency", "kernel": "replay_kernel", "avg_ms": avg_rep_ms,
+    replay_roof = None if not rep_n else {"bound": "latency", "kernel": "replay_kernel", "avg_ms": avg_rep_ms,
                    "ns_per_event_per_replay": 1e6 * avg_rep_ms / (events_per_step / n_rep),
                    "hbm_gbs": alg_bytes / (avg_rep_ms / 1e3) / 1e9, "launches_timed": rep_n,
                    "share_of_step": avg_rep_ms * args.steps / ms if ms else None,
                    "key_stream_avg_ms": ks_ms / max(ks_n, 1), "ttft_median_avg_ms": md_ms / max(md_n, 1)}
-    if rank != 0:
-        return
-    cpu = None if (args.no_cpu_baseline or world > 1) else cpu_baseline_replay(trs, reps)
     peaks = {}
     try:
         peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
     except Exception:
         pass
+    hbm_peak = peaks.get("hbm_gbs") or 6800.0
+    avg_rf = rf_ms / max(rf_n, 1)
+    achieved = rank_bytes / (avg_rf / 1e3) / 1e9
+    roofline = {"bound": "hbm", "kernel": "rank_filter_kernel", "achieved": achieved, "peak": hbm_peak,
+                "unit": "GB/s", "frac": achieved / hbm_peak,
+                "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs, burst copy)" if peaks.get("hbm_gbs")
+                else "fallback 6.8 TB/s", "traffic": None, "avg_ms": avg_rf, "launches_timed": rf_n,
+                "algorithmic_bytes_per_launch": rank_bytes,
+                "bytes_per_record": RANK_BYTES_PER_RECORD, "records_per_launch": len(r_params) * RANK_N}
+    call_ms = (rs_ms + rf_ms + rn_ms) / max(rf_n, 1)
+    rank_leg = {"metric": "rank-kernel HBM GB/s", "sets_per_call": len(r_params), "records_per_set": RANK_N,
+                "k": 1024, "budgets_gib": list(RANK_BUDGETS_GIB),
+                "call_ms": call_ms, "call_gbs": rank_bytes / (call_ms / 1e3) / 1e9,
+                "call_frac_of_peak": rank_bytes / (call_ms / 1e3) / 1e9 / hbm_peak,
+                "records_per_s": len(r_params) * RANK_N / (call_ms / 1e3),
+                "sample_ms": rs_ms / max(rs_n, 1), "filter_ms": avg_rf, "finish_ms": rn_ms / max(rn_n, 1)}
+    if rank != 0:
+        return
+    cpu = None if (args.no_cpu_baseline or world > 1) else cpu_baseline_replay(trs, reps)
     line = {"metric": METRIC, "value": value, "unit": "events/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int64", "data": "synthetic",
@@ -263,9 +346,11 @@ def main():
                                    "paper-scale coding trace, 131072 B/token, SPEAR+TIDE)",
                        "replays": n_rep, "events_per_step": events_per_step,
                        "l2": "flushed before every step (256 MiB write, inside the timed region)"},
-            "roofline": None, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roofline, "rank": rank_leg, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches, "clocks": clocks,
             "peaks": {"hbm_gbs": peaks.get("hbm_gbs"), "source": "MEASURED_PEAKS.json"}}
+    if cpu is not None:
+        cpu["rank"] = cpu_baseline_rank(rec, sigma)
     print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()

@@ -287,7 +287,10 @@ int unison_hazard_lut(const uint32_t *turns_dev, uint64_t n_sessions, uint32_t b
  * (caller-owned).  gap_q: gap average in us (eq. gapq, < 2^31); last_ret:
  * last completion time (carried, not read by the score); turn: register turn
  * t; kv_tok: resident tokens; tier: 1 fast, 2 HBM, other = not resident;
- * flags: bit0 pinned (mid-turn), bit1 done (completed session).  n < 2^31. */
+ * flags: bit0 pinned (mid-turn), bit1 done (completed session).  1 <= n <= 2^24
+ * (the index is packed into 24 bits of the ranking key); gap_q, turn, tier
+ * and flags must start on 16-byte boundaries (they are streamed with bulk
+ * copies), else UNISON_ERR_ARG. */
 typedef struct {
   const uint32_t *gap_q;
   const uint32_t *last_ret;
@@ -301,11 +304,12 @@ typedef struct {
 typedef struct {
   uint16_t sigma_q[51];        /* survival table (unison_hazard_lut), host copy  */
   uint16_t reserved0;
-  uint32_t k;                  /* victims wanted, 0 .. 4096                      */
+  uint32_t k;                  /* victims wanted, 0 .. 4096 (else _RANGE)        */
   uint64_t penalty_q;          /* P_Z, < 2^32                                    */
   uint64_t budget_bytes;       /* TIDE budget for this set                       */
   uint32_t kv_bytes_per_token; /* 1 .. 2^24                                      */
-  uint32_t max_moves;          /* capacity of promote[] and demote[]             */
+  uint32_t max_moves;          /* cap on promotions (and on promote[] / demote[] */
+                               /* capacity), 0 .. 4096                           */
   uint64_t free_fast_tok;      /* free fast-tier capacity, tokens                */
   uint64_t free_hbm_tok;       /* free HBM capacity, tokens                      */
 } unison_rank_params;

@@ -318,3 +318,54 @@ def replay_batch_noalloc(traces: Sequence[Trace], params: Sequence[dict], result
                                            None if log is None else log.data_ptr(), log_capacity,
                                            _stream_handle(stream))
     _check("unison_replay_batch_noalloc", rc)
+
+
+# --------------------------------------------------------------- ranking --
+def records_to_device(rec, device="cuda"):
+    """Copy a synth.Records-like object (numpy SoA) to device tensors (bit
+    patterns in signed torch dtypes)."""
+    import torch
+    conv = lambda a, dt: torch.from_numpy(np.ascontiguousarray(a).view(dt)).to(device)
+    return dict(gap_q=conv(rec.gap_q.astype(np.uint32), np.int32), last_ret=conv(rec.last_ret.astype(np.uint32), np.int32),
+                turn=conv(rec.turn.astype(np.uint16), np.int16), kv_tok=conv(rec.kv_tok.astype(np.uint32), np.int32),
+                tier=conv(rec.tier.astype(np.uint8), np.uint8), flags=conv(rec.flags.astype(np.uint8), np.uint8))
+
+
+def rank_outputs(n: int, k: int, max_moves: int, keys: bool = False, device="cuda"):
+    import torch
+    z = lambda m, dt: torch.zeros(max(m, 1), dtype=dt, device=device)
+    return dict(victims=z(k, torch.int32), promote=z(max_moves, torch.int32), demote=z(max_moves, torch.int32),
+                counts=z(4, torch.int32), moved=z(1, torch.int64), keys=z(n, torch.int64) if keys else None)
+
+
+def rank_batch(sets: Sequence[dict], params: Sequence[dict], outs: Sequence[dict], stream=None) -> None:
+    """unison_rank_batch over device record sets; params per set: sigma_q[51],
+    k, penalty_q, budget_bytes, kv_bytes_per_token, max_moves, free_fast_tok,
+    free_hbm_tok."""
+    n = len(sets)
+    rs = (Records * n)()
+    ps = (RankParams * n)()
+    os_ = (RankOut * n)()
+    for i, (r, p, o) in enumerate(zip(sets, params, outs)):
+        rs[i] = Records(r["gap_q"].data_ptr(), r["last_ret"].data_ptr(), r["turn"].data_ptr(),
+                        r["kv_tok"].data_ptr(), r["tier"].data_ptr(), r["flags"].data_ptr(), r["gap_q"].numel())
+        sig = (C.c_uint16 * 51)(*[int(x) for x in p["sigma_q"]])
+        ps[i] = RankParams(sig, 0, p.get("k", 0), p.get("penalty_q", 500_000_000), p.get("budget_bytes", 0),
+                           p.get("kv_bytes_per_token", 131072), p.get("max_moves", 0), p.get("free_fast_tok", 0),
+                           p.get("free_hbm_tok", 0))
+        os_[i] = RankOut(o["victims"].data_ptr(), o["promote"].data_ptr(), o["demote"].data_ptr(),
+                         o["counts"].data_ptr(), o["moved"].data_ptr(),
+                         None if o.get("keys") is None else o["keys"].data_ptr())
+    _check("unison_rank_batch", lib().unison_rank_batch(rs, ps, os_, n, _stream_handle(stream)))
+
+
+def rank_result(o: dict) -> dict:
+    """Host copy of one set's outputs."""
+    c = o["counts"].cpu().numpy().astype(np.uint32)
+    res = dict(victims=o["victims"].cpu().numpy().astype(np.uint32)[: c[0]],
+               promote=o["promote"].cpu().numpy().astype(np.uint32)[: c[1]],
+               demote=o["demote"].cpu().numpy().astype(np.uint32)[: c[2]],
+               moved_bytes=int(o["moved"].cpu().numpy().astype(np.uint64)[0]), status=int(c[3]))
+    if o.get("keys") is not None:
+        res["keys"] = o["keys"].cpu().numpy().view(np.uint64)
+    return res

@@ -1,6 +1,1217 @@
-// placeholder: the standalone ranking kernels are added next
+// Standalone ranking of large live sets (the scan of Sec. IV-D, eqs. pipe and
+// scan, generalised from one argmax to a top-k) and the TIDE fill of
+// Sec. III-C (eqs. budget, promote, demote) over the same ranking.
+//
+// Every record gets a packed comparable key ck = score40 << 24 | ~index24:
+// unsigned order on ck is the ranking order (larger score first, ties to
+// the smaller index).  Three ordered selections are needed per live set:
+//   V  victims: unpinned resident records, largest ck first (top-k);
+//   D  fast-tier demotion candidates: unpinned fast-tier records, largest first;
+//   P  HBM promotion candidates: unpinned HBM records, smallest ck first.
+// Kernels, in launch order:
+//   rank_sample_kernel   16 CTAs per set: exact order statistics of a
+//                        jittered stratified sample give each list a threshold, turned
+//                        into per-turn thresholds on the gap average (the
+//                        score is monotone in the gap for a fixed turn, so
+//                        the streaming test needs no division).
+//   rank_filter_kernel   one pass over every record (8 B each: gap average,
+//                        turn, flags, tier), emitting the exact values of the
+//                        records that pass a threshold.
+//   rank_finish_kernel   one CTA per set: exact top-M of the candidates by
+//                        radix select, bitonic sort, the victims, and the
+//                        fill as warp prefix scans.  If a list's candidates
+//                        overflowed or fell short, the CTA re-selects that
+//                        list exactly by streaming the whole set.
+#include <algorithm>
+#include <type_traits>
+#include <vector>
+
 #include "common.cuh"
-extern "C" int unison_rank_batch(const unison_records *, const unison_rank_params *, const unison_rank_out *, int,
-                                 void *) {
-  return UNISON_ERR_ARG;
+#include "profile.cuh"
+
+using namespace unison;
+
+namespace {
+
+constexpr int kLists = 3;  // 0 = V, 1 = D, 2 = P
+constexpr uint32_t kSample = 16384;
+constexpr uint32_t kSmemCand = 16384;
+constexpr uint32_t kCandCap = 65536;
+constexpr uint32_t kMaxSel = 4096;
+constexpr uint32_t kFinishThreads = 1024;
+constexpr uint32_t kFull = 0xFFFFFFFFu;
+
+struct RankWork {
+  unsigned int cand[kLists];
+  unsigned int status;  // UNISON_ERR_TIMEOUT if a bounded wait gave up
+  unsigned long long elig[kLists];
+  unsigned int ticket;  // sample CTAs finished
+  unsigned int pad2;
+};
+
+constexpr uint32_t kSampleCtas = 16;     // sample CTAs per set
+constexpr uint32_t kSampleThreads = 1024;
+constexpr uint32_t kMaxR = 256;          // largest sample rank used for a threshold
+
+struct RankSet {
+  const uint32_t *gap;
+  const uint16_t *turn;
+  const uint32_t *kv;
+  const uint8_t *tier;
+  const uint8_t *flags;
+  uint32_t n, k, max_moves, kvb;
+  uint64_t penalty, budget, free_s, free_h;
+  uint32_t *victims, *promote, *demote, *counts;
+  uint64_t *moved, *keys;
+  uint32_t tile0, ntiles;
+  uint32_t sigma[kLutN];
+  uint32_t pad;
+  // scratch (per set)
+  RankWork *work;
+  uint64_t *cand;    // [3][kCandCap]
+  uint64_t *sorted;  // [3][kMaxSel]
+  uint2 *gthr;       // [3][51] (gA, gB)
+  uint64_t *thr;     // [3] threshold in list-value space; [3+L] = active flag
+  uint64_t *t2;      // [51]
+  uint64_t *magic;   // [51]
+  uint64_t *part;    // [3][kSampleCtas][kMaxR] per-CTA top values of the sample
+};
+
+// ---------------------------------------------------------------- keys ----
+// floor(x / s) for x < 2^43 and 2 <= s < 2^12 by one multiply-high
+// (Granlund and Montgomery, PLDI 1994, Thm 4.2 with N = 43): with
+// l = ceil(log2 s) and m = ceil(2^(43+l) / s), floor(x/s) = floor(x m / 2^(43+l));
+// storing m << (21 - l) turns that into the high word of a 64x64 product.
+__host__ __device__ inline uint64_t magic_for(uint32_t s) {
+  uint32_t l = 0;
+  while ((1u << l) < s) l++;
+  // m = ceil(2^(43+l) / s) fits 44 bits; compute without 128-bit division.
+  const uint64_t num = 1ull << (43 + l);  // 43 + l <= 55
+  const uint64_t m = (num + s - 1) / s;
+  return m << (21 - l);
+}
+
+__device__ __forceinline__ uint64_t score_of(uint32_t g, uint32_t t, bool done, const uint64_t *t2,
+                                             const uint64_t *magic) {
+  if (done) return ~0ull;
+  return __umul64hi((uint64_t)g * kLambda, magic[t]) + t2[t];
+}
+
+__device__ __forceinline__ uint64_t ck_of(uint64_t score, uint32_t idx) {
+  const uint64_t k40 = score == ~0ull ? kKeyMax40 : score;
+  return (k40 << 24) | ((~idx) & kIdMask);
+}
+
+__device__ __forceinline__ uint32_t elig_mask(uint8_t fl, uint8_t tr) {
+  if (fl & 1) return 0;  // pinned: never ranked for eviction or migration
+  uint32_t m = 0;
+  if (tr == 1) m = 1u | 2u;
+  if (tr == 2) m = 1u | 4u;
+  return m;
+}
+
+// Smallest gap average whose score reaches K at turn index t.
+__device__ __forceinline__ uint32_t g_at_least(uint64_t K, uint32_t sigma, uint64_t t2) {
+  if (K <= t2) return 0;
+  const uint64_t m = K - t2;
+  const uint64_t g = (m * sigma + kLambda - 1) / kLambda;
+  return g > 0xFFFFFFFFull ? 0xFFFFFFFFu : (uint32_t)g;
+}
+
+// -------------------------------------------------------- block helpers ----
+// Value with the given rank (1 = largest) among get(0..n-1) -- MSB-first
+// radix select, 8 bits per pass.  All threads of the block call it and get
+// the same value.
+template <typename Get>
+__device__ uint64_t block_select_rank(Get get, uint32_t n, uint32_t rank, unsigned int *hist,
+                                      unsigned long long *bcast) {
+  // bytes on which every value agrees need no pass: start at the highest
+  // byte where some two values differ
+  unsigned long long a = ~0ull, o = 0ull;
+  for (uint32_t i = threadIdx.x; i < n; i += blockDim.x) {
+    const uint64_t v = get(i);
+    a &= v;
+    o |= v;
+  }
+  for (int s = 16; s; s >>= 1) {
+    a &= __shfl_xor_sync(0xFFFFFFFFu, a, s);
+    o |= __shfl_xor_sync(0xFFFFFFFFu, o, s);
+  }
+  if (threadIdx.x == 0) {
+    bcast[0] = ~0ull;
+    bcast[1] = 0ull;
+  }
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) {
+    atomicAnd(&bcast[0], a);
+    atomicOr(&bcast[1], o);
+  }
+  __syncthreads();
+  const uint64_t same = ~(bcast[0] ^ bcast[1]);  // bits equal in every value
+  const uint64_t common = bcast[0] & same;
+  int top = 7;
+  while (top > 0 && ((same >> (8 * top)) & 0xFF) == 0xFF) top--;
+  __syncthreads();
+  uint64_t mask = top < 7 ? (~0ull << (8 * (top + 1))) : 0ull;
+  uint64_t prefix = common & mask;
+  uint32_t need = rank;
+  for (int b = top; b >= 0; b--) {
+    for (uint32_t i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    for (uint32_t base = 0; base < n; base += blockDim.x) {
+      const uint32_t i = base + threadIdx.x;
+      bool in = false;
+      uint32_t d = 0;
+      if (i < n) {
+        const uint64_t v = get(i);
+        in = (v & mask) == prefix;
+        d = (uint32_t)(v >> (8 * b)) & 0xFF;
+      }
+      // lanes with the same digit add once per group
+      const unsigned act = __ballot_sync(0xFFFFFFFFu, in);
+      if (in) {
+        const unsigned grp = __match_any_sync(act, d);
+        if ((__ffs(grp) - 1) == (int)(threadIdx.x & 31)) atomicAdd(&hist[d], (unsigned)__popc(grp));
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x < 32) {
+      // lane l owns digits 255-8l .. 248-8l (descending); find the digit where
+      // the count of larger-or-equal values first reaches `need`
+      const int l = threadIdx.x;
+      uint32_t c[8], tot = 0;
+#pragma unroll
+      for (int q = 0; q < 8; q++) {
+        c[q] = hist[255 - 8 * l - q];
+        tot += c[q];
+      }
+      uint32_t incl = tot;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, incl, o);
+        if (l >= o) incl += y;
+      }
+      const uint32_t excl = incl - tot;
+      const unsigned hit = __ballot_sync(0xFFFFFFFFu, excl < need && incl >= need);
+      if (l == __ffs(hit) - 1) {
+        uint32_t cum = excl;
+        for (int q = 0; q < 8; q++) {
+          if (cum + c[q] >= need) {
+            bcast[0] = (unsigned long long)(255 - 8 * l - q);
+            bcast[1] = need - cum;
+            break;
+          }
+          cum += c[q];
+        }
+      }
+    }
+    __syncthreads();
+    prefix |= (uint64_t)bcast[0] << (8 * b);
+    mask |= 0xFFull << (8 * b);
+    need = (uint32_t)bcast[1];
+    __syncthreads();
+  }
+  return prefix;
+}
+
+// Bitonic sort, descending, of a[0..n) padded with zeros to a power of two.
+__device__ void block_sort_desc(uint64_t *a, uint32_t n) {
+  uint32_t p = 1;
+  while (p < n) p <<= 1;
+  for (uint32_t i = n + threadIdx.x; i < p; i += blockDim.x) a[i] = 0;
+  __syncthreads();
+  for (uint32_t k = 2; k <= p; k <<= 1) {
+    for (uint32_t j = k >> 1; j > 0; j >>= 1) {
+      for (uint32_t i = threadIdx.x; i < p; i += blockDim.x) {
+        const uint32_t ij = i ^ j;
+        if (ij > i) {
+          const uint64_t x = a[i], y = a[ij];
+          const bool desc = (i & k) == 0;
+          if (desc ? (x < y) : (x > y)) {
+            a[i] = y;
+            a[ij] = x;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+}
+
+__device__ __forceinline__ uint64_t list_val(uint64_t ck, int L) { return L == 2 ? ~ck : ck; }
+
+// ------------------------------------------------------------- sample ----
+// Sample size and per-list ranks: ns records (ns/8 runs of 8, one run per
+// stratum) and rank r_L = ceil(target_L * ns / n), with ns chosen so that no
+// r_L exceeds kMaxR; target_L = 6 M_L + 2048 candidates for M_L needed.
+__device__ __forceinline__ uint64_t umin64(uint64_t a, uint64_t b) { return a < b ? a : b; }
+__device__ __forceinline__ uint64_t list_target(const RankSet &S, int L) {
+  const uint32_t M = (L == 0) ? S.k : S.max_moves;
+  return 6ull * M + 2048;
+}
+__device__ __forceinline__ bool list_active(const RankSet &S, int L) {
+  const uint32_t M = (L == 0) ? S.k : S.max_moves;
+  return M > 0 && (L == 0 || S.budget > 0);
+}
+__device__ __forceinline__ uint32_t sample_size(const RankSet &S) {
+  const uint32_t n = S.n;
+  if (n <= kSample) return 0;  // whole set: every eligible record is a candidate
+  uint64_t tmax = 0;
+  for (int L = 0; L < kLists; L++)
+    if (list_active(S, L) && list_target(S, L) > tmax) tmax = list_target(S, L);
+  if (tmax == 0) return 0;
+  uint64_t ns = ((uint64_t)kMaxR * n) / tmax;
+  ns = ns < kSample ? ns : kSample;
+  ns &= ~(uint64_t)(8 * kSampleCtas - 1);  // whole runs, evenly split over the CTAs
+  return (uint32_t)ns;
+}
+
+// The value of rank r (1 = largest) among the block's values v (one per
+// thread; `has` false for threads without one), built MSB first: a bit is
+// kept when at least r values reach the prefix with that bit set.  Bits on
+// which all values agree are taken directly.  All threads get the result.
+__device__ uint64_t block_rank_bitwise(uint64_t v, bool has, uint32_t r, unsigned long long *sh) {
+  if (threadIdx.x == 0) {
+    sh[0] = ~0ull;
+    sh[1] = 0ull;
+  }
+  __syncthreads();
+  unsigned long long a = has ? v : ~0ull, o = has ? v : 0ull;
+  for (int s = 16; s; s >>= 1) {
+    a &= __shfl_xor_sync(0xFFFFFFFFu, a, s);
+    o |= __shfl_xor_sync(0xFFFFFFFFu, o, s);
+  }
+  if ((threadIdx.x & 31) == 0) {
+    atomicAnd(&sh[0], a);
+    atomicOr(&sh[1], o);
+  }
+  __syncthreads();
+  const uint64_t same = ~(sh[0] ^ sh[1]);
+  uint64_t T = sh[0] & same;  // bits every value shares
+  __syncthreads();
+  for (int b = 63; b >= 0; b--) {
+    if ((same >> b) & 1) continue;
+    const uint64_t cand = T | (1ull << b);  // undecided lower bits of T are still 0
+    const int cnt = __syncthreads_count(has && v >= cand);
+    if ((uint32_t)cnt >= r) T = cand;
+  }
+  return T;
+}
+
+__global__ void __launch_bounds__(1024) rank_sample_kernel(const RankSet *sets) {
+  const RankSet &S = sets[blockIdx.y];
+  const uint32_t c = blockIdx.x;  // this CTA's share of the sample
+  __shared__ uint64_t t2s[kLutN], mgs[kLutN];
+  __shared__ unsigned long long sh[2];
+  __shared__ unsigned int is_last, wpos;
+  if (threadIdx.x < kLutN) {
+    const uint32_t sg = S.sigma[threadIdx.x];
+    t2s[threadIdx.x] = ((uint64_t)(kLambda - sg) * S.penalty) / kLambda;  // eq. (t2)
+    mgs[threadIdx.x] = magic_for(sg);
+  }
+  __syncthreads();
+  const uint32_t n = S.n;
+  const uint32_t ns = sample_size(S);
+  const uint32_t per = ns / kSampleCtas;  // samples of this CTA (<= 1024, a multiple of 8)
+  // 1. one sample per thread: run j covers stratum j of ns/8, 8 records at a hashed offset
+  uint64_t ck = 0;
+  uint32_t m = 0;
+  if (ns && threadIdx.x < per) {
+    const uint32_t nruns = ns / 8, run = c * (per / 8) + threadIdx.x / 8, o = threadIdx.x % 8;
+    const uint64_t lo = ((uint64_t)run * n) / nruns, hi = ((uint64_t)(run + 1) * n) / nruns;
+    uint32_t h = run * 0x9E3779B1u;
+    h ^= h >> 16;
+    h *= 0x85EBCA6Bu;
+    h ^= h >> 13;
+    const uint32_t span = (uint32_t)(hi - lo) - 8;  // strata hold at least 8 records
+    const uint32_t r = (uint32_t)(lo + (h % (span + 1))) + o;
+    const uint8_t fl = S.flags[r], tr = S.tier[r];
+    const uint32_t t = min((uint32_t)S.turn[r], kTMax);
+    ck = ck_of(score_of(S.gap[r], t, (fl & 2) != 0, t2s, mgs), r);
+    m = elig_mask(fl, tr);
+  }
+  // 2. per list: this CTA's top r values (exactly r, values are distinct)
+  for (int L = 0; L < kLists; L++) {
+    if (!ns || !list_active(S, L)) continue;
+    const uint32_t r = (uint32_t)umin64((list_target(S, L) * ns + n - 1) / n, kMaxR);
+    const bool has = (m >> L) & 1;
+    const uint64_t v = has ? list_val(ck, L) : 0ull;
+    const uint32_t navail = (uint32_t)__syncthreads_count(has);
+    uint64_t *dst = S.part + ((size_t)L * kSampleCtas + c) * kMaxR;
+    if (threadIdx.x == 0) wpos = 0;
+    if (navail <= r) {
+      __syncthreads();
+      if (has) {
+        const uint32_t w = atomicAdd(&wpos, 1u);
+        if (w < r) dst[w] = v;
+      }
+      __syncthreads();
+      for (uint32_t q = navail + threadIdx.x; q < r; q += blockDim.x) dst[q] = 0ull;
+    } else {
+      const uint64_t T = block_rank_bitwise(v, has, r, sh);
+      if (has && v >= T) {
+        const uint32_t w = atomicAdd(&wpos, 1u);
+        if (w < r) dst[w] = v;
+      }
+    }
+    __syncthreads();
+  }
+  // 3. the last CTA to finish merges the partial lists and sets the thresholds
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) is_last = (atomicAdd(&S.work->ticket, 1u) == kSampleCtas - 1);
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  if (threadIdx.x < kLutN) {
+    S.t2[threadIdx.x] = t2s[threadIdx.x];
+    S.magic[threadIdx.x] = mgs[threadIdx.x];
+  }
+  for (int L = 0; L < kLists; L++) {
+    const bool active = list_active(S, L);
+    uint64_t thrv = 0;  // 0: accept every eligible record
+    if (ns && active) {
+      const uint32_t r = (uint32_t)umin64((list_target(S, L) * ns + n - 1) / n, kMaxR);
+      // kSampleCtas * r <= 4096 values: one per thread (with the shared-bit
+      // skip) when they fit in the block, else four per thread
+      const uint32_t nv = kSampleCtas * r;
+      uint64_t T = 0;
+      if (nv <= blockDim.x) {
+        const uint32_t idx = threadIdx.x;
+        uint64_t v = idx < nv ? __ldcg(&S.part[((size_t)L * kSampleCtas + idx / r) * kMaxR + idx % r]) : 0ull;
+        const bool has = idx < nv && v != 0ull;
+        T = block_rank_bitwise(v, has, r, sh);
+        if (__syncthreads_count(has) < (int)r) T = 0;
+      } else {
+        uint64_t vq[4];
+        bool hq[4];
+        for (int q = 0; q < 4; q++) {
+          const uint32_t idx = threadIdx.x + 1024u * q;
+          hq[q] = idx < nv;
+          vq[q] = hq[q] ? __ldcg(&S.part[((size_t)L * kSampleCtas + idx / r) * kMaxR + idx % r]) : 0ull;
+          hq[q] = hq[q] && vq[q] != 0ull;
+        }
+        for (int b = 63; b >= 0; b--) {
+          const uint64_t cand = T | (1ull << b);
+          int cnt = 0;
+          for (int q = 0; q < 4; q++) cnt += __syncthreads_count(hq[q] && vq[q] >= cand);
+          if ((uint32_t)cnt >= r) T = cand;
+        }
+      }
+      thrv = T;  // 0 when fewer than r eligible samples
+    }
+    if (threadIdx.x == 0) {
+      S.thr[L] = thrv;
+      S.thr[kLists + L] = active ? 1 : 0;
+    }
+    if (threadIdx.x < kLutN) {
+      const uint32_t t = threadIdx.x;
+      const uint64_t thr_ck = (L == 2) ? ~thrv : thrv;
+      const uint64_t K = thr_ck >> 24;
+      S.gthr[L * kLutN + t] = make_uint2(g_at_least(K, S.sigma[t], t2s[t]), g_at_least(K + 1, S.sigma[t], t2s[t]));
+    }
+    __syncthreads();
+  }
+}
+
+// ------------------------------------------------------------- filter ----
+__device__ __forceinline__ int set_of_tile(const RankSet *sets, int n_sets, uint32_t tile) {
+  int lo = 0, hi = n_sets - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (sets[mid].tile0 <= tile) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+struct SetConst {
+  uint32_t loV, loD, loP;      // index thresholds of the tie on the threshold key
+  uint32_t dV, dD;             // completed records pass V / D iff lo >= dV / dD
+  int32_t dP;                  // completed records pass P iff lo <= dP
+  uint32_t act;                // active lists (bit L)
+  uint32_t never;              // bit 2L: column A of list L passes no gap; bit 2L+1: column B
+};
+
+// ---- TMA 1-D bulk copies and mbarriers (inline PTX, sm_90+) ----
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count));
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_addr(dst)),
+      "l"(src), "r"(bytes), "r"(smem_addr(bar))
+      : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// Bounded wait on an mbarrier phase; false when the bound ran out.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity) {
+  for (uint32_t it = 0; it < (1u << 22); it++)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
+}
+
+constexpr int kStages = 2;
+constexpr uint32_t kRec = 16;                         // records per consumer thread per tile
+constexpr uint32_t kConsumers = 256;                  // consumer threads (8 warps)
+constexpr uint32_t kBigTile = kConsumers * kRec;      // 4096 records per tile
+constexpr uint32_t kFilterCtaThreads = kConsumers + 32;  // + one producer warp
+struct __align__(128) FilterStage {
+  uint32_t gap[kBigTile];
+  uint16_t turn[kBigTile];
+  uint8_t flags[kBigTile];
+  uint8_t tier[kBigTile];
+};
+constexpr size_t kFilterSmem = sizeof(FilterStage) * kStages;
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+// Barrier 1 over the consumer warps only (the producer warp never joins it).
+__device__ __forceinline__ void consumers_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kConsumers) : "memory"); }
+// A tile is copied by TMA when it is whole (the arrays' 16-byte alignment is
+// checked by the host); the last, partial tile of a set is read directly.
+__device__ __forceinline__ bool tile_is_bulk(const RankSet &S, uint32_t tile) {
+  return (tile - S.tile0 + 1) * kBigTile <= S.n;
+}
+
+__device__ __forceinline__ int set_of(const RankSet *sets, int si, uint32_t tile) {
+  while (tile >= sets[si].tile0 + sets[si].ntiles) si++;
+  return si;
+}
+
+// Thresholds of one set into shared memory (consumer threads call it).  Per
+// turn index: vd = (gA_V, gB_V, gA_D, gB_D), pp = (gA_P, gB_P); an inactive
+// list gets bounds no gap passes.
+__device__ void load_set(const RankSet &S, uint4 *vd, uint2 *pp, uint64_t *t2s, uint64_t *mgs, SetConst &c,
+                         unsigned int *never_sh) {
+  consumers_sync();
+  if (threadIdx.x == 0) *never_sh = 0x3Fu;
+  consumers_sync();
+  const bool aV = S.thr[kLists + 0] != 0, aD = S.thr[kLists + 1] != 0, aP = S.thr[kLists + 2] != 0;
+  if (threadIdx.x < kLutN) {
+    const uint32_t t = threadIdx.x;
+    const uint2 a0 = S.gthr[t], a1 = S.gthr[kLutN + t], a2 = S.gthr[2 * kLutN + t];
+    const uint4 v = make_uint4(aV ? a0.x : kFull, aV ? a0.y : kFull, aD ? a1.x : kFull, aD ? a1.y : kFull);
+    const uint2 w = aP ? a2 : make_uint2(0u, 0u);
+    vd[t] = v;
+    pp[t] = w;
+    t2s[t] = S.t2[t];
+    mgs[t] = S.magic[t];
+    // gaps are below 2^31: a V/D bound of 2^31 or more, or a P bound of 0, passes nothing
+    const uint32_t nv = (v.x >= 0x80000000u ? 1u : 0u) | (v.y >= 0x80000000u ? 2u : 0u) |
+                        (v.z >= 0x80000000u ? 4u : 0u) | (v.w >= 0x80000000u ? 8u : 0u) |
+                        (w.x == 0u ? 16u : 0u) | (w.y == 0u ? 32u : 0u);
+    atomicAnd(never_sh, nv);
+  }
+  uint32_t lo[kLists], dok[kLists];
+#pragma unroll
+  for (int L = 0; L < kLists; L++) {
+    const uint64_t thrv = S.thr[L];
+    const uint64_t thr_ck = (L == 2) ? ~thrv : thrv;
+    const uint64_t K = thr_ck >> 24;
+    lo[L] = (uint32_t)(thr_ck & kIdMask);
+    // a completed record has the maximal key 2^40 - 1: 2 = always passes,
+    // 1 = passes on the index part, 0 = never
+    dok[L] = (L == 2) ? (kKeyMax40 == K ? 1u : 0u) : (kKeyMax40 > K ? 2u : (kKeyMax40 == K ? 1u : 0u));
+  }
+  c.loV = lo[0];
+  c.loD = lo[1];
+  c.loP = lo[2];
+  c.dV = !aV ? 0x1000000u : (dok[0] == 2 ? 0u : (dok[0] == 1 ? lo[0] : 0x1000000u));
+  c.dD = !aD ? 0x1000000u : (dok[1] == 2 ? 0u : (dok[1] == 1 ? lo[1] : 0x1000000u));
+  c.dP = (aP && dok[2] == 1) ? (int32_t)lo[2] : -1;
+  c.act = (aV ? 1u : 0u) | (aD ? 2u : 0u) | (aP ? 4u : 0u);
+  consumers_sync();
+  c.never = *never_sh;
+}
+
+__device__ __forceinline__ void flush_elig(const RankSet &P, uint32_t &eD, uint32_t &eP, int lane) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    eD += __shfl_xor_sync(kFull, eD, o);
+    eP += __shfl_xor_sync(kFull, eP, o);
+  }
+  if (lane == 0) {
+    atomicAdd(&P.work->elig[0], (unsigned long long)(eD + eP));
+    atomicAdd(&P.work->elig[1], (unsigned long long)eD);
+    atomicAdd(&P.work->elig[2], (unsigned long long)eP);
+  }
+  eD = eP = 0;
+}
+
+// Persistent streaming pass.  Each CTA owns a contiguous range of tiles; its
+// producer warp keeps kStages tiles in flight with TMA bulk copies into
+// shared memory ("full" barriers), and its eight consumer warps test every
+// record of each tile against the set's thresholds, then hand the stage back
+// ("empty" barriers).  Every wait is bounded; a CTA that gives up records
+// UNISON_ERR_TIMEOUT, lets its own copies land (bounded) and returns.
+__global__ void __launch_bounds__(kFilterCtaThreads, 3) rank_filter_kernel(const RankSet *sets, int n_sets,
+                                                                        uint32_t total_tiles) {
+  extern __shared__ __align__(128) unsigned char fsm[];
+  FilterStage *stage = reinterpret_cast<FilterStage *>(fsm);
+  __shared__ __align__(8) uint64_t full[kStages], empty[kStages];
+  __shared__ uint4 vd[kLutN];
+  __shared__ uint2 pp[kLutN];
+  __shared__ uint64_t t2s[kLutN], mgs[kLutN];
+  __shared__ unsigned int never_sh;
+  const uint32_t t_begin = (uint32_t)(((uint64_t)blockIdx.x * total_tiles) / gridDim.x);
+  const uint32_t t_end = (uint32_t)(((uint64_t)(blockIdx.x + 1) * total_tiles) / gridDim.x);
+  if (t_begin >= t_end) return;
+  if (threadIdx.x == 0) {
+    for (int q = 0; q < kStages; q++) {
+      mbar_init(&full[q], 1);
+      mbar_init(&empty[q], kConsumers / 32);
+    }
+    fence_mbar_init();
+  }
+  __syncthreads();
+  const int si0 = set_of_tile(sets, n_sets, t_begin);
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x >= kConsumers) {
+    // ---------------- producer warp (one lane issues)
+    if (lane != 0) return;
+    int si = si0;
+    uint32_t fills[kStages] = {};  // bulk copies issued into each stage (one full-barrier phase each)
+    uint32_t issued = 0;           // bit q: the last copy into stage q may still be in flight
+    bool failed = false;
+    for (uint32_t i = 0, tile = t_begin; tile < t_end; i++, tile++) {
+      const int q = (int)(i % kStages);
+      if (i >= (uint32_t)kStages) {
+        // wait until the consumers released this stage's previous tile
+        if (!mbar_wait_bounded(&empty[q], ((i / kStages) - 1) & 1)) {
+          failed = true;
+          break;
+        }
+        issued &= ~(1u << q);
+      }
+      si = set_of(sets, si, tile);
+      const RankSet &T = sets[si];
+      if (!tile_is_bulk(T, tile)) continue;
+      const uint32_t base = (tile - T.tile0) * kBigTile;
+      FilterStage &d = stage[q];
+      fence_proxy_async();
+      mbar_expect_tx(&full[q], kBigTile * 8);
+      bulk_g2s(d.gap, T.gap + base, kBigTile * 4, &full[q]);
+      bulk_g2s(d.turn, T.turn + base, kBigTile * 2, &full[q]);
+      bulk_g2s(d.flags, T.flags + base, kBigTile, &full[q]);
+      bulk_g2s(d.tier, T.tier + base, kBigTile, &full[q]);
+      issued |= 1u << q;
+      fills[q]++;
+    }
+    if (failed) {
+      atomicExch(&sets[si0].work->status, (unsigned int)UNISON_ERR_TIMEOUT);
+      // consumers that still wait will time out too; let this CTA's copies land
+      // (phase fills-1 of each stage's full barrier) before the CTA exits
+      for (int q = 0; q < kStages; q++)
+        if ((issued >> q) & 1) mbar_wait_bounded(&full[q], (fills[q] - 1) & 1);
+    }
+    return;
+  }
+
+  // ---------------- consumer warps
+  int si = si0, lsi = -1;
+  SetConst c;
+  uint32_t eD = 0, eP = 0;
+  uint32_t fph = 0;  // bit q: parity of the next full-barrier phase of stage q (flips per bulk tile)
+  // this set's hot descriptor fields, cached when the set changes (pointers
+  // used only on rare paths are read from the descriptor there)
+  uint32_t s_n = 0, s_tile0 = 0, s_end = 0;
+  bool s_keys = false;
+  for (uint32_t i = 0, tile = t_begin; tile < t_end; i++, tile++) {
+    const int q = (int)(i % kStages);
+    if (lsi < 0 || tile >= s_end) {
+      si = set_of(sets, si, tile);
+      const RankSet &S = sets[si];
+      if (lsi >= 0) flush_elig(sets[lsi], eD, eP, lane);
+      load_set(S, vd, pp, t2s, mgs, c, &never_sh);
+      lsi = si;
+      s_n = S.n;
+      s_tile0 = S.tile0;
+      s_end = S.tile0 + S.ntiles;
+      s_keys = S.keys != nullptr;
+    }
+    const uint32_t tb = (tile - s_tile0) * kBigTile;
+    const bool bulk = tb + kBigTile <= s_n;
+    const uint32_t r0 = threadIdx.x * kRec;
+    uint32_t g[kRec], tw[kRec / 2], fw[kRec / 4], rw[kRec / 4];
+    uint32_t cnt = kRec;
+    if (bulk) {
+      // a timed-out wait is reported, not collective: every wait here is
+      // bounded, so the CTA still ends (with undefined results)
+      if (!mbar_wait_bounded(&full[q], (fph >> q) & 1))
+        atomicExch(&sets[si0].work->status, (unsigned int)UNISON_ERR_TIMEOUT);
+      fph ^= 1u << q;
+      const FilterStage &d = stage[q];
+#pragma unroll
+      for (int v = 0; v < (int)(kRec / 4); v++) {
+        const uint4 gq = *reinterpret_cast<const uint4 *>(d.gap + r0 + 4 * v);
+        g[4 * v] = gq.x; g[4 * v + 1] = gq.y; g[4 * v + 2] = gq.z; g[4 * v + 3] = gq.w;
+      }
+#pragma unroll
+      for (int v = 0; v < (int)(kRec / 8); v++) {
+        const uint4 tq = *reinterpret_cast<const uint4 *>(d.turn + r0 + 8 * v);
+        tw[4 * v] = tq.x; tw[4 * v + 1] = tq.y; tw[4 * v + 2] = tq.z; tw[4 * v + 3] = tq.w;
+      }
+      const uint4 fq = *reinterpret_cast<const uint4 *>(d.flags + r0);
+      const uint4 rq = *reinterpret_cast<const uint4 *>(d.tier + r0);
+      fw[0] = fq.x; fw[1] = fq.y; fw[2] = fq.z; fw[3] = fq.w;
+      rw[0] = rq.x; rw[1] = rq.y; rw[2] = rq.z; rw[3] = rq.w;
+      // the stage's data is in registers: hand it back to the producer
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[q]);
+    } else {
+      const RankSet &S = sets[si];
+      const uint32_t *s_gap = S.gap;
+      const uint16_t *s_turn = S.turn;
+      const uint8_t *s_flags = S.flags, *s_tier = S.tier;
+      const uint32_t base = tb + r0;
+      cnt = base < s_n ? min(s_n - base, kRec) : 0;
+#pragma unroll
+      for (int v = 0; v < (int)(kRec / 2); v++) tw[v] = 0;
+#pragma unroll
+      for (int v = 0; v < (int)(kRec / 4); v++) {
+        fw[v] = 0x01010101u;  // padding reads as pinned: never eligible
+        rw[v] = 0;
+      }
+#pragma unroll
+      for (uint32_t k = 0; k < kRec; k++) {
+        g[k] = 0;
+        if (k < cnt) {
+          g[k] = s_gap[base + k];
+          tw[k >> 1] |= (uint32_t)s_turn[base + k] << (16 * (k & 1));
+          const uint32_t sh = 8 * (k & 3);
+          fw[k >> 2] = (fw[k >> 2] & ~(0xFFu << sh)) | ((uint32_t)s_flags[base + k] << sh);
+          rw[k >> 2] = (rw[k >> 2] & ~(0xFFu << sh)) | ((uint32_t)s_tier[base + k] << sh);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[q]);
+    }
+    const uint32_t base = tb + r0;
+    // Per-record masks, four records per 32-bit word (SWAR): eligible for V
+    // (unpinned resident), D (unpinned fast tier), P (unpinned HBM tier), and
+    // completed.  movemask turns 0x00/0xFF bytes into one bit per record.
+    uint32_t mEV = 0, mED = 0, mEP = 0, mDone = 0;
+#pragma unroll
+    for (int w = 0; w < (int)(kRec / 4); w++) {
+      const uint32_t unp = __vcmpeq4(fw[w] & 0x01010101u, 0u);
+      const uint32_t isS = __vcmpeq4(rw[w], 0x01010101u), isH = __vcmpeq4(rw[w], 0x02020202u);
+      const uint32_t dn = __vcmpne4(fw[w] & 0x02020202u, 0u);
+      auto movemask = [](uint32_t x) { return ((x & 0x01010101u) * 0x01020408u) >> 24; };
+      const uint32_t eDw = unp & isS, ePw = unp & isH;
+      eD += __popc(eDw) >> 3;
+      eP += __popc(ePw) >> 3;
+      mED |= movemask(eDw) << (4 * w);
+      mEP |= movemask(ePw) << (4 * w);
+      mEV |= movemask(eDw | ePw) << (4 * w);
+      mDone |= movemask(dn) << (4 * w);
+    }
+    // Index conditions over this tile: record indices rise through the tile,
+    // so lo = ~index falls from lo_hi to lo_lo and each tie condition on lo
+    // holds for all, none or a prefix of the tile.
+    const uint32_t tcount = min(kBigTile, s_n - tb);
+    const uint32_t lo_hi = (~tb) & kIdMask, lo_lo = (~(tb + tcount - 1)) & kIdMask;
+    // 0 none, 1 all, 2 mixed
+    auto ge_class = [&](uint32_t x) { return lo_lo >= x ? 1u : (lo_hi < x ? 0u : 2u); };                   // lo >= x
+    auto le_class = [&](int64_t x) { return (int64_t)lo_hi <= x ? 1u : ((int64_t)lo_lo > x ? 0u : 2u); };  // lo <= x
+    const uint32_t iV = ge_class(c.loV), iD = ge_class(c.loD), iP = le_class((int64_t)c.loP);
+    const uint32_t dV = ge_class(c.dV), dD = ge_class(c.dD), dP = le_class((int64_t)c.dP);
+    const bool mixed = ((c.act & 1) && (iV == 2 || dV == 2)) || ((c.act & 2) && (iD == 2 || dD == 2)) ||
+                       ((c.act & 4) && (iP == 2 || dP == 2));
+    uint32_t mV = 0, mD = 0, mP = 0;  // candidate bit per record, per list
+    if (!mixed) {
+      // column per list: V/D pass at g >= gA when the index part holds, else g >= gB;
+      // P passes at g < gB when it holds, else g < gA
+      const bool colV = iV == 1, colD = iD == 1, colP = iP == 1;
+      const bool nvV = !(c.act & 1) || ((c.never >> (colV ? 0 : 1)) & 1);
+      const bool nvD = !(c.act & 2) || ((c.never >> (colD ? 2 : 3)) & 1);
+      const bool nvP = !(c.act & 4) || ((c.never >> (colP ? 5 : 4)) & 1);
+      // completed records: one uniform answer per list for the whole tile
+      if ((c.act & 1) && dV == 1) mV = mDone;
+      if ((c.act & 2) && dD == 1) mD = mDone;
+      if ((c.act & 4) && dP == 1) mP = mDone;
+      if (!(nvV && nvD && nvP)) {
+        uint32_t nV = 0, nD = 0, nP = 0;  // live records' tests
+#pragma unroll
+        for (uint32_t k = 0; k < kRec; k++) {
+          const uint32_t t = min((tw[k >> 1] >> (16 * (k & 1))) & 0xFFFF, kTMax);
+          const uint32_t gg = g[k];
+          if (!(nvV && nvD)) {
+            const uint4 a = vd[t];
+            nV |= (uint32_t)(!nvV && gg >= (colV ? a.x : a.y)) << k;
+            nD |= (uint32_t)(!nvD && gg >= (colD ? a.z : a.w)) << k;
+          }
+          if (!nvP) {
+            const uint2 b = pp[t];
+            nP |= (uint32_t)(gg < (colP ? b.y : b.x)) << k;
+          }
+        }
+        mV |= nV & ~mDone;
+        mD |= nD & ~mDone;
+        mP |= nP & ~mDone;
+      }
+    } else {
+#pragma unroll
+      for (uint32_t k = 0; k < kRec; k++) {
+        const bool done = (mDone >> k) & 1;
+        const uint32_t t = min((tw[k >> 1] >> (16 * (k & 1))) & 0xFFFF, kTMax);
+        const uint32_t gg = g[k];
+        const uint32_t lo = (~(base + k)) & kIdMask;
+        const uint4 a = vd[t];
+        const uint2 b = pp[t];
+        const bool pV = done ? lo >= c.dV : (gg >= a.y || (gg >= a.x && lo >= c.loV));
+        const bool pD = done ? lo >= c.dD : (gg >= a.w || (gg >= a.z && lo >= c.loD));
+        const bool pP = done ? (int32_t)lo <= c.dP : (gg < b.x || (gg < b.y && lo <= c.loP));
+        mV |= (uint32_t)pV << k;
+        mD |= (uint32_t)pD << k;
+        mP |= (uint32_t)pP << k;
+      }
+    }
+    mV &= mEV;
+    mD &= mED;
+    mP &= mEP;
+    // emit candidates' exact values (warp-aggregated appends)
+#pragma unroll
+    for (int L = 0; L < kLists; L++) {
+      const uint32_t mm = L == 0 ? mV : (L == 1 ? mD : mP);
+      const uint32_t mine = __popc(mm);
+      if (!__any_sync(kFull, mine != 0)) continue;
+      uint32_t incl = mine;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += y;
+      }
+      const uint32_t total = __shfl_sync(kFull, incl, 31);
+      uint32_t basepos = 0;
+      if (lane == 31) basepos = atomicAdd(&sets[si].work->cand[L], total);
+      basepos = __shfl_sync(kFull, basepos, 31);
+      uint32_t pos = basepos + incl - mine;
+#pragma unroll
+      for (uint32_t k = 0; k < kRec; k++) {
+        if ((mm >> k) & 1) {
+          if (pos < kCandCap) {
+            const uint32_t t = min((tw[k >> 1] >> (16 * (k & 1))) & 0xFFFF, kTMax);
+            const uint64_t ck = ck_of(score_of(g[k], t, (mDone >> k) & 1, t2s, mgs), base + k);
+            sets[si].cand[(size_t)L * kCandCap + pos] = list_val(ck, L);
+          }
+          pos++;
+        }
+      }
+    }
+    if (s_keys) {
+      uint64_t *keys = sets[si].keys;
+#pragma unroll
+      for (uint32_t k = 0; k < kRec; k++) {
+        if (k >= cnt) break;
+        const uint32_t t = min((tw[k >> 1] >> (16 * (k & 1))) & 0xFFFF, kTMax);
+        keys[base + k] = score_of(g[k], t, (mDone >> k) & 1, t2s, mgs);
+      }
+    }
+  }
+  if (lsi >= 0) flush_elig(sets[lsi], eD, eP, lane);
+}
+
+// ------------------------------------------------------------- finish ----
+// Exact top-M of list L over the whole set by one CTA, streaming records and
+// keeping a pool of at most M + 4096 values (the fallback path).
+__device__ uint32_t stream_topM(const RankSet &S, int L, uint32_t M, uint64_t *pool, const uint64_t *t2s,
+                                const uint64_t *mgs, unsigned int *hist, unsigned long long *bcast,
+                                unsigned int *cnt) {
+  if (threadIdx.x == 0) *cnt = 0;
+  uint64_t floorv = 0;  // accept values strictly above (0 = accept all but 0)
+  bool have_floor = false;
+  __syncthreads();
+  for (uint32_t b = 0; b < S.n; b += 4 * blockDim.x) {
+    for (uint32_t q = 0; q < 4; q++) {
+      const uint32_t r = b + q * blockDim.x + threadIdx.x;
+      if (r < S.n) {
+        const uint32_t m = elig_mask(S.flags[r], S.tier[r]);
+        if ((m >> L) & 1) {
+          const uint32_t t = min((uint32_t)S.turn[r], kTMax);
+          const uint64_t v = list_val(ck_of(score_of(S.gap[r], t, (S.flags[r] & 2) != 0, t2s, mgs), r), L);
+          if (!have_floor || v > floorv) {
+            const uint32_t pos = atomicAdd(cnt, 1u);
+            if (pos < kSmemCand) pool[pos] = v;
+          }
+        }
+      }
+    }
+    __syncthreads();
+    const uint32_t c = min(*cnt, kSmemCand);
+    if (c > M) {
+      const uint64_t th = block_select_rank([&](uint32_t i) { return pool[i]; }, c, M, hist, bcast);
+      // compact in place: values >= th (exactly M, values are unique)
+      __syncthreads();
+      if (threadIdx.x == 0) *cnt = 0;
+      __syncthreads();
+      // two-step compaction through registers to avoid overwriting unread values
+      uint64_t keep[8];
+      uint32_t nk = 0;
+      for (uint32_t i = threadIdx.x; i < c; i += blockDim.x) {
+        const uint64_t v = pool[i];
+        if (v >= th && nk < 8) keep[nk++] = v;
+      }
+      __syncthreads();
+      for (uint32_t i = 0; i < nk; i++) pool[atomicAdd(cnt, 1u)] = keep[i];
+      __syncthreads();
+      floorv = th;
+      have_floor = true;
+    }
+    __syncthreads();
+  }
+  __syncthreads();
+  return min(*cnt, M);
+}
+
+__global__ void __launch_bounds__(kFinishThreads) rank_finish_kernel(const RankSet *sets) {
+  const RankSet &S = sets[blockIdx.x];
+  extern __shared__ __align__(16) unsigned char smem[];
+  uint64_t *buf = reinterpret_cast<uint64_t *>(smem);   // [kSmemCand]
+  uint64_t *sel = buf + kSmemCand;                      // [kMaxSel]
+  __shared__ uint64_t t2s[kLutN], mgs[kLutN];
+  __shared__ unsigned int hist[256];
+  __shared__ unsigned long long bcast[2];
+  __shared__ unsigned int cnt;
+  __shared__ uint32_t mL[kLists];
+  if (threadIdx.x < kLutN) {
+    t2s[threadIdx.x] = S.t2[threadIdx.x];
+    mgs[threadIdx.x] = S.magic[threadIdx.x];
+  }
+  __syncthreads();
+  for (int L = 0; L < kLists; L++) {
+    const bool active = S.thr[kLists + L] != 0;
+    const uint32_t Mw = (L == 0) ? S.k : S.max_moves;
+    const unsigned long long e = S.work->elig[L];
+    const uint32_t M = active ? (uint32_t)min((unsigned long long)Mw, e) : 0u;
+    const uint32_t emitted = S.work->cand[L];
+    uint32_t got = 0;
+    if (M > 0) {
+      const uint64_t *cand = S.cand + (size_t)L * kCandCap;
+      if (emitted <= kCandCap && emitted >= M) {
+        const uint32_t c = emitted;
+        const uint64_t *src = cand;
+        if (c <= kSmemCand) {
+          for (uint32_t i = threadIdx.x; i < c; i += blockDim.x) buf[i] = cand[i];
+          __syncthreads();
+          src = buf;
+        }
+        uint64_t th = 0;
+        if (c > M) th = block_select_rank([&](uint32_t i) { return src[i]; }, c, M, hist, bcast);
+        if (threadIdx.x == 0) cnt = 0;
+        __syncthreads();
+        for (uint32_t i = threadIdx.x; i < c; i += blockDim.x) {
+          const uint64_t v = src[i];
+          if (c <= M || v >= th) {
+            const uint32_t pos = atomicAdd(&cnt, 1u);
+            if (pos < kMaxSel) sel[pos] = v;
+          }
+        }
+        __syncthreads();
+        got = min(cnt, M);
+      } else {
+        // candidates overflowed the buffer or fell short of M: exact re-selection
+        got = stream_topM(S, L, M, buf, t2s, mgs, hist, bcast, &cnt);
+        for (uint32_t i = threadIdx.x; i < got; i += blockDim.x) sel[i] = buf[i];
+        __syncthreads();
+      }
+      block_sort_desc(sel, got);
+      for (uint32_t i = threadIdx.x; i < got; i += blockDim.x) S.sorted[(size_t)L * kMaxSel + i] = sel[i];
+    }
+    if (threadIdx.x == 0) mL[L] = got;
+    __syncthreads();
+  }
+  const uint64_t *V = S.sorted, *D = S.sorted + kMaxSel, *P = S.sorted + 2 * kMaxSel;
+  const uint32_t nv = mL[0], nd = mL[1], np = mL[2];
+  for (uint32_t i = threadIdx.x; i < nv; i += blockDim.x) S.victims[i] = (~(uint32_t)V[i]) & kIdMask;
+
+  // TIDE fill.  Stage P (ascending ck) and D (descending ck) with their sizes.
+  // Layout inside the dynamic area (the selection buffers are free now):
+  // pck, dck, dck2: kMaxSel u64 each; psz, dsz, dsz2: kMaxSel u32 each.
+  uint64_t *pck = buf;
+  uint64_t *dck = buf + kMaxSel;
+  uint64_t *dck2 = buf + 2 * kMaxSel;
+  uint32_t *psz = reinterpret_cast<uint32_t *>(buf + 3 * kMaxSel);
+  uint32_t *dsz = psz + kMaxSel;
+  uint32_t *dsz2 = dsz + kMaxSel;
+  for (uint32_t i = threadIdx.x; i < np; i += blockDim.x) {
+    const uint64_t ck = ~P[i];
+    pck[i] = ck;
+    psz[i] = S.kv[(~(uint32_t)ck) & kIdMask];
+  }
+  for (uint32_t i = threadIdx.x; i < nd; i += blockDim.x) {
+    dck[i] = D[i];
+    dsz[i] = S.kv[(~(uint32_t)D[i]) & kIdMask];
+  }
+  __syncthreads();
+  __shared__ uint32_t n1s, npairs;
+  __shared__ unsigned long long rem_s, fs_s, fh_s;
+  const uint64_t kvb = S.kvb;
+  const int lane = threadIdx.x & 31;
+  if (threadIdx.x < 32) {
+    // phase 1: promotions into free fast-tier space, least evictable first
+    uint64_t rem = S.budget, fs = S.free_s, fh = S.free_h;
+    uint32_t n1 = 0;
+    const uint32_t lim = min(np, S.max_moves);
+    bool stop = (S.thr[kLists + 2] == 0);
+    while (!stop && n1 < lim) {
+      const uint32_t j = n1 + lane;
+      const uint64_t sz = j < lim ? psz[j] : 0;
+      uint64_t by = sz * kvb, cs = sz;
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint64_t yb = __shfl_up_sync(kFull, by, o), ys = __shfl_up_sync(kFull, cs, o);
+        if (lane >= o) {
+          by += yb;
+          cs += ys;
+        }
+      }
+      const bool ok = j < lim && by <= rem && cs <= fs;
+      const uint32_t okm = __ballot_sync(kFull, ok);
+      const uint32_t take = __ffs(~okm) - 1;  // ok is a prefix (sums only grow)
+      const uint32_t tk = okm == kFull ? 32u : take;
+      if (tk > 0) {
+        const uint64_t tb = __shfl_sync(kFull, by, tk - 1), ts = __shfl_sync(kFull, cs, tk - 1);
+        rem -= tb;
+        fs -= ts;
+        fh += ts;
+      }
+      n1 += tk;
+      if (tk < 32) stop = true;
+    }
+    if (lane == 0) {
+      n1s = n1;
+      rem_s = rem;
+      fs_s = fs;
+      fh_s = fh;
+    }
+  }
+  __syncthreads();
+  const uint32_t n1 = n1s;
+  // phase 2 demotion order: fast-tier candidates merged with the promoted ones
+  // (only the first lim2 positions can be paired)
+  const uint32_t cap2 = S.max_moves > n1 ? S.max_moves - n1 : 0;
+  const uint32_t nd2 = min(nd + n1, cap2);
+  for (uint32_t i = threadIdx.x; i < nd; i += blockDim.x) {
+    const uint64_t x = dck[i];
+    uint32_t lo = 0, hi = n1;  // promoted (descending = P[n1-1..0]) greater than x
+    while (lo < hi) {
+      const uint32_t mid = (lo + hi) >> 1;
+      if (pck[n1 - 1 - mid] > x) lo = mid + 1; else hi = mid;
+    }
+    if (i + lo < nd2) {
+      dck2[i + lo] = x;
+      dsz2[i + lo] = dsz[i];
+    }
+  }
+  for (uint32_t q = threadIdx.x; q < n1; q += blockDim.x) {
+    const uint64_t x = pck[n1 - 1 - q];
+    uint32_t lo = 0, hi = nd;  // D entries greater than x
+    while (lo < hi) {
+      const uint32_t mid = (lo + hi) >> 1;
+      if (dck[mid] > x) lo = mid + 1; else hi = mid;
+    }
+    if (q + lo < nd2) {
+      dck2[q + lo] = x;
+      dsz2[q + lo] = psz[n1 - 1 - q];
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    uint64_t rem = rem_s, fs = fs_s, fh = fh_s;
+    uint32_t pairs = 0;
+    const uint32_t lim = min(np - min(np, n1), nd2);
+    bool stop = (S.thr[kLists + 2] == 0) || (S.thr[kLists + 1] == 0);
+    while (!stop && pairs < lim) {
+      const uint32_t j = pairs + lane;
+      bool order_ok = false;
+      uint64_t sp = 0, sd = 0;
+      if (j < lim) {
+        sp = psz[n1 + j];
+        sd = dsz2[j];
+        order_ok = dck2[j] > pck[n1 + j];
+      }
+      uint64_t by = (sp + sd) * kvb;
+      long long ds = (long long)sp - (long long)sd;  // fast tier gains sp, loses sd
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint64_t yb = __shfl_up_sync(kFull, by, o);
+        const long long yd = __shfl_up_sync(kFull, ds, o);
+        if (lane >= o) {
+          by += yb;
+          ds += yd;
+        }
+      }
+      const bool ok = j < lim && order_ok && by <= rem && (ds <= 0 || (uint64_t)ds <= fs) &&
+                      (ds >= 0 || (uint64_t)(-ds) <= fh);
+      const uint32_t okm = __ballot_sync(kFull, ok);
+      const uint32_t tk = okm == kFull ? 32u : (uint32_t)(__ffs(~okm) - 1);
+      if (tk > 0) {
+        const uint64_t tb = __shfl_sync(kFull, by, tk - 1);
+        const long long td = __shfl_sync(kFull, ds, tk - 1);
+        rem -= tb;
+        if (td >= 0) {
+          fs -= (uint64_t)td;
+          fh += (uint64_t)td;
+        } else {
+          fs += (uint64_t)(-td);
+          fh -= (uint64_t)(-td);
+        }
+      }
+      pairs += tk;
+      if (tk < 32) stop = true;
+    }
+    if (lane == 0) {
+      npairs = pairs;
+      rem_s = rem;
+    }
+  }
+  __syncthreads();
+  const uint32_t pairs = npairs;
+  for (uint32_t i = threadIdx.x; i < n1 + pairs; i += blockDim.x) S.promote[i] = (~(uint32_t)pck[i]) & kIdMask;
+  for (uint32_t i = threadIdx.x; i < pairs; i += blockDim.x) S.demote[i] = (~(uint32_t)dck2[i]) & kIdMask;
+  if (threadIdx.x == 0) {
+    S.counts[0] = nv;
+    S.counts[1] = n1 + pairs;
+    S.counts[2] = pairs;
+    S.counts[3] = S.work->status ? S.work->status : (unsigned int)UNISON_OK;
+    S.moved[0] = S.budget - rem_s;
+  }
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+}  // namespace
+
+extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_params *params,
+                                 const unison_rank_out *outs, int n_sets, void *cuda_stream) {
+  if (n_sets < 0 || (n_sets > 0 && (!sets || !params || !outs))) return UNISON_ERR_ARG;
+  if (n_sets == 0) return UNISON_OK;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  std::vector<RankSet> hs(n_sets);
+  uint32_t tiles = 0;
+  for (int i = 0; i < n_sets; i++) {
+    const unison_records &r = sets[i];
+    const unison_rank_params &p = params[i];
+    const unison_rank_out &o = outs[i];
+    if (r.n == 0 || r.n > (1ull << 24)) return UNISON_ERR_RANGE;
+    if (!r.gap_q || !r.turn || !r.kv_tok || !r.tier || !r.flags) return UNISON_ERR_ARG;
+    if (!aligned(r.gap_q, 16) || !aligned(r.turn, 16) || !aligned(r.tier, 16) || !aligned(r.flags, 16))
+      return UNISON_ERR_ARG;
+    if (p.k > kMaxSel || p.max_moves > kMaxSel) return UNISON_ERR_RANGE;
+    if (p.penalty_q >= (1ull << 32) || p.kv_bytes_per_token == 0 || p.kv_bytes_per_token > (1u << 24))
+      return UNISON_ERR_RANGE;
+    if (!o.counts || !o.moved_bytes || (p.k && !o.victims) || (p.max_moves && (!o.promote || !o.demote)))
+      return UNISON_ERR_ARG;
+    for (int t = 0; t < (int)kLutN; t++)
+      if (p.sigma_q[t] < kEpsQ || p.sigma_q[t] > kLambda) return UNISON_ERR_RANGE;
+    RankSet &s = hs[i];
+    s.gap = r.gap_q;
+    s.turn = r.turn;
+    s.kv = r.kv_tok;
+    s.tier = r.tier;
+    s.flags = r.flags;
+    s.n = (uint32_t)r.n;
+    s.k = p.k;
+    s.max_moves = p.max_moves;
+    s.kvb = p.kv_bytes_per_token;
+    s.penalty = p.penalty_q;
+    s.budget = p.budget_bytes;
+    s.free_s = p.free_fast_tok;
+    s.free_h = p.free_hbm_tok;
+    s.victims = o.victims;
+    s.promote = o.promote;
+    s.demote = o.demote;
+    s.counts = o.counts;
+    s.moved = o.moved_bytes;
+    s.keys = o.keys;
+    s.tile0 = tiles;
+    s.ntiles = (uint32_t)((r.n + kBigTile - 1) / kBigTile);
+    tiles += s.ntiles;
+    for (int t = 0; t < (int)kLutN; t++) s.sigma[t] = p.sigma_q[t];
+    s.pad = 0;
+  }
+  // scratch: descriptors, then per set: work, thresholds, tables, sorted lists, candidates
+  const size_t per_set = align_up(sizeof(RankWork), 256) + align_up(sizeof(uint64_t) * 2 * kLists, 256) +
+                         align_up(sizeof(uint2) * kLists * kLutN, 256) + 2 * align_up(sizeof(uint64_t) * kLutN, 256) +
+                         align_up(sizeof(uint64_t) * kLists * kMaxSel, 256) +
+                         align_up(sizeof(uint64_t) * kLists * kCandCap, 256) +
+                         align_up(sizeof(uint64_t) * kLists * kSampleCtas * kMaxR, 256);
+  const size_t desc_b = align_up(sizeof(RankSet) * n_sets, 256);
+  char *scratch = nullptr;
+  if (cudaMallocAsync(reinterpret_cast<void **>(&scratch), desc_b + per_set * n_sets, stream) != cudaSuccess) {
+    cudaGetLastError();
+    return UNISON_ERR_OOM;
+  }
+  for (int i = 0; i < n_sets; i++) {
+    char *p = scratch + desc_b + per_set * i;
+    RankSet &s = hs[i];
+    s.work = reinterpret_cast<RankWork *>(p);
+    p += align_up(sizeof(RankWork), 256);
+    s.thr = reinterpret_cast<uint64_t *>(p);
+    p += align_up(sizeof(uint64_t) * 2 * kLists, 256);
+    s.gthr = reinterpret_cast<uint2 *>(p);
+    p += align_up(sizeof(uint2) * kLists * kLutN, 256);
+    s.t2 = reinterpret_cast<uint64_t *>(p);
+    p += align_up(sizeof(uint64_t) * kLutN, 256);
+    s.magic = reinterpret_cast<uint64_t *>(p);
+    p += align_up(sizeof(uint64_t) * kLutN, 256);
+    s.sorted = reinterpret_cast<uint64_t *>(p);
+    p += align_up(sizeof(uint64_t) * kLists * kMaxSel, 256);
+    s.cand = reinterpret_cast<uint64_t *>(p);
+    p += align_up(sizeof(uint64_t) * kLists * kCandCap, 256);
+    s.part = reinterpret_cast<uint64_t *>(p);
+  }
+  int rc = UNISON_OK;
+  auto ck = [&](cudaError_t e) {
+    if (e != cudaSuccess && rc == UNISON_OK) rc = UNISON_ERR_CUDA;
+  };
+  RankSet *d_sets = reinterpret_cast<RankSet *>(scratch);
+  ck(cudaMemcpyAsync(d_sets, hs.data(), sizeof(RankSet) * n_sets, cudaMemcpyHostToDevice, stream));
+  for (int i = 0; i < n_sets; i++) ck(cudaMemsetAsync(hs[i].work, 0, sizeof(RankWork), stream));
+  const size_t smem_finish = sizeof(uint64_t) * (kSmemCand + kMaxSel);
+  // persistent filter: as many CTAs as fit at once, each over a contiguous tile range
+  int dev = 0, n_sm = 0, per_sm = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+  ck(cudaFuncSetAttribute(rank_filter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFilterSmem));
+  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rank_filter_kernel, kFilterCtaThreads, kFilterSmem);
+  const uint32_t grid_filter = std::max(1u, std::min<uint32_t>(tiles, (uint32_t)std::max(1, n_sm * per_sm)));
+  ck(cudaFuncSetAttribute(rank_finish_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_finish));
+  {
+    ProfSpan span("rank_sample", stream);
+    rank_sample_kernel<<<dim3(kSampleCtas, n_sets), kSampleThreads, 0, stream>>>(d_sets);
+  }
+  {
+    ProfSpan span("rank_filter", stream);
+    rank_filter_kernel<<<grid_filter, kFilterCtaThreads, kFilterSmem, stream>>>(d_sets, n_sets, tiles);
+  }
+  {
+    ProfSpan span("rank_finish", stream);
+    rank_finish_kernel<<<n_sets, kFinishThreads, smem_finish, stream>>>(d_sets);
+  }
+  count_launches(3);
+  ck(cudaGetLastError());
+  ck(cudaFreeAsync(scratch, stream));
+  return rc;
 }

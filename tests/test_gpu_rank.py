@@ -1,0 +1,193 @@
+"""GPU parity of the standalone ranking (victims, TIDE fill, keys) against the
+CPU oracle: bit-exact on every output index and key."""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+P_Z = 500_000_000
+KVB = 131072
+GIB = 1 << 30
+
+
+@pytest.fixture(scope="module")
+def B():
+    from paper_2609_09643_gb300 import native
+    native.build()
+    from paper_2609_09643_gb300 import binding
+    return binding
+
+
+@pytest.fixture(scope="module")
+def sigma():
+    _, s = oracle.hazard_lut(synth.geometric_turns(1, 1415, 23.7, 2, 200))
+    return s
+
+
+def run(B, recs, params, keys=False):
+    import torch
+    devs = [B.records_to_device(r) for r in recs]
+    outs = [B.rank_outputs(r.n, p["k"], p["max_moves"], keys) for r, p in zip(recs, params)]
+    B.rank_batch(devs, params, outs)
+    torch.cuda.synchronize()
+    return [B.rank_result(o) for o in outs]
+
+
+def check(r, rec, p, keys=False):
+    o = oracle.rank(rec, p["sigma_q"], p["penalty_q"], p["k"], p["budget_bytes"], p["kv_bytes_per_token"],
+                    p["free_fast_tok"], p["free_hbm_tok"], keys=keys, max_moves=max(p["max_moves"], 1))
+    if p["max_moves"] == 0:
+        o["promote"] = o["promote"][:0]
+        o["demote"] = o["demote"][:0]
+        o["moved_bytes"] = 0
+    assert r["status"] == 0
+    assert np.array_equal(r["victims"], o["victims"]), "victims"
+    assert np.array_equal(r["promote"], o["promote"]), ("promote", r["promote"][:8], o["promote"][:8])
+    assert np.array_equal(r["demote"], o["demote"]), ("demote", r["demote"][:8], o["demote"][:8])
+    assert r["moved_bytes"] == o["moved_bytes"], "moved"
+    if keys:
+        assert np.array_equal(r["keys"], o["keys"]), "keys"
+
+
+def prm(sig, k=1024, budget=16 * GIB, max_moves=1024, free_s=0, free_h=1 << 40):
+    return dict(sigma_q=sig, k=k, penalty_q=P_Z, budget_bytes=budget, kv_bytes_per_token=KVB, max_moves=max_moves,
+                free_fast_tok=free_s, free_hbm_tok=free_h)
+
+
+@pytest.mark.parametrize("n", [1, 7, 1000, 2047, 2049, 4096, 16384])
+def test_small_sets_all_candidates(B, sigma, n):
+    rec = synth.make_records(n, n)
+    ps = [prm(sigma, k=k, budget=b, free_s=fs) for k, b, fs in
+          [(1, 1 * GIB, 0), (5, 64 * GIB, 0), (1024, 4 * GIB, 30000), (4096, 1 << 50, 10 ** 7)]]
+    res = run(B, [rec] * len(ps), ps, keys=True)
+    for r, p in zip(res, ps):
+        check(r, rec, p, keys=True)
+
+
+@pytest.mark.parametrize("n", [16385, 1 << 17, 1 << 18, 1 << 20])
+def test_sampled_sizes(B, sigma, n):
+    rec = synth.make_records(11, n)
+    ps = [prm(sigma, k=k, budget=b) for k, b in [(1, 1 * GIB), (64, 8 * GIB), (1024, 64 * GIB)]]
+    res = run(B, [rec] * len(ps), ps, keys=(n <= (1 << 18)))
+    for r, p in zip(res, ps):
+        check(r, rec, p, keys=(n <= (1 << 18)))
+
+
+def test_full_size_2p24(B, sigma):
+    """The largest live set (2^24 records): victims, fill and every key."""
+    rec = synth.make_records(4, 1 << 24)
+    p = prm(sigma, k=1024, budget=64 * GIB)
+    r = run(B, [rec], [p], keys=True)[0]
+    check(r, rec, p, keys=True)
+
+
+def _sorted_records(n, ascending=True):
+    rec = synth.make_records(5, n)
+    order = np.argsort(rec.gap_q.astype(np.int64), kind="stable")
+    if not ascending:
+        order = order[::-1]
+    f = lambda a: np.ascontiguousarray(a[order])
+    rec2 = synth.Records(f(rec.gap_q), f(rec.last_ret), np.zeros(n, np.uint16), f(rec.kv_tok), f(rec.tier),
+                         (f(rec.flags) & 1).astype(np.uint8))
+    return rec2
+
+
+@pytest.mark.parametrize("asc", [True, False])
+def test_adversarial_order(B, sigma, asc):
+    """Records sorted by key put every top record in one region: the sampled
+    thresholds miss and the exact re-selection must still give the answer."""
+    rec = _sorted_records(1 << 20, asc)
+    ps = [prm(sigma, k=1024, budget=64 * GIB), prm(sigma, k=3000, budget=1 << 50, max_moves=4096)]
+    for r, p in zip(run(B, [rec] * 2, ps), ps):
+        check(r, rec, p)
+
+
+def test_massive_ties(B, sigma):
+    n = 300000
+    rec = synth.make_records(6, n)
+    rec = synth.Records(np.zeros(n, np.uint32), rec.last_ret, np.zeros(n, np.uint16), rec.kv_tok, rec.tier,
+                        np.zeros(n, np.uint8))
+    ps = [prm(sigma, k=777, budget=64 * GIB), prm(sigma, k=4096, budget=1 << 45, free_s=50000, max_moves=4096)]
+    for r, p in zip(run(B, [rec] * 2, ps, keys=True), ps):
+        check(r, rec, p, keys=True)
+
+
+def test_degenerate_sets(B, sigma):
+    n = 50000
+    base = synth.make_records(8, n)
+    all_pinned = synth.Records(base.gap_q, base.last_ret, base.turn, base.kv_tok, base.tier,
+                               np.ones(n, np.uint8))
+    all_fast = synth.Records(base.gap_q, base.last_ret, base.turn, base.kv_tok, np.ones(n, np.uint8), base.flags)
+    none_res = synth.Records(base.gap_q, base.last_ret, base.turn, base.kv_tok, np.zeros(n, np.uint8), base.flags)
+    cases = [(all_pinned, prm(sigma)), (all_fast, prm(sigma)), (none_res, prm(sigma)),
+             (base, prm(sigma, k=0, budget=0, max_moves=0)), (base, prm(sigma, budget=0)),
+             (base, prm(sigma, max_moves=3)), (base, prm(sigma, free_h=0)), (base, prm(sigma, budget=1))]
+    res = run(B, [c[0] for c in cases], [c[1] for c in cases])
+    for r, (rec, p) in zip(res, cases):
+        check(r, rec, p)
+
+
+def test_phase1_promotions(B, sigma):
+    rec = synth.make_records(9, 200000)
+    ps = [prm(sigma, budget=b, free_s=fs, max_moves=mm) for b, fs, mm in
+          [(64 * GIB, 60000, 1024), (1 << 50, 10 ** 6, 4096), (1 << 50, 10 ** 9, 64), (2 * GIB, 10 ** 9, 4096)]]
+    for r, p in zip(run(B, [rec] * 4, ps), ps):
+        check(r, rec, p)
+
+
+def test_batch_of_mixed_sets(B, sigma):
+    recs = [synth.make_records(20 + i, n) for i, n in enumerate([100, 20000, 1 << 18, 3000, 1 << 19])]
+    ps = [prm(sigma, k=k, budget=(1 << i) * GIB) for i, k in enumerate([3, 50, 1024, 4096, 700])]
+    for r, rec, p in zip(run(B, recs, ps, keys=True), recs, ps):
+        check(r, rec, p, keys=True)
+
+
+def test_keys_exact_at_division_boundaries(B):
+    """Every sigma in [41, 4095] (through a table of 51 distinct values per
+    run), gaps at multiples of sigma and just below, and the largest gap."""
+    import torch
+    rs = np.random.default_rng(3)
+    for run_i in range(4):
+        sig = np.sort(rs.choice(np.arange(41, 4096), size=51, replace=False))[::-1].astype(np.uint16)
+        if run_i == 0:
+            sig[0], sig[1] = 4095, 41
+        gs, ts = [], []
+        for t in range(51):
+            s = int(sig[t])
+            q = rs.integers(0, (2 ** 31 - 1) * 4095 // s, 200)
+            for x in np.concatenate([q * s, q * s + s - 1]):
+                g = int(x) // 4095
+                for dg in (-1, 0, 1):
+                    if 0 <= g + dg < 2 ** 31:
+                        gs.append(g + dg)
+                        ts.append(t)
+            gs += [0, 1, 2 ** 31 - 1]
+            ts += [t, t, t]
+        n = len(gs)
+        rec = synth.Records(np.array(gs, np.uint32), np.zeros(n, np.uint32), np.array(ts, np.uint16),
+                            np.full(n, 100, np.uint32), np.full(n, 2, np.uint8), np.zeros(n, np.uint8))
+        p = dict(sigma_q=sig, k=10, penalty_q=(1 << 32) - 1, budget_bytes=0, kv_bytes_per_token=1, max_moves=0,
+                 free_fast_tok=0, free_hbm_tok=0)
+        r = run(B, [rec], [p], keys=True)[0]
+        o = oracle.rank(rec, sig, p["penalty_q"], 10, 0, 1, 0, 0, keys=True)
+        assert np.array_equal(r["keys"], o["keys"])
+
+
+def test_rank_rejects_bad_args(B, sigma):
+    import torch
+    rec = synth.make_records(1, 100)
+    d = B.records_to_device(rec)
+    for bad in (dict(k=5000), dict(max_moves=5000), dict(penalty_q=1 << 32), dict(kv_bytes_per_token=0)):
+        p = prm(sigma)
+        p.update(bad)
+        with pytest.raises(B.UnisonError):
+            B.rank_batch([d], [p], [B.rank_outputs(100, 5000, 5000)])
+    bad_sig = prm(np.full(51, 40, np.uint16))
+    with pytest.raises(B.UnisonError):
+        B.rank_batch([d], [bad_sig], [B.rank_outputs(100, 1024, 1024)])
+    off = dict(d, gap_q=d["gap_q"][1:])  # misaligned
+    with pytest.raises(B.UnisonError):
+        B.rank_batch([off], [prm(sigma)], [B.rank_outputs(99, 1024, 1024)])
