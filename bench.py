@@ -39,6 +39,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--rank-only", action="store_true", help="time only the ranking leg (profiling)")
+    ap.add_argument("--replay-only", action="store_true", help="time only the replay leg (profiling)")
+    ap.add_argument("--replays", type=int, default=1024, help="first N replays of the sweep (profiling)")
     ap.add_argument("--rank-n", type=int, default=1 << 24, help="records per live set")
     ap.add_argument("--rank-sets", type=int, default=7, help="live sets per call (<= 7)")
     return ap.parse_args()
@@ -217,6 +219,10 @@ def main():
     from paper_2609_09643_gb300 import binding as B
 
     trs, reps, lib_params = sweep_workload(rank)
+    if args.replays < len(reps):  # evenly spread subset, for profiling runs
+        pick = [int(i * len(reps) / args.replays) for i in range(args.replays)]
+        reps = [reps[i] for i in pick]
+        lib_params = [lib_params[i] for i in pick]
     stream = torch.cuda.current_stream()
     handles = [B.Trace(t).upload(stream) for t in trs]
     n_rep = len(lib_params)
@@ -240,7 +246,8 @@ def main():
         flush.zero_()
         if not args.rank_only:
             B.replay_batch_async(handles, lib_params, res_dev, stream=stream)
-        B.rank_batch(rank_sets, r_params, rank_outs, stream=stream)
+        if not args.replay_only:
+            B.rank_batch(rank_sets, r_params, rank_outs, stream=stream)
 
     for _ in range(args.warmup):
         step()
@@ -248,7 +255,8 @@ def main():
     if not args.rank_only:
         res = B.results_from_tensor(res_dev)
         assert all(r["status"] == 0 for r in res), "replay status"
-    assert all(B.rank_result(o)["status"] == 0 for o in rank_outs), "rank status"
+    if not args.replay_only:
+        assert all(B.rank_result(o)["status"] == 0 for o in rank_outs), "rank status"
 
     def barrier():
         if world > 1:
@@ -321,15 +329,15 @@ def main():
     except Exception:
         pass
     hbm_peak = peaks.get("hbm_gbs") or 6800.0
-    avg_rf = rf_ms / max(rf_n, 1)
-    achieved = rank_bytes / (avg_rf / 1e3) / 1e9
+    avg_rf = rf_ms / max(rf_n, 1) if rf_n else float("nan")
+    achieved = rank_bytes / (avg_rf / 1e3) / 1e9 if rf_n else float("nan")
     roofline = {"bound": "hbm", "kernel": "rank_filter_kernel", "achieved": achieved, "peak": hbm_peak,
                 "unit": "GB/s", "frac": achieved / hbm_peak,
                 "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs, burst copy)" if peaks.get("hbm_gbs")
                 else "fallback 6.8 TB/s", "traffic": None, "avg_ms": avg_rf, "launches_timed": rf_n,
                 "algorithmic_bytes_per_launch": rank_bytes,
                 "bytes_per_record": RANK_BYTES_PER_RECORD, "records_per_launch": len(r_params) * RANK_N}
-    call_ms = (rs_ms + rf_ms + rn_ms) / max(rf_n, 1)
+    call_ms = (rs_ms + rf_ms + rn_ms) / max(rf_n, 1) if rf_n else float("nan")
     rank_leg = {"metric": "rank-kernel HBM GB/s", "sets_per_call": len(r_params), "records_per_set": RANK_N,
                 "k": 1024, "budgets_gib": list(RANK_BUDGETS_GIB),
                 "call_ms": call_ms, "call_gbs": rank_bytes / (call_ms / 1e3) / 1e9,

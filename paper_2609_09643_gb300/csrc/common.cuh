@@ -63,6 +63,7 @@ struct unison_trace {
   size_t off_ev = 0;        // uint4[E]: time32, session|flags, in_tok, out_tok
   size_t off_prev_out = 0;  // u32[E]: l^out of the previous turn (arrivals)
   size_t off_nref = 0;      // u32[E]: event index of the next arrival (arrivals)
+  size_t off_prev_ev = 0;   // u32[E]: event index of the previous completion (arrivals of turn >= 1)
   size_t off_turn_ev = 0;   // u32[2T]: arrival and completion event of each turn
   size_t off_turn_t = 0;    // u32[2T]: arrival and completion time32 of each turn
   size_t off_turn_off = 0;  // u32[S+1]: session turn offsets

@@ -26,7 +26,7 @@ void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_rela
 
 ProfSpan::ProfSpan(const char *name, cudaStream_t s) : stream_(s) {
   std::lock_guard<std::mutex> lk(g_mu);
-  if (!g_on) return;
+  if (!g_on || !name || !*name) return;
   if (cudaEventCreate(&a_) != cudaSuccess || cudaEventCreate(&b_) != cudaSuccess) {
     cudaGetLastError();
     return;

@@ -33,9 +33,6 @@ namespace {
 
 constexpr uint32_t kFull = 0xFFFFFFFFu;
 constexpr uint32_t kTierNone = 0, kTierS = 1, kTierH = 2;
-constexpr uint32_t kAuxPinned = 1u, kAuxPromoted = 2u;
-constexpr uint16_t kMapNone = 0xFFFFu;
-constexpr uint32_t kEntryBytes = 20;  // hi, lo, size, aux, ret (u32 each)
 
 struct ComboDesc {
   const uint32_t *turn_ev;   // [2T]
@@ -47,15 +44,18 @@ struct ComboDesc {
   uint64_t penalty_q;
   uint16_t *sigma;  // [51]
   uint64_t *t2;     // [51]
-  uint64_t *pkey;   // [E]
-  uint32_t *gq;     // [E]
+  uint64_t *pkey;   // [E] key after the event
+  uint32_t *gq;     // [E] gap average after the event
+  uint64_t *pkb;    // [E] key before the event (arrivals of turn >= 1)
 };
 
 struct ReplayDesc {
   const uint4 *ev;
   const uint32_t *prev_out;
   const uint32_t *nref;
+  const uint32_t *prev_ev;  // previous completion event of each arrival's session
   const uint64_t *pkey;  // key stream (SPEAR policies) or null
+  const uint64_t *pkb;   // key before each arrival (SPEAR policies) or null
   const uint32_t *gq;    // gap-average stream (TIDE policies) or null
   uint64_t *ttft;        // [n_turns]
   uint32_t *glist;       // resident lists in global memory, or null (shared)
@@ -67,7 +67,7 @@ struct ReplayDesc {
   uint64_t prefill_ns;    // ns per prefill token
   uint32_t n_events, n_turns, n_sessions, policy;
   uint32_t max_sessions, kvb, ttl, load;
-  uint32_t rcap_s, rcap_h, use_map, pad;
+  uint32_t rcap_s, rcap_h;
 };
 
 // --------------------------------------------------------------------------
@@ -142,7 +142,7 @@ __global__ void key_stream_kernel(const ComboDesc *combos) {
   if (s >= c.n_sessions) return;
   const uint32_t b = c.turn_off[s], ts = c.tps[s];
   const uint64_t a_num = c.ema_num, a_rest = c.ema_den - c.ema_num, a_den = c.ema_den;
-  uint64_t g = 0;
+  uint64_t g = 0, prev_pk = 0;
   uint32_t prev_c = 0;
   for (uint32_t k = 0; k < ts; k++) {
     const uint32_t ti = b + k;
@@ -158,387 +158,386 @@ __global__ void key_stream_kernel(const ComboDesc *combos) {
     const uint32_t ea = c.turn_ev[2 * ti], ec = c.turn_ev[2 * ti + 1];
     c.pkey[ea] = pk;
     c.gq[ea] = (uint32_t)g;
-    c.pkey[ec] = (k + 1 == ts) ? pack_key(kKeyMax40, s) : pk;
+    c.pkb[ea] = prev_pk;  // the key the session carried into this arrival
+    prev_pk = (k + 1 == ts) ? pack_key(kKeyMax40, s) : pk;
+    c.pkey[ec] = prev_pk;
     c.gq[ec] = (uint32_t)g;
   }
 }
 
 // --------------------------------------------------------------------------
-// Resident lists: one per tier, structure of arrays, unordered (removal
-// swaps in the last entry).  All list state is warp-uniform; lane 0 writes.
+// Resident sessions.  The unpinned residents of each tier sit in an array
+// sorted by packed key, ascending: the most evictable is the last entry and
+// the least evictable the first, so every argmax / argmin of Algorithm 1 and
+// of TIDE is an array end.  Pinned (mid-turn) residents, which no decision
+// may touch, sit in a small unordered list.  Keys change only at a session's
+// own events, so an arriving session is found by binary search on the key it
+// was given at its previous event.  Entries (16 B):
+//   sorted: {key lo, key hi, size | promoted << 31, last return time}
+//   pinned: {key lo, key hi, size, session | tier << 30}
+// All list state is warp-uniform; lane 0 writes single entries, all lanes
+// move blocks (warp-parallel shifts, top or bottom chunk first).
 // --------------------------------------------------------------------------
-struct TierList {
-  uint32_t *hi, *lo, *size, *aux, *ret;
+constexpr uint32_t kPromotedBit = 0x80000000u;
+constexpr uint32_t kSizeMask = 0x7FFFFFFFu;
+
+struct Sorted {
+  uint4 *e;
   uint32_t n, cap;
-  uint64_t used, pinned;  // tokens resident / tokens of pinned residents
 };
 
-struct Pick {
-  int slot;
-  uint64_t pk;
-};
+__device__ __forceinline__ uint64_t ekey(uint4 v) { return ((uint64_t)v.y << 32) | v.x; }
 
-__device__ __forceinline__ uint64_t entry_key(const TierList &L, uint32_t i) {
-  return ((uint64_t)L.hi[i] << 32) | L.lo[i];
+// Number of entries with key < k (warp-uniform result).
+__device__ __forceinline__ uint32_t lower_bound(const Sorted &T, uint64_t k, int lane) {
+  uint32_t lo = 0, hi = T.n;  // the answer lies in [lo, hi]
+  while (hi - lo > 32) {
+    const uint32_t step = (hi - lo + 31) / 32;
+    const uint32_t i = lo + lane * step;
+    const bool less = i < hi && ekey(T.e[i]) < k;
+    const uint32_t cnt = __popc(__ballot_sync(kFull, less));  // 'less' holds for a prefix of lanes
+    const uint32_t nlo = cnt ? lo + (cnt - 1) * step + 1 : lo;
+    const uint32_t nhi = min(hi, lo + cnt * step);
+    lo = nlo;
+    hi = nhi;
+  }
+  const uint32_t i = lo + lane;
+  return lo + __popc(__ballot_sync(kFull, i < hi && ekey(T.e[i]) < k));
 }
 
-// Most evictable unpinned entry (largest packed key); slot -1 if none.
-__device__ __forceinline__ Pick argmax_unpinned(const TierList &L, int lane) {
-  uint64_t best = 0;
-  int bi = -1;
-  for (uint32_t i = lane; i < L.n; i += 32) {
-    const uint32_t a = L.aux[i];
-    const uint64_t k = entry_key(L, i);
-    if (!(a & kAuxPinned) && k > best) {
-      best = k;
-      bi = (int)i;
+// Move e[lo, hi) by delta places (delta > 0 toward the end), warp-parallel.
+__device__ __forceinline__ void shift_block(uint4 *e, uint32_t lo, uint32_t hi, int32_t delta, int lane) {
+  if (lo >= hi || delta == 0) return;
+  if (delta > 0) {  // top chunk first
+    uint32_t top = hi;
+    while (top > lo) {
+      const uint32_t bot = top - lo > 128 ? top - 128 : lo;
+      uint4 v[4];
+#pragma unroll
+      for (int j = 0; j < 4; j++) {
+        const uint32_t i = bot + lane + 32 * j;
+        if (i < top) v[j] = e[i];
+      }
+      __syncwarp();
+#pragma unroll
+      for (int j = 0; j < 4; j++) {
+        const uint32_t i = bot + lane + 32 * j;
+        if (i < top) e[i + delta] = v[j];
+      }
+      __syncwarp();
+      top = bot;
+    }
+  } else {  // bottom chunk first
+    uint32_t bot = lo;
+    while (bot < hi) {
+      const uint32_t top = hi - bot > 128 ? bot + 128 : hi;
+      uint4 v[4];
+#pragma unroll
+      for (int j = 0; j < 4; j++) {
+        const uint32_t i = bot + lane + 32 * j;
+        if (i < top) v[j] = e[i];
+      }
+      __syncwarp();
+#pragma unroll
+      for (int j = 0; j < 4; j++) {
+        const uint32_t i = bot + lane + 32 * j;
+        if (i < top) e[(int32_t)i + delta] = v[j];
+      }
+      __syncwarp();
+      bot = top;
     }
   }
-  const uint32_t h = (uint32_t)(best >> 32);
-  const uint32_t mh = __reduce_max_sync(kFull, h);
-  const uint32_t l = (h == mh) ? (uint32_t)best : 0u;
-  const uint32_t ml = __reduce_max_sync(kFull, l);
-  const uint64_t m = ((uint64_t)mh << 32) | ml;
-  Pick p{-1, 0};
-  if (m == 0) return p;  // valid packed keys are never 0 (inverted id >= 1)
-  const uint32_t who = __ballot_sync(kFull, bi >= 0 && best == m);
-  p.slot = __shfl_sync(kFull, bi, __ffs(who) - 1);
-  p.pk = m;
-  return p;
-}
-
-// Least evictable unpinned entry (smallest packed key); slot -1 if none.
-__device__ __forceinline__ Pick argmin_unpinned(const TierList &L, int lane) {
-  uint64_t best = ~0ull;
-  int bi = -1;
-  for (uint32_t i = lane; i < L.n; i += 32) {
-    const uint32_t a = L.aux[i];
-    const uint64_t k = entry_key(L, i);
-    if (!(a & kAuxPinned) && (bi < 0 || k < best)) {
-      best = k;
-      bi = (int)i;
-    }
-  }
-  Pick p{-1, 0};
-  const uint32_t any = __ballot_sync(kFull, bi >= 0);
-  if (!any) return p;
-  const uint32_t h = bi >= 0 ? (uint32_t)(best >> 32) : kFull;
-  const uint32_t mh = __reduce_min_sync(kFull, h);
-  const uint32_t l = (bi >= 0 && h == mh) ? (uint32_t)best : kFull;
-  const uint32_t ml = __reduce_min_sync(kFull, l);
-  const uint64_t m = ((uint64_t)mh << 32) | ml;
-  const uint32_t who = __ballot_sync(kFull, bi >= 0 && best == m);
-  p.slot = __shfl_sync(kFull, bi, __ffs(who) - 1);
-  p.pk = m;
-  return p;
 }
 
 struct ReplayState {
-  TierList S, H;
-  uint16_t *map;  // session -> (tier bit 15 | slot), or null
+  Sorted S, H;      // unpinned residents per tier
+  uint4 *pin;       // pinned residents
+  uint32_t npin, pin_cap;
+  uint4 *tmp;       // TIDE staging: [0, cap_s) promoted, [cap_s, 2 cap_s) demoted
+  uint64_t used_s, used_h, pinned_s, pinned_h;  // tokens
   unison_decision *log;
   uint64_t log_cap;
   uint32_t e;  // current event index
   int status;
-  uint32_t pinned_cnt;
-  // counters
-  unison_replay_result c;
+  uint64_t hash, log_len;  // decision stream state
+  // counters (warp-uniform registers: every lane keeps the same copy)
+  uint32_t n_warm, n_cold, n_hit_s, n_hit_h, n_miss, n_bypass, n_place_s, n_place_h;
+  uint32_t n_evict, n_demote, n_promote, n_tide_demote, n_expire, n_tide_calls, n_pth;
+  uint64_t tok_hit_s, tok_hit_h, tok_miss, tok_computed, tok_needed, dma_bytes;
 };
+
+#define CNT(st, field, v) ((st).field += (v))
 
 __device__ __forceinline__ void log_dec(ReplayState &st, uint32_t kind, uint32_t s, int lane) {
   const uint64_t w = ((uint64_t)st.e << 32) | ((uint64_t)kind << 24) | s;
-  st.c.decision_hash = (st.c.decision_hash ^ w) * kFnvPrime;
+  st.hash = (st.hash ^ w) * kFnvPrime;
   if (st.log) {
-    if (st.c.log_len < st.log_cap) {
+    if (st.log_len < st.log_cap) {
       if (lane == 0) {
         unison_decision d;
         d.event = st.e;
         d.kind_session = (kind << 24) | s;
-        st.log[st.c.log_len] = d;
+        st.log[st.log_len] = d;
       }
     } else if (st.status == UNISON_OK) {
       st.status = UNISON_ERR_LOG_FULL;
     }
   }
-  st.c.log_len++;
+  st.log_len++;
 }
 
-__device__ __forceinline__ bool tl_append(ReplayState &st, TierList &L, uint32_t tier, uint64_t pk, uint32_t size,
-                                          uint32_t aux, uint32_t ret, int lane) {
-  if (L.n >= L.cap) {
+__device__ __forceinline__ bool sorted_insert(ReplayState &st, Sorted &T, uint4 v, int lane) {
+  if (T.n >= T.cap) {
     st.status = UNISON_ERR_CAPACITY;
     return false;
   }
-  const uint32_t i = L.n;
-  if (lane == 0) {
-    L.hi[i] = (uint32_t)(pk >> 32);
-    L.lo[i] = (uint32_t)pk;
-    L.size[i] = size;
-    L.aux[i] = aux;
-    L.ret[i] = ret;
-    if (st.map) st.map[packed_id(pk)] = (uint16_t)((tier == kTierH ? 0x8000u : 0u) | i);
-  }
-  L.n++;
-  L.used += size;
-  if (aux & kAuxPinned) L.pinned += size;
+  const uint32_t p = lower_bound(T, ekey(v), lane);
+  shift_block(T.e, p, T.n, 1, lane);
+  if (lane == 0) T.e[p] = v;
   __syncwarp();
+  T.n++;
   return true;
 }
 
-__device__ __forceinline__ void tl_remove(ReplayState &st, TierList &L, uint32_t tier, uint32_t i, int lane) {
-  const uint32_t last = L.n - 1;
-  const uint32_t sz = L.size[i], ax = L.aux[i], lo = L.lo[i];
-  const uint32_t lhi = L.hi[last], llo = L.lo[last], lsz = L.size[last], lax = L.aux[last], lret = L.ret[last];
-  __syncwarp();
-  if (lane == 0) {
-    if (i != last) {
-      L.hi[i] = lhi;
-      L.lo[i] = llo;
-      L.size[i] = lsz;
-      L.aux[i] = lax;
-      L.ret[i] = lret;
-      if (st.map) st.map[(~llo) & kIdMask] = (uint16_t)((tier == kTierH ? 0x8000u : 0u) | i);
-    }
-    if (st.map) st.map[(~lo) & kIdMask] = kMapNone;
-  }
-  L.n = last;
-  L.used -= sz;
-  if (ax & kAuxPinned) L.pinned -= sz;
-  __syncwarp();
+__device__ __forceinline__ void sorted_erase(Sorted &T, uint32_t p, int lane) {
+  shift_block(T.e, p + 1, T.n, -1, lane);
+  T.n--;
 }
 
-// Where session s is resident: tier (0 none) and slot.
-__device__ __forceinline__ void locate(const ReplayState &st, uint32_t s, uint32_t &tier, uint32_t &slot, int lane) {
-  if (st.map) {
-    const uint16_t v = st.map[s];
-    if (v == kMapNone) {
-      tier = kTierNone;
-      slot = 0;
-    } else {
-      tier = (v & 0x8000u) ? kTierH : kTierS;
-      slot = v & 0x7FFFu;
-    }
-    return;
-  }
-  const uint32_t want = (~s) & kIdMask;
-  int mine = -1;
-  for (uint32_t i = lane; i < st.S.n; i += 32)
-    if ((st.S.lo[i] & kIdMask) == want) mine = (int)i;
-  uint32_t b = __ballot_sync(kFull, mine >= 0);
-  if (b) {
-    tier = kTierS;
-    slot = (uint32_t)__shfl_sync(kFull, mine, __ffs(b) - 1);
-    return;
-  }
-  for (uint32_t i = lane; i < st.H.n; i += 32)
-    if ((st.H.lo[i] & kIdMask) == want) mine = (int)i;
-  b = __ballot_sync(kFull, mine >= 0);
-  if (b) {
-    tier = kTierH;
-    slot = (uint32_t)__shfl_sync(kFull, mine, __ffs(b) - 1);
-    return;
-  }
-  tier = kTierNone;
-  slot = 0;
+__device__ __forceinline__ uint4 sorted_pop_back(Sorted &T) {
+  const uint4 v = T.e[T.n - 1];
+  __syncwarp();
+  T.n--;
+  return v;
 }
 
-// Evict entry `slot` of a tier (log EVICT / EXPIRE).
-__device__ __forceinline__ void evict_entry(ReplayState &st, TierList &L, uint32_t tier, uint32_t slot, uint32_t kind,
-                                            int lane) {
-  const uint32_t id = (~L.lo[slot]) & kIdMask;
-  tl_remove(st, L, tier, slot, lane);
-  log_dec(st, kind, id, lane);
-  if (kind == UNISON_KIND_EXPIRE)
-    st.c.expire++;
-  else
-    st.c.evict++;
-}
+__device__ __forceinline__ uint32_t esize(uint4 v) { return v.z & kSizeMask; }
 
 // A session demoted out of the fast tier enters HBM, displacing the most
 // evictable unpinned HBM sessions, or is dropped when it is itself the most
 // evictable of (unpinned HBM) + {itself}.
-__device__ __forceinline__ bool admit_demoted(ReplayState &st, const ReplayDesc &D, uint64_t pk, uint32_t size,
-                                              uint32_t aux, uint32_t ret, int lane) {
-  const uint32_t id = packed_id(pk);
-  if (st.H.pinned > D.cap_h || size > D.cap_h - st.H.pinned) {
+__device__ __forceinline__ bool admit_demoted(ReplayState &st, const ReplayDesc &D, uint4 d, int lane) {
+  const uint32_t id = packed_id(ekey(d));
+  const uint32_t size = esize(d);
+  if (st.pinned_h > D.cap_h || size > D.cap_h - st.pinned_h) {
     log_dec(st, UNISON_KIND_EVICT, id, lane);
-    st.c.evict++;
+    CNT(st, n_evict, 1);
     return true;
   }
-  while (st.H.used + size > D.cap_h) {
-    const Pick v = argmax_unpinned(st.H, lane);
-    if (v.slot < 0 || pk > v.pk) {
+  while (st.used_h + size > D.cap_h) {
+    if (st.H.n == 0 || ekey(d) > ekey(st.H.e[st.H.n - 1])) {
       log_dec(st, UNISON_KIND_EVICT, id, lane);
-      st.c.evict++;
+      CNT(st, n_evict, 1);
       return true;
     }
-    evict_entry(st, st.H, kTierH, (uint32_t)v.slot, UNISON_KIND_EVICT, lane);
+    const uint4 v = sorted_pop_back(st.H);
+    st.used_h -= esize(v);
+    log_dec(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
+    CNT(st, n_evict, 1);
   }
-  if (!tl_append(st, st.H, kTierH, pk, size, aux, ret, lane)) return false;
+  if (!sorted_insert(st, st.H, d, lane)) return false;
+  st.used_h += size;
   log_dec(st, UNISON_KIND_DEMOTE, id, lane);
-  st.c.demote++;
+  CNT(st, n_demote, 1);
+  return true;
+}
+
+__device__ __forceinline__ bool pin_append(ReplayState &st, uint64_t pk, uint32_t size, uint32_t s, uint32_t tier,
+                                           int lane) {
+  if (st.npin >= st.pin_cap) {
+    st.status = UNISON_ERR_CAPACITY;
+    return false;
+  }
+  if (lane == 0) st.pin[st.npin] = make_uint4((uint32_t)pk, (uint32_t)(pk >> 32), size, s | (tier << 30));
+  __syncwarp();
+  st.npin++;
   return true;
 }
 
 // Placement of the arriving (pinned) session s with n tokens.
 __device__ __forceinline__ bool place(ReplayState &st, const ReplayDesc &D, uint32_t s, uint64_t pk, uint32_t n,
                                       int lane) {
-  if (D.max_sessions && st.pinned_cnt >= D.max_sessions) {
+  if (D.max_sessions && st.npin >= D.max_sessions) {
     log_dec(st, UNISON_KIND_BYPASS, s, lane);
-    st.c.bypass++;
+    CNT(st, n_bypass, 1);
     return true;
   }
-  if (st.S.pinned <= D.cap_s && n <= D.cap_s - st.S.pinned) {
-    while (st.S.used + n > D.cap_s) {
-      const Pick d = argmax_unpinned(st.S, lane);
-      if (d.slot < 0) {
+  if (st.pinned_s <= D.cap_s && n <= D.cap_s - st.pinned_s) {
+    while (st.used_s + n > D.cap_s) {
+      if (st.S.n == 0) {
         st.status = UNISON_ERR_CAPACITY;
         return false;
       }
-      const uint32_t sd = st.S.size[d.slot], ad = st.S.aux[d.slot], rd = st.S.ret[d.slot];
-      tl_remove(st, st.S, kTierS, (uint32_t)d.slot, lane);
-      if (!admit_demoted(st, D, d.pk, sd, ad, rd, lane)) return false;
+      const uint4 d = sorted_pop_back(st.S);  // most evictable unpinned fast-tier session
+      st.used_s -= esize(d);
+      if (!admit_demoted(st, D, d, lane)) return false;
     }
-    if (!tl_append(st, st.S, kTierS, pk, n, kAuxPinned, 0u, lane)) return false;
+    if (!pin_append(st, pk, n, s, kTierS, lane)) return false;
+    st.used_s += n;
+    st.pinned_s += n;
     log_dec(st, UNISON_KIND_PLACE_S, s, lane);
-    st.c.place_s++;
-  } else if (st.H.pinned <= D.cap_h && n <= D.cap_h - st.H.pinned) {
-    while (st.H.used + n > D.cap_h) {
-      const Pick v = argmax_unpinned(st.H, lane);
-      if (v.slot < 0) {
+    CNT(st, n_place_s, 1);
+  } else if (st.pinned_h <= D.cap_h && n <= D.cap_h - st.pinned_h) {
+    while (st.used_h + n > D.cap_h) {
+      if (st.H.n == 0) {
         st.status = UNISON_ERR_CAPACITY;
         return false;
       }
-      evict_entry(st, st.H, kTierH, (uint32_t)v.slot, UNISON_KIND_EVICT, lane);
+      const uint4 v = sorted_pop_back(st.H);
+      st.used_h -= esize(v);
+      log_dec(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
+      CNT(st, n_evict, 1);
     }
-    if (!tl_append(st, st.H, kTierH, pk, n, kAuxPinned, 0u, lane)) return false;
+    if (!pin_append(st, pk, n, s, kTierH, lane)) return false;
+    st.used_h += n;
+    st.pinned_h += n;
     log_dec(st, UNISON_KIND_PLACE_H, s, lane);
-    st.c.place_h++;
+    CNT(st, n_place_h, 1);
   } else {
     log_dec(st, UNISON_KIND_BYPASS, s, lane);
-    st.c.bypass++;
+    CNT(st, n_bypass, 1);
     return true;
   }
-  st.pinned_cnt++;
   if (D.max_sessions) {
-    while (st.S.n + st.H.n > D.max_sessions) {
-      const Pick a = argmax_unpinned(st.S, lane);
-      const Pick b = argmax_unpinned(st.H, lane);
-      if (a.slot < 0 && b.slot < 0) {
+    while (st.S.n + st.H.n + st.npin > D.max_sessions) {
+      if (st.S.n == 0 && st.H.n == 0) {
         st.status = UNISON_ERR_CAPACITY;
         return false;
       }
-      if (b.slot < 0 || (a.slot >= 0 && a.pk > b.pk))
-        evict_entry(st, st.S, kTierS, (uint32_t)a.slot, UNISON_KIND_EVICT, lane);
+      const bool from_s =
+          st.H.n == 0 || (st.S.n > 0 && ekey(st.S.e[st.S.n - 1]) > ekey(st.H.e[st.H.n - 1]));
+      const uint4 v = sorted_pop_back(from_s ? st.S : st.H);
+      if (from_s)
+        st.used_s -= esize(v);
       else
-        evict_entry(st, st.H, kTierH, (uint32_t)b.slot, UNISON_KIND_EVICT, lane);
+        st.used_h -= esize(v);
+      log_dec(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
+      CNT(st, n_evict, 1);
     }
   }
   return true;
 }
 
-// Move entry `slot` from one tier list to the other, keeping its fields.
-__device__ __forceinline__ bool move_entry(ReplayState &st, TierList &from, uint32_t from_tier, TierList &to,
-                                           uint32_t to_tier, uint32_t slot, uint32_t aux_or, int lane) {
-  const uint64_t pk = entry_key(from, slot);
-  const uint32_t sz = from.size[slot], ax = from.aux[slot], rt = from.ret[slot];
-  tl_remove(st, from, from_tier, slot, lane);
-  return tl_append(st, to, to_tier, pk, sz, ax | aux_or, rt, lane);
-}
-
-// TIDE at a gap_start with budget bytes: promotions into free fast-tier space
-// (least evictable HBM sessions first), then the pair loop of Algorithm 1.
-__device__ __forceinline__ uint64_t tide(ReplayState &st, const ReplayDesc &D, uint64_t budget, int lane) {
+// TIDE at a gap_start with `budget` bytes.  The moves are decided on the
+// sorted arrays in the list form (phase 1: least evictable HBM sessions into
+// free fast-tier space; phase 2: pair the next least evictable HBM session
+// with the most evictable fast-tier one), which makes the same moves as the
+// pair loop of Algorithm 1, and are then applied in bulk.
+__device__ __forceinline__ uint64_t tide(ReplayState &st, const ReplayDesc &D, uint64_t budget, uint32_t rcap_s,
+                                         int lane) {
   uint64_t rem = budget;
   const uint64_t kvb = D.kvb;
-  for (;;) {
-    const Pick p = argmin_unpinned(st.H, lane);
-    if (p.slot < 0) break;
-    const uint32_t sz = st.H.size[p.slot];
-    const uint64_t by = (uint64_t)sz * kvb;
-    if (by > rem || st.S.used + sz > D.cap_s) break;
+  uint32_t n1 = 0;
+  while (n1 < st.H.n) {
+    const uint4 p = st.H.e[n1];
+    const uint64_t sz = esize(p), by = sz * kvb;
+    if (by > rem || st.used_s + sz > D.cap_s) break;
     rem -= by;
-    if (!move_entry(st, st.H, kTierH, st.S, kTierS, (uint32_t)p.slot, kAuxPromoted, lane)) return budget - rem;
-    log_dec(st, UNISON_KIND_PROMOTE, packed_id(p.pk), lane);
-    st.c.promote++;
+    st.used_s += sz;
+    st.used_h -= sz;
+    log_dec(st, UNISON_KIND_PROMOTE, packed_id(ekey(p)), lane);
+    n1++;
   }
+  uint32_t pairs = 0;
   for (;;) {
-    const Pick p = argmin_unpinned(st.H, lane);
-    const Pick d = argmax_unpinned(st.S, lane);
-    if (p.slot < 0 || d.slot < 0) break;
-    if (!(d.pk > p.pk)) break;  // the demoted session must be strictly more evictable
-    const uint32_t sp = st.H.size[p.slot], sd = st.S.size[d.slot];
-    const uint64_t by = ((uint64_t)sp + sd) * kvb;
+    if (n1 + pairs >= st.H.n || pairs >= st.S.n) break;
+    const uint4 p = st.H.e[n1 + pairs];
+    const uint4 d = st.S.e[st.S.n - 1 - pairs];
+    // the next most evictable of (fast tier + promoted) is a promoted session
+    // when the largest promoted key beats d: then it cannot beat p, stop
+    if (n1 > 0 && ekey(st.H.e[n1 - 1]) > ekey(d)) break;
+    if (!(ekey(d) > ekey(p))) break;
+    const uint64_t sp = esize(p), sd = esize(d), by = (sp + sd) * kvb;
     if (by > rem) break;
-    if (st.S.used - sd + sp > D.cap_s) break;
-    if (st.H.used - sp + sd > D.cap_h) break;
+    if (st.used_s - sd + sp > D.cap_s) break;
+    if (st.used_h - sp + sd > D.cap_h) break;
     rem -= by;
-    if (!move_entry(st, st.H, kTierH, st.S, kTierS, (uint32_t)p.slot, kAuxPromoted, lane)) return budget - rem;
-    // the promoted entry was appended at the end of S; d's slot is unchanged
-    if (!move_entry(st, st.S, kTierS, st.H, kTierH, (uint32_t)d.slot, 0u, lane)) return budget - rem;
-    log_dec(st, UNISON_KIND_PROMOTE, packed_id(p.pk), lane);
-    log_dec(st, UNISON_KIND_TIDE_DEMOTE, packed_id(d.pk), lane);
-    st.c.promote++;
-    st.c.tide_demote++;
+    st.used_s = st.used_s - sd + sp;
+    st.used_h = st.used_h - sp + sd;
+    log_dec(st, UNISON_KIND_PROMOTE, packed_id(ekey(p)), lane);
+    log_dec(st, UNISON_KIND_TIDE_DEMOTE, packed_id(ekey(d)), lane);
+    pairs++;
   }
+  const uint32_t m = n1 + pairs;
+  CNT(st, n_promote, m);
+  CNT(st, n_tide_demote, pairs);
+  if (m == 0) return 0;
+  if (m > rcap_s || pairs > rcap_s) {
+    st.status = UNISON_ERR_CAPACITY;
+    return budget - rem;
+  }
+  // stage the moved entries, then fix both arrays
+  uint4 *pro = st.tmp, *dem = st.tmp + rcap_s;
+  for (uint32_t i = lane; i < m; i += 32) {
+    uint4 v = st.H.e[i];
+    v.z |= kPromotedBit;
+    pro[i] = v;
+  }
+  for (uint32_t i = lane; i < pairs; i += 32) dem[i] = st.S.e[st.S.n - pairs + i];
+  __syncwarp();
+  shift_block(st.H.e, m, st.H.n, -(int32_t)m, lane);
+  st.H.n -= m;
+  st.S.n -= pairs;
+  for (uint32_t i = 0; i < m; i++)
+    if (!sorted_insert(st, st.S, pro[i], lane)) return budget - rem;
+  for (uint32_t i = 0; i < pairs; i++)
+    if (!sorted_insert(st, st.H, dem[i], lane)) return budget - rem;
   return budget - rem;
 }
 
 // Timeout: expire unpinned residents idle >= ttl, smallest session id first.
+// Under recency keys the last return time falls as the key grows, so the
+// expired sessions of a tier are a top suffix of its array.
 __device__ __forceinline__ void expire_idle(ReplayState &st, uint32_t now, uint32_t ttl, int lane) {
   for (;;) {
-    uint32_t bid = kFull, bslot = 0, btier = 0;
-    for (uint32_t i = lane; i < st.S.n; i += 32) {
-      const uint32_t id = (~st.S.lo[i]) & kIdMask;
-      if (!(st.S.aux[i] & kAuxPinned) && now - st.S.ret[i] >= ttl && id < bid) {
+    // expired suffix lengths
+    uint32_t cs = 0, ch = 0;
+    while (cs < st.S.n && now - st.S.e[st.S.n - 1 - cs].w >= ttl) cs++;
+    while (ch < st.H.n && now - st.H.e[st.H.n - 1 - ch].w >= ttl) ch++;
+    if (cs + ch == 0) return;
+    // smallest session id among them
+    uint32_t bid = kFull, bpos = 0, btier = 0;
+    for (uint32_t i = lane; i < cs + ch; i += 32) {
+      const bool inS = i < cs;
+      const uint32_t pos = inS ? st.S.n - 1 - i : st.H.n - 1 - (i - cs);
+      const uint32_t id = packed_id(ekey(inS ? st.S.e[pos] : st.H.e[pos]));
+      if (id < bid) {
         bid = id;
-        bslot = i;
-        btier = kTierS;
+        bpos = pos;
+        btier = inS ? kTierS : kTierH;
       }
     }
-    for (uint32_t i = lane; i < st.H.n; i += 32) {
-      const uint32_t id = (~st.H.lo[i]) & kIdMask;
-      if (!(st.H.aux[i] & kAuxPinned) && now - st.H.ret[i] >= ttl && id < bid) {
-        bid = id;
-        bslot = i;
-        btier = kTierH;
-      }
-    }
-    const uint32_t m = __reduce_min_sync(kFull, bid);
-    if (m == kFull) return;
-    const int src = __ffs(__ballot_sync(kFull, bid == m)) - 1;
-    const uint32_t slot = __shfl_sync(kFull, bslot, src), tier = __shfl_sync(kFull, btier, src);
+    const uint32_t mid = __reduce_min_sync(kFull, bid);
+    const int src = __ffs(__ballot_sync(kFull, bid == mid)) - 1;
+    const uint32_t pos = __shfl_sync(kFull, bpos, src), tier = __shfl_sync(kFull, btier, src);
+    Sorted &T = tier == kTierS ? st.S : st.H;
+    const uint32_t sz = esize(T.e[pos]);
+    __syncwarp();
     if (tier == kTierS)
-      evict_entry(st, st.S, kTierS, slot, UNISON_KIND_EXPIRE, lane);
+      st.used_s -= sz;
     else
-      evict_entry(st, st.H, kTierH, slot, UNISON_KIND_EXPIRE, lane);
+      st.used_h -= sz;
+    sorted_erase(T, pos, lane);
+    log_dec(st, UNISON_KIND_EXPIRE, mid, lane);
+    CNT(st, n_expire, 1);
   }
 }
 
-// Completion of a resident session's turn: unpin, refresh its key, stamp
-// its last return time.
-__device__ __forceinline__ void unpin(ReplayState &st, TierList &L, uint32_t slot, bool spear_keys, bool belady,
-                                      uint64_t cu_pk, uint32_t j, uint32_t e, uint32_t s, uint32_t now, int lane) {
-  const uint32_t ax = L.aux[slot], sz = L.size[slot];
-  uint64_t pk = entry_key(L, slot);
-  const uint64_t spk = __shfl_sync(kFull, cu_pk, j);
-  if (spear_keys)
-    pk = spk;
-  else if (!belady)
-    pk = pack_key(0xFFFFFFFFull - e, s);
-  __syncwarp();
-  if (lane == 0) {
-    L.aux[slot] = ax & ~kAuxPinned;
-    L.ret[slot] = now;
-    L.hi[slot] = (uint32_t)(pk >> 32);
-    L.lo[slot] = (uint32_t)pk;
-  }
-  if (ax & kAuxPinned) {
-    L.pinned -= sz;
-    st.pinned_cnt--;
-  }
-  __syncwarp();
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src)
+               : "memory");
 }
+__device__ __forceinline__ void cp_async8(void *dst, const void *src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async4(void *dst, const void *src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_one() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
 __device__ __forceinline__ bool has_tide(uint32_t policy) {
   return policy == UNISON_SPEAR_TIDE || policy == UNISON_LRU_TIDE;
@@ -548,42 +547,36 @@ template <bool kGlobalLists>
 __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, const uint32_t *order) {
   extern __shared__ __align__(16) unsigned char smem[];
   const int lane = threadIdx.x & 31;
-  const ReplayDesc D = descs[order[blockIdx.x]];
+  __shared__ ReplayDesc Dsh;
+  if (lane == 0) Dsh = descs[order[blockIdx.x]];
+  __syncwarp();
+  const ReplayDesc &D = Dsh;
 
   ReplayState st;
-  unsigned char *base = kGlobalLists ? reinterpret_cast<unsigned char *>(D.glist) : smem;
   {
-    uint32_t *p = reinterpret_cast<uint32_t *>(base);
-    const uint32_t cs = D.rcap_s, ch = D.rcap_h;
-    st.S.hi = p; p += cs;
-    st.S.lo = p; p += cs;
-    st.S.size = p; p += cs;
-    st.S.aux = p; p += cs;
-    st.S.ret = p; p += cs;
-    st.H.hi = p; p += ch;
-    st.H.lo = p; p += ch;
-    st.H.size = p; p += ch;
-    st.H.aux = p; p += ch;
-    st.H.ret = p; p += ch;
-    st.map = D.use_map ? reinterpret_cast<uint16_t *>(p) : nullptr;
+    uint4 *p = reinterpret_cast<uint4 *>(kGlobalLists ? reinterpret_cast<unsigned char *>(D.glist) : smem);
+    st.S.e = p;
+    p += D.rcap_s;
+    st.H.e = p;
+    p += D.rcap_h;
+    st.pin = p;
+    p += D.rcap_s + D.rcap_h;
+    st.tmp = p;
     st.S.n = st.H.n = 0;
-    st.S.cap = cs;
-    st.H.cap = ch;
-    st.S.used = st.S.pinned = st.H.used = st.H.pinned = 0;
-  }
-  if (st.map) {
-    for (uint32_t i = lane; i < D.n_sessions; i += 32) st.map[i] = kMapNone;
-    __syncwarp();
+    st.S.cap = D.rcap_s;
+    st.H.cap = D.rcap_h;
+    st.npin = 0;
+    st.pin_cap = D.rcap_s + D.rcap_h;
+    st.used_s = st.used_h = st.pinned_s = st.pinned_h = 0;
   }
   st.log = D.log;
   st.log_cap = D.log_cap;
   st.status = UNISON_OK;
-  st.pinned_cnt = 0;
-  {
-    unison_replay_result z = {};
-    st.c = z;
-  }
-  st.c.decision_hash = kFnvOffset;
+  st.hash = kFnvOffset;
+  st.log_len = 0;
+  st.n_warm = st.n_cold = st.n_hit_s = st.n_hit_h = st.n_miss = st.n_bypass = st.n_place_s = st.n_place_h = 0;
+  st.n_evict = st.n_demote = st.n_promote = st.n_tide_demote = st.n_expire = st.n_tide_calls = st.n_pth = 0;
+  st.tok_hit_s = st.tok_hit_h = st.tok_miss = st.tok_computed = st.tok_needed = st.dma_bytes = 0;
 
   const uint32_t policy = D.policy;
   const bool spear_keys = policy == UNISON_SPEAR || policy == UNISON_SPEAR_TIDE;
@@ -593,84 +586,122 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
 
   // TTFT queue (Sec. V-A): arrivals compressed by the load factor.
   uint64_t rel_us = 0, q_free = 0;
-  uint32_t prev_now = 0, n_arr = 0;
+  uint32_t prev_now = 0, n_arr = 0, n_ev = 0;
+  const uint32_t load = D.load;
+  const uint64_t ns_per_us = (1000u % load == 0) ? 1000u / load : 0u;  // 0: divide exactly
   unsigned long long s_lo = 0, s_hi = 0;
   bool dma_busy = false;
   uint32_t busy_until = 0;
 
-  // Event prefetch: lane i holds event base + i of the current batch.
+  // Event prefetch: the next batch of 32 events is copied into a shared-memory
+  // double buffer with cp.async while the current batch is processed.
+  __shared__ __align__(16) uint4 sev[2][32];
+  __shared__ __align__(16) uint32_t sprev[2][32], spev[2][32], snref[2][32], sgq[2][32];
+  __shared__ __align__(16) unsigned long long spk[2][32], spkb[2][32];
   const uint32_t E = D.n_events;
-  uint4 nx_ev = make_uint4(0, 0, 0, 0);
-  uint32_t nx_prev = 0, nx_nref = kNoRef, nx_gq = 0;
-  uint64_t nx_pk = 0;
-  auto fetch = [&](uint32_t b) {
+  auto fetch = [&](uint32_t b, int bi) {
     const uint32_t i = b + lane;
     if (i < E) {
-      nx_ev = __ldg(&D.ev[i]);
-      nx_prev = __ldg(&D.prev_out[i]);
-      if (belady) nx_nref = __ldg(&D.nref[i]);
-      if (spear_keys) nx_pk = __ldg(&D.pkey[i]);
-      if (tide_on) nx_gq = __ldg(&D.gq[i]);
+      cp_async16(&sev[bi][lane], &D.ev[i]);
+      cp_async4(&sprev[bi][lane], &D.prev_out[i]);
+      cp_async4(&spev[bi][lane], &D.prev_ev[i]);
+      if (belady) cp_async4(&snref[bi][lane], &D.nref[i]);
+      if (spear_keys) {
+        cp_async8(&spk[bi][lane], &D.pkey[i]);
+        cp_async8(&spkb[bi][lane], &D.pkb[i]);
+      }
+      if (tide_on) cp_async4(&sgq[bi][lane], &D.gq[i]);
     }
+    cp_async_commit();
   };
-  fetch(0);
-  if (E) prev_now = __shfl_sync(kFull, nx_ev.x, 0);
+  fetch(0, 0);
+  cp_async_wait_all();
+  __syncwarp();
+  if (E) prev_now = sev[0][0].x;
 
-  for (uint32_t b = 0; b < E && st.status != UNISON_ERR_CAPACITY; b += 32) {
-    const uint4 cu_ev = nx_ev;
-    const uint32_t cu_prev = nx_prev, cu_nref = nx_nref, cu_gq = nx_gq;
-    const uint64_t cu_pk = nx_pk;
-    if (b + 32 < E) fetch(b + 32);
+  int bi = 0;
+  for (uint32_t b = 0; b < E && st.status != UNISON_ERR_CAPACITY; b += 32, bi ^= 1) {
+    if (b + 32 < E) {
+      fetch(b + 32, bi ^ 1);
+      cp_async_wait_one();  // this batch's copies have landed
+    } else {
+      cp_async_wait_all();
+    }
+    __syncwarp();
     const uint32_t cnt = min(32u, E - b);
     for (uint32_t j = 0; j < cnt; j++) {
       const uint32_t e = b + j;
-      const uint32_t now = __shfl_sync(kFull, cu_ev.x, j);
-      const uint32_t w1 = __shfl_sync(kFull, cu_ev.y, j);
+      const uint4 ev = sev[bi][j];
+      const uint32_t now = ev.x;
+      const uint32_t w1 = ev.y;
       const uint32_t s = w1 & kIdMask;
       const bool arrival = (w1 & kEvArrival) != 0;
       const bool edge = (w1 & kEvEdge) != 0;
       st.e = e;
-      st.c.events++;
+      n_ev++;
       rel_us += (uint32_t)(now - prev_now);
       prev_now = now;
       if (timeout) expire_idle(st, now, D.ttl, lane);
       if (dma_busy && (int32_t)(now - busy_until) >= 0) dma_busy = false;
 
-      uint32_t tier, slot;
-      locate(st, s, tier, slot, lane);
       if (arrival) {
-        const uint32_t in = __shfl_sync(kFull, cu_ev.z, j);
-        const uint32_t out = __shfl_sync(kFull, cu_ev.w, j);
-        const uint32_t prev = __shfl_sync(kFull, cu_prev, j);
+        const uint32_t in = ev.z;
+        const uint32_t out = ev.w;
+        const uint32_t prev = sprev[bi][j];
+        // where is s?  search both tiers for the key of its previous event
+        uint32_t tier = kTierNone;
+        uint4 ent = make_uint4(0, 0, 0, 0);
+        uint32_t pos = 0;
+        if (!edge) {
+          uint64_t pkb;
+          if (spear_keys)
+            pkb = spkb[bi][j];
+          else if (belady)
+            pkb = pack_key(e, s);  // the previous arrival's next reference is this event
+          else
+            pkb = pack_key(0xFFFFFFFFull - spev[bi][j], s);
+          pos = lower_bound(st.S, pkb, lane);
+          if (pos < st.S.n && ekey(st.S.e[pos]) == pkb) {
+            tier = kTierS;
+            ent = st.S.e[pos];
+          } else {
+            pos = lower_bound(st.H, pkb, lane);
+            if (pos < st.H.n && ekey(st.H.e[pos]) == pkb) {
+              tier = kTierH;
+              ent = st.H.e[pos];
+            }
+          }
+          __syncwarp();
+        }
         uint64_t prefill;
         if (edge) {
           log_dec(st, UNISON_KIND_COLD, s, lane);
-          st.c.cold++;
+          CNT(st, n_cold, 1);
           prefill = in;
         } else {
-          st.c.req_warm++;
-          st.c.tok_needed += in;
+          CNT(st, n_warm, 1);
+          CNT(st, tok_needed, in);
           if (tier == kTierS) {
             log_dec(st, UNISON_KIND_HIT_S, s, lane);
-            st.c.hit_s++;
-            st.c.tok_hit_s += prev;
+            CNT(st, n_hit_s, 1);
+            CNT(st, tok_hit_s, prev);
             prefill = in - prev;
-            if (st.S.aux[slot] & kAuxPromoted) st.c.promoted_then_hit_s++;
+            if (ent.z & kPromotedBit) CNT(st, n_pth, 1);
           } else if (tier == kTierH) {
             log_dec(st, UNISON_KIND_HIT_H, s, lane);
-            st.c.hit_h++;
-            st.c.tok_hit_h += prev;
+            CNT(st, n_hit_h, 1);
+            CNT(st, tok_hit_h, prev);
             prefill = in - prev;
           } else {
             log_dec(st, UNISON_KIND_MISS, s, lane);
-            st.c.miss++;
-            st.c.tok_miss += prev;
+            CNT(st, n_miss, 1);
+            CNT(st, tok_miss, prev);
             prefill = in;
           }
-          st.c.tok_computed += prefill;
+          CNT(st, tok_computed, prefill);
         }
         {
-          const uint64_t arr = rel_us * 1000ull / D.load;
+          const uint64_t arr = ns_per_us ? rel_us * ns_per_us : rel_us * 1000ull / load;
           if (q_free < arr) q_free = arr;
           q_free += prefill * D.prefill_ns;
           const uint64_t v = q_free - arr;
@@ -680,30 +711,57 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
           s_hi += (lo2 < s_lo);
           s_lo = lo2;
         }
-        if (tier == kTierS)
-          tl_remove(st, st.S, kTierS, slot, lane);
-        else if (tier == kTierH)
-          tl_remove(st, st.H, kTierH, slot, lane);
+        if (tier == kTierS) {
+          st.used_s -= esize(ent);
+          sorted_erase(st.S, pos, lane);
+        } else if (tier == kTierH) {
+          st.used_h -= esize(ent);
+          sorted_erase(st.H, pos, lane);
+        }
         uint64_t pk;
         if (spear_keys)
-          pk = __shfl_sync(kFull, cu_pk, j);
+          pk = spk[bi][j];
         else if (belady) {
-          const uint32_t nr = __shfl_sync(kFull, cu_nref, j);
+          const uint32_t nr = snref[bi][j];
           pk = pack_key(nr == kNoRef ? kKeyMax40 : (uint64_t)nr, s);
         } else
           pk = pack_key(0xFFFFFFFFull - e, s);
         if (!place(st, D, s, pk, out, lane)) break;
       } else {
-        if (tier == kTierS)
-          unpin(st, st.S, slot, spear_keys, belady, cu_pk, j, e, s, now, lane);
-        else if (tier == kTierH)
-          unpin(st, st.H, slot, spear_keys, belady, cu_pk, j, e, s, now, lane);
+        // completion: unpin (if resident) and rank the session with its new key
+        int mine = -1;
+        for (uint32_t i = lane; i < st.npin; i += 32)
+          if ((st.pin[i].w & kIdMask) == s) mine = (int)i;
+        const uint32_t who = __ballot_sync(kFull, mine >= 0);
+        if (who) {
+          const uint32_t pi = (uint32_t)__shfl_sync(kFull, mine, __ffs(who) - 1);
+          const uint4 pe = st.pin[pi];
+          const uint4 last = st.pin[st.npin - 1];
+          __syncwarp();
+          if (lane == 0) st.pin[pi] = last;
+          __syncwarp();
+          st.npin--;
+          const uint32_t tier = pe.w >> 30, sz = pe.z;
+          uint64_t pk = ((uint64_t)pe.y << 32) | pe.x;
+          if (spear_keys)
+            pk = spk[bi][j];
+          else if (!belady)
+            pk = pack_key(0xFFFFFFFFull - e, s);
+          const uint4 v = make_uint4((uint32_t)pk, (uint32_t)(pk >> 32), sz, now);
+          if (tier == kTierS) {
+            st.pinned_s -= sz;
+            if (!sorted_insert(st, st.S, v, lane)) break;
+          } else {
+            st.pinned_h -= sz;
+            if (!sorted_insert(st, st.H, v, lane)) break;
+          }
+        }
         if (!edge && tide_on && !dma_busy) {
-          const uint64_t g = __shfl_sync(kFull, cu_gq, j);
+          const uint64_t g = sgq[bi][j];
           const uint64_t budget = g * D.dma;
-          st.c.tide_calls++;
-          const uint64_t moved = tide(st, D, budget, lane);
-          st.c.dma_bytes += moved;
+          CNT(st, n_tide_calls, 1);
+          const uint64_t moved = tide(st, D, budget, D.rcap_s, lane);
+          CNT(st, dma_bytes, moved);
           if (moved > 0 && D.dma > 0) {
             dma_busy = true;
             busy_until = now + (uint32_t)((moved + D.dma - 1) / D.dma);
@@ -713,12 +771,39 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
       }
     }
   }
-  st.c.ttft_n = n_arr;
-  st.c.ttft_sum_lo = s_lo;
-  st.c.ttft_sum_hi = s_hi;
-  st.c.ttft_p50_ns = 0;
-  st.c.status = st.status;
-  if (lane == 0) *D.result = st.c;
+  if (lane == 0) {
+    unison_replay_result r = {};
+    r.events = n_ev;
+    r.req_warm = st.n_warm;
+    r.cold = st.n_cold;
+    r.hit_s = st.n_hit_s;
+    r.hit_h = st.n_hit_h;
+    r.miss = st.n_miss;
+    r.bypass = st.n_bypass;
+    r.place_s = st.n_place_s;
+    r.place_h = st.n_place_h;
+    r.evict = st.n_evict;
+    r.demote = st.n_demote;
+    r.promote = st.n_promote;
+    r.tide_demote = st.n_tide_demote;
+    r.expire = st.n_expire;
+    r.tok_hit_s = st.tok_hit_s;
+    r.tok_hit_h = st.tok_hit_h;
+    r.tok_miss = st.tok_miss;
+    r.tok_computed = st.tok_computed;
+    r.tok_needed = st.tok_needed;
+    r.dma_bytes = st.dma_bytes;
+    r.tide_calls = st.n_tide_calls;
+    r.promoted_then_hit_s = st.n_pth;
+    r.ttft_sum_lo = s_lo;
+    r.ttft_sum_hi = s_hi;
+    r.ttft_p50_ns = 0;
+    r.ttft_n = n_arr;
+    r.decision_hash = st.hash;
+    r.log_len = st.log_len;
+    r.status = st.status;
+    *D.result = r;
+  }
 }
 
 // Lower median (element floor((n-1)/2) in sorted order) by MSB-first radix select.
@@ -808,106 +893,98 @@ extern "C" int unison_hazard_lut(const uint32_t *turns_dev, uint64_t n_sessions,
   return cudaGetLastError() == cudaSuccess ? UNISON_OK : UNISON_ERR_CUDA;
 }
 
-extern "C" int unison_replay_batch(const unison_trace *const *traces, int n_traces,
-                                   const unison_replay_params *params, int n_replays,
-                                   unison_replay_result *results_dev, unison_replay_result *results_host,
-                                   unison_decision *log_dev, uint64_t log_capacity_per_replay, void *cuda_stream) {
-  if (!traces || n_traces <= 0 || !params || n_replays < 0) return UNISON_ERR_ARG;
-  if (n_replays == 0) return UNISON_OK;
-  if (!results_dev && !results_host) return UNISON_ERR_ARG;
-  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return UNISON_ERR_CUDA;
-  for (int i = 0; i < n_traces; i++)
-    if (!traces[i] || !traces[i]->d_block || traces[i]->device != dev) return UNISON_ERR_ARG;
-  for (int r = 0; r < n_replays; r++) {
-    const int rc = check_params(params[r], n_traces);
-    if (rc != UNISON_OK) return rc;
-  }
-  int smem_optin = 0;
-  cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-  const size_t smem_limit = (size_t)smem_optin > 1024 ? (size_t)smem_optin - 1024 : 0;
+namespace {
 
-  // Key streams: one per (trace, EMA weight, bucket, P_Z) used by a policy that needs them.
-  std::map<std::tuple<uint32_t, uint32_t, uint32_t, uint32_t, uint64_t>, int> combo_of;
+// Scratch layout and launch plan of one batch (shared by both entry points).
+struct ReplayPlan {
   std::vector<std::tuple<uint32_t, uint32_t, uint32_t, uint32_t, uint64_t>> combos;
-  std::vector<int> replay_combo(n_replays, -1);
+  std::vector<int> replay_combo;
+  size_t off_desc = 0, off_order = 0, off_combo = 0, bytes = 0;
+  std::vector<size_t> off_lut, off_stream, off_ttft, off_glist;
+  std::vector<uint32_t> rcap_s, rcap_h, in_smem, in_global;
+  size_t max_smem = 0;
+};
+
+// Resident-list capacity of a tier: at most one entry per session and no more
+// than the tier's token capacity over the smallest l^out of the trace (+1
+// for the transient extra entry while a pair is swapped).
+uint32_t list_cap(uint64_t cap_tok, const unison_trace *tr) {
+  const uint64_t mo = std::max<uint32_t>(tr->min_out_tok, 1);
+  return (uint32_t)std::min<uint64_t>(tr->n_sessions, cap_tok / mo) + 1;
+}
+
+// 16-byte entries: fast and HBM arrays, the pinned list (both tiers) and the
+// TIDE staging area (two fast-tier capacities).
+size_t list_bytes(uint32_t cs, uint32_t ch) { return 16ull * (4ull * cs + 2ull * ch); }
+
+void plan_replays(const unison_trace *const *traces, const unison_replay_params *params, int n_replays,
+                  size_t smem_limit, bool results_in_scratch, ReplayPlan &P, size_t &off_res) {
+  std::map<std::tuple<uint32_t, uint32_t, uint32_t, uint32_t, uint64_t>, int> combo_of;
+  P.replay_combo.assign(n_replays, -1);
   for (int r = 0; r < n_replays; r++) {
     const unison_replay_params &p = params[r];
     if (!needs_stream(p.policy)) continue;
     auto key = std::make_tuple(p.trace_idx, p.ema_num, p.ema_den, p.hazard_bucket, p.penalty_q);
     auto it = combo_of.find(key);
     if (it == combo_of.end()) {
-      it = combo_of.emplace(key, (int)combos.size()).first;
-      combos.push_back(key);
+      it = combo_of.emplace(key, (int)P.combos.size()).first;
+      P.combos.push_back(key);
     }
-    replay_combo[r] = it->second;
+    P.replay_combo[r] = it->second;
   }
-
-  // Scratch layout.
   size_t off = 0;
-  const size_t off_desc = off;
+  P.off_desc = off;
   off = align_up(off + sizeof(ReplayDesc) * n_replays, 256);
-  const size_t off_order = off;
+  P.off_order = off;
   off = align_up(off + sizeof(uint32_t) * 2 * n_replays, 256);
-  const size_t off_combo = off;
-  off = align_up(off + sizeof(ComboDesc) * combos.size() + 1, 256);
-  std::vector<size_t> off_lut(combos.size()), off_stream(combos.size());
-  for (size_t c = 0; c < combos.size(); c++) {
-    off_lut[c] = off;
+  P.off_combo = off;
+  off = align_up(off + sizeof(ComboDesc) * P.combos.size() + 1, 256);
+  P.off_lut.resize(P.combos.size());
+  P.off_stream.resize(P.combos.size());
+  for (size_t c = 0; c < P.combos.size(); c++) {
+    P.off_lut[c] = off;
     off = align_up(off + 128 + 51 * 8, 256);
-    const uint64_t E = traces[std::get<0>(combos[c])]->n_events;
-    off_stream[c] = off;
-    off = align_up(off + 12 * E, 256);
+    const uint64_t E = traces[std::get<0>(P.combos[c])]->n_events;
+    P.off_stream[c] = off;
+    off = align_up(off + align_up(12 * E, 8) + 8 * E, 256);
   }
-  std::vector<size_t> off_ttft(n_replays), off_glist(n_replays, 0);
-  std::vector<uint32_t> rcap_s(n_replays), rcap_h(n_replays), use_map(n_replays), smem_bytes(n_replays);
-  std::vector<uint32_t> in_smem, in_global;
-  size_t max_smem = 0;
+  P.off_ttft.assign(n_replays, 0);
+  P.off_glist.assign(n_replays, 0);
+  P.rcap_s.resize(n_replays);
+  P.rcap_h.resize(n_replays);
   for (int r = 0; r < n_replays; r++) {
     const unison_replay_params &p = params[r];
     const unison_trace *tr = traces[p.trace_idx];
-    const uint64_t cs = p.cap_fast_bytes / p.kv_bytes_per_token, ch = p.cap_hbm_bytes / p.kv_bytes_per_token;
-    const uint64_t mo = std::max<uint32_t>(tr->min_out_tok, 1);
-    rcap_s[r] = (uint32_t)std::min<uint64_t>(tr->n_sessions, cs / mo) + 1;
-    rcap_h[r] = (uint32_t)std::min<uint64_t>(tr->n_sessions, ch / mo) + 1;
-    const size_t lists = (size_t)kEntryBytes * (rcap_s[r] + rcap_h[r]);
-    const size_t map_b = align_up(2ull * tr->n_sessions, 16);
-    const bool map_ok = rcap_s[r] <= 0x7FFF && rcap_h[r] <= 0x7FFF;
-    if (map_ok && lists + map_b <= smem_limit && map_b <= 32768) {
-      use_map[r] = 1;
-      smem_bytes[r] = (uint32_t)(lists + map_b);
+    P.rcap_s[r] = list_cap(p.cap_fast_bytes / p.kv_bytes_per_token, tr);
+    P.rcap_h[r] = list_cap(p.cap_hbm_bytes / p.kv_bytes_per_token, tr);
+    const size_t lists = list_bytes(P.rcap_s[r], P.rcap_h[r]);
+    if (lists <= smem_limit) {
+      P.in_smem.push_back((uint32_t)r);
+      P.max_smem = std::max<size_t>(P.max_smem, lists);
     } else {
-      use_map[r] = 0;
-      smem_bytes[r] = (uint32_t)lists;
-    }
-    if (smem_bytes[r] <= smem_limit) {
-      in_smem.push_back((uint32_t)r);
-      max_smem = std::max<size_t>(max_smem, smem_bytes[r]);
-    } else {
-      use_map[r] = 0;
-      in_global.push_back((uint32_t)r);
-      off_glist[r] = off;
+      P.in_global.push_back((uint32_t)r);
+      P.off_glist[r] = off;
       off = align_up(off + lists, 256);
     }
-    off_ttft[r] = off;
+    P.off_ttft[r] = off;
     off = align_up(off + 8 * (tr->n_turns + 1), 256);
   }
-  size_t off_res = 0;
-  if (!results_dev) {
+  off_res = 0;
+  if (results_in_scratch) {
     off_res = off;
     off = align_up(off + sizeof(unison_replay_result) * n_replays, 256);
   }
-  char *scratch = nullptr;
-  if (cudaMallocAsync(reinterpret_cast<void **>(&scratch), off, stream) != cudaSuccess) {
-    cudaGetLastError();
-    return UNISON_ERR_OOM;
-  }
-  unison_replay_result *res = results_dev ? results_dev : reinterpret_cast<unison_replay_result *>(scratch + off_res);
+  P.bytes = off;
+}
 
-  std::vector<ComboDesc> hc(combos.size());
-  for (size_t c = 0; c < combos.size(); c++) {
-    const unison_trace *tr = traces[std::get<0>(combos[c])];
+// Fill the descriptors for a plan placed at `scratch`.
+void fill_descs(const unison_trace *const *traces, const unison_replay_params *params, int n_replays,
+                const ReplayPlan &P, char *scratch, unison_replay_result *res, unison_decision *log_dev,
+                uint64_t log_cap, std::vector<ComboDesc> &hc, std::vector<ReplayDesc> &hd,
+                std::vector<uint32_t> &order) {
+  hc.resize(P.combos.size());
+  for (size_t c = 0; c < P.combos.size(); c++) {
+    const unison_trace *tr = traces[std::get<0>(P.combos[c])];
     ComboDesc &d = hc[c];
     d.turn_ev = tr->d<uint32_t>(tr->off_turn_ev);
     d.turn_t = tr->d<uint32_t>(tr->off_turn_t);
@@ -915,17 +992,18 @@ extern "C" int unison_replay_batch(const unison_trace *const *traces, int n_trac
     d.tps = tr->d<uint32_t>(tr->off_tps);
     d.n_sessions = tr->n_sessions;
     d.n_events = (uint32_t)tr->n_events;
-    d.ema_num = std::get<1>(combos[c]);
-    d.ema_den = std::get<2>(combos[c]);
-    d.bucket = std::get<3>(combos[c]);
+    d.ema_num = std::get<1>(P.combos[c]);
+    d.ema_den = std::get<2>(P.combos[c]);
+    d.bucket = std::get<3>(P.combos[c]);
     d.pad = 0;
-    d.penalty_q = std::get<4>(combos[c]);
-    d.sigma = reinterpret_cast<uint16_t *>(scratch + off_lut[c]);
-    d.t2 = reinterpret_cast<uint64_t *>(scratch + off_lut[c] + 128);
-    d.pkey = reinterpret_cast<uint64_t *>(scratch + off_stream[c]);
-    d.gq = reinterpret_cast<uint32_t *>(scratch + off_stream[c] + 8 * tr->n_events);
+    d.penalty_q = std::get<4>(P.combos[c]);
+    d.sigma = reinterpret_cast<uint16_t *>(scratch + P.off_lut[c]);
+    d.t2 = reinterpret_cast<uint64_t *>(scratch + P.off_lut[c] + 128);
+    d.pkey = reinterpret_cast<uint64_t *>(scratch + P.off_stream[c]);
+    d.gq = reinterpret_cast<uint32_t *>(scratch + P.off_stream[c] + 8 * tr->n_events);
+    d.pkb = reinterpret_cast<uint64_t *>(scratch + P.off_stream[c] + align_up(12 * tr->n_events, 8));
   }
-  std::vector<ReplayDesc> hd(n_replays);
+  hd.resize(n_replays);
   for (int r = 0; r < n_replays; r++) {
     const unison_replay_params &p = params[r];
     const unison_trace *tr = traces[p.trace_idx];
@@ -933,12 +1011,14 @@ extern "C" int unison_replay_batch(const unison_trace *const *traces, int n_trac
     d.ev = tr->d<uint4>(tr->off_ev);
     d.prev_out = tr->d<uint32_t>(tr->off_prev_out);
     d.nref = tr->d<uint32_t>(tr->off_nref);
-    d.pkey = replay_combo[r] >= 0 ? hc[replay_combo[r]].pkey : nullptr;
-    d.gq = replay_combo[r] >= 0 ? hc[replay_combo[r]].gq : nullptr;
-    d.ttft = reinterpret_cast<uint64_t *>(scratch + off_ttft[r]);
-    d.glist = off_glist[r] ? reinterpret_cast<uint32_t *>(scratch + off_glist[r]) : nullptr;
-    d.log = log_dev ? log_dev + (uint64_t)r * log_capacity_per_replay : nullptr;
-    d.log_cap = log_dev ? log_capacity_per_replay : 0;
+    d.prev_ev = tr->d<uint32_t>(tr->off_prev_ev);
+    d.pkey = P.replay_combo[r] >= 0 ? hc[P.replay_combo[r]].pkey : nullptr;
+    d.gq = P.replay_combo[r] >= 0 ? hc[P.replay_combo[r]].gq : nullptr;
+    d.pkb = P.replay_combo[r] >= 0 ? hc[P.replay_combo[r]].pkb : nullptr;
+    d.ttft = reinterpret_cast<uint64_t *>(scratch + P.off_ttft[r]);
+    d.glist = P.off_glist[r] ? reinterpret_cast<uint32_t *>(scratch + P.off_glist[r]) : nullptr;
+    d.log = log_dev ? log_dev + (uint64_t)r * log_cap : nullptr;
+    d.log_cap = log_dev ? log_cap : 0;
     d.result = res + r;
     d.cap_s = p.cap_fast_bytes / p.kv_bytes_per_token;
     d.cap_h = p.cap_hbm_bytes / p.kv_bytes_per_token;
@@ -952,61 +1032,113 @@ extern "C" int unison_replay_batch(const unison_trace *const *traces, int n_trac
     d.kvb = p.kv_bytes_per_token;
     d.ttl = p.ttl_us;
     d.load = p.ttft_load;
-    d.rcap_s = rcap_s[r];
-    d.rcap_h = rcap_h[r];
-    d.use_map = use_map[r];
-    d.pad = 0;
+    d.rcap_s = P.rcap_s[r];
+    d.rcap_h = P.rcap_h[r];
   }
-  std::vector<uint32_t> order;
-  order.insert(order.end(), in_smem.begin(), in_smem.end());
-  order.insert(order.end(), in_global.begin(), in_global.end());
+  order.clear();
+  order.insert(order.end(), P.in_smem.begin(), P.in_smem.end());
+  order.insert(order.end(), P.in_global.begin(), P.in_global.end());
+}
 
+// Queue the kernels of a planned batch on `stream`.
+int launch_replays(const ReplayPlan &P, char *scratch, const std::vector<ComboDesc> &hc,
+                   const std::vector<ReplayDesc> &hd, const std::vector<uint32_t> &order, int n_replays,
+                   cudaStream_t stream, bool profile) {
   int rc = UNISON_OK;
   auto ck = [&](cudaError_t e) {
     if (e != cudaSuccess && rc == UNISON_OK) rc = UNISON_ERR_CUDA;
   };
-  ReplayDesc *d_desc = reinterpret_cast<ReplayDesc *>(scratch + off_desc);
-  uint32_t *d_order = reinterpret_cast<uint32_t *>(scratch + off_order);
-  ComboDesc *d_combo = reinterpret_cast<ComboDesc *>(scratch + off_combo);
+  ReplayDesc *d_desc = reinterpret_cast<ReplayDesc *>(scratch + P.off_desc);
+  uint32_t *d_order = reinterpret_cast<uint32_t *>(scratch + P.off_order);
+  ComboDesc *d_combo = reinterpret_cast<ComboDesc *>(scratch + P.off_combo);
   ck(cudaMemcpyAsync(d_desc, hd.data(), sizeof(ReplayDesc) * n_replays, cudaMemcpyHostToDevice, stream));
   ck(cudaMemcpyAsync(d_order, order.data(), sizeof(uint32_t) * order.size(), cudaMemcpyHostToDevice, stream));
-  if (!combos.empty()) {
-    ck(cudaMemcpyAsync(d_combo, hc.data(), sizeof(ComboDesc) * combos.size(), cudaMemcpyHostToDevice, stream));
-    hazard_lut_kernel<<<(unsigned)combos.size(), 256, 0, stream>>>(d_combo);
+  if (!P.combos.empty()) {
+    ck(cudaMemcpyAsync(d_combo, hc.data(), sizeof(ComboDesc) * P.combos.size(), cudaMemcpyHostToDevice, stream));
+    hazard_lut_kernel<<<(unsigned)P.combos.size(), 256, 0, stream>>>(d_combo);
     uint32_t max_s = 0;
     for (auto &c : hc) max_s = std::max(max_s, c.n_sessions);
-    dim3 g((max_s + 127) / 128, (unsigned)combos.size());
+    dim3 g((max_s + 127) / 128, (unsigned)P.combos.size());
     {
-      ProfSpan span("key_stream", stream);
+      ProfSpan span(profile ? "key_stream" : "", stream);
       key_stream_kernel<<<g, 128, 0, stream>>>(d_combo);
     }
     count_launches(2);
     ck(cudaGetLastError());
   }
   {
-    ProfSpan span("replay", stream);
-    if (!in_smem.empty()) {
-      ck(cudaFuncSetAttribute(replay_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)max_smem));
-      replay_kernel<false><<<(unsigned)in_smem.size(), 32, max_smem, stream>>>(d_desc, d_order);
+    ProfSpan span(profile ? "replay" : "", stream);
+    if (!P.in_smem.empty()) {
+      ck(cudaFuncSetAttribute(replay_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P.max_smem));
+      replay_kernel<false><<<(unsigned)P.in_smem.size(), 32, P.max_smem, stream>>>(d_desc, d_order);
       count_launches(1);
       ck(cudaGetLastError());
     }
-    if (!in_global.empty()) {
-      replay_kernel<true><<<(unsigned)in_global.size(), 32, 0, stream>>>(d_desc, d_order + in_smem.size());
+    if (!P.in_global.empty()) {
+      replay_kernel<true><<<(unsigned)P.in_global.size(), 32, 0, stream>>>(d_desc, d_order + P.in_smem.size());
       count_launches(1);
       ck(cudaGetLastError());
     }
   }
   {
-    ProfSpan span("ttft_median", stream);
+    ProfSpan span(profile ? "ttft_median" : "", stream);
     ttft_median_kernel<<<(unsigned)n_replays, 256, 0, stream>>>(d_desc, (uint32_t)n_replays);
   }
   count_launches(1);
   ck(cudaGetLastError());
-  if (results_host)
-    ck(cudaMemcpyAsync(results_host, res, sizeof(unison_replay_result) * n_replays, cudaMemcpyDeviceToHost, stream));
-  ck(cudaFreeAsync(scratch, stream));
-  if (results_host) ck(cudaStreamSynchronize(stream));
+  return rc;
+}
+
+int check_batch(const unison_trace *const *traces, int n_traces, const unison_replay_params *params, int n_replays,
+                int &dev, size_t &smem_limit) {
+  if (!traces || n_traces <= 0 || !params || n_replays < 0) return UNISON_ERR_ARG;
+  if (cudaGetDevice(&dev) != cudaSuccess) return UNISON_ERR_CUDA;
+  for (int i = 0; i < n_traces; i++)
+    if (!traces[i] || !traces[i]->d_block || traces[i]->device != dev) return UNISON_ERR_ARG;
+  for (int r = 0; r < n_replays; r++) {
+    const int rc = check_params(params[r], n_traces);
+    if (rc != UNISON_OK) return rc;
+  }
+  int smem_optin = 0;
+  cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  smem_limit = (size_t)smem_optin > 1024 ? (size_t)smem_optin - 1024 : 0;
+  return UNISON_OK;
+}
+
+}  // namespace
+
+extern "C" int unison_replay_batch(const unison_trace *const *traces, int n_traces,
+                                   const unison_replay_params *params, int n_replays,
+                                   unison_replay_result *results_dev, unison_replay_result *results_host,
+                                   unison_decision *log_dev, uint64_t log_capacity_per_replay, void *cuda_stream) {
+  int dev = 0;
+  size_t smem_limit = 0;
+  int rc = check_batch(traces, n_traces, params, n_replays, dev, smem_limit);
+  if (rc != UNISON_OK) return rc;
+  if (n_replays == 0) return UNISON_OK;
+  if (!results_dev && !results_host) return UNISON_ERR_ARG;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  ReplayPlan P;
+  size_t off_res = 0;
+  plan_replays(traces, params, n_replays, smem_limit, results_dev == nullptr, P, off_res);
+  char *scratch = nullptr;
+  if (cudaMallocAsync(reinterpret_cast<void **>(&scratch), P.bytes, stream) != cudaSuccess) {
+    cudaGetLastError();
+    return UNISON_ERR_OOM;
+  }
+  unison_replay_result *res = results_dev ? results_dev : reinterpret_cast<unison_replay_result *>(scratch + off_res);
+  std::vector<ComboDesc> hc;
+  std::vector<ReplayDesc> hd;
+  std::vector<uint32_t> order;
+  fill_descs(traces, params, n_replays, P, scratch, res, log_dev, log_capacity_per_replay, hc, hd, order);
+  rc = launch_replays(P, scratch, hc, hd, order, n_replays, stream, true);
+  if (results_host &&
+      cudaMemcpyAsync(results_host, res, sizeof(unison_replay_result) * n_replays, cudaMemcpyDeviceToHost, stream) !=
+          cudaSuccess &&
+      rc == UNISON_OK)
+    rc = UNISON_ERR_CUDA;
+  if (cudaFreeAsync(scratch, stream) != cudaSuccess && rc == UNISON_OK) rc = UNISON_ERR_CUDA;
+  if (results_host && cudaStreamSynchronize(stream) != cudaSuccess && rc == UNISON_OK) rc = UNISON_ERR_CUDA;
   return rc;
 }
 
@@ -1071,190 +1203,35 @@ extern "C" int unison_replay_batch_noalloc(const unison_trace *const *traces, in
                                            unison_replay_result *results_dev, unison_replay_result *results_host,
                                            unison_decision *log_dev, uint64_t log_capacity_per_replay,
                                            void *cuda_stream) {
-  if (!traces || n_traces <= 0 || !params || n_replays < 0) return UNISON_ERR_ARG;
+  int dev = 0;
+  size_t smem_limit = 0;
+  int rc = check_batch(traces, n_traces, params, n_replays, dev, smem_limit);
+  if (rc != UNISON_OK) return rc;
   if (n_replays == 0) return UNISON_OK;
   if (!results_dev) return UNISON_ERR_ARG;  // the caller provides the output buffer
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return UNISON_ERR_CUDA;
-  for (int i = 0; i < n_traces; i++)
-    if (!traces[i] || !traces[i]->d_block || traces[i]->device != dev) return UNISON_ERR_ARG;
-  for (int r = 0; r < n_replays; r++) {
-    const int rc = check_params(params[r], n_traces);
-    if (rc != UNISON_OK) return rc;
-  }
   char *scratch = nullptr;
-  {
-    const int rc = noalloc_scratch_address(&scratch);
-    if (rc != UNISON_OK) return rc;
-  }
-  int smem_optin = 0;
-  cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-  const size_t smem_limit = (size_t)smem_optin > 1024 ? (size_t)smem_optin - 1024 : 0;
-
-  std::map<std::tuple<uint32_t, uint32_t, uint32_t, uint32_t, uint64_t>, int> combo_of;
-  std::vector<std::tuple<uint32_t, uint32_t, uint32_t, uint32_t, uint64_t>> combos;
-  std::vector<int> replay_combo(n_replays, -1);
-  for (int r = 0; r < n_replays; r++) {
-    const unison_replay_params &p = params[r];
-    if (!needs_stream(p.policy)) continue;
-    auto key = std::make_tuple(p.trace_idx, p.ema_num, p.ema_den, p.hazard_bucket, p.penalty_q);
-    auto it = combo_of.find(key);
-    if (it == combo_of.end()) {
-      it = combo_of.emplace(key, (int)combos.size()).first;
-      combos.push_back(key);
-    }
-    replay_combo[r] = it->second;
-  }
-
-  // Same layout as unison_replay_batch, without the results region.
-  size_t off = 0;
-  const size_t off_desc = off;
-  off = align_up(off + sizeof(ReplayDesc) * n_replays, 256);
-  const size_t off_order = off;
-  off = align_up(off + sizeof(uint32_t) * 2 * n_replays, 256);
-  const size_t off_combo = off;
-  off = align_up(off + sizeof(ComboDesc) * combos.size() + 1, 256);
-  std::vector<size_t> off_lut(combos.size()), off_stream(combos.size());
-  for (size_t c = 0; c < combos.size(); c++) {
-    off_lut[c] = off;
-    off = align_up(off + 128 + 51 * 8, 256);
-    const uint64_t E = traces[std::get<0>(combos[c])]->n_events;
-    off_stream[c] = off;
-    off = align_up(off + 12 * E, 256);
-  }
-  std::vector<size_t> off_ttft(n_replays), off_glist(n_replays, 0);
-  std::vector<uint32_t> rcap_s(n_replays), rcap_h(n_replays), use_map(n_replays), smem_bytes(n_replays);
-  std::vector<uint32_t> in_smem, in_global;
-  size_t max_smem = 0;
-  for (int r = 0; r < n_replays; r++) {
-    const unison_replay_params &p = params[r];
-    const unison_trace *tr = traces[p.trace_idx];
-    const uint64_t cs = p.cap_fast_bytes / p.kv_bytes_per_token, ch = p.cap_hbm_bytes / p.kv_bytes_per_token;
-    const uint64_t mo = std::max<uint32_t>(tr->min_out_tok, 1);
-    rcap_s[r] = (uint32_t)std::min<uint64_t>(tr->n_sessions, cs / mo) + 1;
-    rcap_h[r] = (uint32_t)std::min<uint64_t>(tr->n_sessions, ch / mo) + 1;
-    const size_t lists = (size_t)kEntryBytes * (rcap_s[r] + rcap_h[r]);
-    const size_t map_b = align_up(2ull * tr->n_sessions, 16);
-    const bool map_ok = rcap_s[r] <= 0x7FFF && rcap_h[r] <= 0x7FFF;
-    if (map_ok && lists + map_b <= smem_limit && map_b <= 32768) {
-      use_map[r] = 1;
-      smem_bytes[r] = (uint32_t)(lists + map_b);
-    } else {
-      use_map[r] = 0;
-      smem_bytes[r] = (uint32_t)lists;
-    }
-    if (smem_bytes[r] <= smem_limit) {
-      in_smem.push_back((uint32_t)r);
-      max_smem = std::max<size_t>(max_smem, smem_bytes[r]);
-    } else {
-      use_map[r] = 0;
-      in_global.push_back((uint32_t)r);
-      off_glist[r] = off;
-      off = align_up(off + lists, 256);
-    }
-    off_ttft[r] = off;
-    off = align_up(off + 8 * (tr->n_turns + 1), 256);
-  }
-  if (off > UNISON_NOALLOC_SCRATCH_BYTES) return UNISON_ERR_RANGE;  // batch too large for the fixed scratch
-
+  rc = noalloc_scratch_address(&scratch);
+  if (rc != UNISON_OK) return rc;
+  ReplayPlan P;
+  size_t off_res = 0;
+  plan_replays(traces, params, n_replays, smem_limit, false, P, off_res);
+  if (P.bytes > UNISON_NOALLOC_SCRATCH_BYTES) return UNISON_ERR_RANGE;  // batch too large for the fixed scratch
   // Every scratch region is written before it is read within one call (the
-  // descriptors by the copies below, the tables and streams by their kernels,
-  // TTFT values and lists by the event loop), so nothing left by an earlier
-  // call is ever read and no region needs clearing.
-  std::vector<ComboDesc> hc(combos.size());
-  for (size_t c = 0; c < combos.size(); c++) {
-    const unison_trace *tr = traces[std::get<0>(combos[c])];
-    ComboDesc &d = hc[c];
-    d.turn_ev = tr->d<uint32_t>(tr->off_turn_ev);
-    d.turn_t = tr->d<uint32_t>(tr->off_turn_t);
-    d.turn_off = tr->d<uint32_t>(tr->off_turn_off);
-    d.tps = tr->d<uint32_t>(tr->off_tps);
-    d.n_sessions = tr->n_sessions;
-    d.n_events = (uint32_t)tr->n_events;
-    d.ema_num = std::get<1>(combos[c]);
-    d.ema_den = std::get<2>(combos[c]);
-    d.bucket = std::get<3>(combos[c]);
-    d.pad = 0;
-    d.penalty_q = std::get<4>(combos[c]);
-    d.sigma = reinterpret_cast<uint16_t *>(scratch + off_lut[c]);
-    d.t2 = reinterpret_cast<uint64_t *>(scratch + off_lut[c] + 128);
-    d.pkey = reinterpret_cast<uint64_t *>(scratch + off_stream[c]);
-    d.gq = reinterpret_cast<uint32_t *>(scratch + off_stream[c] + 8 * tr->n_events);
-  }
-  std::vector<ReplayDesc> hd(n_replays);
-  for (int r = 0; r < n_replays; r++) {
-    const unison_replay_params &p = params[r];
-    const unison_trace *tr = traces[p.trace_idx];
-    ReplayDesc &d = hd[r];
-    d.ev = tr->d<uint4>(tr->off_ev);
-    d.prev_out = tr->d<uint32_t>(tr->off_prev_out);
-    d.nref = tr->d<uint32_t>(tr->off_nref);
-    d.pkey = replay_combo[r] >= 0 ? hc[replay_combo[r]].pkey : nullptr;
-    d.gq = replay_combo[r] >= 0 ? hc[replay_combo[r]].gq : nullptr;
-    d.ttft = reinterpret_cast<uint64_t *>(scratch + off_ttft[r]);
-    d.glist = off_glist[r] ? reinterpret_cast<uint32_t *>(scratch + off_glist[r]) : nullptr;
-    d.log = log_dev ? log_dev + (uint64_t)r * log_capacity_per_replay : nullptr;
-    d.log_cap = log_dev ? log_capacity_per_replay : 0;
-    d.result = results_dev + r;
-    d.cap_s = p.cap_fast_bytes / p.kv_bytes_per_token;
-    d.cap_h = p.cap_hbm_bytes / p.kv_bytes_per_token;
-    d.dma = p.dma_bytes_per_us;
-    d.prefill_ns = p.t_p_ps_per_tok / 1000;
-    d.n_events = (uint32_t)tr->n_events;
-    d.n_turns = (uint32_t)tr->n_turns;
-    d.n_sessions = tr->n_sessions;
-    d.policy = p.policy;
-    d.max_sessions = p.max_sessions;
-    d.kvb = p.kv_bytes_per_token;
-    d.ttl = p.ttl_us;
-    d.load = p.ttft_load;
-    d.rcap_s = rcap_s[r];
-    d.rcap_h = rcap_h[r];
-    d.use_map = use_map[r];
-    d.pad = 0;
-  }
+  // descriptors by the copies in launch_replays, the tables and streams by
+  // their kernels, TTFT values and lists by the event loop), so nothing left
+  // by an earlier call is ever read and no region needs clearing.
+  std::vector<ComboDesc> hc;
+  std::vector<ReplayDesc> hd;
   std::vector<uint32_t> order;
-  order.insert(order.end(), in_smem.begin(), in_smem.end());
-  order.insert(order.end(), in_global.begin(), in_global.end());
-
-  int rc = UNISON_OK;
-  auto ck = [&](cudaError_t e) {
-    if (e != cudaSuccess && rc == UNISON_OK) rc = UNISON_ERR_CUDA;
-  };
-  ReplayDesc *d_desc = reinterpret_cast<ReplayDesc *>(scratch + off_desc);
-  uint32_t *d_order = reinterpret_cast<uint32_t *>(scratch + off_order);
-  ComboDesc *d_combo = reinterpret_cast<ComboDesc *>(scratch + off_combo);
-  ck(cudaMemcpyAsync(d_desc, hd.data(), sizeof(ReplayDesc) * n_replays, cudaMemcpyHostToDevice, stream));
-  ck(cudaMemcpyAsync(d_order, order.data(), sizeof(uint32_t) * order.size(), cudaMemcpyHostToDevice, stream));
-  if (!combos.empty()) {
-    ck(cudaMemcpyAsync(d_combo, hc.data(), sizeof(ComboDesc) * combos.size(), cudaMemcpyHostToDevice, stream));
-    hazard_lut_kernel<<<(unsigned)combos.size(), 256, 0, stream>>>(d_combo);
-    uint32_t max_s = 0;
-    for (auto &c : hc) max_s = std::max(max_s, c.n_sessions);
-    dim3 g((max_s + 127) / 128, (unsigned)combos.size());
-    key_stream_kernel<<<g, 128, 0, stream>>>(d_combo);
-    count_launches(2);
-    ck(cudaGetLastError());
-  }
-  if (!in_smem.empty()) {
-    ck(cudaFuncSetAttribute(replay_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)max_smem));
-    replay_kernel<false><<<(unsigned)in_smem.size(), 32, max_smem, stream>>>(d_desc, d_order);
-    count_launches(1);
-    ck(cudaGetLastError());
-  }
-  if (!in_global.empty()) {
-    replay_kernel<true><<<(unsigned)in_global.size(), 32, 0, stream>>>(d_desc, d_order + in_smem.size());
-    count_launches(1);
-    ck(cudaGetLastError());
-  }
-  ttft_median_kernel<<<(unsigned)n_replays, 256, 0, stream>>>(d_desc, (uint32_t)n_replays);
-  count_launches(1);
-  ck(cudaGetLastError());
+  fill_descs(traces, params, n_replays, P, scratch, results_dev, log_dev, log_capacity_per_replay, hc, hd, order);
+  rc = launch_replays(P, scratch, hc, hd, order, n_replays, stream, false);
   if (results_host) {
-    ck(cudaMemcpyAsync(results_host, results_dev, sizeof(unison_replay_result) * n_replays, cudaMemcpyDeviceToHost,
-                       stream));
-    ck(cudaStreamSynchronize(stream));
+    if (cudaMemcpyAsync(results_host, results_dev, sizeof(unison_replay_result) * n_replays, cudaMemcpyDeviceToHost,
+                        stream) != cudaSuccess &&
+        rc == UNISON_OK)
+      rc = UNISON_ERR_CUDA;
+    if (cudaStreamSynchronize(stream) != cudaSuccess && rc == UNISON_OK) rc = UNISON_ERR_CUDA;
   }
   return rc;
 }

@@ -111,6 +111,7 @@ extern "C" int unison_trace_create(const unison_turns *turns, unison_trace **out
   tr->off_ev = off;        off = align_up(off + 16 * E, 256);
   tr->off_prev_out = off;  off = align_up(off + 4 * E, 256);
   tr->off_nref = off;      off = align_up(off + 4 * E, 256);
+  tr->off_prev_ev = off;   off = align_up(off + 4 * E, 256);
   tr->off_turn_ev = off;   off = align_up(off + 8 * T, 256);
   tr->off_turn_t = off;    off = align_up(off + 8 * T, 256);
   tr->off_turn_off = off;  off = align_up(off + 4 * (S + 1), 256);
@@ -134,6 +135,7 @@ extern "C" int unison_trace_create(const unison_turns *turns, unison_trace **out
   uint4 *hev = tr->h<uint4>(tr->off_ev);
   uint32_t *prev_out = tr->h<uint32_t>(tr->off_prev_out);
   uint32_t *nref = tr->h<uint32_t>(tr->off_nref);
+  uint32_t *prev_ev = tr->h<uint32_t>(tr->off_prev_ev);
   uint32_t *turn_ev = tr->h<uint32_t>(tr->off_turn_ev);
   uint32_t *turn_t = tr->h<uint32_t>(tr->off_turn_t);
   uint32_t *toff = tr->h<uint32_t>(tr->off_turn_off);
@@ -168,9 +170,11 @@ extern "C" int unison_trace_create(const unison_turns *turns, unison_trace **out
   for (uint64_t e = 0; e < E; e++) {
     const HostEvent &x = ev[e];
     nref[e] = kNoRef;
+    prev_ev[e] = kNoRef;
     if (x.arrival) {
       const uint64_t ti = turns->turn_off[x.session] + x.turn;
       if (x.turn + 1 < tps[x.session]) nref[e] = turn_ev[2 * (ti + 1)];
+      if (x.turn > 0) prev_ev[e] = turn_ev[2 * (ti - 1) + 1];
     }
   }
   *out = tr;
