@@ -429,7 +429,6 @@ struct SetConst {
   uint32_t dV, dD;             // completed records pass V / D iff lo >= dV / dD
   int32_t dP;                  // completed records pass P iff lo <= dP
   uint32_t act;                // active lists (bit L)
-  uint32_t never;              // bit 2L: column A of list L passes no gap; bit 2L+1: column B
 };
 
 // ---- TMA 1-D bulk copies and mbarriers (inline PTX, sm_90+) ----
@@ -469,10 +468,26 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity
   return false;
 }
 
-constexpr int kStages = 2;
-constexpr uint32_t kRec = 16;                         // records per consumer thread per tile
-constexpr uint32_t kConsumers = 256;                  // consumer threads (8 warps)
+#ifndef UNISON_FILTER_STAGES
+#define UNISON_FILTER_STAGES 2
+#endif
+#ifndef UNISON_FILTER_REC
+#define UNISON_FILTER_REC 16
+#endif
+#ifndef UNISON_FILTER_CONSUMERS
+#define UNISON_FILTER_CONSUMERS 256
+#endif
+#ifndef UNISON_FILTER_MINBLOCKS
+#define UNISON_FILTER_MINBLOCKS 3
+#endif
+constexpr int kStages = UNISON_FILTER_STAGES;          // tiles in flight per CTA
+constexpr uint32_t kRec = UNISON_FILTER_REC;           // records per consumer thread per tile
+constexpr uint32_t kConsumers = UNISON_FILTER_CONSUMERS;  // consumer threads
 constexpr uint32_t kBigTile = kConsumers * kRec;      // 4096 records per tile
+constexpr uint32_t kGroups = kRec / 4;                 // groups of four records per thread
+constexpr uint32_t kGroupStride = kConsumers * 4;      // records between a thread's groups
+static_assert(kRec % 4 == 0 && kRec <= 32, "records per thread: a multiple of 4, at most 32");
+static_assert(kConsumers >= kLutN * 5, "one consumer thread per bound-table entry");
 constexpr uint32_t kFilterCtaThreads = kConsumers + 32;  // + one producer warp
 struct __align__(128) FilterStage {
   uint32_t gap[kBigTile];
@@ -487,6 +502,16 @@ __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
 }
 // Barrier 1 over the consumer warps only (the producer warp never joins it).
 __device__ __forceinline__ void consumers_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kConsumers) : "memory"); }
+// Barrier 1 with an OR reduction of p over the consumer threads.
+__device__ __forceinline__ bool consumers_sync_or(bool p) {
+  uint32_t r;
+  asm volatile(
+      "{\n .reg .pred pi, po;\n setp.ne.u32 pi, %1, 0;\n bar.red.or.pred po, 1, %2, pi;\n selp.u32 %0, 1, 0, po;\n}"
+      : "=r"(r)
+      : "r"((uint32_t)p), "n"(kConsumers)
+      : "memory");
+  return r != 0;
+}
 // A tile is copied by TMA when it is whole (the arrays' 16-byte alignment is
 // checked by the host); the last, partial tile of a set is read directly.
 __device__ __forceinline__ bool tile_is_bulk(const RankSet &S, uint32_t tile) {
@@ -501,26 +526,16 @@ __device__ __forceinline__ int set_of(const RankSet *sets, int si, uint32_t tile
 // Thresholds of one set into shared memory (consumer threads call it).  Per
 // turn index: vd = (gA_V, gB_V, gA_D, gB_D), pp = (gA_P, gB_P); an inactive
 // list gets bounds no gap passes.
-__device__ void load_set(const RankSet &S, uint4 *vd, uint2 *pp, uint64_t *t2s, uint64_t *mgs, SetConst &c,
-                         unsigned int *never_sh) {
-  consumers_sync();
-  if (threadIdx.x == 0) *never_sh = 0x3Fu;
-  consumers_sync();
+__device__ void load_set(const RankSet &S, uint4 *vd, uint2 *pp, uint64_t *t2s, uint64_t *mgs, SetConst &c) {
+  consumers_sync();  // everyone is done with the previous set's tables
   const bool aV = S.thr[kLists + 0] != 0, aD = S.thr[kLists + 1] != 0, aP = S.thr[kLists + 2] != 0;
   if (threadIdx.x < kLutN) {
     const uint32_t t = threadIdx.x;
     const uint2 a0 = S.gthr[t], a1 = S.gthr[kLutN + t], a2 = S.gthr[2 * kLutN + t];
-    const uint4 v = make_uint4(aV ? a0.x : kFull, aV ? a0.y : kFull, aD ? a1.x : kFull, aD ? a1.y : kFull);
-    const uint2 w = aP ? a2 : make_uint2(0u, 0u);
-    vd[t] = v;
-    pp[t] = w;
+    vd[t] = make_uint4(aV ? a0.x : kFull, aV ? a0.y : kFull, aD ? a1.x : kFull, aD ? a1.y : kFull);
+    pp[t] = aP ? a2 : make_uint2(0u, 0u);
     t2s[t] = S.t2[t];
     mgs[t] = S.magic[t];
-    // gaps are below 2^31: a V/D bound of 2^31 or more, or a P bound of 0, passes nothing
-    const uint32_t nv = (v.x >= 0x80000000u ? 1u : 0u) | (v.y >= 0x80000000u ? 2u : 0u) |
-                        (v.z >= 0x80000000u ? 4u : 0u) | (v.w >= 0x80000000u ? 8u : 0u) |
-                        (w.x == 0u ? 16u : 0u) | (w.y == 0u ? 32u : 0u);
-    atomicAnd(never_sh, nv);
   }
   uint32_t lo[kLists], dok[kLists];
 #pragma unroll
@@ -541,30 +556,15 @@ __device__ void load_set(const RankSet &S, uint4 *vd, uint2 *pp, uint64_t *t2s, 
   c.dP = (aP && dok[2] == 1) ? (int32_t)lo[2] : -1;
   c.act = (aV ? 1u : 0u) | (aD ? 2u : 0u) | (aP ? 4u : 0u);
   consumers_sync();
-  c.never = *never_sh;
 }
 
-__device__ __forceinline__ void flush_elig(const RankSet &P, uint32_t &eD, uint32_t &eP, int lane) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) {
-    eD += __shfl_xor_sync(kFull, eD, o);
-    eP += __shfl_xor_sync(kFull, eP, o);
-  }
-  if (lane == 0) {
-    atomicAdd(&P.work->elig[0], (unsigned long long)(eD + eP));
-    atomicAdd(&P.work->elig[1], (unsigned long long)eD);
-    atomicAdd(&P.work->elig[2], (unsigned long long)eP);
-  }
-  eD = eP = 0;
-}
-
-// Persistent streaming pass.  Each CTA owns a contiguous range of tiles; its
+// Persistent streaming pass.  Each CTA takes every gridDim-th tile; its
 // producer warp keeps kStages tiles in flight with TMA bulk copies into
-// shared memory ("full" barriers), and its eight consumer warps test every
-// record of each tile against the set's thresholds, then hand the stage back
-// ("empty" barriers).  Every wait is bounded; a CTA that gives up records
+// shared memory ("full" barriers), and its consumer warps copy each tile to
+// registers, hand the stage back ("empty" barriers) and test every record
+// against the set's thresholds.  Every wait is bounded; a CTA that gives up records
 // UNISON_ERR_TIMEOUT, lets its own copies land (bounded) and returns.
-__global__ void __launch_bounds__(kFilterCtaThreads, 3) rank_filter_kernel(const RankSet *sets, int n_sets,
+__global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) rank_filter_kernel(const RankSet *sets, int n_sets,
                                                                         uint32_t total_tiles) {
   extern __shared__ __align__(128) unsigned char fsm[];
   FilterStage *stage = reinterpret_cast<FilterStage *>(fsm);
@@ -572,9 +572,12 @@ __global__ void __launch_bounds__(kFilterCtaThreads, 3) rank_filter_kernel(const
   __shared__ uint4 vd[kLutN];
   __shared__ uint2 pp[kLutN];
   __shared__ uint64_t t2s[kLutN], mgs[kLutN];
-  __shared__ unsigned int never_sh;
-  const uint32_t t_begin = (uint32_t)(((uint64_t)blockIdx.x * total_tiles) / gridDim.x);
-  const uint32_t t_end = (uint32_t)(((uint64_t)(blockIdx.x + 1) * total_tiles) / gridDim.x);
+  __shared__ uint2 ftab[kLutN * 5];
+  // Tiles are dealt round-robin: CTA b takes tiles b, b + grid, ...  Records
+  // that pass a threshold cluster by index (ties on a key go to the smaller
+  // index, so a threshold on a tied key admits an index prefix); dealing the
+  // tiles spreads that work over all CTAs.
+  const uint32_t t_begin = blockIdx.x, t_step = gridDim.x, t_end = total_tiles;
   if (t_begin >= t_end) return;
   if (threadIdx.x == 0) {
     for (int q = 0; q < kStages; q++) {
@@ -594,7 +597,7 @@ __global__ void __launch_bounds__(kFilterCtaThreads, 3) rank_filter_kernel(const
     uint32_t fills[kStages] = {};  // bulk copies issued into each stage (one full-barrier phase each)
     uint32_t issued = 0;           // bit q: the last copy into stage q may still be in flight
     bool failed = false;
-    for (uint32_t i = 0, tile = t_begin; tile < t_end; i++, tile++) {
+    for (uint32_t i = 0, tile = t_begin; tile < t_end; i++, tile += t_step) {
       const int q = (int)(i % kStages);
       if (i >= (uint32_t)kStages) {
         // wait until the consumers released this stage's previous tile
@@ -629,32 +632,89 @@ __global__ void __launch_bounds__(kFilterCtaThreads, 3) rank_filter_kernel(const
   }
 
   // ---------------- consumer warps
+  // Consumer thread ct owns, in each tile, kGroups groups of four consecutive
+  // records, group gi starting at record gi * kGroupStride + 4 * ct: every
+  // shared-memory read of the stage is lane-contiguous (no bank conflicts).
+  const uint32_t ct = threadIdx.x;
   int si = si0, lsi = -1;
   SetConst c;
-  uint32_t eD = 0, eP = 0;
   uint32_t fph = 0;  // bit q: parity of the next full-barrier phase of stage q (flips per bulk tile)
   // this set's hot descriptor fields, cached when the set changes (pointers
   // used only on rare paths are read from the descriptor there)
   uint32_t s_n = 0, s_tile0 = 0, s_end = 0;
   bool s_keys = false;
-  for (uint32_t i = 0, tile = t_begin; tile < t_end; i++, tile++) {
+  // Segment: a run of tiles over which every index condition of the set has
+  // one class (all, none or mixed).  Within a set each condition changes class
+  // at most twice (at the tile holding its boundary and the one after), so a
+  // set has at most 13 segments.
+  uint32_t seg_end = 0;  // first tile of the next segment
+  bool seg_mixed = false, seg_none = false;
+  for (uint32_t i = 0, tile = t_begin; tile < t_end; i++, tile += t_step) {
     const int q = (int)(i % kStages);
     if (lsi < 0 || tile >= s_end) {
       si = set_of(sets, si, tile);
       const RankSet &S = sets[si];
-      if (lsi >= 0) flush_elig(sets[lsi], eD, eP, lane);
-      load_set(S, vd, pp, t2s, mgs, c, &never_sh);
+      load_set(S, vd, pp, t2s, mgs, c);
       lsi = si;
       s_n = S.n;
       s_tile0 = S.tile0;
       s_end = S.tile0 + S.ntiles;
       s_keys = S.keys != nullptr;
+      seg_end = tile;  // force a new segment
     }
     const uint32_t tb = (tile - s_tile0) * kBigTile;
+    if (tile >= seg_end) {
+      // Index conditions over this tile: record indices rise through the
+      // tile, so lo = ~index falls from lo_hi to lo_lo and each tie condition
+      // on lo holds for all, none or a part of the tile.
+      const uint32_t tcount = min(kBigTile, s_n - tb);
+      const uint32_t lo_hi = (~tb) & kIdMask, lo_lo = (~(tb + tcount - 1)) & kIdMask;
+      // 0 none, 1 all, 2 mixed
+      auto ge_class = [&](uint32_t x) { return lo_lo >= x ? 1u : (lo_hi < x ? 0u : 2u); };                   // lo >= x
+      auto le_class = [&](int64_t x) { return (int64_t)lo_hi <= x ? 1u : ((int64_t)lo_lo > x ? 0u : 2u); };  // lo <= x
+      const uint32_t iV = ge_class(c.loV), iD = ge_class(c.loD), iP = le_class((int64_t)c.loP);
+      const uint32_t dV = ge_class(c.dV), dD = ge_class(c.dD), dP = le_class((int64_t)c.dP);
+      seg_mixed = ((c.act & 1) && (iV == 2 || dV == 2)) || ((c.act & 2) && (iD == 2 || dD == 2)) ||
+                  ((c.act & 4) && (iP == 2 || dP == 2));
+      // next tile where a condition can change class: lo >= x holds for
+      // indices up to kIdMask - x, lo <= x from kIdMask - x on; the change
+      // points are the tile holding that index and the tile after it
+      const uint32_t r = tile - s_tile0;
+      uint32_t nxt = s_end - s_tile0;
+      auto upd = [&](int64_t lo_bound) {
+        const int64_t b = (int64_t)kIdMask - lo_bound;
+        if (b < 0 || b >= (int64_t)s_n) return;
+        const uint32_t tbnd = (uint32_t)b / kBigTile;
+        if (tbnd > r) nxt = min(nxt, tbnd);
+        else if (tbnd + 1 > r) nxt = min(nxt, tbnd + 1);
+      };
+      upd(c.loV); upd(c.loD); upd(c.loP); upd(c.dV); upd(c.dD); upd(c.dP);
+      seg_end = s_tile0 + nxt;
+      // Per-segment bound table over (turn index, record class): a record of
+      // class cls at turn index t may be a candidate of some list iff
+      // g >= x or g < y.  Classes: 0 not eligible, 1 live fast tier, 2 live
+      // HBM tier, 3 completed fast tier, 4 completed HBM tier.
+      consumers_sync();  // everyone is done with the previous table
+      bool live = false;
+      if (!seg_mixed && ct < kLutN * 5) {
+        const uint32_t t = ct / 5, cls = ct % 5;
+        const uint4 a = vd[t];
+        const uint2 bb = pp[t];
+        const uint32_t bV = iV == 1 ? a.x : a.y, bD = iD == 1 ? a.z : a.w, bP = iP == 1 ? bb.y : bb.x;
+        const bool pdV = (c.act & 1) && dV == 1, pdD = (c.act & 2) && dD == 1, pdP = (c.act & 4) && dP == 1;
+        uint2 e = make_uint2(kFull, 0u);
+        if (cls == 1) e = make_uint2(min(bV, bD), 0u);
+        if (cls == 2) e = make_uint2(bV, bP);
+        if (cls == 3) e = make_uint2(pdV || pdD ? 0u : kFull, 0u);
+        if (cls == 4) e = make_uint2(pdV ? 0u : kFull, pdP ? kFull : 0u);
+        ftab[ct] = e;
+        // gaps are below 2^31: x >= 2^31 and y == 0 admit nothing
+        live = e.x < 0x80000000u || e.y != 0u;
+      }
+      seg_none = !consumers_sync_or(live) && !seg_mixed;
+    }
     const bool bulk = tb + kBigTile <= s_n;
-    const uint32_t r0 = threadIdx.x * kRec;
-    uint32_t g[kRec], tw[kRec / 2], fw[kRec / 4], rw[kRec / 4];
-    uint32_t cnt = kRec;
+    uint32_t g[kRec], tw[kRec / 2], fw[kGroups], rw[kGroups];
     if (bulk) {
       // a timed-out wait is reported, not collective: every wait here is
       // bounded, so the CTA still ends (with undefined results)
@@ -663,19 +723,15 @@ __global__ void __launch_bounds__(kFilterCtaThreads, 3) rank_filter_kernel(const
       fph ^= 1u << q;
       const FilterStage &d = stage[q];
 #pragma unroll
-      for (int v = 0; v < (int)(kRec / 4); v++) {
-        const uint4 gq = *reinterpret_cast<const uint4 *>(d.gap + r0 + 4 * v);
-        g[4 * v] = gq.x; g[4 * v + 1] = gq.y; g[4 * v + 2] = gq.z; g[4 * v + 3] = gq.w;
+      for (int gi = 0; gi < (int)kGroups; gi++) {
+        const uint32_t o = gi * kGroupStride + 4 * ct;
+        const uint4 gq = *reinterpret_cast<const uint4 *>(d.gap + o);
+        g[4 * gi] = gq.x; g[4 * gi + 1] = gq.y; g[4 * gi + 2] = gq.z; g[4 * gi + 3] = gq.w;
+        const uint2 tq = *reinterpret_cast<const uint2 *>(d.turn + o);
+        tw[2 * gi] = tq.x; tw[2 * gi + 1] = tq.y;
+        fw[gi] = *reinterpret_cast<const uint32_t *>(d.flags + o);
+        rw[gi] = *reinterpret_cast<const uint32_t *>(d.tier + o);
       }
-#pragma unroll
-      for (int v = 0; v < (int)(kRec / 8); v++) {
-        const uint4 tq = *reinterpret_cast<const uint4 *>(d.turn + r0 + 8 * v);
-        tw[4 * v] = tq.x; tw[4 * v + 1] = tq.y; tw[4 * v + 2] = tq.z; tw[4 * v + 3] = tq.w;
-      }
-      const uint4 fq = *reinterpret_cast<const uint4 *>(d.flags + r0);
-      const uint4 rq = *reinterpret_cast<const uint4 *>(d.tier + r0);
-      fw[0] = fq.x; fw[1] = fq.y; fw[2] = fq.z; fw[3] = fq.w;
-      rw[0] = rq.x; rw[1] = rq.y; rw[2] = rq.z; rw[3] = rq.w;
       // the stage's data is in registers: hand it back to the producer
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty[q]);
@@ -684,138 +740,102 @@ __global__ void __launch_bounds__(kFilterCtaThreads, 3) rank_filter_kernel(const
       const uint32_t *s_gap = S.gap;
       const uint16_t *s_turn = S.turn;
       const uint8_t *s_flags = S.flags, *s_tier = S.tier;
-      const uint32_t base = tb + r0;
-      cnt = base < s_n ? min(s_n - base, kRec) : 0;
 #pragma unroll
-      for (int v = 0; v < (int)(kRec / 2); v++) tw[v] = 0;
+      for (int gi = 0; gi < (int)kGroups; gi++) {
+        tw[2 * gi] = tw[2 * gi + 1] = 0;
+        fw[gi] = 0x01010101u;  // padding reads as pinned: never eligible
+        rw[gi] = 0;
 #pragma unroll
-      for (int v = 0; v < (int)(kRec / 4); v++) {
-        fw[v] = 0x01010101u;  // padding reads as pinned: never eligible
-        rw[v] = 0;
-      }
-#pragma unroll
-      for (uint32_t k = 0; k < kRec; k++) {
-        g[k] = 0;
-        if (k < cnt) {
-          g[k] = s_gap[base + k];
-          tw[k >> 1] |= (uint32_t)s_turn[base + k] << (16 * (k & 1));
-          const uint32_t sh = 8 * (k & 3);
-          fw[k >> 2] = (fw[k >> 2] & ~(0xFFu << sh)) | ((uint32_t)s_flags[base + k] << sh);
-          rw[k >> 2] = (rw[k >> 2] & ~(0xFFu << sh)) | ((uint32_t)s_tier[base + k] << sh);
+        for (uint32_t m = 0; m < 4; m++) {
+          const uint32_t idx = tb + gi * kGroupStride + 4 * ct + m;
+          g[4 * gi + m] = 0;
+          if (idx < s_n) {
+            g[4 * gi + m] = s_gap[idx];
+            tw[2 * gi + (m >> 1)] |= (uint32_t)s_turn[idx] << (16 * (m & 1));
+            const uint32_t sh = 8 * m;
+            fw[gi] = (fw[gi] & ~(0xFFu << sh)) | ((uint32_t)s_flags[idx] << sh);
+            rw[gi] = (rw[gi] & ~(0xFFu << sh)) | ((uint32_t)s_tier[idx] << sh);
+          }
         }
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty[q]);
     }
-    const uint32_t base = tb + r0;
-    // Per-record masks, four records per 32-bit word (SWAR): eligible for V
-    // (unpinned resident), D (unpinned fast tier), P (unpinned HBM tier), and
-    // completed.  movemask turns 0x00/0xFF bytes into one bit per record.
-    uint32_t mEV = 0, mED = 0, mEP = 0, mDone = 0;
+    auto turn_of = [&](uint32_t k) { return min((tw[k >> 1] >> (16 * (k & 1))) & 0xFFFF, kTMax); };
+    auto index_of = [&](uint32_t k) { return tb + (k >> 2) * kGroupStride + 4 * ct + (k & 3); };
+    // 1. candidate bit per record (any list): one table lookup per record
+    uint32_t cm = 0;
+    if (seg_mixed) {
+      cm = (1u << kRec) - 1;  // index conditions vary inside the tile: test every record exactly
+    } else if (!seg_none) {
+      const unsigned char *tab = reinterpret_cast<const unsigned char *>(ftab);
 #pragma unroll
-    for (int w = 0; w < (int)(kRec / 4); w++) {
-      const uint32_t unp = __vcmpeq4(fw[w] & 0x01010101u, 0u);
-      const uint32_t isS = __vcmpeq4(rw[w], 0x01010101u), isH = __vcmpeq4(rw[w], 0x02020202u);
-      const uint32_t dn = __vcmpne4(fw[w] & 0x02020202u, 0u);
-      auto movemask = [](uint32_t x) { return ((x & 0x01010101u) * 0x01020408u) >> 24; };
-      const uint32_t eDw = unp & isS, ePw = unp & isH;
-      eD += __popc(eDw) >> 3;
-      eP += __popc(ePw) >> 3;
-      mED |= movemask(eDw) << (4 * w);
-      mEP |= movemask(ePw) << (4 * w);
-      mEV |= movemask(eDw | ePw) << (4 * w);
-      mDone |= movemask(dn) << (4 * w);
+      for (int gi = 0; gi < (int)kGroups; gi++) {
+        // class * 8 per record, four records per word (SWAR)
+        const uint32_t unp = __vcmpeq4(fw[gi] & 0x01010101u, 0u);
+        const uint32_t isS = __vcmpeq4(rw[gi], 0x01010101u), isH = __vcmpeq4(rw[gi], 0x02020202u);
+        const uint32_t dn = __vcmpne4(fw[gi] & 0x02020202u, 0u);
+        const uint32_t c8 = (unp & ((isS & 0x08080808u) | (isH & 0x10101010u))) +
+                            (unp & dn & (isS | isH) & 0x10101010u);
+#pragma unroll
+        for (uint32_t m = 0; m < 4; m++) {
+          const uint32_t k = 4 * gi + m;
+          const uint2 e = *reinterpret_cast<const uint2 *>(tab + turn_of(k) * 40 + ((c8 >> (8 * m)) & 0xFF));
+          cm |= (uint32_t)(g[k] >= e.x || g[k] < e.y) << k;
+        }
+      }
     }
-    // Index conditions over this tile: record indices rise through the tile,
-    // so lo = ~index falls from lo_hi to lo_lo and each tie condition on lo
-    // holds for all, none or a prefix of the tile.
-    const uint32_t tcount = min(kBigTile, s_n - tb);
-    const uint32_t lo_hi = (~tb) & kIdMask, lo_lo = (~(tb + tcount - 1)) & kIdMask;
-    // 0 none, 1 all, 2 mixed
-    auto ge_class = [&](uint32_t x) { return lo_lo >= x ? 1u : (lo_hi < x ? 0u : 2u); };                   // lo >= x
-    auto le_class = [&](int64_t x) { return (int64_t)lo_hi <= x ? 1u : ((int64_t)lo_lo > x ? 0u : 2u); };  // lo <= x
-    const uint32_t iV = ge_class(c.loV), iD = ge_class(c.loD), iP = le_class((int64_t)c.loP);
-    const uint32_t dV = ge_class(c.dV), dD = ge_class(c.dD), dP = le_class((int64_t)c.dP);
-    const bool mixed = ((c.act & 1) && (iV == 2 || dV == 2)) || ((c.act & 2) && (iD == 2 || dD == 2)) ||
-                       ((c.act & 4) && (iP == 2 || dP == 2));
-    uint32_t mV = 0, mD = 0, mP = 0;  // candidate bit per record, per list
-    if (!mixed) {
-      // column per list: V/D pass at g >= gA when the index part holds, else g >= gB;
-      // P passes at g < gB when it holds, else g < gA
-      const bool colV = iV == 1, colD = iD == 1, colP = iP == 1;
-      const bool nvV = !(c.act & 1) || ((c.never >> (colV ? 0 : 1)) & 1);
-      const bool nvD = !(c.act & 2) || ((c.never >> (colD ? 2 : 3)) & 1);
-      const bool nvP = !(c.act & 4) || ((c.never >> (colP ? 5 : 4)) & 1);
-      // completed records: one uniform answer per list for the whole tile
-      if ((c.act & 1) && dV == 1) mV = mDone;
-      if ((c.act & 2) && dD == 1) mD = mDone;
-      if ((c.act & 4) && dP == 1) mP = mDone;
-      if (!(nvV && nvD && nvP)) {
-        uint32_t nV = 0, nD = 0, nP = 0;  // live records' tests
+    // 2. exact per-list tests of the flagged records (rare outside mixed tiles)
+    if (__any_sync(kFull, cm != 0)) {
+      uint32_t mV = 0, mD = 0, mP = 0;  // candidate bit per record, per list
+      if (cm) {
 #pragma unroll
         for (uint32_t k = 0; k < kRec; k++) {
-          const uint32_t t = min((tw[k >> 1] >> (16 * (k & 1))) & 0xFFFF, kTMax);
-          const uint32_t gg = g[k];
-          if (!(nvV && nvD)) {
-            const uint4 a = vd[t];
-            nV |= (uint32_t)(!nvV && gg >= (colV ? a.x : a.y)) << k;
-            nD |= (uint32_t)(!nvD && gg >= (colD ? a.z : a.w)) << k;
-          }
-          if (!nvP) {
-            const uint2 b = pp[t];
-            nP |= (uint32_t)(gg < (colP ? b.y : b.x)) << k;
-          }
+          if (!((cm >> k) & 1)) continue;
+          const uint32_t fl = (fw[k >> 2] >> (8 * (k & 3))) & 0xFF, tr = (rw[k >> 2] >> (8 * (k & 3))) & 0xFF;
+          const uint32_t em = elig_mask((uint8_t)fl, (uint8_t)tr);
+          const bool done = (fl & 2) != 0;
+          const uint32_t t = turn_of(k), gg = g[k];
+          const uint32_t lo = (~index_of(k)) & kIdMask;
+          const uint4 a = vd[t];
+          const uint2 b = pp[t];
+          const bool pV = done ? lo >= c.dV : (gg >= a.y || (gg >= a.x && lo >= c.loV));
+          const bool pD = done ? lo >= c.dD : (gg >= a.w || (gg >= a.z && lo >= c.loD));
+          const bool pP = done ? (int32_t)lo <= c.dP : (gg < b.x || (gg < b.y && lo <= c.loP));
+          mV |= (uint32_t)(pV && (em & 1)) << k;
+          mD |= (uint32_t)(pD && (em & 2)) << k;
+          mP |= (uint32_t)(pP && (em & 4)) << k;
         }
-        mV |= nV & ~mDone;
-        mD |= nD & ~mDone;
-        mP |= nP & ~mDone;
       }
-    } else {
+      // emit candidates' exact values (warp-aggregated appends)
 #pragma unroll
-      for (uint32_t k = 0; k < kRec; k++) {
-        const bool done = (mDone >> k) & 1;
-        const uint32_t t = min((tw[k >> 1] >> (16 * (k & 1))) & 0xFFFF, kTMax);
-        const uint32_t gg = g[k];
-        const uint32_t lo = (~(base + k)) & kIdMask;
-        const uint4 a = vd[t];
-        const uint2 b = pp[t];
-        const bool pV = done ? lo >= c.dV : (gg >= a.y || (gg >= a.x && lo >= c.loV));
-        const bool pD = done ? lo >= c.dD : (gg >= a.w || (gg >= a.z && lo >= c.loD));
-        const bool pP = done ? (int32_t)lo <= c.dP : (gg < b.x || (gg < b.y && lo <= c.loP));
-        mV |= (uint32_t)pV << k;
-        mD |= (uint32_t)pD << k;
-        mP |= (uint32_t)pP << k;
-      }
-    }
-    mV &= mEV;
-    mD &= mED;
-    mP &= mEP;
-    // emit candidates' exact values (warp-aggregated appends)
+      for (int L = 0; L < kLists; L++) {
+        const uint32_t mm = L == 0 ? mV : (L == 1 ? mD : mP);
+        const uint32_t mine = __popc(mm);
+        if (!__any_sync(kFull, mine != 0)) continue;
+        uint32_t incl = mine;
 #pragma unroll
-    for (int L = 0; L < kLists; L++) {
-      const uint32_t mm = L == 0 ? mV : (L == 1 ? mD : mP);
-      const uint32_t mine = __popc(mm);
-      if (!__any_sync(kFull, mine != 0)) continue;
-      uint32_t incl = mine;
+        for (int o = 1; o < 32; o <<= 1) {
+          const uint32_t y = __shfl_up_sync(kFull, incl, o);
+          if (lane >= o) incl += y;
+        }
+        const uint32_t total = __shfl_sync(kFull, incl, 31);
+        uint32_t basepos = 0;
+        if (lane == 31) basepos = atomicAdd(&sets[si].work->cand[L], total);
+        basepos = __shfl_sync(kFull, basepos, 31);
+        uint32_t pos = basepos + incl - mine;
+        if (mm) {
+          uint64_t *dst = sets[si].cand + (size_t)L * kCandCap;
 #pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint32_t y = __shfl_up_sync(kFull, incl, o);
-        if (lane >= o) incl += y;
-      }
-      const uint32_t total = __shfl_sync(kFull, incl, 31);
-      uint32_t basepos = 0;
-      if (lane == 31) basepos = atomicAdd(&sets[si].work->cand[L], total);
-      basepos = __shfl_sync(kFull, basepos, 31);
-      uint32_t pos = basepos + incl - mine;
-#pragma unroll
-      for (uint32_t k = 0; k < kRec; k++) {
-        if ((mm >> k) & 1) {
-          if (pos < kCandCap) {
-            const uint32_t t = min((tw[k >> 1] >> (16 * (k & 1))) & 0xFFFF, kTMax);
-            const uint64_t ck = ck_of(score_of(g[k], t, (mDone >> k) & 1, t2s, mgs), base + k);
-            sets[si].cand[(size_t)L * kCandCap + pos] = list_val(ck, L);
+          for (uint32_t k = 0; k < kRec; k++) {
+            if ((mm >> k) & 1) {
+              if (pos < kCandCap) {
+                const bool dn = (fw[k >> 2] >> (8 * (k & 3) + 1)) & 1;
+                dst[pos] = list_val(ck_of(score_of(g[k], turn_of(k), dn, t2s, mgs), index_of(k)), L);
+              }
+              pos++;
+            }
           }
-          pos++;
         }
       }
     }
@@ -823,13 +843,14 @@ __global__ void __launch_bounds__(kFilterCtaThreads, 3) rank_filter_kernel(const
       uint64_t *keys = sets[si].keys;
 #pragma unroll
       for (uint32_t k = 0; k < kRec; k++) {
-        if (k >= cnt) break;
-        const uint32_t t = min((tw[k >> 1] >> (16 * (k & 1))) & 0xFFFF, kTMax);
-        keys[base + k] = score_of(g[k], t, (mDone >> k) & 1, t2s, mgs);
+        const uint32_t idx = index_of(k);
+        if (idx < s_n) {
+          const bool dn = (fw[k >> 2] >> (8 * (k & 3) + 1)) & 1;
+          keys[idx] = score_of(g[k], turn_of(k), dn, t2s, mgs);
+        }
       }
     }
   }
-  if (lsi >= 0) flush_elig(sets[lsi], eD, eP, lane);
 }
 
 // ------------------------------------------------------------- finish ----
@@ -902,13 +923,18 @@ __global__ void __launch_bounds__(kFinishThreads) rank_finish_kernel(const RankS
   for (int L = 0; L < kLists; L++) {
     const bool active = S.thr[kLists + L] != 0;
     const uint32_t Mw = (L == 0) ? S.k : S.max_moves;
-    const unsigned long long e = S.work->elig[L];
-    const uint32_t M = active ? (uint32_t)min((unsigned long long)Mw, e) : 0u;
     const uint32_t emitted = S.work->cand[L];
+    // Candidates are every eligible record at or beyond the threshold.  They
+    // certify the top Mw when there are at least Mw of them, or when the
+    // threshold admitted every eligible record; otherwise (or when the buffer
+    // overflowed) the list is re-selected exactly from the whole set.
+    const bool all_admitted = S.thr[L] == 0;
+    const bool certified = emitted <= kCandCap && (emitted >= Mw || all_admitted);
+    const uint32_t M = !active ? 0u : (certified ? min(Mw, emitted) : Mw);
     uint32_t got = 0;
     if (M > 0) {
       const uint64_t *cand = S.cand + (size_t)L * kCandCap;
-      if (emitted <= kCandCap && emitted >= M) {
+      if (certified) {
         const uint32_t c = emitted;
         const uint64_t *src = cand;
         if (c <= kSmemCand) {
