@@ -9,19 +9,20 @@
 //   D  fast-tier demotion candidates: unpinned fast-tier records, largest first;
 //   P  HBM promotion candidates: unpinned HBM records, smallest ck first.
 // Kernels, in launch order:
-//   rank_sample_kernel   16 CTAs per set: exact order statistics of a
-//                        jittered stratified sample give each list a threshold, turned
+//   rank_sample_kernel   16 CTAs per set: order statistics of a jittered
+//                        stratified sample give each list a threshold, turned
 //                        into per-turn thresholds on the gap average (the
 //                        score is monotone in the gap for a fixed turn, so
 //                        the streaming test needs no division).
 //   rank_filter_kernel   one pass over every record (8 B each: gap average,
 //                        turn, flags, tier), emitting the exact values of the
 //                        records that pass a threshold.
-//   rank_finish_kernel   one CTA per set: exact top-M of the candidates by
-//                        radix select, bitonic sort, the victims, and the
-//                        fill as warp prefix scans.  If a list's candidates
-//                        overflowed or fell short, the CTA re-selects that
-//                        list exactly by streaming the whole set.
+//   rank_finish_kernel   one CTA per (list, set): exact top-M of the list's
+//                        candidates by radix select and a bitonic sort; if
+//                        the candidates overflowed or fell short, the CTA
+//                        re-selects the list exactly by streaming the whole
+//                        set.  The set's last CTA writes the victims and runs
+//                        the fill as warp prefix scans.
 #include <algorithm>
 #include <type_traits>
 #include <vector>
@@ -42,11 +43,11 @@ constexpr uint32_t kFinishThreads = 1024;
 constexpr uint32_t kFull = 0xFFFFFFFFu;
 
 struct RankWork {
-  unsigned int cand[kLists];
-  unsigned int status;  // UNISON_ERR_TIMEOUT if a bounded wait gave up
-  unsigned long long elig[kLists];
-  unsigned int ticket;  // sample CTAs finished
-  unsigned int pad2;
+  unsigned int cand[kLists];  // candidates emitted per list
+  unsigned int status;        // UNISON_ERR_TIMEOUT if a bounded wait gave up
+  unsigned int got[kLists];   // selected entries per list (finish)
+  unsigned int ticket;        // finish CTAs done with their list
+  unsigned int sticket;       // sample CTAs done
 };
 
 constexpr uint32_t kSampleCtas = 16;     // sample CTAs per set
@@ -74,7 +75,8 @@ struct RankSet {
   uint64_t *thr;     // [3] threshold in list-value space; [3+L] = active flag
   uint64_t *t2;      // [51]
   uint64_t *magic;   // [51]
-  uint64_t *part;    // [3][kSampleCtas][kMaxR] per-CTA top values of the sample
+  uint32_t *part;    // [3][kSampleCtas][kMaxR] per-CTA top summaries of the sample
+  uint32_t *part_n;  // [3][kSampleCtas] entries in each
 };
 
 // ---------------------------------------------------------------- keys ----
@@ -214,14 +216,38 @@ __device__ uint64_t block_select_rank(Get get, uint32_t n, uint32_t rank, unsign
   return prefix;
 }
 
-// Bitonic sort, descending, of a[0..n) padded with zeros to a power of two.
+// Bitonic sort, descending, of a[0..n) padded with zeros to a power of two
+// (at least 32).  Element i sits in lane i % 32 of its warp, so every
+// compare-exchange at distance below 32 runs in registers with shuffles; only
+// distances of 32 and more go through shared memory, one barrier each.
 __device__ void block_sort_desc(uint64_t *a, uint32_t n) {
-  uint32_t p = 1;
+  if (n <= 1) return;
+  uint32_t p = 32;
   while (p < n) p <<= 1;
   for (uint32_t i = n + threadIdx.x; i < p; i += blockDim.x) a[i] = 0;
   __syncthreads();
-  for (uint32_t k = 2; k <= p; k <<= 1) {
-    for (uint32_t j = k >> 1; j > 0; j >>= 1) {
+  // stages k = kmin..kmax, distances below 32, in registers
+  auto reg_steps = [&](uint32_t kmin, uint32_t kmax) {
+    for (uint32_t base = 0; base < p; base += blockDim.x) {
+      const uint32_t i = base + threadIdx.x;
+      if (i < p) {  // p and blockDim are multiples of 32: whole warps
+        uint64_t x = a[i];
+        for (uint32_t k = kmin; k <= kmax; k <<= 1) {
+          const bool desc = (i & k) == 0;
+          for (uint32_t j = min(k >> 1, 16u); j > 0; j >>= 1) {
+            const uint64_t y = __shfl_xor_sync(0xFFFFFFFFu, x, j);
+            const bool lower = (i & j) == 0;
+            x = (lower == desc) ? (x > y ? x : y) : (x < y ? x : y);
+          }
+        }
+        a[i] = x;
+      }
+    }
+    __syncthreads();
+  };
+  reg_steps(2, 32);
+  for (uint32_t k = 64; k <= p; k <<= 1) {
+    for (uint32_t j = k >> 1; j >= 32; j >>= 1) {
       for (uint32_t i = threadIdx.x; i < p; i += blockDim.x) {
         const uint32_t ij = i ^ j;
         if (ij > i) {
@@ -235,6 +261,7 @@ __device__ void block_sort_desc(uint64_t *a, uint32_t n) {
       }
       __syncthreads();
     }
+    reg_steps(k, k);
   }
 }
 
@@ -266,58 +293,143 @@ __device__ __forceinline__ uint32_t sample_size(const RankSet &S) {
   return (uint32_t)ns;
 }
 
-// The value of rank r (1 = largest) among the block's values v (one per
-// thread; `has` false for threads without one), built MSB first: a bit is
-// kept when at least r values reach the prefix with that bit set.  Bits on
-// which all values agree are taken directly.  All threads get the result.
-__device__ uint64_t block_rank_bitwise(uint64_t v, bool has, uint32_t r, unsigned long long *sh) {
-  if (threadIdx.x == 0) {
-    sh[0] = ~0ull;
-    sh[1] = 0ull;
-  }
-  __syncthreads();
-  unsigned long long a = has ? v : ~0ull, o = has ? v : 0ull;
-  for (int s = 16; s; s >>= 1) {
-    a &= __shfl_xor_sync(0xFFFFFFFFu, a, s);
-    o |= __shfl_xor_sync(0xFFFFFFFFu, o, s);
-  }
-  if ((threadIdx.x & 31) == 0) {
-    atomicAnd(&sh[0], a);
-    atomicOr(&sh[1], o);
-  }
-  __syncthreads();
-  const uint64_t same = ~(sh[0] ^ sh[1]);
-  uint64_t T = sh[0] & same;  // bits every value shares
-  __syncthreads();
-  for (int b = 63; b >= 0; b--) {
-    if ((same >> b) & 1) continue;
-    const uint64_t cand = T | (1ull << b);  // undecided lower bits of T are still 0
-    const int cnt = __syncthreads_count(has && v >= cand);
-    if ((uint32_t)cnt >= r) T = cand;
-  }
-  return T;
+// 32-bit order-preserving summary of a list value v = key40 << 24 | low24:
+// key40 >> 9 below the maximal key, and 2^31 | low24 on it (completed
+// sessions all carry the maximal key, so only their index orders them).
+// summary(a) <= summary(b) whenever a <= b; summary_floor(f) is the smallest
+// list value whose summary is f.
+__device__ __forceinline__ uint32_t summary_of(uint64_t v) {
+  const uint64_t K = v >> 24;
+  return K == kKeyMax40 ? (0x80000000u | (uint32_t)(v & kIdMask)) : (uint32_t)(K >> 9);
+}
+__device__ __forceinline__ uint64_t summary_floor(uint32_t f) {
+  return (f & 0x80000000u) ? ((kKeyMax40 << 24) | (f & kIdMask)) : ((uint64_t)f << 33);
 }
 
-__global__ void __launch_bounds__(1024) rank_sample_kernel(const RankSet *sets) {
+// Joint MSB-first radix select over the block, 8-bit digits: for every list
+// L in `sel`, the value of rank need[L] (1 = largest) among the values
+// v[L][q] whose bit L * Q + q of `has` is set (Q values per thread per list).
+// All threads get the results in out[L].
+template <int Q>
+__device__ void joint_select32(const uint32_t (&v)[kLists][Q], uint32_t has, uint32_t sel,
+                               const uint32_t (&need_in)[kLists], uint32_t (&out)[kLists],
+                               unsigned int (*hist)[256], unsigned int *sel_digit, unsigned int *sel_need) {
+  const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t need[kLists], prefix[kLists];
+#pragma unroll
+  for (int L = 0; L < kLists; L++) {
+    need[L] = need_in[L];
+    prefix[L] = 0;
+  }
+  for (int b = 3; b >= 0; b--) {
+    const uint32_t mask = b == 3 ? 0u : (~0u << (8 * (b + 1)));
+    for (uint32_t i = threadIdx.x; i < kLists * 256; i += blockDim.x) (&hist[0][0])[i] = 0;
+    __syncthreads();
+#pragma unroll
+    for (int L = 0; L < kLists; L++) {
+      if (!((sel >> L) & 1)) continue;  // block-uniform
+#pragma unroll
+      for (int q = 0; q < Q; q++) {
+        const bool in = ((has >> (L * Q + q)) & 1) && (v[L][q] & mask) == prefix[L];
+        const uint32_t d = (v[L][q] >> (8 * b)) & 0xFF;
+        // lanes with the same digit add once per group
+        const unsigned ain = __ballot_sync(kFull, in);
+        if (in) {
+          const unsigned grp = __match_any_sync(ain, d);
+          if ((__ffs(grp) - 1) == (int)lane) atomicAdd(&hist[L][d], (unsigned)__popc(grp));
+        }
+      }
+    }
+    __syncthreads();
+    if (warp < (uint32_t)kLists && ((sel >> warp) & 1)) {
+      // lane l owns digits 255-8l .. 248-8l (descending): find the digit where
+      // the count of larger-or-equal values first reaches need
+      const int L = warp;
+      uint32_t nd = 0;
+#pragma unroll
+      for (int LL = 0; LL < kLists; LL++)
+        if (LL == L) nd = need[LL];
+      uint32_t c[8], tot = 0;
+#pragma unroll
+      for (int qq = 0; qq < 8; qq++) {
+        c[qq] = hist[L][255 - 8 * lane - qq];
+        tot += c[qq];
+      }
+      uint32_t incl = tot;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(kFull, incl, o);
+        if ((int)lane >= o) incl += y;
+      }
+      const uint32_t excl = incl - tot;
+      const unsigned hit = __ballot_sync(kFull, excl < nd && incl >= nd);
+      if ((int)lane == __ffs(hit) - 1) {
+        uint32_t cum = excl;
+#pragma unroll
+        for (int qq = 0; qq < 8; qq++) {
+          if (cum + c[qq] >= nd) {
+            sel_digit[L] = 255 - 8 * lane - qq;
+            sel_need[L] = nd - cum;
+            cum = 0xFFFFFFFFu;  // found: no later digit matches
+            break;
+          }
+          cum += c[qq];
+        }
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int L = 0; L < kLists; L++) {
+      if (!((sel >> L) & 1)) continue;
+      prefix[L] |= sel_digit[L] << (8 * b);
+      need[L] = sel_need[L];
+    }
+    __syncthreads();  // sel_* are rewritten by the next pass
+  }
+#pragma unroll
+  for (int L = 0; L < kLists; L++) out[L] = prefix[L];
+}
+
+// kSampleCtas CTAs per set.  1. One sample per thread: run j of ns/8 covers
+// stratum j (records [j n / (ns/8), (j+1) n / (ns/8))), 8 consecutive
+// records at a hashed offset inside it.  2. Per list, each CTA keeps the top
+// r_L summaries of its eligible samples (all of them when it has fewer).
+// 3. The last CTA to finish selects the summary of rank r_L among those
+// partial lists -- the rank-r_L summary of the whole sample -- and turns it
+// into the list's threshold: the smallest list value with that summary (at
+// least r_L samples reach it), plus, per turn index, the smallest gap whose
+// key reaches the threshold's key (gA) or exceeds it (gB).
+__global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankSet *sets) {
   const RankSet &S = sets[blockIdx.y];
   const uint32_t c = blockIdx.x;  // this CTA's share of the sample
   __shared__ uint64_t t2s[kLutN], mgs[kLutN];
-  __shared__ unsigned long long sh[2];
-  __shared__ unsigned int is_last, wpos;
-  if (threadIdx.x < kLutN) {
-    const uint32_t sg = S.sigma[threadIdx.x];
-    t2s[threadIdx.x] = ((uint64_t)(kLambda - sg) * S.penalty) / kLambda;  // eq. (t2)
-    mgs[threadIdx.x] = magic_for(sg);
+  __shared__ unsigned int hist[kLists][256];
+  __shared__ unsigned int ecount[kLists], sel_digit[kLists], sel_need[kLists], wpos[kLists];
+  __shared__ unsigned int is_last;
+  const uint32_t tid = threadIdx.x, lane = tid & 31;
+  if (tid < kLutN) {
+    const uint32_t sg = S.sigma[tid];
+    t2s[tid] = ((uint64_t)(kLambda - sg) * S.penalty) / kLambda;  // eq. (t2)
+    mgs[tid] = magic_for(sg);
+  }
+  if (tid < kLists) {
+    ecount[tid] = 0;
+    wpos[tid] = 0;
   }
   __syncthreads();
   const uint32_t n = S.n;
   const uint32_t ns = sample_size(S);
   const uint32_t per = ns / kSampleCtas;  // samples of this CTA (<= 1024, a multiple of 8)
-  // 1. one sample per thread: run j covers stratum j of ns/8, 8 records at a hashed offset
-  uint64_t ck = 0;
+  const uint32_t act = (list_active(S, 0) ? 1u : 0u) | (list_active(S, 1) ? 2u : 0u) | (list_active(S, 2) ? 4u : 0u);
+  uint32_t rL[kLists];
+#pragma unroll
+  for (int L = 0; L < kLists; L++)
+    rL[L] = (ns && ((act >> L) & 1)) ? (uint32_t)umin64((list_target(S, L) * ns + n - 1) / n, kMaxR) : 0u;
+  // 1. this thread's sample
+  uint32_t f[kLists][1] = {{0}, {0}, {0}};
   uint32_t m = 0;
-  if (ns && threadIdx.x < per) {
-    const uint32_t nruns = ns / 8, run = c * (per / 8) + threadIdx.x / 8, o = threadIdx.x % 8;
+  if (tid < per) {
+    const uint32_t nruns = ns / 8, run = c * (per / 8) + tid / 8, o = tid % 8;
     const uint64_t lo = ((uint64_t)run * n) / nruns, hi = ((uint64_t)(run + 1) * n) / nruns;
     uint32_t h = run * 0x9E3779B1u;
     h ^= h >> 16;
@@ -327,90 +439,94 @@ __global__ void __launch_bounds__(1024) rank_sample_kernel(const RankSet *sets) 
     const uint32_t r = (uint32_t)(lo + (h % (span + 1))) + o;
     const uint8_t fl = S.flags[r], tr = S.tier[r];
     const uint32_t t = min((uint32_t)S.turn[r], kTMax);
-    ck = ck_of(score_of(S.gap[r], t, (fl & 2) != 0, t2s, mgs), r);
-    m = elig_mask(fl, tr);
+    const uint64_t ck = ck_of(score_of(S.gap[r], t, (fl & 2) != 0, t2s, mgs), r);
+    m = elig_mask(fl, tr) & act;
+#pragma unroll
+    for (int L = 0; L < kLists; L++) f[L][0] = summary_of(list_val(ck, L));
   }
-  // 2. per list: this CTA's top r values (exactly r, values are distinct)
+#pragma unroll
   for (int L = 0; L < kLists; L++) {
-    if (!ns || !list_active(S, L)) continue;
-    const uint32_t r = (uint32_t)umin64((list_target(S, L) * ns + n - 1) / n, kMaxR);
+    const uint32_t cnt = __popc(__ballot_sync(kFull, (m >> L) & 1));
+    if (lane == 0 && cnt) atomicAdd(&ecount[L], cnt);
+  }
+  __syncthreads();
+  // 2. per list: this CTA's top r_L (the summary of rank r_L, then the values
+  // above it and enough copies of it)
+  uint32_t sel = 0, need[kLists], T[kLists] = {0, 0, 0};
+#pragma unroll
+  for (int L = 0; L < kLists; L++) {
+    need[L] = rL[L];
+    if (rL[L] && ecount[L] > rL[L]) sel |= 1u << L;
+  }
+  if (sel) joint_select32<1>(f, m, sel, need, T, hist, sel_digit, sel_need);
+#pragma unroll
+  for (int L = 0; L < kLists; L++) {
+    if (!rL[L]) continue;
+    uint32_t *dst = S.part + ((size_t)L * kSampleCtas + c) * kMaxR;
+    const bool all = !((sel >> L) & 1);  // keep every eligible sample
     const bool has = (m >> L) & 1;
-    const uint64_t v = has ? list_val(ck, L) : 0ull;
-    const uint32_t navail = (uint32_t)__syncthreads_count(has);
-    uint64_t *dst = S.part + ((size_t)L * kSampleCtas + c) * kMaxR;
-    if (threadIdx.x == 0) wpos = 0;
-    if (navail <= r) {
-      __syncthreads();
-      if (has) {
-        const uint32_t w = atomicAdd(&wpos, 1u);
-        if (w < r) dst[w] = v;
-      }
-      __syncthreads();
-      for (uint32_t q = navail + threadIdx.x; q < r; q += blockDim.x) dst[q] = 0ull;
-    } else {
-      const uint64_t T = block_rank_bitwise(v, has, r, sh);
-      if (has && v >= T) {
-        const uint32_t w = atomicAdd(&wpos, 1u);
-        if (w < r) dst[w] = v;
-      }
-    }
+    if (has && (all || f[L][0] > T[L])) dst[atomicAdd(&wpos[L], 1u)] = f[L][0];
     __syncthreads();
+    if (tid == 0) {
+      const uint32_t above = wpos[L];
+      const uint32_t total = all ? above : rL[L];
+      for (uint32_t q = above; q < total; q++) dst[q] = T[L];  // ties at the rank-r_L summary
+      S.part_n[L * kSampleCtas + c] = total;
+    }
   }
   // 3. the last CTA to finish merges the partial lists and sets the thresholds
   __threadfence();
   __syncthreads();
-  if (threadIdx.x == 0) is_last = (atomicAdd(&S.work->ticket, 1u) == kSampleCtas - 1);
+  if (tid == 0) is_last = (atomicAdd(&S.work->sticket, 1u) == kSampleCtas - 1);
   __syncthreads();
   if (!is_last) return;
   __threadfence();
-  if (threadIdx.x < kLutN) {
-    S.t2[threadIdx.x] = t2s[threadIdx.x];
-    S.magic[threadIdx.x] = mgs[threadIdx.x];
+  if (tid < kLutN) {
+    S.t2[tid] = t2s[tid];
+    S.magic[tid] = mgs[tid];
   }
+  // kSampleCtas * r_L <= 4096 entries per list: four per thread
+  uint32_t v4[kLists][4];
+  uint32_t has4 = 0;
+#pragma unroll
   for (int L = 0; L < kLists; L++) {
-    const bool active = list_active(S, L);
-    uint64_t thrv = 0;  // 0: accept every eligible record
-    if (ns && active) {
-      const uint32_t r = (uint32_t)umin64((list_target(S, L) * ns + n - 1) / n, kMaxR);
-      // kSampleCtas * r <= 4096 values: one per thread (with the shared-bit
-      // skip) when they fit in the block, else four per thread
-      const uint32_t nv = kSampleCtas * r;
-      uint64_t T = 0;
-      if (nv <= blockDim.x) {
-        const uint32_t idx = threadIdx.x;
-        uint64_t v = idx < nv ? __ldcg(&S.part[((size_t)L * kSampleCtas + idx / r) * kMaxR + idx % r]) : 0ull;
-        const bool has = idx < nv && v != 0ull;
-        T = block_rank_bitwise(v, has, r, sh);
-        if (__syncthreads_count(has) < (int)r) T = 0;
-      } else {
-        uint64_t vq[4];
-        bool hq[4];
-        for (int q = 0; q < 4; q++) {
-          const uint32_t idx = threadIdx.x + 1024u * q;
-          hq[q] = idx < nv;
-          vq[q] = hq[q] ? __ldcg(&S.part[((size_t)L * kSampleCtas + idx / r) * kMaxR + idx % r]) : 0ull;
-          hq[q] = hq[q] && vq[q] != 0ull;
-        }
-        for (int b = 63; b >= 0; b--) {
-          const uint64_t cand = T | (1ull << b);
-          int cnt = 0;
-          for (int q = 0; q < 4; q++) cnt += __syncthreads_count(hq[q] && vq[q] >= cand);
-          if ((uint32_t)cnt >= r) T = cand;
-        }
+#pragma unroll
+    for (int q = 0; q < 4; q++) v4[L][q] = 0;
+    if (!rL[L]) continue;
+    // entry e of the concatenation: CTA e / kMaxR, slot e % kMaxR
+#pragma unroll
+    for (int q = 0; q < 4; q++) {
+      const uint32_t e = tid + 1024u * q;
+      const uint32_t cc = e / kMaxR, slot = e % kMaxR;
+      if (cc < kSampleCtas && slot < __ldcg(&S.part_n[L * kSampleCtas + cc])) {
+        v4[L][q] = __ldcg(&S.part[((size_t)L * kSampleCtas + cc) * kMaxR + slot]);
+        has4 |= 1u << (L * 4 + q);
       }
-      thrv = T;  // 0 when fewer than r eligible samples
     }
-    if (threadIdx.x == 0) {
+  }
+  uint32_t sel2 = 0;
+#pragma unroll
+  for (int L = 0; L < kLists; L++) {
+    if (!rL[L]) continue;
+    uint32_t cnt = 0;
+    for (uint32_t cc = 0; cc < kSampleCtas; cc++) cnt += __ldcg(&S.part_n[L * kSampleCtas + cc]);
+    if (cnt >= rL[L]) sel2 |= 1u << L;
+  }
+  uint32_t T2[kLists] = {0, 0, 0};
+  if (sel2) joint_select32<4>(v4, has4, sel2, rL, T2, hist, sel_digit, sel_need);
+#pragma unroll
+  for (int L = 0; L < kLists; L++) {
+    // 0 (fewer than r_L eligible samples, or none taken): accept every eligible record
+    const uint64_t thrv = ((sel2 >> L) & 1) ? summary_floor(T2[L]) : 0ull;
+    if (tid == 0) {
       S.thr[L] = thrv;
-      S.thr[kLists + L] = active ? 1 : 0;
+      S.thr[kLists + L] = (act >> L) & 1;
     }
-    if (threadIdx.x < kLutN) {
-      const uint32_t t = threadIdx.x;
+    if (tid < kLutN) {
       const uint64_t thr_ck = (L == 2) ? ~thrv : thrv;
       const uint64_t K = thr_ck >> 24;
-      S.gthr[L * kLutN + t] = make_uint2(g_at_least(K, S.sigma[t], t2s[t]), g_at_least(K + 1, S.sigma[t], t2s[t]));
+      S.gthr[L * kLutN + tid] = make_uint2(g_at_least(K, S.sigma[tid], t2s[tid]), g_at_least(K + 1, S.sigma[tid], t2s[tid]));
     }
-    __syncthreads();
   }
 }
 
@@ -906,21 +1022,21 @@ __device__ uint32_t stream_topM(const RankSet &S, int L, uint32_t M, uint64_t *p
 }
 
 __global__ void __launch_bounds__(kFinishThreads) rank_finish_kernel(const RankSet *sets) {
-  const RankSet &S = sets[blockIdx.x];
+  const RankSet &S = sets[blockIdx.y];
+  const int L = blockIdx.x;  // this CTA's list
   extern __shared__ __align__(16) unsigned char smem[];
   uint64_t *buf = reinterpret_cast<uint64_t *>(smem);   // [kSmemCand]
   uint64_t *sel = buf + kSmemCand;                      // [kMaxSel]
   __shared__ uint64_t t2s[kLutN], mgs[kLutN];
   __shared__ unsigned int hist[256];
   __shared__ unsigned long long bcast[2];
-  __shared__ unsigned int cnt;
-  __shared__ uint32_t mL[kLists];
+  __shared__ unsigned int cnt, is_last;
   if (threadIdx.x < kLutN) {
     t2s[threadIdx.x] = S.t2[threadIdx.x];
     mgs[threadIdx.x] = S.magic[threadIdx.x];
   }
   __syncthreads();
-  for (int L = 0; L < kLists; L++) {
+  {
     const bool active = S.thr[kLists + L] != 0;
     const uint32_t Mw = (L == 0) ? S.k : S.max_moves;
     const uint32_t emitted = S.work->cand[L];
@@ -964,12 +1080,18 @@ __global__ void __launch_bounds__(kFinishThreads) rank_finish_kernel(const RankS
       block_sort_desc(sel, got);
       for (uint32_t i = threadIdx.x; i < got; i += blockDim.x) S.sorted[(size_t)L * kMaxSel + i] = sel[i];
     }
-    if (threadIdx.x == 0) mL[L] = got;
-    __syncthreads();
+    if (threadIdx.x == 0) S.work->got[L] = got;
   }
+  // the last of the set's list CTAs does the victims and the fill
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) is_last = (atomicAdd(&S.work->ticket, 1u) == (unsigned)kLists - 1);
+  __syncthreads();
+  if (!is_last) return;
+  __threadfence();
+  const uint32_t nv = __ldcg(&S.work->got[0]), nd = __ldcg(&S.work->got[1]), np = __ldcg(&S.work->got[2]);
   const uint64_t *V = S.sorted, *D = S.sorted + kMaxSel, *P = S.sorted + 2 * kMaxSel;
-  const uint32_t nv = mL[0], nd = mL[1], np = mL[2];
-  for (uint32_t i = threadIdx.x; i < nv; i += blockDim.x) S.victims[i] = (~(uint32_t)V[i]) & kIdMask;
+  for (uint32_t i = threadIdx.x; i < nv; i += blockDim.x) S.victims[i] = (~(uint32_t)__ldcg(&V[i])) & kIdMask;
 
   // TIDE fill.  Stage P (ascending ck) and D (descending ck) with their sizes.
   // Layout inside the dynamic area (the selection buffers are free now):
@@ -981,13 +1103,14 @@ __global__ void __launch_bounds__(kFinishThreads) rank_finish_kernel(const RankS
   uint32_t *dsz = psz + kMaxSel;
   uint32_t *dsz2 = dsz + kMaxSel;
   for (uint32_t i = threadIdx.x; i < np; i += blockDim.x) {
-    const uint64_t ck = ~P[i];
+    const uint64_t ck = ~__ldcg(&P[i]);
     pck[i] = ck;
     psz[i] = S.kv[(~(uint32_t)ck) & kIdMask];
   }
   for (uint32_t i = threadIdx.x; i < nd; i += blockDim.x) {
-    dck[i] = D[i];
-    dsz[i] = S.kv[(~(uint32_t)D[i]) & kIdMask];
+    const uint64_t d = __ldcg(&D[i]);
+    dck[i] = d;
+    dsz[i] = S.kv[(~(uint32_t)d) & kIdMask];
   }
   __syncthreads();
   __shared__ uint32_t n1s, npairs;
@@ -1177,12 +1300,14 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
     for (int t = 0; t < (int)kLutN; t++) s.sigma[t] = p.sigma_q[t];
     s.pad = 0;
   }
-  // scratch: descriptors, then per set: work, thresholds, tables, sorted lists, candidates
+  // scratch: descriptors, then per set: work, thresholds, tables, sorted
+  // lists, candidates, the sample's partial lists
   const size_t per_set = align_up(sizeof(RankWork), 256) + align_up(sizeof(uint64_t) * 2 * kLists, 256) +
                          align_up(sizeof(uint2) * kLists * kLutN, 256) + 2 * align_up(sizeof(uint64_t) * kLutN, 256) +
                          align_up(sizeof(uint64_t) * kLists * kMaxSel, 256) +
                          align_up(sizeof(uint64_t) * kLists * kCandCap, 256) +
-                         align_up(sizeof(uint64_t) * kLists * kSampleCtas * kMaxR, 256);
+                         align_up(sizeof(uint32_t) * kLists * kSampleCtas * kMaxR, 256) +
+                         align_up(sizeof(uint32_t) * kLists * kSampleCtas, 256);
   const size_t desc_b = align_up(sizeof(RankSet) * n_sets, 256);
   char *scratch = nullptr;
   if (cudaMallocAsync(reinterpret_cast<void **>(&scratch), desc_b + per_set * n_sets, stream) != cudaSuccess) {
@@ -1206,7 +1331,9 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
     p += align_up(sizeof(uint64_t) * kLists * kMaxSel, 256);
     s.cand = reinterpret_cast<uint64_t *>(p);
     p += align_up(sizeof(uint64_t) * kLists * kCandCap, 256);
-    s.part = reinterpret_cast<uint64_t *>(p);
+    s.part = reinterpret_cast<uint32_t *>(p);
+    p += align_up(sizeof(uint32_t) * kLists * kSampleCtas * kMaxR, 256);
+    s.part_n = reinterpret_cast<uint32_t *>(p);
   }
   int rc = UNISON_OK;
   auto ck = [&](cudaError_t e) {
@@ -1216,7 +1343,7 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
   ck(cudaMemcpyAsync(d_sets, hs.data(), sizeof(RankSet) * n_sets, cudaMemcpyHostToDevice, stream));
   for (int i = 0; i < n_sets; i++) ck(cudaMemsetAsync(hs[i].work, 0, sizeof(RankWork), stream));
   const size_t smem_finish = sizeof(uint64_t) * (kSmemCand + kMaxSel);
-  // persistent filter: as many CTAs as fit at once, each over a contiguous tile range
+  // persistent filter: as many CTAs as fit at once, tiles dealt round-robin
   int dev = 0, n_sm = 0, per_sm = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
@@ -1234,7 +1361,7 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
   }
   {
     ProfSpan span("rank_finish", stream);
-    rank_finish_kernel<<<n_sets, kFinishThreads, smem_finish, stream>>>(d_sets);
+    rank_finish_kernel<<<dim3(kLists, n_sets), kFinishThreads, smem_finish, stream>>>(d_sets);
   }
   count_launches(3);
   ck(cudaGetLastError());
