@@ -785,7 +785,10 @@ int or_rank(const or_records *r, const uint16_t *sigma_q51, uint64_t penalty_q, 
   *n_victims = (uint32_t)nv;
 
   qsort(P, np, sizeof(uint32_t), cmp_rank_asc);
-  uint64_t rem = budget_bytes, fs = free_s_tok, fh = free_h_tok, j = 0, npro = 0, ndem = 0;
+  /* Free space is tracked exactly (128 bits): the capacity tests are on the
+   * integers, whatever the free space passed in. */
+  unsigned __int128 fs = free_s_tok, fh = free_h_tok;
+  uint64_t rem = budget_bytes, j = 0, npro = 0, ndem = 0;
   while (j < np && npro < max_moves) { /* phase 1 */
     uint64_t sz = r->kv_tok[P[j]], by = sz * kv_bytes_per_token;
     if (by > rem || sz > fs) break;

@@ -485,9 +485,13 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
     S.t2[tid] = t2s[tid];
     S.magic[tid] = mgs[tid];
   }
-  // kSampleCtas * r_L <= 4096 entries per list: four per thread
+  // entry counts of the partial lists, then kSampleCtas * r_L <= 4096
+  // entries per list: four per thread
+  __shared__ unsigned int pn[kLists * kSampleCtas];
+  if (tid < kLists * kSampleCtas) pn[tid] = __ldcg(&S.part_n[tid]);
+  __syncthreads();
   uint32_t v4[kLists][4];
-  uint32_t has4 = 0;
+  uint32_t has4 = 0, sel2 = 0;
 #pragma unroll
   for (int L = 0; L < kLists; L++) {
 #pragma unroll
@@ -498,18 +502,13 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
     for (int q = 0; q < 4; q++) {
       const uint32_t e = tid + 1024u * q;
       const uint32_t cc = e / kMaxR, slot = e % kMaxR;
-      if (cc < kSampleCtas && slot < __ldcg(&S.part_n[L * kSampleCtas + cc])) {
+      if (cc < kSampleCtas && slot < pn[L * kSampleCtas + cc]) {
         v4[L][q] = __ldcg(&S.part[((size_t)L * kSampleCtas + cc) * kMaxR + slot]);
         has4 |= 1u << (L * 4 + q);
       }
     }
-  }
-  uint32_t sel2 = 0;
-#pragma unroll
-  for (int L = 0; L < kLists; L++) {
-    if (!rL[L]) continue;
     uint32_t cnt = 0;
-    for (uint32_t cc = 0; cc < kSampleCtas; cc++) cnt += __ldcg(&S.part_n[L * kSampleCtas + cc]);
+    for (uint32_t cc = 0; cc < kSampleCtas; cc++) cnt += pn[L * kSampleCtas + cc];
     if (cnt >= rL[L]) sel2 |= 1u << L;
   }
   uint32_t T2[kLists] = {0, 0, 0};
@@ -970,6 +969,82 @@ __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) ra
 }
 
 // ------------------------------------------------------------- finish ----
+constexpr uint32_t kIpt = kMaxSel / kFinishThreads;  // fill items per thread
+static_assert(kMaxSel % kFinishThreads == 0 && kFinishThreads == 1024, "fill scan layout");
+
+// Byte sums of up to 4096 moves reach 2^70: kept as lo + 2^64 hi.
+struct Sum {
+  uint64_t lo;
+  uint32_t hi;
+};
+__device__ __forceinline__ Sum sum_add(Sum x, Sum y) {
+  const uint64_t lo = x.lo + y.lo;
+  return Sum{lo, x.hi + y.hi + (lo < x.lo ? 1u : 0u)};
+}
+__device__ __forceinline__ bool sum_le(Sum x, uint64_t cap) { return x.hi == 0 && x.lo <= cap; }
+__device__ __forceinline__ Sum shfl_up_sum(Sum x, int o) {
+  return Sum{__shfl_up_sync(kFull, x.lo, o), __shfl_up_sync(kFull, x.hi, o)};
+}
+
+// Block-wide inclusive prefix sums over items j = kIpt * tid + i of a and b.
+__device__ void block_scan_pairs(Sum (&a)[kIpt], int64_t (&b)[kIpt], Sum *wa, int64_t *wb) {
+  const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (uint32_t i = 1; i < kIpt; i++) {
+    a[i] = sum_add(a[i], a[i - 1]);
+    b[i] += b[i - 1];
+  }
+  Sum ia = a[kIpt - 1];
+  int64_t ib = b[kIpt - 1];
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const Sum ya = shfl_up_sum(ia, o);
+    const int64_t yb = __shfl_up_sync(kFull, ib, o);
+    if ((int)lane >= o) {
+      ia = sum_add(ia, ya);
+      ib += yb;
+    }
+  }
+  Sum ea = shfl_up_sum(ia, 1);
+  int64_t eb = __shfl_up_sync(kFull, ib, 1);
+  if (lane == 0) {
+    ea = Sum{0, 0};
+    eb = 0;
+  }
+  if (lane == 31) {
+    wa[warp] = ia;
+    wb[warp] = ib;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    Sum xa = wa[lane];
+    int64_t xb = wb[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const Sum ya = shfl_up_sum(xa, o);
+      const int64_t yb = __shfl_up_sync(kFull, xb, o);
+      if ((int)lane >= o) {
+        xa = sum_add(xa, ya);
+        xb += yb;
+      }
+    }
+    const Sum pa = shfl_up_sum(xa, 1);
+    const int64_t pb = __shfl_up_sync(kFull, xb, 1);
+    __syncwarp();
+    wa[lane] = lane ? pa : Sum{0, 0};
+    wb[lane] = lane ? pb : 0ll;
+  }
+  __syncthreads();
+  const Sum oa = sum_add(wa[warp], ea);
+  const int64_t ob = wb[warp] + eb;
+#pragma unroll
+  for (uint32_t i = 0; i < kIpt; i++) {
+    a[i] = sum_add(a[i], oa);
+    b[i] += ob;
+  }
+  __syncthreads();  // wa, wb free again
+}
+
 // Exact top-M of list L over the whole set by one CTA, streaming records and
 // keeping a pool of at most M + 4096 values (the fallback path).
 __device__ uint32_t stream_topM(const RankSet &S, int L, uint32_t M, uint64_t *pool, const uint64_t *t2s,
@@ -1113,49 +1188,46 @@ __global__ void __launch_bounds__(kFinishThreads) rank_finish_kernel(const RankS
     dsz[i] = S.kv[(~(uint32_t)d) & kIdMask];
   }
   __syncthreads();
-  __shared__ uint32_t n1s, npairs;
-  __shared__ unsigned long long rem_s, fs_s, fh_s;
+  // Both fill phases take items in order and stop at the first that does not
+  // fit; with the state after j items a function of prefix sums over items
+  // 0..j, each phase is one block scan and a minimum over the failing items.
+  __shared__ Sum wa[32];
+  __shared__ int64_t wb[32];
+  __shared__ unsigned int first_bad;
+  __shared__ unsigned long long at_a;
+  __shared__ long long at_b;
   const uint64_t kvb = S.kvb;
-  const int lane = threadIdx.x & 31;
-  if (threadIdx.x < 32) {
-    // phase 1: promotions into free fast-tier space, least evictable first
-    uint64_t rem = S.budget, fs = S.free_s, fh = S.free_h;
-    uint32_t n1 = 0;
-    const uint32_t lim = min(np, S.max_moves);
-    bool stop = (S.thr[kLists + 2] == 0);
-    while (!stop && n1 < lim) {
-      const uint32_t j = n1 + lane;
-      const uint64_t sz = j < lim ? psz[j] : 0;
-      uint64_t by = sz * kvb, cs = sz;
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint64_t yb = __shfl_up_sync(kFull, by, o), ys = __shfl_up_sync(kFull, cs, o);
-        if (lane >= o) {
-          by += yb;
-          cs += ys;
-        }
-      }
-      const bool ok = j < lim && by <= rem && cs <= fs;
-      const uint32_t okm = __ballot_sync(kFull, ok);
-      const uint32_t take = __ffs(~okm) - 1;  // ok is a prefix (sums only grow)
-      const uint32_t tk = okm == kFull ? 32u : take;
-      if (tk > 0) {
-        const uint64_t tb = __shfl_sync(kFull, by, tk - 1), ts = __shfl_sync(kFull, cs, tk - 1);
-        rem -= tb;
-        fs -= ts;
-        fh += ts;
-      }
-      n1 += tk;
-      if (tk < 32) stop = true;
-    }
-    if (lane == 0) {
-      n1s = n1;
-      rem_s = rem;
-      fs_s = fs;
-      fh_s = fh;
-    }
+  const uint32_t tid = threadIdx.x;
+  Sum a[kIpt];
+  int64_t b[kIpt];
+  // phase 1: promotions into free fast-tier space, least evictable first
+  const uint32_t lim1 = (S.thr[kLists + 2] == 0) ? 0u : min(np, S.max_moves);
+#pragma unroll
+  for (uint32_t i = 0; i < kIpt; i++) {
+    const uint32_t j = kIpt * tid + i;
+    const uint64_t sz = j < lim1 ? psz[j] : 0;
+    a[i] = Sum{sz * kvb, 0};  // bytes moved
+    b[i] = (int64_t)sz;  // fast-tier tokens taken
+  }
+  if (tid == 0) first_bad = lim1;
+  block_scan_pairs(a, b, wa, wb);
+#pragma unroll
+  for (uint32_t i = 0; i < kIpt; i++) {
+    const uint32_t j = kIpt * tid + i;
+    if (j < lim1 && !(sum_le(a[i], S.budget) && (uint64_t)b[i] <= S.free_s)) atomicMin(&first_bad, j);
   }
   __syncthreads();
-  const uint32_t n1 = n1s;
+  const uint32_t n1 = first_bad;
+#pragma unroll
+  for (uint32_t i = 0; i < kIpt; i++)
+    if (n1 > 0 && kIpt * tid + i == n1 - 1) {
+      at_a = a[i].lo;
+      at_b = b[i];
+    }
+  __syncthreads();
+  const uint64_t rem = S.budget - (n1 ? at_a : 0ull);
+  const uint64_t fs = S.free_s - (n1 ? (uint64_t)at_b : 0ull), fh = S.free_h + (n1 ? (uint64_t)at_b : 0ull);
+  __syncthreads();
   // phase 2 demotion order: fast-tier candidates merged with the promoted ones
   // (only the first lim2 positions can be paired)
   const uint32_t cap2 = S.max_moves > n1 ? S.max_moves - n1 : 0;
@@ -1185,56 +1257,41 @@ __global__ void __launch_bounds__(kFinishThreads) rank_finish_kernel(const RankS
     }
   }
   __syncthreads();
-  if (threadIdx.x < 32) {
-    uint64_t rem = rem_s, fs = fs_s, fh = fh_s;
-    uint32_t pairs = 0;
-    const uint32_t lim = min(np - min(np, n1), nd2);
-    bool stop = (S.thr[kLists + 2] == 0) || (S.thr[kLists + 1] == 0);
-    while (!stop && pairs < lim) {
-      const uint32_t j = pairs + lane;
-      bool order_ok = false;
-      uint64_t sp = 0, sd = 0;
-      if (j < lim) {
-        sp = psz[n1 + j];
-        sd = dsz2[j];
-        order_ok = dck2[j] > pck[n1 + j];
-      }
-      uint64_t by = (sp + sd) * kvb;
-      long long ds = (long long)sp - (long long)sd;  // fast tier gains sp, loses sd
-      for (int o = 1; o < 32; o <<= 1) {
-        const uint64_t yb = __shfl_up_sync(kFull, by, o);
-        const long long yd = __shfl_up_sync(kFull, ds, o);
-        if (lane >= o) {
-          by += yb;
-          ds += yd;
-        }
-      }
-      const bool ok = j < lim && order_ok && by <= rem && (ds <= 0 || (uint64_t)ds <= fs) &&
-                      (ds >= 0 || (uint64_t)(-ds) <= fh);
-      const uint32_t okm = __ballot_sync(kFull, ok);
-      const uint32_t tk = okm == kFull ? 32u : (uint32_t)(__ffs(~okm) - 1);
-      if (tk > 0) {
-        const uint64_t tb = __shfl_sync(kFull, by, tk - 1);
-        const long long td = __shfl_sync(kFull, ds, tk - 1);
-        rem -= tb;
-        if (td >= 0) {
-          fs -= (uint64_t)td;
-          fh += (uint64_t)td;
-        } else {
-          fs += (uint64_t)(-td);
-          fh -= (uint64_t)(-td);
-        }
-      }
-      pairs += tk;
-      if (tk < 32) stop = true;
+  // phase 2: pair P[n1 + j] (next least evictable HBM record) with the j-th
+  // most evictable fast-tier entry while the demoted one ranks above the
+  // promoted one and the budget and both tiers' capacities hold
+  const bool p2 = (S.thr[kLists + 2] != 0) && (S.thr[kLists + 1] != 0);
+  const uint32_t lim2 = p2 ? min(np - min(np, n1), nd2) : 0u;
+  bool order_ok[kIpt];
+#pragma unroll
+  for (uint32_t i = 0; i < kIpt; i++) {
+    const uint32_t j = kIpt * tid + i;
+    uint64_t sp = 0, sd = 0;
+    order_ok[i] = false;
+    if (j < lim2) {
+      sp = psz[n1 + j];
+      sd = dsz2[j];
+      order_ok[i] = dck2[j] > pck[n1 + j];
     }
-    if (lane == 0) {
-      npairs = pairs;
-      rem_s = rem;
-    }
+    a[i] = Sum{(sp + sd) * kvb, 0};         // bytes moved by the pair
+    b[i] = (int64_t)sp - (int64_t)sd;      // fast tier gains sp, loses sd
+  }
+  if (tid == 0) first_bad = lim2;
+  block_scan_pairs(a, b, wa, wb);
+#pragma unroll
+  for (uint32_t i = 0; i < kIpt; i++) {
+    const uint32_t j = kIpt * tid + i;
+    const bool ok = order_ok[i] && sum_le(a[i], rem) && (b[i] <= 0 || (uint64_t)b[i] <= fs) &&
+                    (b[i] >= 0 || (uint64_t)(-b[i]) <= fh);
+    if (j < lim2 && !ok) atomicMin(&first_bad, j);
   }
   __syncthreads();
-  const uint32_t pairs = npairs;
+  const uint32_t pairs = first_bad;
+#pragma unroll
+  for (uint32_t i = 0; i < kIpt; i++)
+    if (pairs > 0 && kIpt * tid + i == pairs - 1) at_a = a[i].lo;
+  __syncthreads();
+  const uint64_t rem_end = rem - (pairs ? at_a : 0ull);
   for (uint32_t i = threadIdx.x; i < n1 + pairs; i += blockDim.x) S.promote[i] = (~(uint32_t)pck[i]) & kIdMask;
   for (uint32_t i = threadIdx.x; i < pairs; i += blockDim.x) S.demote[i] = (~(uint32_t)dck2[i]) & kIdMask;
   if (threadIdx.x == 0) {
@@ -1242,7 +1299,7 @@ __global__ void __launch_bounds__(kFinishThreads) rank_finish_kernel(const RankS
     S.counts[1] = n1 + pairs;
     S.counts[2] = pairs;
     S.counts[3] = S.work->status ? S.work->status : (unsigned int)UNISON_OK;
-    S.moved[0] = S.budget - rem_s;
+    S.moved[0] = S.budget - rem_end;
   }
 }
 

@@ -138,6 +138,31 @@ def test_phase1_promotions(B, sigma):
         check(r, rec, p)
 
 
+def test_fill_byte_sums_beyond_2p64(B, sigma):
+    """Sizes near 2^32 tokens at 2^24 bytes per token and the largest budget:
+    the running byte sums pass 2^64 within a few hundred moves, in phase 1
+    (free fast-tier space, random sizes) and in the pair loop (equal sizes,
+    one promotion's worth of free space)."""
+    n = 100000
+    base = synth.make_records(10, n)
+    big = synth.rng.randint(11, 0, np.arange(n, dtype=np.uint64), 1 << 31, (1 << 32) - 1).astype(np.uint32)
+    rnd = synth.Records(base.gap_q, base.last_ret, base.turn, big, base.tier, base.flags)
+    flat = synth.Records(base.gap_q, base.last_ret, base.turn, np.full(n, 0xFFFFFFFF, np.uint32), base.tier,
+                         base.flags)
+    top = (1 << 64) - 1
+    cases = [(rnd, 1 << 62, 1 << 62), (rnd, top, top), (flat, 0xFFFFFFFF, 1 << 62), (flat, 0, top)]
+    recs, ps = [], []
+    for rec, fs, fh in cases:
+        p = prm(sigma, k=64, budget=top, max_moves=4096, free_s=fs, free_h=fh)
+        p["kv_bytes_per_token"] = 1 << 24
+        recs.append(rec)
+        ps.append(p)
+    res = run(B, recs, ps)
+    for r, rec, p in zip(res, recs, ps):
+        check(r, rec, p)
+    assert len(res[0]["promote"]) > 100 and len(res[2]["demote"]) > 100
+
+
 def test_batch_of_mixed_sets(B, sigma):
     recs = [synth.make_records(20 + i, n) for i, n in enumerate([100, 20000, 1 << 18, 3000, 1 << 19])]
     ps = [prm(sigma, k=k, budget=(1 << i) * GIB) for i, k in enumerate([3, 50, 1024, 4096, 700])]
