@@ -66,15 +66,19 @@ struct RankSet {
   uint64_t *moved, *keys;
   uint32_t tile0, ntiles;
   uint32_t sigma[kLutN];
-  uint32_t pad;
+  // per-set constants, computed on the host
+  uint32_t ns, nruns, sq, srem;  // sample size, its runs of 8, n = sq * nruns + srem
+  uint32_t act;                  // active lists (bit L)
+  uint32_t rL[kLists];           // sample rank of each list's threshold
+  uint64_t t2v[kLutN];           // eq. (t2) per turn index
+  uint64_t mgv[kLutN];           // division magic of sigma per turn index
   // scratch (per set)
   RankWork *work;
   uint64_t *cand;    // [3][kCandCap]
   uint64_t *sorted;  // [3][kMaxSel]
+  uint32_t *ssz;     // [3][kMaxSel] KV tokens of the sorted entries (D and P)
   uint2 *gthr;       // [3][51] (gA, gB)
   uint64_t *thr;     // [3] threshold in list-value space; [3+L] = active flag
-  uint64_t *t2;      // [51]
-  uint64_t *magic;   // [51]
   uint32_t *part;    // [3][kSampleCtas][kMaxR] per-CTA top summaries of the sample
   uint32_t *part_n;  // [3][kSampleCtas] entries in each
 };
@@ -123,10 +127,11 @@ __device__ __forceinline__ uint32_t g_at_least(uint64_t K, uint32_t sigma, uint6
 // -------------------------------------------------------- block helpers ----
 // Value with the given rank (1 = largest) among get(0..n-1) -- MSB-first
 // radix select, 8 bits per pass.  All threads of the block call it and get
-// the same value.
+// the same value.  hist[2][256] and pick[2][2] are double-buffered, so a
+// pass takes two barriers.
 template <typename Get>
-__device__ uint64_t block_select_rank(Get get, uint32_t n, uint32_t rank, unsigned int *hist,
-                                      unsigned long long *bcast) {
+__device__ uint64_t block_select_rank(Get get, uint32_t n, uint32_t rank, unsigned int (*hist)[256],
+                                      unsigned int (*pick)[2], unsigned long long *bcast) {
   // bytes on which every value agrees need no pass: start at the highest
   // byte where some two values differ
   unsigned long long a = ~0ull, o = 0ull;
@@ -143,6 +148,7 @@ __device__ uint64_t block_select_rank(Get get, uint32_t n, uint32_t rank, unsign
     bcast[0] = ~0ull;
     bcast[1] = 0ull;
   }
+  for (uint32_t i = threadIdx.x; i < 2 * 256; i += blockDim.x) (&hist[0][0])[i] = 0;
   __syncthreads();
   if ((threadIdx.x & 31) == 0) {
     atomicAnd(&bcast[0], a);
@@ -153,13 +159,11 @@ __device__ uint64_t block_select_rank(Get get, uint32_t n, uint32_t rank, unsign
   const uint64_t common = bcast[0] & same;
   int top = 7;
   while (top > 0 && ((same >> (8 * top)) & 0xFF) == 0xFF) top--;
-  __syncthreads();
   uint64_t mask = top < 7 ? (~0ull << (8 * (top + 1))) : 0ull;
   uint64_t prefix = common & mask;
   uint32_t need = rank;
   for (int b = top; b >= 0; b--) {
-    for (uint32_t i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
-    __syncthreads();
+    const int pb = b & 1;
     for (uint32_t base = 0; base < n; base += blockDim.x) {
       const uint32_t i = base + threadIdx.x;
       bool in = false;
@@ -173,7 +177,7 @@ __device__ uint64_t block_select_rank(Get get, uint32_t n, uint32_t rank, unsign
       const unsigned act = __ballot_sync(0xFFFFFFFFu, in);
       if (in) {
         const unsigned grp = __match_any_sync(act, d);
-        if ((__ffs(grp) - 1) == (int)(threadIdx.x & 31)) atomicAdd(&hist[d], (unsigned)__popc(grp));
+        if ((__ffs(grp) - 1) == (int)(threadIdx.x & 31)) atomicAdd(&hist[pb][d], (unsigned)__popc(grp));
       }
     }
     __syncthreads();
@@ -184,7 +188,7 @@ __device__ uint64_t block_select_rank(Get get, uint32_t n, uint32_t rank, unsign
       uint32_t c[8], tot = 0;
 #pragma unroll
       for (int q = 0; q < 8; q++) {
-        c[q] = hist[255 - 8 * l - q];
+        c[q] = hist[pb][255 - 8 * l - q];
         tot += c[q];
       }
       uint32_t incl = tot;
@@ -197,71 +201,81 @@ __device__ uint64_t block_select_rank(Get get, uint32_t n, uint32_t rank, unsign
       const unsigned hit = __ballot_sync(0xFFFFFFFFu, excl < need && incl >= need);
       if (l == __ffs(hit) - 1) {
         uint32_t cum = excl;
+#pragma unroll
         for (int q = 0; q < 8; q++) {
           if (cum + c[q] >= need) {
-            bcast[0] = (unsigned long long)(255 - 8 * l - q);
-            bcast[1] = need - cum;
+            pick[pb][0] = 255 - 8 * l - q;
+            pick[pb][1] = need - cum;
+            cum = 0xFFFFFFFFu;  // found: no later digit matches
             break;
           }
           cum += c[q];
         }
       }
     }
+    // the other histogram was last read before the barrier above
+    for (uint32_t i = threadIdx.x; i < 256; i += blockDim.x) hist[pb ^ 1][i] = 0;
     __syncthreads();
-    prefix |= (uint64_t)bcast[0] << (8 * b);
+    prefix |= (uint64_t)pick[pb][0] << (8 * b);
     mask |= 0xFFull << (8 * b);
-    need = (uint32_t)bcast[1];
-    __syncthreads();
+    need = pick[pb][1];
   }
+  __syncthreads();  // hist, pick and bcast free for the caller
   return prefix;
 }
 
-// Bitonic sort, descending, of a[0..n) padded with zeros to a power of two
-// (at least 32).  Element i sits in lane i % 32 of its warp, so every
-// compare-exchange at distance below 32 runs in registers with shuffles; only
-// distances of 32 and more go through shared memory, one barrier each.
-__device__ void block_sort_desc(uint64_t *a, uint32_t n) {
+// Sort, descending, of a[0..n) padded with zeros to a power of two p >= 32
+// (tmp: p more entries of scratch).  Each warp sorts runs of 32 in registers
+// (bitonic network over shuffles); then runs are merged pairwise, log2(p/32)
+// levels of one barrier each: an element of the left run lands at its index
+// plus the number of right-run elements above it, an element of the right
+// run at its index plus the number of left-run elements at or above it, both
+// counts by binary search in the other (sorted) run.
+__device__ void block_sort_desc(uint64_t *a, uint32_t n, uint64_t *tmp) {
   if (n <= 1) return;
   uint32_t p = 32;
   while (p < n) p <<= 1;
   for (uint32_t i = n + threadIdx.x; i < p; i += blockDim.x) a[i] = 0;
   __syncthreads();
-  // stages k = kmin..kmax, distances below 32, in registers
-  auto reg_steps = [&](uint32_t kmin, uint32_t kmax) {
-    for (uint32_t base = 0; base < p; base += blockDim.x) {
-      const uint32_t i = base + threadIdx.x;
-      if (i < p) {  // p and blockDim are multiples of 32: whole warps
-        uint64_t x = a[i];
-        for (uint32_t k = kmin; k <= kmax; k <<= 1) {
-          const bool desc = (i & k) == 0;
-          for (uint32_t j = min(k >> 1, 16u); j > 0; j >>= 1) {
-            const uint64_t y = __shfl_xor_sync(0xFFFFFFFFu, x, j);
-            const bool lower = (i & j) == 0;
-            x = (lower == desc) ? (x > y ? x : y) : (x < y ? x : y);
-          }
-        }
-        a[i] = x;
+  const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  for (uint32_t r = warp; r < p / 32; r += nw) {
+    uint64_t x = a[r * 32 + lane];
+#pragma unroll
+    for (uint32_t k = 2; k <= 32; k <<= 1) {
+      const bool desc = (lane & k) == 0;
+#pragma unroll
+      for (uint32_t j = k >> 1; j > 0; j >>= 1) {
+        const uint64_t y = __shfl_xor_sync(0xFFFFFFFFu, x, j);
+        const bool lower = (lane & j) == 0;
+        x = (lower == desc) ? (x > y ? x : y) : (x < y ? x : y);
       }
+    }
+    a[r * 32 + lane] = x;
+  }
+  __syncthreads();
+  uint64_t *src = a, *dst = tmp;
+  for (uint32_t m = 32; m < p; m <<= 1) {
+    for (uint32_t i = threadIdx.x; i < p; i += blockDim.x) {
+      const uint64_t v = src[i];
+      const uint32_t run0 = i & ~(2 * m - 1);
+      const bool left = (i & m) == 0;
+      const uint64_t *other = src + run0 + (left ? m : 0);
+      uint32_t lo = 0, hi = m;  // other-run elements placed before v: a prefix
+      while (lo < hi) {
+        const uint32_t mid = (lo + hi) >> 1;
+        const uint64_t w = other[mid];
+        if (left ? (w > v) : (w >= v)) lo = mid + 1; else hi = mid;
+      }
+      dst[run0 + (i & (m - 1)) + lo] = v;
     }
     __syncthreads();
-  };
-  reg_steps(2, 32);
-  for (uint32_t k = 64; k <= p; k <<= 1) {
-    for (uint32_t j = k >> 1; j >= 32; j >>= 1) {
-      for (uint32_t i = threadIdx.x; i < p; i += blockDim.x) {
-        const uint32_t ij = i ^ j;
-        if (ij > i) {
-          const uint64_t x = a[i], y = a[ij];
-          const bool desc = (i & k) == 0;
-          if (desc ? (x < y) : (x > y)) {
-            a[i] = y;
-            a[ij] = x;
-          }
-        }
-      }
-      __syncthreads();
-    }
-    reg_steps(k, k);
+    uint64_t *t = src;
+    src = dst;
+    dst = t;
+  }
+  if (src != a) {
+    for (uint32_t i = threadIdx.x; i < p; i += blockDim.x) a[i] = src[i];
+    __syncthreads();
   }
 }
 
@@ -271,16 +285,16 @@ __device__ __forceinline__ uint64_t list_val(uint64_t ck, int L) { return L == 2
 // Sample size and per-list ranks: ns records (ns/8 runs of 8, one run per
 // stratum) and rank r_L = ceil(target_L * ns / n), with ns chosen so that no
 // r_L exceeds kMaxR; target_L = 6 M_L + 2048 candidates for M_L needed.
-__device__ __forceinline__ uint64_t umin64(uint64_t a, uint64_t b) { return a < b ? a : b; }
-__device__ __forceinline__ uint64_t list_target(const RankSet &S, int L) {
+__host__ __device__ __forceinline__ uint64_t umin64(uint64_t a, uint64_t b) { return a < b ? a : b; }
+__host__ __device__ __forceinline__ uint64_t list_target(const RankSet &S, int L) {
   const uint32_t M = (L == 0) ? S.k : S.max_moves;
   return 6ull * M + 2048;
 }
-__device__ __forceinline__ bool list_active(const RankSet &S, int L) {
+__host__ __device__ __forceinline__ bool list_active(const RankSet &S, int L) {
   const uint32_t M = (L == 0) ? S.k : S.max_moves;
   return M > 0 && (L == 0 || S.budget > 0);
 }
-__device__ __forceinline__ uint32_t sample_size(const RankSet &S) {
+__host__ __device__ __forceinline__ uint32_t sample_size(const RankSet &S) {
   const uint32_t n = S.n;
   if (n <= kSample) return 0;  // whole set: every eligible record is a candidate
   uint64_t tmax = 0;
@@ -309,11 +323,13 @@ __device__ __forceinline__ uint64_t summary_floor(uint32_t f) {
 // Joint MSB-first radix select over the block, 8-bit digits: for every list
 // L in `sel`, the value of rank need[L] (1 = largest) among the values
 // v[L][q] whose bit L * Q + q of `has` is set (Q values per thread per list).
-// All threads get the results in out[L].
+// All threads get the results in out[L].  Histograms and digit picks are
+// double-buffered (hist[2][kLists][256], pick[2][2 * kLists]), so a pass
+// takes two barriers.
 template <int Q>
 __device__ void joint_select32(const uint32_t (&v)[kLists][Q], uint32_t has, uint32_t sel,
                                const uint32_t (&need_in)[kLists], uint32_t (&out)[kLists],
-                               unsigned int (*hist)[256], unsigned int *sel_digit, unsigned int *sel_need) {
+                               unsigned int (*hist)[kLists][256], unsigned int (*pick)[2 * kLists]) {
   const uint32_t lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   uint32_t need[kLists], prefix[kLists];
 #pragma unroll
@@ -321,10 +337,11 @@ __device__ void joint_select32(const uint32_t (&v)[kLists][Q], uint32_t has, uin
     need[L] = need_in[L];
     prefix[L] = 0;
   }
+  for (uint32_t i = threadIdx.x; i < 2 * kLists * 256; i += blockDim.x) (&hist[0][0][0])[i] = 0;
+  __syncthreads();
   for (int b = 3; b >= 0; b--) {
+    const int pb = b & 1;
     const uint32_t mask = b == 3 ? 0u : (~0u << (8 * (b + 1)));
-    for (uint32_t i = threadIdx.x; i < kLists * 256; i += blockDim.x) (&hist[0][0])[i] = 0;
-    __syncthreads();
 #pragma unroll
     for (int L = 0; L < kLists; L++) {
       if (!((sel >> L) & 1)) continue;  // block-uniform
@@ -336,7 +353,7 @@ __device__ void joint_select32(const uint32_t (&v)[kLists][Q], uint32_t has, uin
         const unsigned ain = __ballot_sync(kFull, in);
         if (in) {
           const unsigned grp = __match_any_sync(ain, d);
-          if ((__ffs(grp) - 1) == (int)lane) atomicAdd(&hist[L][d], (unsigned)__popc(grp));
+          if ((__ffs(grp) - 1) == (int)lane) atomicAdd(&hist[pb][L][d], (unsigned)__popc(grp));
         }
       }
     }
@@ -352,7 +369,7 @@ __device__ void joint_select32(const uint32_t (&v)[kLists][Q], uint32_t has, uin
       uint32_t c[8], tot = 0;
 #pragma unroll
       for (int qq = 0; qq < 8; qq++) {
-        c[qq] = hist[L][255 - 8 * lane - qq];
+        c[qq] = hist[pb][L][255 - 8 * lane - qq];
         tot += c[qq];
       }
       uint32_t incl = tot;
@@ -368,8 +385,8 @@ __device__ void joint_select32(const uint32_t (&v)[kLists][Q], uint32_t has, uin
 #pragma unroll
         for (int qq = 0; qq < 8; qq++) {
           if (cum + c[qq] >= nd) {
-            sel_digit[L] = 255 - 8 * lane - qq;
-            sel_need[L] = nd - cum;
+            pick[pb][L] = 255 - 8 * lane - qq;
+            pick[pb][kLists + L] = nd - cum;
             cum = 0xFFFFFFFFu;  // found: no later digit matches
             break;
           }
@@ -377,15 +394,18 @@ __device__ void joint_select32(const uint32_t (&v)[kLists][Q], uint32_t has, uin
         }
       }
     }
+    // the other histogram was last read before the barrier above: clear it
+    // for the next pass
+    for (uint32_t i = threadIdx.x; i < kLists * 256; i += blockDim.x) (&hist[pb ^ 1][0][0])[i] = 0;
     __syncthreads();
 #pragma unroll
     for (int L = 0; L < kLists; L++) {
       if (!((sel >> L) & 1)) continue;
-      prefix[L] |= sel_digit[L] << (8 * b);
-      need[L] = sel_need[L];
+      prefix[L] |= pick[pb][L] << (8 * b);
+      need[L] = pick[pb][kLists + L];
     }
-    __syncthreads();  // sel_* are rewritten by the next pass
   }
+  __syncthreads();  // hist and pick free for the caller
 #pragma unroll
   for (int L = 0; L < kLists; L++) out[L] = prefix[L];
 }
@@ -403,40 +423,39 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
   const RankSet &S = sets[blockIdx.y];
   const uint32_t c = blockIdx.x;  // this CTA's share of the sample
   __shared__ uint64_t t2s[kLutN], mgs[kLutN];
-  __shared__ unsigned int hist[kLists][256];
-  __shared__ unsigned int ecount[kLists], sel_digit[kLists], sel_need[kLists], wpos[kLists];
+  __shared__ unsigned int hist[2][kLists][256];
+  __shared__ unsigned int pick[2][2 * kLists];
+  __shared__ unsigned int ecount[kLists], wpos[kLists];
   __shared__ unsigned int is_last;
   const uint32_t tid = threadIdx.x, lane = tid & 31;
   if (tid < kLutN) {
-    const uint32_t sg = S.sigma[tid];
-    t2s[tid] = ((uint64_t)(kLambda - sg) * S.penalty) / kLambda;  // eq. (t2)
-    mgs[tid] = magic_for(sg);
+    t2s[tid] = S.t2v[tid];
+    mgs[tid] = S.mgv[tid];
   }
   if (tid < kLists) {
     ecount[tid] = 0;
     wpos[tid] = 0;
   }
   __syncthreads();
-  const uint32_t n = S.n;
-  const uint32_t ns = sample_size(S);
+  const uint32_t ns = S.ns, act = S.act;
   const uint32_t per = ns / kSampleCtas;  // samples of this CTA (<= 1024, a multiple of 8)
-  const uint32_t act = (list_active(S, 0) ? 1u : 0u) | (list_active(S, 1) ? 2u : 0u) | (list_active(S, 2) ? 4u : 0u);
   uint32_t rL[kLists];
 #pragma unroll
-  for (int L = 0; L < kLists; L++)
-    rL[L] = (ns && ((act >> L) & 1)) ? (uint32_t)umin64((list_target(S, L) * ns + n - 1) / n, kMaxR) : 0u;
+  for (int L = 0; L < kLists; L++) rL[L] = S.rL[L];
   // 1. this thread's sample
   uint32_t f[kLists][1] = {{0}, {0}, {0}};
   uint32_t m = 0;
   if (tid < per) {
-    const uint32_t nruns = ns / 8, run = c * (per / 8) + tid / 8, o = tid % 8;
-    const uint64_t lo = ((uint64_t)run * n) / nruns, hi = ((uint64_t)(run + 1) * n) / nruns;
+    // stratum bounds floor(run n / nruns) with n = sq nruns + srem, in 32 bits
+    const uint32_t nruns = S.nruns, run = c * (per / 8) + tid / 8, o = tid % 8;
+    const uint32_t lo = run * S.sq + (run * S.srem) / nruns;
+    const uint32_t hi = (run + 1) * S.sq + ((run + 1) * S.srem) / nruns;
     uint32_t h = run * 0x9E3779B1u;
     h ^= h >> 16;
     h *= 0x85EBCA6Bu;
     h ^= h >> 13;
-    const uint32_t span = (uint32_t)(hi - lo) - 8;  // strata hold at least 8 records
-    const uint32_t r = (uint32_t)(lo + (h % (span + 1))) + o;
+    const uint32_t span = hi - lo - 8;  // strata hold at least 8 records
+    const uint32_t r = lo + (h % (span + 1)) + o;
     const uint8_t fl = S.flags[r], tr = S.tier[r];
     const uint32_t t = min((uint32_t)S.turn[r], kTMax);
     const uint64_t ck = ck_of(score_of(S.gap[r], t, (fl & 2) != 0, t2s, mgs), r);
@@ -458,21 +477,30 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
     need[L] = rL[L];
     if (rL[L] && ecount[L] > rL[L]) sel |= 1u << L;
   }
-  if (sel) joint_select32<1>(f, m, sel, need, T, hist, sel_digit, sel_need);
+  if (sel) joint_select32<1>(f, m, sel, need, T, hist, pick);
 #pragma unroll
   for (int L = 0; L < kLists; L++) {
     if (!rL[L]) continue;
-    uint32_t *dst = S.part + ((size_t)L * kSampleCtas + c) * kMaxR;
     const bool all = !((sel >> L) & 1);  // keep every eligible sample
     const bool has = (m >> L) & 1;
-    if (has && (all || f[L][0] > T[L])) dst[atomicAdd(&wpos[L], 1u)] = f[L][0];
-    __syncthreads();
-    if (tid == 0) {
-      const uint32_t above = wpos[L];
-      const uint32_t total = all ? above : rL[L];
-      for (uint32_t q = above; q < total; q++) dst[q] = T[L];  // ties at the rank-r_L summary
-      S.part_n[L * kSampleCtas + c] = total;
-    }
+    const bool above = has && (all || f[L][0] > T[L]);
+    const unsigned bal = __ballot_sync(kFull, above);
+    unsigned wbase = 0;
+    if (lane == 0 && bal) wbase = atomicAdd(&wpos[L], (unsigned)__popc(bal));
+    wbase = __shfl_sync(kFull, wbase, 0);
+    uint32_t *dst = S.part + ((size_t)L * kSampleCtas + c) * kMaxR;
+    if (above) dst[wbase + __popc(bal & ((1u << lane) - 1))] = f[L][0];
+  }
+  __syncthreads();
+  // ties at the rank-r_L summary fill each partial list up to r_L entries
+#pragma unroll
+  for (int L = 0; L < kLists; L++) {
+    if (!rL[L]) continue;
+    const bool all = !((sel >> L) & 1);
+    const uint32_t nab = wpos[L], total = all ? nab : rL[L];
+    uint32_t *dst = S.part + ((size_t)L * kSampleCtas + c) * kMaxR;
+    for (uint32_t q = nab + tid; q < total; q += kSampleThreads) dst[q] = T[L];
+    if (tid == 0) S.part_n[L * kSampleCtas + c] = total;
   }
   // 3. the last CTA to finish merges the partial lists and sets the thresholds
   __threadfence();
@@ -481,38 +509,46 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
   __syncthreads();
   if (!is_last) return;
   __threadfence();
-  if (tid < kLutN) {
-    S.t2[tid] = t2s[tid];
-    S.magic[tid] = mgs[tid];
-  }
   // entry counts of the partial lists, then kSampleCtas * r_L <= 4096
-  // entries per list: four per thread
+  // entries per list: one per thread when they fit, else four per thread
   __shared__ unsigned int pn[kLists * kSampleCtas];
   if (tid < kLists * kSampleCtas) pn[tid] = __ldcg(&S.part_n[tid]);
   __syncthreads();
-  uint32_t v4[kLists][4];
-  uint32_t has4 = 0, sel2 = 0;
+  uint32_t rmax = 0, sel2 = 0;
 #pragma unroll
   for (int L = 0; L < kLists; L++) {
-#pragma unroll
-    for (int q = 0; q < 4; q++) v4[L][q] = 0;
+    rmax = max(rmax, rL[L]);
     if (!rL[L]) continue;
-    // entry e of the concatenation: CTA e / kMaxR, slot e % kMaxR
-#pragma unroll
-    for (int q = 0; q < 4; q++) {
-      const uint32_t e = tid + 1024u * q;
-      const uint32_t cc = e / kMaxR, slot = e % kMaxR;
-      if (cc < kSampleCtas && slot < pn[L * kSampleCtas + cc]) {
-        v4[L][q] = __ldcg(&S.part[((size_t)L * kSampleCtas + cc) * kMaxR + slot]);
-        has4 |= 1u << (L * 4 + q);
-      }
-    }
     uint32_t cnt = 0;
     for (uint32_t cc = 0; cc < kSampleCtas; cc++) cnt += pn[L * kSampleCtas + cc];
     if (cnt >= rL[L]) sel2 |= 1u << L;
   }
   uint32_t T2[kLists] = {0, 0, 0};
-  if (sel2) joint_select32<4>(v4, has4, sel2, rL, T2, hist, sel_digit, sel_need);
+  auto merge = [&](auto qtag) {
+    constexpr int Q = decltype(qtag)::value;
+    uint32_t vq[kLists][Q];
+    uint32_t hq = 0;
+#pragma unroll
+    for (int L = 0; L < kLists; L++) {
+#pragma unroll
+      for (int q = 0; q < Q; q++) {
+        vq[L][q] = 0;
+        // entry e of the concatenation: CTA e / r_L, slot e % r_L
+        const uint32_t e = tid + kSampleThreads * q;
+        if (!rL[L]) continue;
+        const uint32_t cc = e / rL[L], slot = e % rL[L];
+        if (cc < kSampleCtas && slot < pn[L * kSampleCtas + cc]) {
+          vq[L][q] = __ldcg(&S.part[((size_t)L * kSampleCtas + cc) * kMaxR + slot]);
+          hq |= 1u << (L * Q + q);
+        }
+      }
+    }
+    joint_select32<Q>(vq, hq, sel2, rL, T2, hist, pick);
+  };
+  if (sel2) {
+    if (kSampleCtas * rmax <= kSampleThreads) merge(std::integral_constant<int, 1>());
+    else merge(std::integral_constant<int, 4>());
+  }
 #pragma unroll
   for (int L = 0; L < kLists; L++) {
     // 0 (fewer than r_L eligible samples, or none taken): accept every eligible record
@@ -649,8 +685,8 @@ __device__ void load_set(const RankSet &S, uint4 *vd, uint2 *pp, uint64_t *t2s, 
     const uint2 a0 = S.gthr[t], a1 = S.gthr[kLutN + t], a2 = S.gthr[2 * kLutN + t];
     vd[t] = make_uint4(aV ? a0.x : kFull, aV ? a0.y : kFull, aD ? a1.x : kFull, aD ? a1.y : kFull);
     pp[t] = aP ? a2 : make_uint2(0u, 0u);
-    t2s[t] = S.t2[t];
-    mgs[t] = S.magic[t];
+    t2s[t] = S.t2v[t];
+    mgs[t] = S.mgv[t];
   }
   uint32_t lo[kLists], dok[kLists];
 #pragma unroll
@@ -1048,8 +1084,8 @@ __device__ void block_scan_pairs(Sum (&a)[kIpt], int64_t (&b)[kIpt], Sum *wa, in
 // Exact top-M of list L over the whole set by one CTA, streaming records and
 // keeping a pool of at most M + 4096 values (the fallback path).
 __device__ uint32_t stream_topM(const RankSet &S, int L, uint32_t M, uint64_t *pool, const uint64_t *t2s,
-                                const uint64_t *mgs, unsigned int *hist, unsigned long long *bcast,
-                                unsigned int *cnt) {
+                                const uint64_t *mgs, unsigned int (*hist)[256], unsigned int (*pick)[2],
+                                unsigned long long *bcast, unsigned int *cnt) {
   if (threadIdx.x == 0) *cnt = 0;
   uint64_t floorv = 0;  // accept values strictly above (0 = accept all but 0)
   bool have_floor = false;
@@ -1072,7 +1108,7 @@ __device__ uint32_t stream_topM(const RankSet &S, int L, uint32_t M, uint64_t *p
     __syncthreads();
     const uint32_t c = min(*cnt, kSmemCand);
     if (c > M) {
-      const uint64_t th = block_select_rank([&](uint32_t i) { return pool[i]; }, c, M, hist, bcast);
+      const uint64_t th = block_select_rank([&](uint32_t i) { return pool[i]; }, c, M, hist, pick, bcast);
       // compact in place: values >= th (exactly M, values are unique)
       __syncthreads();
       if (threadIdx.x == 0) *cnt = 0;
@@ -1103,12 +1139,14 @@ __global__ void __launch_bounds__(kFinishThreads) rank_finish_kernel(const RankS
   uint64_t *buf = reinterpret_cast<uint64_t *>(smem);   // [kSmemCand]
   uint64_t *sel = buf + kSmemCand;                      // [kMaxSel]
   __shared__ uint64_t t2s[kLutN], mgs[kLutN];
-  __shared__ unsigned int hist[256];
+  __shared__ unsigned int hist[2][256];
+  __shared__ unsigned int pick[2][2];
   __shared__ unsigned long long bcast[2];
+  __shared__ __align__(8) uint64_t cbar;
   __shared__ unsigned int cnt, is_last;
   if (threadIdx.x < kLutN) {
-    t2s[threadIdx.x] = S.t2[threadIdx.x];
-    mgs[threadIdx.x] = S.magic[threadIdx.x];
+    t2s[threadIdx.x] = S.t2v[threadIdx.x];
+    mgs[threadIdx.x] = S.mgv[threadIdx.x];
   }
   __syncthreads();
   {
@@ -1129,31 +1167,56 @@ __global__ void __launch_bounds__(kFinishThreads) rank_finish_kernel(const RankS
         const uint32_t c = emitted;
         const uint64_t *src = cand;
         if (c <= kSmemCand) {
-          for (uint32_t i = threadIdx.x; i < c; i += blockDim.x) buf[i] = cand[i];
+          // one bulk copy (an even count: 16-byte multiple; the buffer holds
+          // kCandCap >= c + 1 entries)
+          const uint32_t bytes = ((c + 1) & ~1u) * 8u;
+          if (threadIdx.x == 0) {
+            mbar_init(&cbar, 1);
+            fence_mbar_init();
+            mbar_expect_tx(&cbar, bytes);
+            bulk_g2s(buf, cand, bytes, &cbar);
+          }
           __syncthreads();
+          if (!mbar_wait_bounded(&cbar, 0)) {
+            atomicExch(&S.work->status, (unsigned int)UNISON_ERR_TIMEOUT);
+            mbar_wait_bounded(&cbar, 0);  // let the copy land before the buffer is reused
+          }
           src = buf;
         }
         uint64_t th = 0;
-        if (c > M) th = block_select_rank([&](uint32_t i) { return src[i]; }, c, M, hist, bcast);
+        if (c > M) th = block_select_rank([&](uint32_t i) { return src[i]; }, c, M, hist, pick, bcast);
         if (threadIdx.x == 0) cnt = 0;
         __syncthreads();
-        for (uint32_t i = threadIdx.x; i < c; i += blockDim.x) {
-          const uint64_t v = src[i];
-          if (c <= M || v >= th) {
-            const uint32_t pos = atomicAdd(&cnt, 1u);
-            if (pos < kMaxSel) sel[pos] = v;
-          }
+        // keep the values at or above the rank-M value (exactly M: values are
+        // unique), warp-aggregated appends
+        const uint32_t lane = threadIdx.x & 31;
+        for (uint32_t base = 0; base < c; base += blockDim.x) {
+          const uint32_t i = base + threadIdx.x;
+          const uint64_t v = i < c ? src[i] : 0ull;
+          const bool keep = i < c && (c <= M || v >= th);
+          const unsigned bal = __ballot_sync(kFull, keep);
+          unsigned wb = 0;
+          if (lane == 0 && bal) wb = atomicAdd(&cnt, (unsigned)__popc(bal));
+          wb = __shfl_sync(kFull, wb, 0);
+          const uint32_t pos = wb + __popc(bal & ((1u << lane) - 1));
+          if (keep && pos < kMaxSel) sel[pos] = v;
         }
         __syncthreads();
         got = min(cnt, M);
       } else {
         // candidates overflowed the buffer or fell short of M: exact re-selection
-        got = stream_topM(S, L, M, buf, t2s, mgs, hist, bcast, &cnt);
+        got = stream_topM(S, L, M, buf, t2s, mgs, hist, pick, bcast, &cnt);
         for (uint32_t i = threadIdx.x; i < got; i += blockDim.x) sel[i] = buf[i];
         __syncthreads();
       }
-      block_sort_desc(sel, got);
-      for (uint32_t i = threadIdx.x; i < got; i += blockDim.x) S.sorted[(size_t)L * kMaxSel + i] = sel[i];
+      block_sort_desc(sel, got, buf);
+      for (uint32_t i = threadIdx.x; i < got; i += blockDim.x) {
+        const uint64_t v = sel[i];
+        S.sorted[(size_t)L * kMaxSel + i] = v;
+        // the fill reads the moved records' sizes: look them up here, in
+        // parallel with the other lists
+        if (L != 0) S.ssz[(size_t)L * kMaxSel + i] = S.kv[(~(uint32_t)(L == 2 ? ~v : v)) & kIdMask];
+      }
     }
     if (threadIdx.x == 0) S.work->got[L] = got;
   }
@@ -1178,14 +1241,12 @@ __global__ void __launch_bounds__(kFinishThreads) rank_finish_kernel(const RankS
   uint32_t *dsz = psz + kMaxSel;
   uint32_t *dsz2 = dsz + kMaxSel;
   for (uint32_t i = threadIdx.x; i < np; i += blockDim.x) {
-    const uint64_t ck = ~__ldcg(&P[i]);
-    pck[i] = ck;
-    psz[i] = S.kv[(~(uint32_t)ck) & kIdMask];
+    pck[i] = ~__ldcg(&P[i]);
+    psz[i] = __ldcg(&S.ssz[2 * kMaxSel + i]);
   }
   for (uint32_t i = threadIdx.x; i < nd; i += blockDim.x) {
-    const uint64_t d = __ldcg(&D[i]);
-    dck[i] = d;
-    dsz[i] = S.kv[(~(uint32_t)d) & kIdMask];
+    dck[i] = __ldcg(&D[i]);
+    dsz[i] = __ldcg(&S.ssz[kMaxSel + i]);
   }
   __syncthreads();
   // Both fill phases take items in order and stop at the first that does not
@@ -1354,14 +1415,28 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
     s.tile0 = tiles;
     s.ntiles = (uint32_t)((r.n + kBigTile - 1) / kBigTile);
     tiles += s.ntiles;
-    for (int t = 0; t < (int)kLutN; t++) s.sigma[t] = p.sigma_q[t];
-    s.pad = 0;
+    for (int t = 0; t < (int)kLutN; t++) {
+      s.sigma[t] = p.sigma_q[t];
+      s.t2v[t] = ((uint64_t)(kLambda - p.sigma_q[t]) * p.penalty_q) / kLambda;  // eq. (t2)
+      s.mgv[t] = magic_for(p.sigma_q[t]);
+    }
+    s.ns = sample_size(s);
+    s.nruns = s.ns / 8;
+    s.sq = s.nruns ? s.n / s.nruns : 0;
+    s.srem = s.nruns ? s.n % s.nruns : 0;
+    s.act = 0;
+    for (int L = 0; L < kLists; L++) {
+      s.act |= list_active(s, L) ? 1u << L : 0u;
+      s.rL[L] = (s.ns && list_active(s, L))
+                    ? (uint32_t)umin64((list_target(s, L) * s.ns + s.n - 1) / s.n, kMaxR) : 0u;
+    }
   }
   // scratch: descriptors, then per set: work, thresholds, tables, sorted
   // lists, candidates, the sample's partial lists
   const size_t per_set = align_up(sizeof(RankWork), 256) + align_up(sizeof(uint64_t) * 2 * kLists, 256) +
-                         align_up(sizeof(uint2) * kLists * kLutN, 256) + 2 * align_up(sizeof(uint64_t) * kLutN, 256) +
+                         align_up(sizeof(uint2) * kLists * kLutN, 256) +
                          align_up(sizeof(uint64_t) * kLists * kMaxSel, 256) +
+                         align_up(sizeof(uint32_t) * kLists * kMaxSel, 256) +
                          align_up(sizeof(uint64_t) * kLists * kCandCap, 256) +
                          align_up(sizeof(uint32_t) * kLists * kSampleCtas * kMaxR, 256) +
                          align_up(sizeof(uint32_t) * kLists * kSampleCtas, 256);
@@ -1380,12 +1455,10 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
     p += align_up(sizeof(uint64_t) * 2 * kLists, 256);
     s.gthr = reinterpret_cast<uint2 *>(p);
     p += align_up(sizeof(uint2) * kLists * kLutN, 256);
-    s.t2 = reinterpret_cast<uint64_t *>(p);
-    p += align_up(sizeof(uint64_t) * kLutN, 256);
-    s.magic = reinterpret_cast<uint64_t *>(p);
-    p += align_up(sizeof(uint64_t) * kLutN, 256);
     s.sorted = reinterpret_cast<uint64_t *>(p);
     p += align_up(sizeof(uint64_t) * kLists * kMaxSel, 256);
+    s.ssz = reinterpret_cast<uint32_t *>(p);
+    p += align_up(sizeof(uint32_t) * kLists * kMaxSel, 256);
     s.cand = reinterpret_cast<uint64_t *>(p);
     p += align_up(sizeof(uint64_t) * kLists * kCandCap, 256);
     s.part = reinterpret_cast<uint32_t *>(p);
