@@ -30,6 +30,25 @@ sys.path.insert(0, os.path.join(ROOT, "tests"))
 METRIC = "replay events/s (SPEAR+TIDE batched)"
 
 
+def filter_traffic(records_per_launch: int):
+    """DRAM bytes (read + write) per rank_filter launch from the ncu capture
+    summarised in profiles/rank_filter_2p24_ncu.md, scaled from one 2^24 set
+    to the launch's records; None when rank.cu has changed since the capture
+    (its hash no longer matches the recorded one) or the record is missing."""
+    import hashlib
+    try:
+        text = open(os.path.join(ROOT, "profiles", "rank_filter_2p24_ncu.md")).read()
+        line = next(l for l in text.splitlines() if l.startswith("traffic-record:"))
+        rec = dict(kv.split("=") for kv in line.split()[1:])
+        src = open(os.path.join(ROOT, "paper_2609_09643_gb300", "csrc", "rank.cu"), "rb").read()
+        if hashlib.sha256(src).hexdigest()[:16] != rec["rank.cu-sha256-16"]:
+            return None
+        per_set = int(rec["dram_read_bytes_per_set"]) + int(rec["dram_write_bytes_per_set"])
+        return per_set * records_per_launch / int(rec["records_per_set"])
+    except (OSError, StopIteration, KeyError, ValueError):
+        return None
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -104,11 +123,14 @@ class ClockSampler:
 
 # ------------------------------------------------------------- workloads ----
 def sweep_workload(rank: int):
+    """The 1,024-replay sweep; under torchrun each rank replays it on its own
+    trace seeds (rank 0: seeds 0-7, the single-GPU workload)."""
     from cases import sweep_case, to_lib
+    import synth
+    from paper_2609_09643_gb300 import shard
     trs, reps = sweep_case()
-    if rank:  # weak scaling: each rank replays its own seeds
-        import synth
-        trs = [synth.paper_scale_trace(8 * rank + i, "coding") for i in range(len(trs))]
+    if rank:
+        trs = [synth.paper_scale_trace(s, "coding") for s in shard.rank_seeds(rank)]
     return trs, reps, [to_lib(p, ti) for ti, p in reps]
 
 
@@ -286,11 +308,10 @@ def main():
     rn_ms, rn_n = B.profile_read("rank_finish", reset=True)
     B.profile_enable(False)
     clocks = clk.stop()
-    if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
-    value = world * events_per_step * args.steps / (ms / 1e3) if not args.rank_only else None
+    from paper_2609_09643_gb300 import shard
+    ms = shard.max_over_ranks(ms, device="cuda")
+    units = shard.units_over_ranks(events_per_step, device="cuda")
+    value = shard.job_rate(units, args.steps, ms) if not args.rank_only else None
 
     # end to end through the public API: host trace staging -> device, replay,
     # results back to the host, every step
@@ -313,11 +334,14 @@ def main():
             _ = [B.rank_result(o) for o in rank_outs]
         torch.cuda.synchronize()
         dt = time.perf_counter() - t0
-        e2e = {"value": world * events_per_step * args.steps / dt, "unit": "events/s",
+        e2e = {"value": shard.job_rate(units, args.steps, 1e3 * shard.max_over_ranks(dt, device="cuda")),
+               "unit": "events/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
     avg_rep_ms = rep_ms / max(rep_n, 1) if rep_n else float("nan")
-    alg_bytes = events_per_step * 32  # 16 B event + 4 B prev size + 8 B key + 4 B gap average
+    # 16 B event + 4 B previous size + 8 B key + 4 B gap average + 8 B key
+    # before each arrival (half the events): 36 B/event
+    alg_bytes = events_per_step * 36
     replay_roof = None if not rep_n else {"bound": "latency", "kernel": "replay_kernel", "avg_ms": avg_rep_ms,
                    "ns_per_event_per_replay": 1e6 * avg_rep_ms / (events_per_step / n_rep),
                    "hbm_gbs": alg_bytes / (avg_rep_ms / 1e3) / 1e9, "launches_timed": rep_n,
@@ -334,7 +358,9 @@ def main():
     roofline = {"bound": "hbm", "kernel": "rank_filter_kernel", "achieved": achieved, "peak": hbm_peak,
                 "unit": "GB/s", "frac": achieved / hbm_peak,
                 "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs, burst copy)" if peaks.get("hbm_gbs")
-                else "fallback 6.8 TB/s", "traffic": None, "avg_ms": avg_rf, "launches_timed": rf_n,
+                else "fallback 6.8 TB/s", "traffic": filter_traffic(len(r_params) * RANK_N),
+                "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum of one 2^24 set, scaled by records",
+                "avg_ms": avg_rf, "launches_timed": rf_n,
                 "algorithmic_bytes_per_launch": rank_bytes,
                 "bytes_per_record": RANK_BYTES_PER_RECORD, "records_per_launch": len(r_params) * RANK_N}
     call_ms = (rs_ms + rf_ms + rn_ms) / max(rf_n, 1) if rf_n else float("nan")

@@ -12,10 +12,11 @@
 //                       the event loop re-ranks from these values instead of
 //                       re-dividing every live score at every event; the
 //                       decisions are identical.
-//   replay_kernel       Algorithm 1: one warp per replay, resident sessions of
-//                       each tier held structure-of-arrays in shared memory,
-//                       every decision a warp-wide scan + shuffle/redux argmax
-//                       (or argmin) over the packed 64-bit keys.
+//   replay_kernel       Algorithm 1: one warp per replay; the unpinned
+//                       residents of each tier kept sorted by packed 64-bit
+//                       key in shared memory (the most evictable last), so
+//                       the argmax of a decision is a pop and an update is a
+//                       warp-parallel lower bound plus a block shift.
 //   ttft_median_kernel  Sec. V-A TTFT p50: radix select of the lower median
 //                       over each replay's per-request TTFT values.
 #include <algorithm>
