@@ -62,6 +62,7 @@ def parse():
     ap.add_argument("--replays", type=int, default=1024, help="first N replays of the sweep (profiling)")
     ap.add_argument("--rank-n", type=int, default=1 << 24, help="records per live set")
     ap.add_argument("--rank-sets", type=int, default=7, help="live sets per call (<= 7)")
+    ap.add_argument("--no-rank-sizes", action="store_true", help="skip the live-set size sweep")
     return ap.parse_args()
 
 
@@ -153,6 +154,57 @@ def rank_workload():
 def rank_params(sigma, n_sets=7):
     return [dict(sigma_q=sigma, k=1024, penalty_q=500_000_000, budget_bytes=b << 30, kv_bytes_per_token=131072,
                  max_moves=1024, free_fast_tok=0, free_hbm_tok=1 << 40) for b in RANK_BUDGETS_GIB[:n_sets]]
+
+
+RANK_SIZES = (1 << 10, 1 << 14, 1 << 18, 1 << 20, 1 << 22, 1 << 24)
+RANK_KS = (1, 2, 4, 8, 16, 32, 64, 128, 256, 512, 1024)
+
+
+def rank_size_sweep(B, host_rec, sigma, stream, steps: int = 10, warmup: int = 3):
+    """The live-set sizes of the ranking microbenchmark.  At each size one call
+    ranks enough distinct sets (slices of the 2^24-record set, at most 64) to
+    stream at least 2x the 129 MB L2, so no set is re-read from L2 between
+    calls; k cycles through 1..1,024 and the budget through 1..64 GiB.
+    Call time = CUDA events around the call on its stream."""
+    import torch
+    out = []
+    full = {k: v.to("cuda", non_blocking=True) for k, v in host_rec.items()}
+    total = int(full["gap_q"].numel())
+    for n in RANK_SIZES:
+        n_sets = max(1, min(64, -(-(2 * 129 << 20) // (n * RANK_BYTES_PER_RECORD))))
+        sets, params, outs = [], [], []
+        for i in range(n_sets):
+            off = (i * n) % total if n * n_sets <= total else 0
+            if n * n_sets <= total:
+                sets.append({k: v[off:off + n] for k, v in full.items()})
+            else:  # more records than the 2^24 set holds: separate copies
+                sets.append({k: v[:n].clone() for k, v in full.items()})
+            k = RANK_KS[i % len(RANK_KS)]
+            params.append(dict(sigma_q=sigma, k=k, penalty_q=500_000_000,
+                               budget_bytes=RANK_BUDGETS_GIB[i % len(RANK_BUDGETS_GIB)] << 30,
+                               kv_bytes_per_token=131072, max_moves=1024, free_fast_tok=0, free_hbm_tok=1 << 40))
+            outs.append(B.rank_outputs(n, k, 1024))
+        call = B.rank_prepare(sets, params, outs)  # marshalled once: the loop times the device
+        for _ in range(warmup):
+            call.run(stream)
+        torch.cuda.synchronize()
+        assert all(B.rank_result(o)["status"] == 0 for o in outs), "rank status"
+        B.profile_read("rank_filter", reset=True)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps):
+            call.run(stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        call_us = 1e3 * e0.elapsed_time(e1) / steps
+        f_ms, f_n = B.profile_read("rank_filter", reset=True)
+        recs = n * n_sets
+        gbs = recs * RANK_BYTES_PER_RECORD / (call_us / 1e6) / 1e9
+        out.append({"n": n, "sets_per_call": n_sets, "call_us": call_us,
+                    "filter_us": 1e3 * f_ms / max(f_n, 1) if f_n else None, "call_gbs": gbs,
+                    "l2_resident": recs * RANK_BYTES_PER_RECORD < (2 * 129 << 20)})
+        del call, sets, outs
+    return out
 
 
 def cpu_baseline_replay(trs, reps, budget_s: float = 12.0):
@@ -313,6 +365,15 @@ def main():
     units = shard.units_over_ranks(events_per_step, device="cuda")
     value = shard.job_rate(units, args.steps, ms) if not args.rank_only else None
 
+    sizes = None
+    if not args.replay_only and not args.no_rank_sizes:
+        B.profile_enable(True)
+        sizes = rank_size_sweep(B, host_rec, sigma, stream)
+        B.profile_enable(False)
+        for e in sizes:
+            e["call_frac_of_peak"] = e["call_gbs"] / (json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+                                                      .get("hbm_gbs") or 6800.0)
+
     # end to end through the public API: host trace staging -> device, replay,
     # results back to the host, every step
     e2e = None
@@ -380,7 +441,7 @@ def main():
                                    "paper-scale coding trace, 131072 B/token, SPEAR+TIDE)",
                        "replays": n_rep, "events_per_step": events_per_step,
                        "l2": "flushed before every step (256 MiB write, inside the timed region)"},
-            "roofline": roofline, "rank": rank_leg, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roofline, "rank": rank_leg, "rank_sizes": sizes, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches, "clocks": clocks,
             "peaks": {"hbm_gbs": peaks.get("hbm_gbs"), "source": "MEASURED_PEAKS.json"}}
     if cpu is not None:

@@ -338,25 +338,47 @@ def rank_outputs(n: int, k: int, max_moves: int, keys: bool = False, device="cud
                 counts=z(4, torch.int32), moved=z(1, torch.int64), keys=z(n, torch.int64) if keys else None)
 
 
+class RankCall:
+    """The marshalled arguments of one unison_rank_batch call (ctypes arrays
+    over the tensors' device pointers), reusable while those tensors live."""
+
+    def __init__(self, sets: Sequence[dict], params: Sequence[dict], outs: Sequence[dict]):
+        n = len(sets)
+        self.n = n
+        self.rs = (Records * n)()
+        self.ps = (RankParams * n)()
+        self.os = (RankOut * n)()
+        self._keep = (list(sets), list(outs))  # the pointers stay valid while these live
+        for i, (r, p, o) in enumerate(zip(sets, params, outs)):
+            self.rs[i] = Records(r["gap_q"].data_ptr(), r["last_ret"].data_ptr(), r["turn"].data_ptr(),
+                                 r["kv_tok"].data_ptr(), r["tier"].data_ptr(), r["flags"].data_ptr(),
+                                 r["gap_q"].numel())
+            sig = np.ascontiguousarray(np.asarray(p["sigma_q"], dtype=np.uint16))
+            if sig.shape != (51,):
+                raise ValueError("sigma_q must have 51 entries")
+            self.ps[i] = RankParams((C.c_uint16 * 51).from_buffer_copy(sig.tobytes()), 0, p.get("k", 0),
+                                    p.get("penalty_q", 500_000_000), p.get("budget_bytes", 0),
+                                    p.get("kv_bytes_per_token", 131072), p.get("max_moves", 0),
+                                    p.get("free_fast_tok", 0), p.get("free_hbm_tok", 0))
+            self.os[i] = RankOut(o["victims"].data_ptr(), o["promote"].data_ptr(), o["demote"].data_ptr(),
+                                 o["counts"].data_ptr(), o["moved"].data_ptr(),
+                                 None if o.get("keys") is None else o["keys"].data_ptr())
+
+    def run(self, stream=None) -> None:
+        _check("unison_rank_batch", lib().unison_rank_batch(self.rs, self.ps, self.os, self.n,
+                                                            _stream_handle(stream)))
+
+
+def rank_prepare(sets: Sequence[dict], params: Sequence[dict], outs: Sequence[dict]) -> RankCall:
+    """Marshal a rank call once (see RankCall) for repeated launches."""
+    return RankCall(sets, params, outs)
+
+
 def rank_batch(sets: Sequence[dict], params: Sequence[dict], outs: Sequence[dict], stream=None) -> None:
     """unison_rank_batch over device record sets; params per set: sigma_q[51],
     k, penalty_q, budget_bytes, kv_bytes_per_token, max_moves, free_fast_tok,
     free_hbm_tok."""
-    n = len(sets)
-    rs = (Records * n)()
-    ps = (RankParams * n)()
-    os_ = (RankOut * n)()
-    for i, (r, p, o) in enumerate(zip(sets, params, outs)):
-        rs[i] = Records(r["gap_q"].data_ptr(), r["last_ret"].data_ptr(), r["turn"].data_ptr(),
-                        r["kv_tok"].data_ptr(), r["tier"].data_ptr(), r["flags"].data_ptr(), r["gap_q"].numel())
-        sig = (C.c_uint16 * 51)(*[int(x) for x in p["sigma_q"]])
-        ps[i] = RankParams(sig, 0, p.get("k", 0), p.get("penalty_q", 500_000_000), p.get("budget_bytes", 0),
-                           p.get("kv_bytes_per_token", 131072), p.get("max_moves", 0), p.get("free_fast_tok", 0),
-                           p.get("free_hbm_tok", 0))
-        os_[i] = RankOut(o["victims"].data_ptr(), o["promote"].data_ptr(), o["demote"].data_ptr(),
-                         o["counts"].data_ptr(), o["moved"].data_ptr(),
-                         None if o.get("keys") is None else o["keys"].data_ptr())
-    _check("unison_rank_batch", lib().unison_rank_batch(rs, ps, os_, n, _stream_handle(stream)))
+    RankCall(sets, params, outs).run(stream)
 
 
 def rank_result(o: dict) -> dict:

@@ -24,6 +24,7 @@
 //                        set.  The set's last CTA writes the victims and runs
 //                        the fill as warp prefix scans.
 #include <algorithm>
+#include <mutex>
 #include <type_traits>
 #include <vector>
 
@@ -68,6 +69,8 @@ struct RankSet {
   uint32_t sigma[kLutN];
   // per-set constants, computed on the host
   uint32_t ns, nruns, sq, srem;  // sample size, its runs of 8, n = sq * nruns + srem
+  uint32_t sctas;                // sample CTAs (at most kSampleCtas)
+  uint32_t cta0, nctas;           // filter, group mode: CTAs [cta0, cta0 + nctas) stream this set
   uint32_t act;                  // active lists (bit L)
   uint32_t rL[kLists];           // sample rank of each list's threshold
   uint64_t t2v[kLutN];           // eq. (t2) per turn index
@@ -283,27 +286,45 @@ __device__ __forceinline__ uint64_t list_val(uint64_t ck, int L) { return L == 2
 
 // ------------------------------------------------------------- sample ----
 // Sample size and per-list ranks: ns records (ns/8 runs of 8, one run per
-// stratum) and rank r_L = ceil(target_L * ns / n), with ns chosen so that no
-// r_L exceeds kMaxR; target_L = 6 M_L + 2048 candidates for M_L needed.
+// stratum) and rank r_L = ceil(target_L * ns / n), with ns about kSampleRank
+// times n over the largest target, capped at kSample; the sample is split over
+// ceil(ns / 1024) CTAs.  Candidates above the rank-r_L sample value number
+// about target_L / r_L * Gamma(r_L), and fall short of M_L with probability
+// P(Gamma(r_L) < r_L M_L / target_L).  Targets: 2 M + 1024 while the sample
+// is not capped (r = 32 for the largest list: below 1e-6), else 6 M + 2048
+// (r >= 8 at 2^24 records: about 1e-5).  A shortfall costs time, never
+// exactness (the finish re-selects the list).
+constexpr uint32_t kSampleRank = 32;
 __host__ __device__ __forceinline__ uint64_t umin64(uint64_t a, uint64_t b) { return a < b ? a : b; }
-__host__ __device__ __forceinline__ uint64_t list_target(const RankSet &S, int L) {
-  const uint32_t M = (L == 0) ? S.k : S.max_moves;
-  return 6ull * M + 2048;
-}
 __host__ __device__ __forceinline__ bool list_active(const RankSet &S, int L) {
   const uint32_t M = (L == 0) ? S.k : S.max_moves;
   return M > 0 && (L == 0 || S.budget > 0);
 }
-__host__ __device__ __forceinline__ uint32_t sample_size(const RankSet &S) {
-  const uint32_t n = S.n;
-  if (n <= kSample) return 0;  // whole set: every eligible record is a candidate
+__host__ __device__ __forceinline__ uint64_t list_target_of(const RankSet &S, int L, bool wide) {
+  const uint32_t M = (L == 0) ? S.k : S.max_moves;
+  return wide ? 6ull * M + 2048 : 2ull * M + 1024;
+}
+__host__ __device__ __forceinline__ uint32_t sample_ctas(uint32_t ns) {
+  return ns ? (ns + kSampleThreads - 1) / kSampleThreads : 1u;
+}
+// Sample size for the given targets (0: no sample, the whole set qualifies).
+__host__ __device__ __forceinline__ uint64_t sample_size_raw(const RankSet &S, bool wide) {
+  if (S.n <= kSample) return 0;
   uint64_t tmax = 0;
   for (int L = 0; L < kLists; L++)
-    if (list_active(S, L) && list_target(S, L) > tmax) tmax = list_target(S, L);
+    if (list_active(S, L) && list_target_of(S, L, wide) > tmax) tmax = list_target_of(S, L, wide);
   if (tmax == 0) return 0;
-  uint64_t ns = ((uint64_t)kMaxR * n) / tmax;
-  ns = ns < kSample ? ns : kSample;
-  ns &= ~(uint64_t)(8 * kSampleCtas - 1);  // whole runs, evenly split over the CTAs
+  return ((uint64_t)kSampleRank * S.n) / tmax;
+}
+// The narrow targets unless their sample would exceed the cap.
+__host__ __device__ __forceinline__ bool wide_targets(const RankSet &S) { return sample_size_raw(S, false) > kSample; }
+__host__ __device__ __forceinline__ uint64_t list_target(const RankSet &S, int L) {
+  return list_target_of(S, L, wide_targets(S));
+}
+__host__ __device__ __forceinline__ uint32_t sample_size(const RankSet &S) {
+  uint64_t ns = umin64(sample_size_raw(S, wide_targets(S)), kSample);
+  const uint32_t step = 8 * sample_ctas((uint32_t)ns);
+  ns -= ns % step;  // whole runs, evenly split over the CTAs
   return (uint32_t)ns;
 }
 
@@ -410,7 +431,7 @@ __device__ void joint_select32(const uint32_t (&v)[kLists][Q], uint32_t has, uin
   for (int L = 0; L < kLists; L++) out[L] = prefix[L];
 }
 
-// kSampleCtas CTAs per set.  1. One sample per thread: run j of ns/8 covers
+// S.sctas <= kSampleCtas CTAs per set.  1. One sample per thread: run j of ns/8 covers
 // stratum j (records [j n / (ns/8), (j+1) n / (ns/8))), 8 consecutive
 // records at a hashed offset inside it.  2. Per list, each CTA keeps the top
 // r_L summaries of its eligible samples (all of them when it has fewer).
@@ -422,6 +443,8 @@ __device__ void joint_select32(const uint32_t (&v)[kLists][Q], uint32_t has, uin
 __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankSet *sets) {
   const RankSet &S = sets[blockIdx.y];
   const uint32_t c = blockIdx.x;  // this CTA's share of the sample
+  const uint32_t nct = S.sctas;
+  if (c >= nct) return;           // the set needs fewer CTAs
   __shared__ uint64_t t2s[kLutN], mgs[kLutN];
   __shared__ unsigned int hist[2][kLists][256];
   __shared__ unsigned int pick[2][2 * kLists];
@@ -438,7 +461,7 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
   }
   __syncthreads();
   const uint32_t ns = S.ns, act = S.act;
-  const uint32_t per = ns / kSampleCtas;  // samples of this CTA (<= 1024, a multiple of 8)
+  const uint32_t per = ns / nct;  // samples of this CTA (<= 1024, a multiple of 8)
   uint32_t rL[kLists];
 #pragma unroll
   for (int L = 0; L < kLists; L++) rL[L] = S.rL[L];
@@ -505,14 +528,14 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
   // 3. the last CTA to finish merges the partial lists and sets the thresholds
   __threadfence();
   __syncthreads();
-  if (tid == 0) is_last = (atomicAdd(&S.work->sticket, 1u) == kSampleCtas - 1);
+  if (tid == 0) is_last = (atomicAdd(&S.work->sticket, 1u) == nct - 1);
   __syncthreads();
   if (!is_last) return;
   __threadfence();
   // entry counts of the partial lists, then kSampleCtas * r_L <= 4096
   // entries per list: one per thread when they fit, else four per thread
   __shared__ unsigned int pn[kLists * kSampleCtas];
-  if (tid < kLists * kSampleCtas) pn[tid] = __ldcg(&S.part_n[tid]);
+  if (tid < kLists * kSampleCtas) pn[tid] = (tid % kSampleCtas) < nct ? __ldcg(&S.part_n[tid]) : 0u;
   __syncthreads();
   uint32_t rmax = 0, sel2 = 0;
 #pragma unroll
@@ -537,7 +560,7 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
         const uint32_t e = tid + kSampleThreads * q;
         if (!rL[L]) continue;
         const uint32_t cc = e / rL[L], slot = e % rL[L];
-        if (cc < kSampleCtas && slot < pn[L * kSampleCtas + cc]) {
+        if (cc < nct && slot < pn[L * kSampleCtas + cc]) {
           vq[L][q] = __ldcg(&S.part[((size_t)L * kSampleCtas + cc) * kMaxR + slot]);
           hq |= 1u << (L * Q + q);
         }
@@ -546,7 +569,7 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
     joint_select32<Q>(vq, hq, sel2, rL, T2, hist, pick);
   };
   if (sel2) {
-    if (kSampleCtas * rmax <= kSampleThreads) merge(std::integral_constant<int, 1>());
+    if (nct * rmax <= kSampleThreads) merge(std::integral_constant<int, 1>());
     else merge(std::integral_constant<int, 4>());
   }
 #pragma unroll
@@ -637,6 +660,7 @@ constexpr uint32_t kConsumers = UNISON_FILTER_CONSUMERS;  // consumer threads
 constexpr uint32_t kBigTile = kConsumers * kRec;      // 4096 records per tile
 constexpr uint32_t kGroups = kRec / 4;                 // groups of four records per thread
 constexpr uint32_t kGroupStride = kConsumers * 4;      // records between a thread's groups
+constexpr uint32_t kWarpBuf = 128;                     // flagged records a warp tests per pass
 static_assert(kRec % 4 == 0 && kRec <= 32, "records per thread: a multiple of 4, at most 32");
 static_assert(kConsumers >= kLutN * 5, "one consumer thread per bound-table entry");
 constexpr uint32_t kFilterCtaThreads = kConsumers + 32;  // + one producer warp
@@ -663,12 +687,6 @@ __device__ __forceinline__ bool consumers_sync_or(bool p) {
       : "memory");
   return r != 0;
 }
-// A tile is copied by TMA when it is whole (the arrays' 16-byte alignment is
-// checked by the host); the last, partial tile of a set is read directly.
-__device__ __forceinline__ bool tile_is_bulk(const RankSet &S, uint32_t tile) {
-  return (tile - S.tile0 + 1) * kBigTile <= S.n;
-}
-
 __device__ __forceinline__ int set_of(const RankSet *sets, int si, uint32_t tile) {
   while (tile >= sets[si].tile0 + sets[si].ntiles) si++;
   return si;
@@ -688,24 +706,26 @@ __device__ void load_set(const RankSet &S, uint4 *vd, uint2 *pp, uint64_t *t2s, 
     t2s[t] = S.t2v[t];
     mgs[t] = S.mgv[t];
   }
-  uint32_t lo[kLists], dok[kLists];
+  if (threadIdx.x == 32) {
+    uint32_t lo[kLists], dok[kLists];
 #pragma unroll
-  for (int L = 0; L < kLists; L++) {
-    const uint64_t thrv = S.thr[L];
-    const uint64_t thr_ck = (L == 2) ? ~thrv : thrv;
-    const uint64_t K = thr_ck >> 24;
-    lo[L] = (uint32_t)(thr_ck & kIdMask);
-    // a completed record has the maximal key 2^40 - 1: 2 = always passes,
-    // 1 = passes on the index part, 0 = never
-    dok[L] = (L == 2) ? (kKeyMax40 == K ? 1u : 0u) : (kKeyMax40 > K ? 2u : (kKeyMax40 == K ? 1u : 0u));
+    for (int L = 0; L < kLists; L++) {
+      const uint64_t thrv = S.thr[L];
+      const uint64_t thr_ck = (L == 2) ? ~thrv : thrv;
+      const uint64_t K = thr_ck >> 24;
+      lo[L] = (uint32_t)(thr_ck & kIdMask);
+      // a completed record has the maximal key 2^40 - 1: 2 = always passes,
+      // 1 = passes on the index part, 0 = never
+      dok[L] = (L == 2) ? (kKeyMax40 == K ? 1u : 0u) : (kKeyMax40 > K ? 2u : (kKeyMax40 == K ? 1u : 0u));
+    }
+    c.loV = lo[0];
+    c.loD = lo[1];
+    c.loP = lo[2];
+    c.dV = !aV ? 0x1000000u : (dok[0] == 2 ? 0u : (dok[0] == 1 ? lo[0] : 0x1000000u));
+    c.dD = !aD ? 0x1000000u : (dok[1] == 2 ? 0u : (dok[1] == 1 ? lo[1] : 0x1000000u));
+    c.dP = (aP && dok[2] == 1) ? (int32_t)lo[2] : -1;
+    c.act = (aV ? 1u : 0u) | (aD ? 2u : 0u) | (aP ? 4u : 0u);
   }
-  c.loV = lo[0];
-  c.loD = lo[1];
-  c.loP = lo[2];
-  c.dV = !aV ? 0x1000000u : (dok[0] == 2 ? 0u : (dok[0] == 1 ? lo[0] : 0x1000000u));
-  c.dD = !aD ? 0x1000000u : (dok[1] == 2 ? 0u : (dok[1] == 1 ? lo[1] : 0x1000000u));
-  c.dP = (aP && dok[2] == 1) ? (int32_t)lo[2] : -1;
-  c.act = (aV ? 1u : 0u) | (aD ? 2u : 0u) | (aP ? 4u : 0u);
   consumers_sync();
 }
 
@@ -716,7 +736,7 @@ __device__ void load_set(const RankSet &S, uint4 *vd, uint2 *pp, uint64_t *t2s, 
 // against the set's thresholds.  Every wait is bounded; a CTA that gives up records
 // UNISON_ERR_TIMEOUT, lets its own copies land (bounded) and returns.
 __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) rank_filter_kernel(const RankSet *sets, int n_sets,
-                                                                        uint32_t total_tiles) {
+                                                                        uint32_t total_tiles, int grouped) {
   extern __shared__ __align__(128) unsigned char fsm[];
   FilterStage *stage = reinterpret_cast<FilterStage *>(fsm);
   __shared__ __align__(8) uint64_t full[kStages], empty[kStages];
@@ -724,11 +744,34 @@ __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) ra
   __shared__ uint2 pp[kLutN];
   __shared__ uint64_t t2s[kLutN], mgs[kLutN];
   __shared__ uint2 ftab[kLutN * 5];
-  // Tiles are dealt round-robin: CTA b takes tiles b, b + grid, ...  Records
-  // that pass a threshold cluster by index (ties on a key go to the smaller
-  // index, so a threshold on a tied key admits an index prefix); dealing the
-  // tiles spreads that work over all CTAs.
-  const uint32_t t_begin = blockIdx.x, t_step = gridDim.x, t_end = total_tiles;
+  __shared__ SetConst cset;
+  __shared__ uint16_t wbuf[kConsumers / 32][kWarpBuf];  // per consumer warp: flagged records' offsets
+  // Tiles are dealt round-robin, so the CTAs stream neighbouring tiles at any
+  // moment, and the tiles whose records pass a threshold -- they cluster by
+  // index, since ties on a key go to the smaller index -- spread over CTAs.
+  // Grouped: set s owns CTAs [cta0, cta0 + nctas), which deal its tiles among
+  // themselves (each CTA then loads one set's thresholds once).  Otherwise
+  // (more sets than CTAs) the CTAs deal every set's tiles in one sequence.
+  uint32_t t_begin, t_step, t_end;
+  int si0;
+  if (grouped) {
+    int lo = 0, hi = n_sets - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (sets[mid].cta0 <= blockIdx.x) lo = mid; else hi = mid - 1;
+    }
+    si0 = lo;
+    const RankSet &S = sets[si0];
+    t_begin = S.tile0 + (blockIdx.x - S.cta0);
+    t_step = S.nctas;
+    t_end = S.tile0 + S.ntiles;
+    if (blockIdx.x >= S.cta0 + S.nctas) return;
+  } else {
+    t_begin = blockIdx.x;
+    t_step = gridDim.x;
+    t_end = total_tiles;
+    si0 = -1;
+  }
   if (t_begin >= t_end) return;
   if (threadIdx.x == 0) {
     for (int q = 0; q < kStages; q++) {
@@ -738,7 +781,7 @@ __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) ra
     fence_mbar_init();
   }
   __syncthreads();
-  const int si0 = set_of_tile(sets, n_sets, t_begin);
+  if (si0 < 0) si0 = set_of_tile(sets, n_sets, t_begin);
   const int lane = threadIdx.x & 31;
 
   if (threadIdx.x >= kConsumers) {
@@ -760,8 +803,8 @@ __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) ra
       }
       si = set_of(sets, si, tile);
       const RankSet &T = sets[si];
-      if (!tile_is_bulk(T, tile)) continue;
       const uint32_t base = (tile - T.tile0) * kBigTile;
+      if (base + kBigTile > T.n) continue;  // the partial last tile is read directly
       FilterStage &d = stage[q];
       fence_proxy_async();
       mbar_expect_tx(&full[q], kBigTile * 8);
@@ -787,8 +830,8 @@ __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) ra
   // records, group gi starting at record gi * kGroupStride + 4 * ct: every
   // shared-memory read of the stage is lane-contiguous (no bank conflicts).
   const uint32_t ct = threadIdx.x;
-  int si = si0, lsi = -1;
-  SetConst c;
+  int si = si0;
+  SetConst &c = cset;  // this set's constants, in shared memory
   uint32_t fph = 0;  // bit q: parity of the next full-barrier phase of stage q (flips per bulk tile)
   // this set's hot descriptor fields, cached when the set changes (pointers
   // used only on rare paths are read from the descriptor there)
@@ -802,11 +845,10 @@ __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) ra
   bool seg_mixed = false, seg_none = false;
   for (uint32_t i = 0, tile = t_begin; tile < t_end; i++, tile += t_step) {
     const int q = (int)(i % kStages);
-    if (lsi < 0 || tile >= s_end) {
+    if (i == 0 || tile >= s_end) {
       si = set_of(sets, si, tile);
       const RankSet &S = sets[si];
       load_set(S, vd, pp, t2s, mgs, c);
-      lsi = si;
       s_n = S.n;
       s_tile0 = S.tile0;
       s_end = S.tile0 + S.ntiles;
@@ -883,9 +925,6 @@ __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) ra
         fw[gi] = *reinterpret_cast<const uint32_t *>(d.flags + o);
         rw[gi] = *reinterpret_cast<const uint32_t *>(d.tier + o);
       }
-      // the stage's data is in registers: hand it back to the producer
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&empty[q]);
     } else {
       const RankSet &S = sets[si];
       const uint32_t *s_gap = S.gap;
@@ -909,8 +948,6 @@ __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) ra
           }
         }
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&empty[q]);
     }
     auto turn_of = [&](uint32_t k) { return min((tw[k >> 1] >> (16 * (k & 1))) & 0xFFFF, kTMax); };
     auto index_of = [&](uint32_t k) { return tb + (k >> 2) * kGroupStride + 4 * ct + (k & 3); };
@@ -936,60 +973,7 @@ __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) ra
         }
       }
     }
-    // 2. exact per-list tests of the flagged records (rare outside mixed tiles)
-    if (__any_sync(kFull, cm != 0)) {
-      uint32_t mV = 0, mD = 0, mP = 0;  // candidate bit per record, per list
-      if (cm) {
-#pragma unroll
-        for (uint32_t k = 0; k < kRec; k++) {
-          if (!((cm >> k) & 1)) continue;
-          const uint32_t fl = (fw[k >> 2] >> (8 * (k & 3))) & 0xFF, tr = (rw[k >> 2] >> (8 * (k & 3))) & 0xFF;
-          const uint32_t em = elig_mask((uint8_t)fl, (uint8_t)tr);
-          const bool done = (fl & 2) != 0;
-          const uint32_t t = turn_of(k), gg = g[k];
-          const uint32_t lo = (~index_of(k)) & kIdMask;
-          const uint4 a = vd[t];
-          const uint2 b = pp[t];
-          const bool pV = done ? lo >= c.dV : (gg >= a.y || (gg >= a.x && lo >= c.loV));
-          const bool pD = done ? lo >= c.dD : (gg >= a.w || (gg >= a.z && lo >= c.loD));
-          const bool pP = done ? (int32_t)lo <= c.dP : (gg < b.x || (gg < b.y && lo <= c.loP));
-          mV |= (uint32_t)(pV && (em & 1)) << k;
-          mD |= (uint32_t)(pD && (em & 2)) << k;
-          mP |= (uint32_t)(pP && (em & 4)) << k;
-        }
-      }
-      // emit candidates' exact values (warp-aggregated appends)
-#pragma unroll
-      for (int L = 0; L < kLists; L++) {
-        const uint32_t mm = L == 0 ? mV : (L == 1 ? mD : mP);
-        const uint32_t mine = __popc(mm);
-        if (!__any_sync(kFull, mine != 0)) continue;
-        uint32_t incl = mine;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-          const uint32_t y = __shfl_up_sync(kFull, incl, o);
-          if (lane >= o) incl += y;
-        }
-        const uint32_t total = __shfl_sync(kFull, incl, 31);
-        uint32_t basepos = 0;
-        if (lane == 31) basepos = atomicAdd(&sets[si].work->cand[L], total);
-        basepos = __shfl_sync(kFull, basepos, 31);
-        uint32_t pos = basepos + incl - mine;
-        if (mm) {
-          uint64_t *dst = sets[si].cand + (size_t)L * kCandCap;
-#pragma unroll
-          for (uint32_t k = 0; k < kRec; k++) {
-            if ((mm >> k) & 1) {
-              if (pos < kCandCap) {
-                const bool dn = (fw[k >> 2] >> (8 * (k & 3) + 1)) & 1;
-                dst[pos] = list_val(ck_of(score_of(g[k], turn_of(k), dn, t2s, mgs), index_of(k)), L);
-              }
-              pos++;
-            }
-          }
-        }
-      }
-    }
+    // every record's key, when asked for (from registers)
     if (s_keys) {
       uint64_t *keys = sets[si].keys;
 #pragma unroll
@@ -1001,6 +985,89 @@ __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) ra
         }
       }
     }
+    // The stage is handed back to the producer as soon as this warp no longer
+    // reads it: at once when none of its records is flagged, else after the
+    // exact tests below, which read the flagged records back from the stage.
+    const bool flagged = __any_sync(kFull, cm != 0);
+    if (!flagged) {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&empty[q]);
+      continue;
+    }
+    // 2. exact per-list tests of the flagged records: the warp lists their
+    // offsets in the tile (kWarpBuf a pass), then each lane tests one and
+    // appends its exact value to every list it passes (one atomic per warp
+    // and list).
+    uint16_t *wb = wbuf[ct >> 5];
+    const FilterStage &d = stage[q];
+    const RankSet &S = sets[si];
+    uint32_t rem = cm;
+    while (__any_sync(kFull, rem != 0)) {
+      const uint32_t mine = __popc(rem);
+      uint32_t incl = mine;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += y;
+      }
+      const uint32_t nb = min(__shfl_sync(kFull, incl, 31), kWarpBuf);
+      uint32_t pos = incl - mine, wrote = 0;
+#pragma unroll
+      for (uint32_t k = 0; k < kRec; k++) {
+        if ((rem >> k) & 1) {
+          if (pos < kWarpBuf) {
+            wb[pos] = (uint16_t)((k >> 2) * kGroupStride + 4 * ct + (k & 3));
+            wrote |= 1u << k;
+          }
+          pos++;
+        }
+      }
+      rem &= ~wrote;
+      __syncwarp();
+      for (uint32_t j0 = 0; j0 < nb; j0 += 32) {
+        const uint32_t j = j0 + lane;
+        bool pL[kLists] = {false, false, false};
+        uint64_t ck = 0;
+        if (j < nb) {
+          const uint32_t o = wb[j], idx = tb + o;
+          uint32_t gg, t, fl, tr;
+          if (bulk) {
+            gg = d.gap[o];
+            t = d.turn[o];
+            fl = d.flags[o];
+            tr = d.tier[o];
+          } else {  // the partial last tile: read from the set (padding is pinned)
+            const bool in = idx < s_n;
+            gg = in ? S.gap[idx] : 0u;
+            t = in ? S.turn[idx] : 0u;
+            fl = in ? S.flags[idx] : 1u;
+            tr = in ? S.tier[idx] : 0u;
+          }
+          t = min(t, kTMax);
+          const uint32_t em = elig_mask((uint8_t)fl, (uint8_t)tr);
+          const bool done = (fl & 2) != 0;
+          const uint32_t lo = (~idx) & kIdMask;
+          const uint4 a = vd[t];
+          const uint2 b = pp[t];
+          pL[0] = (em & 1) && (done ? lo >= c.dV : (gg >= a.y || (gg >= a.x && lo >= c.loV)));
+          pL[1] = (em & 2) && (done ? lo >= c.dD : (gg >= a.w || (gg >= a.z && lo >= c.loD)));
+          pL[2] = (em & 4) && (done ? (int32_t)lo <= c.dP : (gg < b.x || (gg < b.y && lo <= c.loP)));
+          if (pL[0] || pL[1] || pL[2]) ck = ck_of(score_of(gg, t, done, t2s, mgs), idx);
+        }
+#pragma unroll
+        for (int L = 0; L < kLists; L++) {
+          const unsigned bal = __ballot_sync(kFull, pL[L]);
+          if (!bal) continue;
+          unsigned base = 0;
+          if (lane == 0) base = atomicAdd(&S.work->cand[L], (unsigned)__popc(bal));
+          base = __shfl_sync(kFull, base, 0);
+          const uint32_t at = base + __popc(bal & ((1u << lane) - 1));
+          if (pL[L] && at < kCandCap) S.cand[(size_t)L * kCandCap + at] = list_val(ck, L);
+        }
+      }
+      __syncwarp();  // the buffer is rewritten by the next pass
+    }
+    if (lane == 0) mbar_arrive(&empty[q]);
   }
 }
 
@@ -1368,6 +1435,42 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
+// Kernel attributes and the filter's resident-CTA count, set up once per
+// device (the attributes belong to the device's context).
+struct LaunchCfg {
+  bool ok = false;
+  uint32_t filter_ctas = 0;
+};
+const LaunchCfg &launch_cfg() {
+  static std::mutex mu;
+  static LaunchCfg cfgs[64];
+  static bool done[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
+    static LaunchCfg bad;
+    return bad;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (!done[dev]) {
+    LaunchCfg c;
+    int n_sm = 0, per_sm = 0;
+    const size_t smem_finish = sizeof(uint64_t) * (kSmemCand + kMaxSel);
+    c.ok = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess &&
+           cudaFuncSetAttribute(rank_filter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)kFilterSmem) == cudaSuccess &&
+           cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rank_filter_kernel, kFilterCtaThreads,
+                                                         kFilterSmem) == cudaSuccess &&
+           cudaFuncSetAttribute(rank_finish_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)smem_finish) == cudaSuccess;
+    if (!c.ok) cudaGetLastError();
+    c.filter_ctas = (uint32_t)std::max(1, n_sm * per_sm);
+    cfgs[dev] = c;
+    done[dev] = c.ok;
+  }
+  return cfgs[dev];
+}
+
 }  // namespace
 
 extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_params *params,
@@ -1415,12 +1518,14 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
     s.tile0 = tiles;
     s.ntiles = (uint32_t)((r.n + kBigTile - 1) / kBigTile);
     tiles += s.ntiles;
+
     for (int t = 0; t < (int)kLutN; t++) {
       s.sigma[t] = p.sigma_q[t];
       s.t2v[t] = ((uint64_t)(kLambda - p.sigma_q[t]) * p.penalty_q) / kLambda;  // eq. (t2)
       s.mgv[t] = magic_for(p.sigma_q[t]);
     }
     s.ns = sample_size(s);
+    s.sctas = sample_ctas(s.ns);
     s.nruns = s.ns / 8;
     s.sq = s.nruns ? s.n / s.nruns : 0;
     s.srem = s.nruns ? s.n % s.nruns : 0;
@@ -1431,26 +1536,28 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
                     ? (uint32_t)umin64((list_target(s, L) * s.ns + s.n - 1) / s.n, kMaxR) : 0u;
     }
   }
-  // scratch: descriptors, then per set: work, thresholds, tables, sorted
-  // lists, candidates, the sample's partial lists
-  const size_t per_set = align_up(sizeof(RankWork), 256) + align_up(sizeof(uint64_t) * 2 * kLists, 256) +
-                         align_up(sizeof(uint2) * kLists * kLutN, 256) +
+  // scratch: descriptors, every set's work words (one memset), then per set:
+  // thresholds, tables, sorted lists and sizes, candidates, the sample's
+  // partial lists
+  const size_t per_set = align_up(sizeof(uint64_t) * 2 * kLists, 256) + align_up(sizeof(uint2) * kLists * kLutN, 256) +
                          align_up(sizeof(uint64_t) * kLists * kMaxSel, 256) +
                          align_up(sizeof(uint32_t) * kLists * kMaxSel, 256) +
                          align_up(sizeof(uint64_t) * kLists * kCandCap, 256) +
                          align_up(sizeof(uint32_t) * kLists * kSampleCtas * kMaxR, 256) +
                          align_up(sizeof(uint32_t) * kLists * kSampleCtas, 256);
   const size_t desc_b = align_up(sizeof(RankSet) * n_sets, 256);
+  const size_t work_b = align_up(sizeof(RankWork) * n_sets, 256);
   char *scratch = nullptr;
-  if (cudaMallocAsync(reinterpret_cast<void **>(&scratch), desc_b + per_set * n_sets, stream) != cudaSuccess) {
+  if (cudaMallocAsync(reinterpret_cast<void **>(&scratch), desc_b + work_b + per_set * n_sets, stream) !=
+      cudaSuccess) {
     cudaGetLastError();
     return UNISON_ERR_OOM;
   }
+  RankWork *works = reinterpret_cast<RankWork *>(scratch + desc_b);
   for (int i = 0; i < n_sets; i++) {
-    char *p = scratch + desc_b + per_set * i;
+    char *p = scratch + desc_b + work_b + per_set * i;
     RankSet &s = hs[i];
-    s.work = reinterpret_cast<RankWork *>(p);
-    p += align_up(sizeof(RankWork), 256);
+    s.work = works + i;
     s.thr = reinterpret_cast<uint64_t *>(p);
     p += align_up(sizeof(uint64_t) * 2 * kLists, 256);
     s.gthr = reinterpret_cast<uint2 *>(p);
@@ -1470,24 +1577,43 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
     if (e != cudaSuccess && rc == UNISON_OK) rc = UNISON_ERR_CUDA;
   };
   RankSet *d_sets = reinterpret_cast<RankSet *>(scratch);
-  ck(cudaMemcpyAsync(d_sets, hs.data(), sizeof(RankSet) * n_sets, cudaMemcpyHostToDevice, stream));
-  for (int i = 0; i < n_sets; i++) ck(cudaMemsetAsync(hs[i].work, 0, sizeof(RankWork), stream));
   const size_t smem_finish = sizeof(uint64_t) * (kSmemCand + kMaxSel);
-  // persistent filter: as many CTAs as fit at once, tiles dealt round-robin
-  int dev = 0, n_sm = 0, per_sm = 0;
-  cudaGetDevice(&dev);
-  cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
-  ck(cudaFuncSetAttribute(rank_filter_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFilterSmem));
-  cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rank_filter_kernel, kFilterCtaThreads, kFilterSmem);
-  const uint32_t grid_filter = std::max(1u, std::min<uint32_t>(tiles, (uint32_t)std::max(1, n_sm * per_sm)));
-  ck(cudaFuncSetAttribute(rank_finish_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_finish));
+  // persistent filter: as many CTAs as fit at once (per device, set up once)
+  const LaunchCfg &cfg = launch_cfg();
+  if (!cfg.ok) {
+    cudaFreeAsync(scratch, stream);
+    return UNISON_ERR_CUDA;
+  }
+  uint32_t grid_filter = std::max(1u, std::min<uint32_t>(tiles, cfg.filter_ctas));
+  // Filter schedule: each set gets a group of CTAs in proportion to its tiles
+  // (at least 1, at most its tile count) when the groups fit in the resident
+  // CTAs; otherwise every CTA deals from all sets' tiles.
+  int grouped = 0;
+  {
+    uint64_t total = 0;
+    for (int i = 0; i < n_sets; i++) {
+      RankSet &s = hs[i];
+      s.nctas = (uint32_t)std::max<uint64_t>(1, ((uint64_t)grid_filter * s.ntiles) / tiles);
+      s.nctas = std::min(s.nctas, s.ntiles);
+      s.cta0 = (uint32_t)total;
+      total += s.nctas;
+    }
+    if (total <= grid_filter) {
+      grouped = 1;
+      grid_filter = (uint32_t)total;
+    }
+  }
+  uint32_t max_sctas = 1;
+  for (int i = 0; i < n_sets; i++) max_sctas = std::max(max_sctas, hs[i].sctas);
+  ck(cudaMemcpyAsync(d_sets, hs.data(), sizeof(RankSet) * n_sets, cudaMemcpyHostToDevice, stream));
+  ck(cudaMemsetAsync(works, 0, sizeof(RankWork) * n_sets, stream));
   {
     ProfSpan span("rank_sample", stream);
-    rank_sample_kernel<<<dim3(kSampleCtas, n_sets), kSampleThreads, 0, stream>>>(d_sets);
+    rank_sample_kernel<<<dim3(max_sctas, n_sets), kSampleThreads, 0, stream>>>(d_sets);
   }
   {
     ProfSpan span("rank_filter", stream);
-    rank_filter_kernel<<<grid_filter, kFilterCtaThreads, kFilterSmem, stream>>>(d_sets, n_sets, tiles);
+    rank_filter_kernel<<<grid_filter, kFilterCtaThreads, kFilterSmem, stream>>>(d_sets, n_sets, tiles, grouped);
   }
   {
     ProfSpan span("rank_finish", stream);
