@@ -200,11 +200,43 @@ def rank_size_sweep(B, host_rec, sigma, stream, steps: int = 10, warmup: int = 3
         f_ms, f_n = B.profile_read("rank_filter", reset=True)
         recs = n * n_sets
         gbs = recs * RANK_BYTES_PER_RECORD / (call_us / 1e6) / 1e9
-        out.append({"n": n, "sets_per_call": n_sets, "call_us": call_us,
-                    "filter_us": 1e3 * f_ms / max(f_n, 1) if f_n else None, "call_gbs": gbs,
+        filter_us = 1e3 * f_ms / max(f_n, 1) if f_n else None
+        out.append({"n": n, "sets_per_call": n_sets, "call_us": call_us, "filter_us": filter_us, "call_gbs": gbs,
+                    "filter_gbs": recs * RANK_BYTES_PER_RECORD / (filter_us / 1e6) / 1e9 if filter_us else None,
                     "l2_resident": recs * RANK_BYTES_PER_RECORD < (2 * 129 << 20)})
         del call, sets, outs
     return out
+
+
+def kendall_fp32_vs_fixed(B, host_rec, sigma, stream, n: int = 1 << 20):
+    """Kendall tau-b between the fixed-point keys the ranking kernel writes
+    (eq. scoreq) and a float32 ranking by the same formula without the
+    fixed-point floors, s = g * Lambda / sigma_q + (Lambda - sigma_q) * P_Z /
+    Lambda (eq. esp; completed sessions rank first in both), on the first n
+    records of the live set.  Reporting only (Sec. IV-C compares the two)."""
+    import numpy as np
+    import torch
+    try:
+        from scipy.stats import kendalltau
+    except ImportError:
+        return None
+    part = {k: v[:n].to("cuda") for k, v in host_rec.items()}
+    p = dict(sigma_q=sigma, k=1, penalty_q=500_000_000, budget_bytes=0, kv_bytes_per_token=131072, max_moves=0,
+             free_fast_tok=0, free_hbm_tok=0)
+    out = B.rank_outputs(n, 1, 0, keys=True)
+    B.rank_prepare([part], [p], [out]).run(stream)
+    torch.cuda.synchronize()
+    fixed = out["keys"].cpu().numpy().view(np.uint64)
+    g = host_rec["gap_q"][:n].numpy().view(np.uint32).astype(np.float32)
+    t = np.minimum(host_rec["turn"][:n].numpy().view(np.uint16), 50)
+    sq = np.asarray(sigma, dtype=np.float32)[t]
+    lam, pz = np.float32(4095.0), np.float32(500_000_000.0)
+    f32 = g * lam / sq + (lam - sq) * pz / lam
+    done = (host_rec["flags"][:n].numpy() & 2) != 0
+    f32 = np.where(done, np.float32(np.inf), f32).astype(np.float32)
+    tau = kendalltau(fixed.astype(np.float64), f32.astype(np.float64))[0]
+    return {"tau_b": float(tau), "records": n, "fixed": "rank kernel keys (eq. scoreq)",
+            "float": "float32 g*Lambda/sigma_q + (Lambda-sigma_q)*P_Z/Lambda"}
 
 
 def cpu_baseline_replay(trs, reps, budget_s: float = 12.0):
@@ -366,13 +398,17 @@ def main():
     value = shard.job_rate(units, args.steps, ms) if not args.rank_only else None
 
     sizes = None
+    tau = None
+    if not args.replay_only:
+        tau = kendall_fp32_vs_fixed(B, host_rec, sigma, stream)
     if not args.replay_only and not args.no_rank_sizes:
         B.profile_enable(True)
         sizes = rank_size_sweep(B, host_rec, sigma, stream)
         B.profile_enable(False)
+        pk = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))).get("hbm_gbs") or 6800.0
         for e in sizes:
-            e["call_frac_of_peak"] = e["call_gbs"] / (json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
-                                                      .get("hbm_gbs") or 6800.0)
+            e["call_frac_of_peak"] = e["call_gbs"] / pk
+            e["filter_frac_of_peak"] = e["filter_gbs"] / pk if e["filter_gbs"] else None
 
     # end to end through the public API: host trace staging -> device, replay,
     # results back to the host, every step
@@ -441,7 +477,7 @@ def main():
                                    "paper-scale coding trace, 131072 B/token, SPEAR+TIDE)",
                        "replays": n_rep, "events_per_step": events_per_step,
                        "l2": "flushed before every step (256 MiB write, inside the timed region)"},
-            "roofline": roofline, "rank": rank_leg, "rank_sizes": sizes, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roofline, "rank": rank_leg, "rank_sizes": sizes, "rank_kendall": tau, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches, "clocks": clocks,
             "peaks": {"hbm_gbs": peaks.get("hbm_gbs"), "source": "MEASURED_PEAKS.json"}}
     if cpu is not None:

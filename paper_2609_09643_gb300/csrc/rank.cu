@@ -954,7 +954,22 @@ __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) ra
     // 1. candidate bit per record (any list): one table lookup per record
     uint32_t cm = 0;
     if (seg_mixed) {
-      cm = (1u << kRec) - 1;  // index conditions vary inside the tile: test every record exactly
+      // index conditions vary inside the tile: flag the records that pass
+      // some list exactly
+#pragma unroll
+      for (uint32_t k = 0; k < kRec; k++) {
+        const uint32_t sh = 8 * (k & 3);
+        const uint32_t fl = (fw[k >> 2] >> sh) & 0xFF, tr = (rw[k >> 2] >> sh) & 0xFF;
+        const uint32_t em = elig_mask((uint8_t)fl, (uint8_t)tr);
+        const bool done = (fl & 2) != 0;
+        const uint32_t gg = g[k], t = turn_of(k), lo = (~index_of(k)) & kIdMask;
+        const uint4 a = vd[t];
+        const uint2 b = pp[t];
+        const bool pV = (em & 1) && (done ? lo >= c.dV : (gg >= a.y || (gg >= a.x && lo >= c.loV)));
+        const bool pD = (em & 2) && (done ? lo >= c.dD : (gg >= a.w || (gg >= a.z && lo >= c.loD)));
+        const bool pP = (em & 4) && (done ? (int32_t)lo <= c.dP : (gg < b.x || (gg < b.y && lo <= c.loP)));
+        cm |= (uint32_t)(pV || pD || pP) << k;
+      }
     } else if (!seg_none) {
       const unsigned char *tab = reinterpret_cast<const unsigned char *>(ftab);
 #pragma unroll
