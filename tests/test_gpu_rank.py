@@ -163,6 +163,18 @@ def test_fill_byte_sums_beyond_2p64(B, sigma):
     assert len(res[0]["promote"]) > 100 and len(res[2]["demote"]) > 100
 
 
+def test_more_sets_than_filter_ctas(B, sigma):
+    """600 sampled sets (more than the filter's resident CTAs): every CTA
+    deals tiles from all sets instead of owning one set's group."""
+    n = 20000
+    recs = [synth.make_records(1000 + i, n) for i in range(600)]
+    ks = [1, 7, 64, 1024]
+    ps = [prm(sigma, k=ks[i % 4], budget=(1 << (i % 7)) * GIB, max_moves=(64, 1024)[i % 2]) for i in range(600)]
+    res = run(B, recs, ps)
+    for i in list(range(0, 600, 37)) + [599]:
+        check(res[i], recs[i], ps[i])
+
+
 def test_batch_of_mixed_sets(B, sigma):
     recs = [synth.make_records(20 + i, n) for i, n in enumerate([100, 20000, 1 << 18, 3000, 1 << 19])]
     ps = [prm(sigma, k=k, budget=(1 << i) * GIB) for i, k in enumerate([3, 50, 1024, 4096, 700])]
