@@ -69,6 +69,8 @@ struct ReplayDesc {
   uint32_t n_events, n_turns, n_sessions, policy;
   uint32_t max_sessions, kvb, ttl, load;
   uint32_t rcap_s, rcap_h;
+  uint32_t tmap;  // 1: a per-session tier byte follows the lists in shared memory
+  uint32_t pad_;
 };
 
 // --------------------------------------------------------------------------
@@ -255,6 +257,7 @@ struct ReplayState {
   uint4 *pin;       // pinned residents
   uint32_t npin, pin_cap;
   uint4 *tmp;       // TIDE staging: [0, cap_s) promoted, [cap_s, 2 cap_s) demoted
+  uint8_t *tmap;    // tier of each unpinned resident session (kTierNone otherwise), or null
   uint64_t used_s, used_h, pinned_s, pinned_h;  // tokens
   unison_decision *log;
   uint64_t log_cap;
@@ -287,7 +290,13 @@ __device__ __forceinline__ void log_dec(ReplayState &st, uint32_t kind, uint32_t
   st.log_len++;
 }
 
-__device__ __forceinline__ bool sorted_insert(ReplayState &st, Sorted &T, uint4 v, int lane) {
+// Tier-map update: every lane stores the same byte, so each lane's later
+// reads see it without a warp barrier.
+__device__ __forceinline__ void set_tier(ReplayState &st, uint32_t id, uint32_t tier) {
+  if (st.tmap) st.tmap[id] = (uint8_t)tier;
+}
+
+__device__ __forceinline__ bool sorted_insert(ReplayState &st, Sorted &T, uint4 v, int lane, uint32_t tier) {
   if (T.n >= T.cap) {
     st.status = UNISON_ERR_CAPACITY;
     return false;
@@ -297,6 +306,7 @@ __device__ __forceinline__ bool sorted_insert(ReplayState &st, Sorted &T, uint4 
   if (lane == 0) T.e[p] = v;
   __syncwarp();
   T.n++;
+  set_tier(st, packed_id(ekey(v)), tier);
   return true;
 }
 
@@ -305,10 +315,11 @@ __device__ __forceinline__ void sorted_erase(Sorted &T, uint32_t p, int lane) {
   T.n--;
 }
 
-__device__ __forceinline__ uint4 sorted_pop_back(Sorted &T) {
+__device__ __forceinline__ uint4 sorted_pop_back(ReplayState &st, Sorted &T) {
   const uint4 v = T.e[T.n - 1];
   __syncwarp();
   T.n--;
+  set_tier(st, packed_id(ekey(v)), kTierNone);
   return v;
 }
 
@@ -331,12 +342,12 @@ __device__ __forceinline__ bool admit_demoted(ReplayState &st, const ReplayDesc 
       CNT(st, n_evict, 1);
       return true;
     }
-    const uint4 v = sorted_pop_back(st.H);
+    const uint4 v = sorted_pop_back(st, st.H);
     st.used_h -= esize(v);
     log_dec(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
     CNT(st, n_evict, 1);
   }
-  if (!sorted_insert(st, st.H, d, lane)) return false;
+  if (!sorted_insert(st, st.H, d, lane, kTierH)) return false;
   st.used_h += size;
   log_dec(st, UNISON_KIND_DEMOTE, id, lane);
   CNT(st, n_demote, 1);
@@ -369,7 +380,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const ReplayDesc &D, uint
         st.status = UNISON_ERR_CAPACITY;
         return false;
       }
-      const uint4 d = sorted_pop_back(st.S);  // most evictable unpinned fast-tier session
+      const uint4 d = sorted_pop_back(st, st.S);  // most evictable unpinned fast-tier session
       st.used_s -= esize(d);
       if (!admit_demoted(st, D, d, lane)) return false;
     }
@@ -384,7 +395,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const ReplayDesc &D, uint
         st.status = UNISON_ERR_CAPACITY;
         return false;
       }
-      const uint4 v = sorted_pop_back(st.H);
+      const uint4 v = sorted_pop_back(st, st.H);
       st.used_h -= esize(v);
       log_dec(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
       CNT(st, n_evict, 1);
@@ -407,7 +418,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const ReplayDesc &D, uint
       }
       const bool from_s =
           st.H.n == 0 || (st.S.n > 0 && ekey(st.S.e[st.S.n - 1]) > ekey(st.H.e[st.H.n - 1]));
-      const uint4 v = sorted_pop_back(from_s ? st.S : st.H);
+      const uint4 v = sorted_pop_back(st, from_s ? st.S : st.H);
       if (from_s)
         st.used_s -= esize(v);
       else
@@ -480,9 +491,9 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const ReplayDesc &D, u
   st.H.n -= m;
   st.S.n -= pairs;
   for (uint32_t i = 0; i < m; i++)
-    if (!sorted_insert(st, st.S, pro[i], lane)) return budget - rem;
+    if (!sorted_insert(st, st.S, pro[i], lane, kTierS)) return budget - rem;
   for (uint32_t i = 0; i < pairs; i++)
-    if (!sorted_insert(st, st.H, dem[i], lane)) return budget - rem;
+    if (!sorted_insert(st, st.H, dem[i], lane, kTierH)) return budget - rem;
   return budget - rem;
 }
 
@@ -519,6 +530,7 @@ __device__ __forceinline__ void expire_idle(ReplayState &st, uint32_t now, uint3
     else
       st.used_h -= sz;
     sorted_erase(T, pos, lane);
+    set_tier(st, mid, kTierNone);
     log_dec(st, UNISON_KIND_EXPIRE, mid, lane);
     CNT(st, n_expire, 1);
   }
@@ -563,6 +575,14 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
     st.pin = p;
     p += D.rcap_s + D.rcap_h;
     st.tmp = p;
+    p += 2 * D.rcap_s;
+    st.tmap = nullptr;
+    if (!kGlobalLists && D.tmap) {
+      st.tmap = reinterpret_cast<uint8_t *>(p);
+      uint32_t *m32 = reinterpret_cast<uint32_t *>(p);
+      for (uint32_t i = lane; i < (D.n_sessions + 3) / 4; i += 32) m32[i] = 0u;
+      __syncwarp();
+    }
     st.S.n = st.H.n = 0;
     st.S.cap = D.rcap_s;
     st.H.cap = D.rcap_h;
@@ -661,11 +681,17 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
             pkb = pack_key(e, s);  // the previous arrival's next reference is this event
           else
             pkb = pack_key(0xFFFFFFFFull - spev[bi][j], s);
-          pos = lower_bound(st.S, pkb, lane);
-          if (pos < st.S.n && ekey(st.S.e[pos]) == pkb) {
-            tier = kTierS;
-            ent = st.S.e[pos];
-          } else {
+          // with the tier map only the session's own tier is searched (and
+          // nothing for a session that is not resident)
+          const uint32_t mt = st.tmap ? st.tmap[s] : (kTierS | kTierH);
+          if (mt & kTierS) {
+            pos = lower_bound(st.S, pkb, lane);
+            if (pos < st.S.n && ekey(st.S.e[pos]) == pkb) {
+              tier = kTierS;
+              ent = st.S.e[pos];
+            }
+          }
+          if (tier == kTierNone && (mt & kTierH)) {
             pos = lower_bound(st.H, pkb, lane);
             if (pos < st.H.n && ekey(st.H.e[pos]) == pkb) {
               tier = kTierH;
@@ -715,9 +741,11 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
         if (tier == kTierS) {
           st.used_s -= esize(ent);
           sorted_erase(st.S, pos, lane);
+          set_tier(st, s, kTierNone);
         } else if (tier == kTierH) {
           st.used_h -= esize(ent);
           sorted_erase(st.H, pos, lane);
+          set_tier(st, s, kTierNone);
         }
         uint64_t pk;
         if (spear_keys)
@@ -751,10 +779,10 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
           const uint4 v = make_uint4((uint32_t)pk, (uint32_t)(pk >> 32), sz, now);
           if (tier == kTierS) {
             st.pinned_s -= sz;
-            if (!sorted_insert(st, st.S, v, lane)) break;
+            if (!sorted_insert(st, st.S, v, lane, kTierS)) break;
           } else {
             st.pinned_h -= sz;
-            if (!sorted_insert(st, st.H, v, lane)) break;
+            if (!sorted_insert(st, st.H, v, lane, kTierH)) break;
           }
         }
         if (!edge && tide_on && !dma_busy) {
@@ -902,7 +930,7 @@ struct ReplayPlan {
   std::vector<int> replay_combo;
   size_t off_desc = 0, off_order = 0, off_combo = 0, bytes = 0;
   std::vector<size_t> off_lut, off_stream, off_ttft, off_glist;
-  std::vector<uint32_t> rcap_s, rcap_h, in_smem, in_global;
+  std::vector<uint32_t> rcap_s, rcap_h, in_smem, in_global, tmap;
   size_t max_smem = 0;
 };
 
@@ -915,7 +943,9 @@ uint32_t list_cap(uint64_t cap_tok, const unison_trace *tr) {
 }
 
 // 16-byte entries: fast and HBM arrays, the pinned list (both tiers) and the
-// TIDE staging area (two fast-tier capacities).
+// TIDE staging area (two fast-tier capacities).  A tier map of one byte per
+// session follows when the trace has at most kTierMapMax sessions.
+constexpr uint32_t kTierMapMax = 32768;
 size_t list_bytes(uint32_t cs, uint32_t ch) { return 16ull * (4ull * cs + 2ull * ch); }
 
 void plan_replays(const unison_trace *const *traces, const unison_replay_params *params, int n_replays,
@@ -953,16 +983,21 @@ void plan_replays(const unison_trace *const *traces, const unison_replay_params 
   P.off_glist.assign(n_replays, 0);
   P.rcap_s.resize(n_replays);
   P.rcap_h.resize(n_replays);
+  P.tmap.assign(n_replays, 0);
   for (int r = 0; r < n_replays; r++) {
     const unison_replay_params &p = params[r];
     const unison_trace *tr = traces[p.trace_idx];
     P.rcap_s[r] = list_cap(p.cap_fast_bytes / p.kv_bytes_per_token, tr);
     P.rcap_h[r] = list_cap(p.cap_hbm_bytes / p.kv_bytes_per_token, tr);
     const size_t lists = list_bytes(P.rcap_s[r], P.rcap_h[r]);
+    // the tier map (one byte per session) when it fits beside the lists
+    const size_t map = align_up(tr->n_sessions, 16);
+    P.tmap[r] = tr->n_sessions <= kTierMapMax && lists + map <= smem_limit;
     if (lists <= smem_limit) {
       P.in_smem.push_back((uint32_t)r);
-      P.max_smem = std::max<size_t>(P.max_smem, lists);
+      P.max_smem = std::max<size_t>(P.max_smem, lists + (P.tmap[r] ? map : 0));
     } else {
+      P.tmap[r] = 0;
       P.in_global.push_back((uint32_t)r);
       P.off_glist[r] = off;
       off = align_up(off + lists, 256);
@@ -1035,6 +1070,8 @@ void fill_descs(const unison_trace *const *traces, const unison_replay_params *p
     d.load = p.ttft_load;
     d.rcap_s = P.rcap_s[r];
     d.rcap_h = P.rcap_h[r];
+    d.tmap = P.tmap[r];
+    d.pad_ = 0;
   }
   order.clear();
   order.insert(order.end(), P.in_smem.begin(), P.in_smem.end());
