@@ -254,6 +254,14 @@ __device__ __noinline__ void shift_block(uint4 *e, uint32_t lo, uint32_t hi, int
   }
 }
 
+// Descriptor fields the placement and fill read on every event, held in
+// registers (the descriptor itself sits in shared memory).
+struct Hot {
+  uint64_t cap_s, cap_h;  // tokens
+  uint64_t kvb, dma;      // bytes per token, bytes per us
+  uint32_t max_sessions;
+};
+
 struct ReplayState {
   Sorted S, H;      // unpinned residents per tier
   uint4 *pin;       // pinned residents
@@ -330,7 +338,7 @@ __device__ __forceinline__ uint32_t esize(uint4 v) { return v.z & kSizeMask; }
 // A session demoted out of the fast tier enters HBM, displacing the most
 // evictable unpinned HBM sessions, or is dropped when it is itself the most
 // evictable of (unpinned HBM) + {itself}.
-__device__ __forceinline__ bool admit_demoted(ReplayState &st, const ReplayDesc &D, uint4 d, int lane) {
+__device__ __forceinline__ bool admit_demoted(ReplayState &st, const Hot &D, uint4 d, int lane) {
   const uint32_t id = packed_id(ekey(d));
   const uint32_t size = esize(d);
   if (st.pinned_h > D.cap_h || size > D.cap_h - st.pinned_h) {
@@ -369,7 +377,7 @@ __device__ __forceinline__ bool pin_append(ReplayState &st, uint64_t pk, uint32_
 }
 
 // Placement of the arriving (pinned) session s with n tokens.
-__device__ __forceinline__ bool place(ReplayState &st, const ReplayDesc &D, uint32_t s, uint64_t pk, uint32_t n,
+__device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s, uint64_t pk, uint32_t n,
                                       int lane) {
   if (D.max_sessions && st.npin >= D.max_sessions) {
     log_dec(st, UNISON_KIND_BYPASS, s, lane);
@@ -437,7 +445,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const ReplayDesc &D, uint
 // free fast-tier space; phase 2: pair the next least evictable HBM session
 // with the most evictable fast-tier one), which makes the same moves as the
 // pair loop of Algorithm 1, and are then applied in bulk.
-__device__ __forceinline__ uint64_t tide(ReplayState &st, const ReplayDesc &D, uint64_t budget, uint32_t rcap_s,
+__device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t budget, uint32_t rcap_s,
                                          int lane) {
   uint64_t rem = budget;
   const uint64_t kvb = D.kvb;
@@ -566,6 +574,7 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
   if (lane == 0) Dsh = descs[order[blockIdx.x]];
   __syncwarp();
   const ReplayDesc &D = Dsh;
+  const Hot hot{D.cap_s, D.cap_h, D.kvb, D.dma, D.max_sessions};
 
   ReplayState st;
   {
@@ -757,7 +766,7 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
           pk = pack_key(nr == kNoRef ? kKeyMax40 : (uint64_t)nr, s);
         } else
           pk = pack_key(0xFFFFFFFFull - e, s);
-        if (!place(st, D, s, pk, out, lane)) break;
+        if (!place(st, hot, s, pk, out, lane)) break;
       } else {
         // completion: unpin (if resident) and rank the session with its new key
         int mine = -1;
@@ -791,7 +800,7 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
           const uint64_t g = sgq[bi][j];
           const uint64_t budget = g * D.dma;
           CNT(st, n_tide_calls, 1);
-          const uint64_t moved = tide(st, D, budget, D.rcap_s, lane);
+          const uint64_t moved = tide(st, hot, budget, D.rcap_s, lane);
           CNT(st, dma_bytes, moved);
           if (moved > 0 && D.dma > 0) {
             dma_busy = true;
