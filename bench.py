@@ -239,6 +239,21 @@ def kendall_fp32_vs_fixed(B, host_rec, sigma, stream, n: int = 1 << 20):
             "float": "float32 g*Lambda/sigma_q + (Lambda-sigma_q)*P_Z/Lambda"}
 
 
+def sweep_ase(B, results, reps, lib_params):
+    """Eq. (ase) over the sweep: its 128 settings (fast/HBM capacity pair x
+    window x bucket) compared on its 8 traces (seed-major replay order)."""
+    n_seeds = 1 + max(ti for ti, _ in reps)
+    per = len(reps) // n_seeds
+    grid = [[B.stats(results[d * per + c], lib_params[d * per + c]) for d in range(n_seeds)] for c in range(per)]
+    vals = B.ase(grid)
+    order = sorted(range(per), key=lambda c: -vals[c])
+    desc = lambda c: {"cap_fast_gib": lib_params[c]["cap_fast_bytes"] >> 30,
+                      "cap_hbm_gib": lib_params[c]["cap_hbm_bytes"] >> 30,
+                      "window": lib_params[c]["ema_den"] - 1, "bucket": lib_params[c]["hazard_bucket"]}
+    return {"settings": per, "traces": n_seeds, "best": [dict(desc(c), ase=vals[c]) for c in order[:3]],
+            "median": sorted(vals)[per // 2], "worst": vals[order[-1]]}
+
+
 def cpu_baseline_replay(trs, reps, budget_s: float = 12.0):
     """The oracle as it stands, single-threaded, on a bounded sample of the
     sweep's replays (spread over the batch) until budget_s of CPU work."""
@@ -358,9 +373,12 @@ def main():
     for _ in range(args.warmup):
         step()
     torch.cuda.synchronize()
+    ase = None
     if not args.rank_only:
         res = B.results_from_tensor(res_dev)
         assert all(r["status"] == 0 for r in res), "replay status"
+        if len(res) == 1024:
+            ase = sweep_ase(B, res, reps, lib_params)
     if not args.replay_only:
         assert all(B.rank_result(o)["status"] == 0 for o in rank_outs), "rank status"
 
@@ -477,7 +495,7 @@ def main():
                                    "paper-scale coding trace, 131072 B/token, SPEAR+TIDE)",
                        "replays": n_rep, "events_per_step": events_per_step,
                        "l2": "flushed before every step (256 MiB write, inside the timed region)"},
-            "roofline": roofline, "rank": rank_leg, "rank_sizes": sizes, "rank_kendall": tau, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roofline, "rank": rank_leg, "rank_sizes": sizes, "rank_kendall": tau, "sweep_ase": ase, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches, "clocks": clocks,
             "peaks": {"hbm_gbs": peaks.get("hbm_gbs"), "source": "MEASURED_PEAKS.json"}}
     if cpu is not None:

@@ -272,6 +272,19 @@ typedef struct {
 } unison_stats_t;
 int unison_stats(const unison_replay_result *r, const unison_replay_params *p, unison_stats_t *out);
 
+/* Agent Serving Effectiveness (Sec. IV-E, eq. ase) of n_configs
+ * configurations compared over n_datasets datasets (traces):
+ *   ASE_c = ( prod_d  HR_cd / HR_d^max  *  AMAT_d^min / AMAT_cd
+ *                     *  TTFT_d^min / TTFT_cd ) ^ (1 / (3 n_datasets)),
+ * the extremes taken over the n_configs configurations of dataset d.
+ * stats: host array [n_configs][n_datasets] of unison_stats outputs (TTFT is
+ * ttft_mean_ns); ase_out: host double[n_configs], each in [0, 1].  Readings:
+ * a ratio 0/0 (every configuration at 0) counts as 1; a zero AMAT or TTFT
+ * minimum against a positive value gives a factor 0, so ASE_c = 0.
+ * n_configs, n_datasets >= 1, else UNISON_ERR_ARG; a negative or non-finite
+ * metric gives UNISON_ERR_RANGE. */
+int unison_ase(const unison_stats_t *stats, int n_configs, int n_datasets, double *ase_out);
+
 /* ============================================================ hazard LUT */
 /* The survival table of eqs. (hazard), (hq), (survq) built on the device
  * from turns-per-session counts: n(t) = #{T_s >= t+1}, d(t) = #{T_s = t+1}

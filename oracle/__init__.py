@@ -80,7 +80,7 @@ def build(force: bool = False) -> str:
     if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
         tmp = _LIB + f".tmp{os.getpid()}"
         subprocess.check_call(["gcc", "-O2", "-std=gnu11", "-ffp-contract=off", "-fPIC", "-shared",
-                               "-o", tmp, _SRC])
+                               "-o", tmp, _SRC, "-lm"])
         os.replace(tmp, _LIB)
     return _LIB
 
@@ -105,6 +105,8 @@ def lib():
             L.or_rank.restype = C.c_int
             L.or_kendall_brute.argtypes = [C.c_void_p, C.c_void_p, C.c_uint64]
             L.or_kendall_brute.restype = C.c_double
+            L.or_ase.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_void_p]
+            L.or_ase.restype = None
             _lib = L
     return _lib
 
@@ -208,3 +210,15 @@ def kendall_brute(x, y) -> float:
     a = np.ascontiguousarray(x, dtype=np.float64)
     b = np.ascontiguousarray(y, dtype=np.float64)
     return float(lib().or_kendall_brute(_ptr(a), _ptr(b), a.shape[0]))
+
+
+def ase(hit_rate, amat, ttft):
+    """Eq. (ase) per configuration: arrays [n_configs][n_datasets] of HR,
+    AMAT and TTFT; returns n_configs values."""
+    hr = np.ascontiguousarray(hit_rate, dtype=np.float64)
+    am = np.ascontiguousarray(amat, dtype=np.float64)
+    tt = np.ascontiguousarray(ttft, dtype=np.float64)
+    nc, nd = hr.shape
+    out = np.zeros(nc, dtype=np.float64)
+    lib().or_ase(_ptr(hr), _ptr(am), _ptr(tt), nc, nd, _ptr(out))
+    return out

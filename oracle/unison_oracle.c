@@ -28,6 +28,7 @@
  *       else H, else bypass.
  *   R10 request accounting (warm = turn >= 1).
  *   R11 TIDE budget in bytes = g_q(us) * dma bytes per us.
+ *   R25 ASE: a metric ratio 0/0 counts as 1.
  *   R12 a completed session stays resident with the maximal key.
  *   R13 DMA busy until now + ceil(moved / dma bytes per us).
  *   R14 TIDE phase 1 (promotion into free fast-tier space) then phase 2
@@ -39,6 +40,7 @@
  *   R19 prefetch accuracy: promoted sessions whose next request hits the
  *       fast tier.
  */
+#include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
@@ -842,4 +844,30 @@ double or_kendall_brute(const double *x, const double *y, uint64_t n) {
   double n0 = c + d + tx, n1 = c + d + ty;
   if (n0 == 0 || n1 == 0) return 0.0;
   return (c - d) / __builtin_sqrt(n0 * n1);
+}
+
+/* ====================================================================== */
+/* Agent Serving Effectiveness (Sec. IV-E, Eq. ase)                        */
+/* ====================================================================== */
+
+/* ASE of each configuration c over datasets d: the 3*nd-th root of the
+ * product, over d, of HR_cd/HR_d^max, AMAT_d^min/AMAT_cd, TTFT_d^min/TTFT_cd
+ * (extremes over the configurations).  Arrays are [nc][nd].  Reading R25: a
+ * ratio 0/0 (every configuration at 0 on that metric) counts as 1. */
+void or_ase(const double *hr, const double *amat, const double *ttft, int nc, int nd, double *out) {
+  for (int c = 0; c < nc; c++) {
+    double prod = 1.0;
+    for (int d = 0; d < nd; d++) {
+      double hr_max = 0.0, amat_min = amat[d], ttft_min = ttft[d];
+      for (int c2 = 0; c2 < nc; c2++) {
+        if (hr[c2 * nd + d] > hr_max) hr_max = hr[c2 * nd + d];
+        if (amat[c2 * nd + d] < amat_min) amat_min = amat[c2 * nd + d];
+        if (ttft[c2 * nd + d] < ttft_min) ttft_min = ttft[c2 * nd + d];
+      }
+      prod *= hr_max == 0.0 ? 1.0 : hr[c * nd + d] / hr_max;
+      prod *= amat[c * nd + d] == 0.0 ? 1.0 : amat_min / amat[c * nd + d];
+      prod *= ttft[c * nd + d] == 0.0 ? 1.0 : ttft_min / ttft[c * nd + d];
+    }
+    out[c] = pow(prod, 1.0 / (3.0 * nd));
+  }
 }

@@ -91,7 +91,7 @@ EXPORTS = ["unison_strerror", "unison_version", "unison_trace_create", "unison_t
            "unison_trace_upload", "unison_trace_free", "unison_trace_info", "unison_trace_device_bytes",
            "unison_replay_batch", "unison_stats", "unison_hazard_lut", "unison_rank_batch",
            "unison_profile_enable", "unison_profile_read", "unison_launch_count",
-           "unison_replay_batch_noalloc"]
+           "unison_replay_batch_noalloc", "unison_ase"]
 
 
 def lib_path() -> str:
@@ -130,6 +130,7 @@ def lib():
             L.unison_profile_read.argtypes = [C.c_char_p, C.POINTER(C.c_double), C.POINTER(C.c_uint64), C.c_int]
             L.unison_launch_count.restype = C.c_uint64
             L.unison_replay_batch_noalloc.argtypes = L.unison_replay_batch.argtypes
+            L.unison_ase.argtypes = [C.POINTER(Stats), C.c_int, C.c_int, C.POINTER(C.c_double)]
             _lib = L
     return _lib
 
@@ -273,6 +274,22 @@ def stats(result: dict, params: dict) -> dict:
     s = Stats()
     _check("unison_stats", lib().unison_stats(C.byref(r), C.byref(p), C.byref(s)))
     return {f: getattr(s, f) for f, _ in Stats._fields_}
+
+
+def ase(stats_grid) -> List[float]:
+    """unison_ase over stats_grid[config][dataset] (dicts as returned by
+    stats(): hit_rate, amat_ps, ttft_mean_ns, ...): one value per config."""
+    nc = len(stats_grid)
+    nd = len(stats_grid[0]) if nc else 0
+    arr = (Stats * (nc * nd))()
+    for c, row in enumerate(stats_grid):
+        if len(row) != nd:
+            raise ValueError("every configuration needs the same datasets")
+        for d, st in enumerate(row):
+            arr[c * nd + d] = Stats(*[float(st.get(f, 0.0)) for f, _ in Stats._fields_])
+    out = (C.c_double * max(nc, 1))()
+    _check("unison_ase", lib().unison_ase(arr, nc, nd, out))
+    return [out[i] for i in range(nc)]
 
 
 def hazard_lut(turns_dev, bucket: int = 1, stream=None):

@@ -20,6 +20,7 @@
 //   ttft_median_kernel  Sec. V-A TTFT p50: radix select of the lower median
 //                       over each replay's per-request TTFT values.
 #include <algorithm>
+#include <cmath>
 #include <map>
 #include <mutex>
 #include <tuple>
@@ -1204,6 +1205,47 @@ extern "C" int unison_stats(const unison_replay_result *r, const unison_replay_p
   const long double sum = (long double)r->ttft_sum_hi * 18446744073709551616.0L + (long double)r->ttft_sum_lo;
   out->ttft_mean_ns = r->ttft_n ? (double)(sum / r->ttft_n) : 0.0;
   out->ttft_p50_ns = (double)r->ttft_p50_ns;
+  return UNISON_OK;
+}
+
+// Eq. (ase), accumulated as a mean of logarithms (many datasets would
+// underflow a plain product).
+extern "C" int unison_ase(const unison_stats_t *stats, int n_configs, int n_datasets, double *ase_out) {
+  if (!stats || !ase_out || n_configs < 1 || n_datasets < 1) return UNISON_ERR_ARG;
+  const size_t nc = (size_t)n_configs, nd = (size_t)n_datasets;
+  for (size_t i = 0; i < nc * nd; i++) {
+    const unison_stats_t &x = stats[i];
+    if (!std::isfinite(x.hit_rate) || !std::isfinite(x.amat_ps) || !std::isfinite(x.ttft_mean_ns) ||
+        x.hit_rate < 0 || x.amat_ps < 0 || x.ttft_mean_ns < 0)
+      return UNISON_ERR_RANGE;
+  }
+  std::vector<double> logsum(nc, 0.0);
+  std::vector<char> zero(nc, 0);
+  for (size_t d = 0; d < nd; d++) {
+    double hr_max = 0.0, amat_min = INFINITY, ttft_min = INFINITY;
+    for (size_t c = 0; c < nc; c++) {
+      const unison_stats_t &x = stats[c * nd + d];
+      hr_max = std::max(hr_max, x.hit_rate);
+      amat_min = std::min(amat_min, x.amat_ps);
+      ttft_min = std::min(ttft_min, x.ttft_mean_ns);
+    }
+    // factor num/den of one metric: 0/0 counts as 1, 0/positive as 0
+    auto factor = [&](size_t c, double num, double den) {
+      if (den == 0.0) return;  // then num == 0 as well (num <= den): 1
+      if (num == 0.0) {
+        zero[c] = 1;
+        return;
+      }
+      logsum[c] += std::log(num / den);
+    };
+    for (size_t c = 0; c < nc; c++) {
+      const unison_stats_t &x = stats[c * nd + d];
+      factor(c, x.hit_rate, hr_max);
+      factor(c, amat_min, x.amat_ps);
+      factor(c, ttft_min, x.ttft_mean_ns);
+    }
+  }
+  for (size_t c = 0; c < nc; c++) ase_out[c] = zero[c] ? 0.0 : std::exp(logsum[c] / (3.0 * (double)nd));
   return UNISON_OK;
 }
 

@@ -119,3 +119,26 @@ def test_stats_definitions(B):
 def test_oracle_library_loads_standalone():
     import oracle
     assert oracle.spear_score(3_000_000, 41) == 794_628_040
+
+
+def test_ase_library_matches_oracle(B):
+    """unison_ase (host function of the library) against the oracle's plain
+    product, and its argument checks."""
+    import oracle
+    rs = np.random.default_rng(7)
+    for nc, nd in ((1, 1), (3, 6), (17, 8)):
+        hr = rs.uniform(0.0, 1.0, (nc, nd))
+        am = rs.uniform(1e5, 1e9, (nc, nd))
+        tt = rs.uniform(1e3, 1e9, (nc, nd))
+        if nc > 2:
+            hr[:, 0] = 0.0
+            am[1, -1] = 0.0
+        grid = [[dict(hit_rate=hr[c, d], amat_ps=am[c, d], ttft_mean_ns=tt[c, d]) for d in range(nd)]
+                for c in range(nc)]
+        got = np.array(B.ase(grid))
+        want = oracle.ase(hr, am, tt)
+        assert np.allclose(got, want, rtol=1e-12, atol=0), (nc, nd, got, want)
+    with pytest.raises(B.UnisonError):
+        B.ase([[dict(hit_rate=-1.0, amat_ps=1.0, ttft_mean_ns=1.0)]])
+    with pytest.raises(B.UnisonError):
+        B.ase([])

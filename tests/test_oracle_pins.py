@@ -427,3 +427,56 @@ def test_kendall_brute_matches_scipy():
         x = rs.integers(0, 20, n).astype(float)
         y = x + rs.normal(0, 3, n).round()
         assert abs(oracle.kendall_brute(x, y) - stats.kendalltau(x, y).statistic) < 1e-12
+
+
+# ------------------------------------------------------------------ ASE --
+def test_ase_hand_values():
+    rows, want = {}, {}
+    for line in _rows("ase_hand.txt"):
+        tag, *rest = line.split()
+        if tag == "row":
+            c, d, hr, am, tt = rest
+            rows[(int(c), int(d))] = (float(hr), float(am), float(tt))
+        else:
+            want[int(rest[0])] = float(rest[1])
+    nc, nd = 1 + max(c for c, _ in rows), 1 + max(d for _, d in rows)
+    grid = np.array([[rows[(c, d)] for d in range(nd)] for c in range(nc)])
+    got = oracle.ase(grid[:, :, 0], grid[:, :, 1], grid[:, :, 2])
+    for c, v in want.items():
+        assert abs(got[c] - v) < 1e-15
+
+
+def _ase_grid(seed, nc=5, nd=4):
+    rs = np.random.default_rng(seed)
+    return rs.uniform(0.05, 0.9, (nc, nd)), rs.uniform(1e5, 1e8, (nc, nd)), rs.uniform(1e3, 1e9, (nc, nd))
+
+
+def test_ase_closed_forms():
+    hr, am, tt = _ase_grid(3)
+    # identical configurations: every ratio is 1
+    one = oracle.ase(np.tile(hr[:1], (4, 1)), np.tile(am[:1], (4, 1)), np.tile(tt[:1], (4, 1)))
+    assert np.allclose(one, 1.0, rtol=0, atol=1e-15)
+    # a configuration at the best value of every metric on every dataset scores 1
+    hr2, am2, tt2 = hr.copy(), am.copy(), tt.copy()
+    hr2[2], am2[2], tt2[2] = hr.max(0), am.min(0), tt.min(0)
+    a = oracle.ase(hr2, am2, tt2)
+    assert abs(a[2] - 1.0) < 1e-15 and (a <= 1.0 + 1e-15).all()
+    # each metric is a ratio within a dataset: scaling it by a per-dataset constant changes nothing
+    s = np.array([3.0, 0.5, 7.0, 11.0])
+    assert np.allclose(oracle.ase(hr * s, am * s, tt / s), oracle.ase(hr, am, tt), rtol=1e-14)
+    # one dataset: the cube root of the three ratios, written out
+    h1, m1, t1 = hr[:, :1], am[:, :1], tt[:, :1]
+    direct = ((h1 / h1.max()) * (m1.min() / m1) * (t1.min() / t1)) ** (1 / 3)
+    assert np.allclose(oracle.ase(h1, m1, t1), direct[:, 0], rtol=1e-14)
+
+
+def test_ase_zero_readings():
+    hr, am, tt = _ase_grid(4, nc=3, nd=2)
+    hr[:, 0] = 0.0                     # no configuration hits on dataset 0: factor 1 for all (0/0)
+    base = oracle.ase(hr, am, tt)
+    hr1 = hr.copy()
+    hr1[:, 0] = 0.5                    # equal positive values are also factor 1
+    assert np.allclose(base, oracle.ase(hr1, am, tt), rtol=1e-14)
+    am[1, 1] = 0.0                     # a zero AMAT minimum: the others' factor is 0
+    z = oracle.ase(hr, am, tt)
+    assert z[0] == 0.0 and z[2] == 0.0 and z[1] > 0.0
