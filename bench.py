@@ -189,7 +189,8 @@ def rank_size_sweep(B, host_rec, sigma, stream, steps: int = 10, warmup: int = 3
             call.run(stream)
         torch.cuda.synchronize()
         assert all(B.rank_result(o)["status"] == 0 for o in outs), "rank status"
-        B.profile_read("rank_filter", reset=True)
+        for kname in ("rank_sample", "rank_filter", "rank_finish"):
+            B.profile_read(kname, reset=True)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for _ in range(steps):
@@ -198,10 +199,13 @@ def rank_size_sweep(B, host_rec, sigma, stream, steps: int = 10, warmup: int = 3
         torch.cuda.synchronize()
         call_us = 1e3 * e0.elapsed_time(e1) / steps
         f_ms, f_n = B.profile_read("rank_filter", reset=True)
+        sm_ms, sm_n = B.profile_read("rank_sample", reset=True)
+        fi_ms, fi_n = B.profile_read("rank_finish", reset=True)
         recs = n * n_sets
         gbs = recs * RANK_BYTES_PER_RECORD / (call_us / 1e6) / 1e9
         filter_us = 1e3 * f_ms / max(f_n, 1) if f_n else None
-        out.append({"n": n, "sets_per_call": n_sets, "call_us": call_us, "filter_us": filter_us, "call_gbs": gbs,
+        out.append({"n": n, "sets_per_call": n_sets, "call_us": call_us, "filter_us": filter_us,
+                    "sample_us": 1e3 * sm_ms / max(sm_n, 1), "finish_us": 1e3 * fi_ms / max(fi_n, 1), "call_gbs": gbs,
                     "filter_gbs": recs * RANK_BYTES_PER_RECORD / (filter_us / 1e6) / 1e9 if filter_us else None,
                     "l2_resident": recs * RANK_BYTES_PER_RECORD < (2 * 129 << 20)})
         del call, sets, outs
@@ -363,12 +367,21 @@ def main():
     rank_outs = [B.rank_outputs(RANK_N, p["k"], p["max_moves"]) for p in r_params]
     rank_bytes = len(r_params) * RANK_N * RANK_BYTES_PER_RECORD
 
-    def step():
+    rank_call = B.rank_prepare(rank_sets, r_params, rank_outs) if not args.replay_only else None
+    rank_marks = []  # (start, end) events around each timed rank call
+
+    def step(mark=False):
         flush.zero_()
         if not args.rank_only:
             B.replay_batch_async(handles, lib_params, res_dev, stream=stream)
         if not args.replay_only:
-            B.rank_batch(rank_sets, r_params, rank_outs, stream=stream)
+            if mark:
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+            rank_call.run(stream)
+            if mark:
+                b.record(stream)
+                rank_marks.append((a, b))
 
     for _ in range(args.warmup):
         step()
@@ -396,7 +409,7 @@ def main():
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(args.steps):
-        step()
+        step(mark=True)
     e1.record(stream)
     torch.cuda.synchronize()
     barrier()
@@ -484,7 +497,10 @@ def main():
                 "call_ms": call_ms, "call_gbs": rank_bytes / (call_ms / 1e3) / 1e9,
                 "call_frac_of_peak": rank_bytes / (call_ms / 1e3) / 1e9 / hbm_peak,
                 "records_per_s": len(r_params) * RANK_N / (call_ms / 1e3),
-                "sample_ms": rs_ms / max(rs_n, 1), "filter_ms": avg_rf, "finish_ms": rn_ms / max(rn_n, 1)}
+                "sample_ms": rs_ms / max(rs_n, 1), "filter_ms": avg_rf, "finish_ms": rn_ms / max(rn_n, 1),
+                # the whole API call on its stream: kernels plus the upload and launch gaps
+                "call_ms_events": (sum(a.elapsed_time(b) for a, b in rank_marks) / len(rank_marks)
+                                   if rank_marks else None)}
     if rank != 0:
         return
     cpu = None if (args.no_cpu_baseline or world > 1) else cpu_baseline_replay(trs, reps)

@@ -24,6 +24,8 @@
 //                        set.  The set's last CTA writes the victims and runs
 //                        the fill as warp prefix scans.
 #include <algorithm>
+#include <map>
+#include <cstring>
 #include <mutex>
 #include <type_traits>
 #include <vector>
@@ -304,8 +306,10 @@ __host__ __device__ __forceinline__ uint64_t list_target_of(const RankSet &S, in
   const uint32_t M = (L == 0) ? S.k : S.max_moves;
   return wide ? 6ull * M + 2048 : 2ull * M + 1024;
 }
-__host__ __device__ __forceinline__ uint32_t sample_ctas(uint32_t ns) {
-  return ns ? (ns + kSampleThreads - 1) / kSampleThreads : 1u;
+// q samples per thread (1 or 4: more samples per CTA make a CTA slower but
+// let many sets' sample CTAs fit in one wave).
+__host__ __device__ __forceinline__ uint32_t sample_ctas(uint32_t ns, uint32_t q) {
+  return ns ? (ns + kSampleThreads * q - 1) / (kSampleThreads * q) : 1u;
 }
 // Sample size for the given targets (0: no sample, the whole set qualifies).
 __host__ __device__ __forceinline__ uint64_t sample_size_raw(const RankSet &S, bool wide) {
@@ -321,9 +325,9 @@ __host__ __device__ __forceinline__ bool wide_targets(const RankSet &S) { return
 __host__ __device__ __forceinline__ uint64_t list_target(const RankSet &S, int L) {
   return list_target_of(S, L, wide_targets(S));
 }
-__host__ __device__ __forceinline__ uint32_t sample_size(const RankSet &S) {
+__host__ __device__ __forceinline__ uint32_t sample_size(const RankSet &S, uint32_t q) {
   uint64_t ns = umin64(sample_size_raw(S, wide_targets(S)), kSample);
-  const uint32_t step = 8 * sample_ctas((uint32_t)ns);
+  const uint32_t step = 8 * sample_ctas((uint32_t)ns, q);
   ns -= ns % step;  // whole runs, evenly split over the CTAs
   return (uint32_t)ns;
 }
@@ -440,6 +444,7 @@ __device__ void joint_select32(const uint32_t (&v)[kLists][Q], uint32_t has, uin
 // into the list's threshold: the smallest list value with that summary (at
 // least r_L samples reach it), plus, per turn index, the smallest gap whose
 // key reaches the threshold's key (gA) or exceeds it (gB).
+template <int Q>
 __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankSet *sets) {
   const RankSet &S = sets[blockIdx.y];
   const uint32_t c = blockIdx.x;  // this CTA's share of the sample
@@ -461,34 +466,45 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
   }
   __syncthreads();
   const uint32_t ns = S.ns, act = S.act;
-  const uint32_t per = ns / nct;  // samples of this CTA (<= 1024, a multiple of 8)
+  const uint32_t per = ns / nct;  // samples of this CTA (<= 1024 Q, a multiple of 8)
   uint32_t rL[kLists];
 #pragma unroll
   for (int L = 0; L < kLists; L++) rL[L] = S.rL[L];
-  // 1. this thread's sample
-  uint32_t f[kLists][1] = {{0}, {0}, {0}};
-  uint32_t m = 0;
-  if (tid < per) {
-    // stratum bounds floor(run n / nruns) with n = sq nruns + srem, in 32 bits
-    const uint32_t nruns = S.nruns, run = c * (per / 8) + tid / 8, o = tid % 8;
-    const uint32_t lo = run * S.sq + (run * S.srem) / nruns;
-    const uint32_t hi = (run + 1) * S.sq + ((run + 1) * S.srem) / nruns;
-    uint32_t h = run * 0x9E3779B1u;
-    h ^= h >> 16;
-    h *= 0x85EBCA6Bu;
-    h ^= h >> 13;
-    const uint32_t span = hi - lo - 8;  // strata hold at least 8 records
-    const uint32_t r = lo + (h % (span + 1)) + o;
-    const uint8_t fl = S.flags[r], tr = S.tier[r];
-    const uint32_t t = min((uint32_t)S.turn[r], kTMax);
-    const uint64_t ck = ck_of(score_of(S.gap[r], t, (fl & 2) != 0, t2s, mgs), r);
-    m = elig_mask(fl, tr) & act;
+  // 1. this thread's samples j = tid + 1024 q: run j / 8 of the CTA's share
+  uint32_t f[kLists][Q];
+  uint32_t m = 0;  // bit L * Q + q: sample q is eligible for list L
 #pragma unroll
-    for (int L = 0; L < kLists; L++) f[L][0] = summary_of(list_val(ck, L));
+  for (int q = 0; q < Q; q++) {
+#pragma unroll
+    for (int L = 0; L < kLists; L++) f[L][q] = 0;
+    const uint32_t jt = tid + kSampleThreads * q;
+    if (jt < per) {
+      // stratum bounds floor(run n / nruns) with n = sq nruns + srem, in 32 bits
+      const uint32_t nruns = S.nruns, run = c * (per / 8) + jt / 8, o = jt % 8;
+      const uint32_t lo = run * S.sq + (run * S.srem) / nruns;
+      const uint32_t hi = (run + 1) * S.sq + ((run + 1) * S.srem) / nruns;
+      uint32_t h = run * 0x9E3779B1u;
+      h ^= h >> 16;
+      h *= 0x85EBCA6Bu;
+      h ^= h >> 13;
+      const uint32_t span = hi - lo - 8;  // strata hold at least 8 records
+      const uint32_t r = lo + (h % (span + 1)) + o;
+      const uint8_t fl = S.flags[r], tr = S.tier[r];
+      const uint32_t t = min((uint32_t)S.turn[r], kTMax);
+      const uint64_t ck = ck_of(score_of(S.gap[r], t, (fl & 2) != 0, t2s, mgs), r);
+      const uint32_t em = elig_mask(fl, tr) & act;
+#pragma unroll
+      for (int L = 0; L < kLists; L++) {
+        f[L][q] = summary_of(list_val(ck, L));
+        m |= ((em >> L) & 1u) << (L * Q + q);
+      }
+    }
   }
 #pragma unroll
   for (int L = 0; L < kLists; L++) {
-    const uint32_t cnt = __popc(__ballot_sync(kFull, (m >> L) & 1));
+    uint32_t cnt = 0;
+#pragma unroll
+    for (int q = 0; q < Q; q++) cnt += __popc(__ballot_sync(kFull, (m >> (L * Q + q)) & 1));
     if (lane == 0 && cnt) atomicAdd(&ecount[L], cnt);
   }
   __syncthreads();
@@ -500,19 +516,22 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
     need[L] = rL[L];
     if (rL[L] && ecount[L] > rL[L]) sel |= 1u << L;
   }
-  if (sel) joint_select32<1>(f, m, sel, need, T, hist, pick);
+  if (sel) joint_select32<Q>(f, m, sel, need, T, hist, pick);
 #pragma unroll
   for (int L = 0; L < kLists; L++) {
     if (!rL[L]) continue;
     const bool all = !((sel >> L) & 1);  // keep every eligible sample
-    const bool has = (m >> L) & 1;
-    const bool above = has && (all || f[L][0] > T[L]);
-    const unsigned bal = __ballot_sync(kFull, above);
-    unsigned wbase = 0;
-    if (lane == 0 && bal) wbase = atomicAdd(&wpos[L], (unsigned)__popc(bal));
-    wbase = __shfl_sync(kFull, wbase, 0);
     uint32_t *dst = S.part + ((size_t)L * kSampleCtas + c) * kMaxR;
-    if (above) dst[wbase + __popc(bal & ((1u << lane) - 1))] = f[L][0];
+#pragma unroll
+    for (int q = 0; q < Q; q++) {
+      const bool has = (m >> (L * Q + q)) & 1;
+      const bool above = has && (all || f[L][q] > T[L]);
+      const unsigned bal = __ballot_sync(kFull, above);
+      unsigned wbase = 0;
+      if (lane == 0 && bal) wbase = atomicAdd(&wpos[L], (unsigned)__popc(bal));
+      wbase = __shfl_sync(kFull, wbase, 0);
+      if (above) dst[wbase + __popc(bal & ((1u << lane) - 1))] = f[L][q];
+    }
   }
   __syncthreads();
   // ties at the rank-r_L summary fill each partial list up to r_L entries
@@ -548,13 +567,13 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
   }
   uint32_t T2[kLists] = {0, 0, 0};
   auto merge = [&](auto qtag) {
-    constexpr int Q = decltype(qtag)::value;
-    uint32_t vq[kLists][Q];
+    constexpr int QM = decltype(qtag)::value;
+    uint32_t vq[kLists][QM];
     uint32_t hq = 0;
 #pragma unroll
     for (int L = 0; L < kLists; L++) {
 #pragma unroll
-      for (int q = 0; q < Q; q++) {
+      for (int q = 0; q < QM; q++) {
         vq[L][q] = 0;
         // entry e of the concatenation: CTA e / r_L, slot e % r_L
         const uint32_t e = tid + kSampleThreads * q;
@@ -562,11 +581,11 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
         const uint32_t cc = e / rL[L], slot = e % rL[L];
         if (cc < nct && slot < pn[L * kSampleCtas + cc]) {
           vq[L][q] = __ldcg(&S.part[((size_t)L * kSampleCtas + cc) * kMaxR + slot]);
-          hq |= 1u << (L * Q + q);
+          hq |= 1u << (L * QM + q);
         }
       }
     }
-    joint_select32<Q>(vq, hq, sel2, rL, T2, hist, pick);
+    joint_select32<QM>(vq, hq, sel2, rL, T2, hist, pick);
   };
   if (sel2) {
     if (nct * rmax <= kSampleThreads) merge(std::integral_constant<int, 1>());
@@ -1450,11 +1469,95 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
+// Device scratch of the ranking calls, kept per (device, stream) and grown
+// when a call needs more: calls on one stream run in order, so each reuses
+// the buffer after the previous one is done with it (stream order), and
+// calls on different streams get different buffers.  Held for the life of
+// the process.
+std::mutex g_scratch_mu;
+std::map<std::pair<int, cudaStream_t>, std::pair<char *, size_t>> g_scratch;
+
+int scratch_acquire(cudaStream_t stream, size_t bytes, char **out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return UNISON_ERR_CUDA;
+  }
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  auto &e = g_scratch[std::make_pair(dev, stream)];
+  if (e.second < bytes) {
+    if (e.first) cudaFreeAsync(e.first, stream);  // ordered after the calls that used it
+    e.first = nullptr;
+    e.second = 0;
+    char *p = nullptr;
+    if (cudaMallocAsync(reinterpret_cast<void **>(&p), bytes, stream) != cudaSuccess) {
+      cudaGetLastError();
+      return UNISON_ERR_OOM;
+    }
+    e.first = p;
+    e.second = bytes;
+  }
+  *out = e.first;
+  return UNISON_OK;
+}
+
+// Pinned host staging for the per-call upload, a ring of buffers per device.
+// A buffer is handed out only after the copy that last read it has finished
+// (its event); staging_release() ends the caller's hold.
+struct Staging {
+  unsigned char *host = nullptr;
+  size_t cap = 0;
+  cudaEvent_t done = nullptr;
+};
+constexpr int kStagingRing = 4;
+std::mutex g_staging_mu;
+Staging g_staging[64][kStagingRing];
+int g_staging_next[64] = {};
+
+int staging_acquire(size_t bytes, unsigned char **host, cudaEvent_t *done) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
+    return UNISON_ERR_CUDA;
+  }
+  g_staging_mu.lock();
+  Staging &b = g_staging[dev][g_staging_next[dev]];
+  g_staging_next[dev] = (g_staging_next[dev] + 1) % kStagingRing;
+  if (b.done && cudaEventSynchronize(b.done) != cudaSuccess) {
+    cudaGetLastError();
+    g_staging_mu.unlock();
+    return UNISON_ERR_CUDA;
+  }
+  if (!b.done && cudaEventCreateWithFlags(&b.done, cudaEventDisableTiming) != cudaSuccess) {
+    cudaGetLastError();
+    b.done = nullptr;
+    g_staging_mu.unlock();
+    return UNISON_ERR_CUDA;
+  }
+  if (b.cap < bytes) {
+    if (b.host) cudaFreeHost(b.host);
+    b.host = nullptr;
+    b.cap = 0;
+    const size_t cap = std::max<size_t>(bytes, 64 << 10);
+    if (cudaMallocHost(reinterpret_cast<void **>(&b.host), cap) != cudaSuccess) {
+      cudaGetLastError();
+      b.host = nullptr;
+      g_staging_mu.unlock();
+      return UNISON_ERR_OOM;
+    }
+    b.cap = cap;
+  }
+  *host = b.host;
+  *done = b.done;
+  return UNISON_OK;  // the lock is held until staging_release()
+}
+void staging_release() { g_staging_mu.unlock(); }
+
 // Kernel attributes and the filter's resident-CTA count, set up once per
 // device (the attributes belong to the device's context).
 struct LaunchCfg {
   bool ok = false;
-  uint32_t filter_ctas = 0;
+  uint32_t filter_ctas = 0, n_sm = 0;
 };
 const LaunchCfg &launch_cfg() {
   static std::mutex mu;
@@ -1480,6 +1583,7 @@ const LaunchCfg &launch_cfg() {
                                 (int)smem_finish) == cudaSuccess;
     if (!c.ok) cudaGetLastError();
     c.filter_ctas = (uint32_t)std::max(1, n_sm * per_sm);
+    c.n_sm = (uint32_t)std::max(1, n_sm);
     cfgs[dev] = c;
     done[dev] = c.ok;
   }
@@ -1539,17 +1643,29 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
       s.t2v[t] = ((uint64_t)(kLambda - p.sigma_q[t]) * p.penalty_q) / kLambda;  // eq. (t2)
       s.mgv[t] = magic_for(p.sigma_q[t]);
     }
-    s.ns = sample_size(s);
-    s.sctas = sample_ctas(s.ns);
+    s.act = 0;
+    for (int L = 0; L < kLists; L++) s.act |= list_active(s, L) ? 1u << L : 0u;
+  }
+  const LaunchCfg &cfg = launch_cfg();
+  if (!cfg.ok) return UNISON_ERR_CUDA;
+  // samples per thread: 1 while every set's sample CTAs fit in one wave (two
+  // 1,024-thread CTAs per SM), else 4
+  uint32_t sq_per = 1;
+  {
+    uint64_t ctas1 = 0;
+    for (int i = 0; i < n_sets; i++) ctas1 += sample_ctas(sample_size(hs[i], 1), 1);
+    if (ctas1 > 2ull * cfg.n_sm) sq_per = 4;
+  }
+  for (int i = 0; i < n_sets; i++) {
+    RankSet &s = hs[i];
+    s.ns = sample_size(s, sq_per);
+    s.sctas = sample_ctas(s.ns, sq_per);
     s.nruns = s.ns / 8;
     s.sq = s.nruns ? s.n / s.nruns : 0;
     s.srem = s.nruns ? s.n % s.nruns : 0;
-    s.act = 0;
-    for (int L = 0; L < kLists; L++) {
-      s.act |= list_active(s, L) ? 1u << L : 0u;
+    for (int L = 0; L < kLists; L++)
       s.rL[L] = (s.ns && list_active(s, L))
                     ? (uint32_t)umin64((list_target(s, L) * s.ns + s.n - 1) / s.n, kMaxR) : 0u;
-    }
   }
   // scratch: descriptors, every set's work words (one memset), then per set:
   // thresholds, tables, sorted lists and sizes, candidates, the sample's
@@ -1563,10 +1679,9 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
   const size_t desc_b = align_up(sizeof(RankSet) * n_sets, 256);
   const size_t work_b = align_up(sizeof(RankWork) * n_sets, 256);
   char *scratch = nullptr;
-  if (cudaMallocAsync(reinterpret_cast<void **>(&scratch), desc_b + work_b + per_set * n_sets, stream) !=
-      cudaSuccess) {
-    cudaGetLastError();
-    return UNISON_ERR_OOM;
+  {
+    const int ar = scratch_acquire(stream, desc_b + work_b + per_set * n_sets, &scratch);
+    if (ar != UNISON_OK) return ar;
   }
   RankWork *works = reinterpret_cast<RankWork *>(scratch + desc_b);
   for (int i = 0; i < n_sets; i++) {
@@ -1594,11 +1709,6 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
   RankSet *d_sets = reinterpret_cast<RankSet *>(scratch);
   const size_t smem_finish = sizeof(uint64_t) * (kSmemCand + kMaxSel);
   // persistent filter: as many CTAs as fit at once (per device, set up once)
-  const LaunchCfg &cfg = launch_cfg();
-  if (!cfg.ok) {
-    cudaFreeAsync(scratch, stream);
-    return UNISON_ERR_CUDA;
-  }
   uint32_t grid_filter = std::max(1u, std::min<uint32_t>(tiles, cfg.filter_ctas));
   // Filter schedule: each set gets a group of CTAs in proportion to its tiles
   // (at least 1, at most its tile count) when the groups fit in the resident
@@ -1620,11 +1730,25 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
   }
   uint32_t max_sctas = 1;
   for (int i = 0; i < n_sets; i++) max_sctas = std::max(max_sctas, hs[i].sctas);
-  ck(cudaMemcpyAsync(d_sets, hs.data(), sizeof(RankSet) * n_sets, cudaMemcpyHostToDevice, stream));
-  ck(cudaMemsetAsync(works, 0, sizeof(RankWork) * n_sets, stream));
+  // descriptors and zeroed work words: one copy from pinned staging
+  {
+    const size_t up = desc_b + sizeof(RankWork) * n_sets;
+    unsigned char *h = nullptr;
+    cudaEvent_t done = nullptr;
+    const int sr = staging_acquire(up, &h, &done);
+    if (sr != UNISON_OK) return sr;
+    std::memcpy(h, hs.data(), sizeof(RankSet) * n_sets);
+    std::memset(h + desc_b, 0, sizeof(RankWork) * n_sets);
+    ck(cudaMemcpyAsync(d_sets, h, up, cudaMemcpyHostToDevice, stream));
+    ck(cudaEventRecord(done, stream));  // the buffer is reused after this copy
+    staging_release();
+  }
   {
     ProfSpan span("rank_sample", stream);
-    rank_sample_kernel<<<dim3(max_sctas, n_sets), kSampleThreads, 0, stream>>>(d_sets);
+    if (sq_per == 1)
+      rank_sample_kernel<1><<<dim3(max_sctas, n_sets), kSampleThreads, 0, stream>>>(d_sets);
+    else
+      rank_sample_kernel<4><<<dim3(max_sctas, n_sets), kSampleThreads, 0, stream>>>(d_sets);
   }
   {
     ProfSpan span("rank_filter", stream);
@@ -1636,6 +1760,5 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
   }
   count_launches(3);
   ck(cudaGetLastError());
-  ck(cudaFreeAsync(scratch, stream));
   return rc;
 }
