@@ -346,6 +346,15 @@ typedef struct {
  * is more evictable).  Results are exact: candidate thresholds come from a
  * sample, and a set whose candidates fall short is re-selected exactly on
  * the device.  sets, params, outs: host arrays [n_sets].  Asynchronous.
+ * Memory: the call's device scratch (about 2.2 MB per set) is kept per
+ * (device, stream) and grown when a call needs more, and the per-call
+ * descriptors go up from a small pinned host ring; both are held for the
+ * life of the process.  Calls on one stream run in order and share that
+ * stream's scratch; calls on different streams use different scratch.
+ * Errors: UNISON_ERR_ARG (null or misaligned arrays), UNISON_ERR_RANGE
+ * (limits above), UNISON_ERR_OOM (scratch or staging), UNISON_ERR_CUDA
+ * (launch); a bounded device wait that gives up sets counts[3] of its set to
+ * UNISON_ERR_TIMEOUT.
  */
 int unison_rank_batch(const unison_records *sets, const unison_rank_params *params,
                       const unison_rank_out *outs, int n_sets, void *cuda_stream);
