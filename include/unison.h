@@ -147,8 +147,17 @@ typedef struct {
   uint64_t t_h_ps_per_tok;
   uint64_t t_p_ps_per_tok;     /* prefill cost; TTFT uses t_p / 1000 ns per token */
   uint32_t ttft_load;          /* arrival compression factor of the TTFT queue    */
-  uint32_t reserved;
+  uint32_t flags;              /* UNISON_HAZARD_ONLINE, or 0                      */
 } unison_replay_params;
+
+/* Online hazard table (Sec. V-F, eq. attainment): instead of the table fitted
+ * on the whole trace, the table starts with no sessions, and the turn count
+ * of each session joins it at that session's final completion, which then
+ * re-ranks every resident under the rebuilt table before the next event.
+ * SPEAR and SPEAR+TIDE only (else UNISON_ERR_ARG); the trace must have at
+ * most 32,768 sessions and the replay's resident lists must fit in shared
+ * memory (else UNISON_ERR_RANGE). */
+#define UNISON_HAZARD_ONLINE 1u
 
 /* Per-replay counters (written by the device). */
 typedef struct {

@@ -50,7 +50,7 @@ class _Params(C.Structure):
                 ("ema_num", C.c_uint32), ("ema_den", C.c_uint32), ("penalty_q", C.c_uint64),
                 ("ttl_us", C.c_uint32), ("ttft_load", C.c_uint32),
                 ("dma_bytes_per_us", C.c_uint64), ("prefill_ns_per_tok", C.c_uint64),
-                ("debug", C.c_uint32), ("pad1", C.c_uint32)]
+                ("debug", C.c_uint32), ("hazard_online", C.c_uint32)]
 
 
 RESULT_FIELDS = ["events", "req_warm", "cold", "hit_s", "hit_h", "miss", "bypass", "place_s",
@@ -131,7 +131,7 @@ def _params_struct(p: dict, debug: bool):
     return _Params(pol, q["hazard_bucket"], q["cap_s_bytes"], q["cap_h_bytes"],
                    q["kv_bytes_per_token"], q["max_sessions"], q["ema_num"], q["ema_den"],
                    q["penalty_q"], q["ttl_us"], q["ttft_load"], q["dma_bytes_per_us"],
-                   q["t_p_ps_per_tok"] // 1000, 1 if debug else 0, 0)
+                   q["t_p_ps_per_tok"] // 1000, 1 if debug else 0, 1 if q.get("hazard_online") else 0)
 
 
 def replay(tr, params: dict, log: bool = False, ttft: bool = False, debug: bool = False,

@@ -29,6 +29,9 @@
  *   R10 request accounting (warm = turn >= 1).
  *   R11 TIDE budget in bytes = g_q(us) * dma bytes per us.
  *   R25 ASE: a metric ratio 0/0 counts as 1.
+ *   R26 online hazard table (Sec. V-F): starts with no sessions; at the final
+ *       completion of a session its turn count T_s is added and the table is
+ *       rebuilt with the quantizer of R5; every later key uses it.
  *   R12 a completed session stays resident with the maximal key.
  *   R13 DMA busy until now + ceil(moved / dma bytes per us).
  *   R14 TIDE phase 1 (promotion into free fast-tier space) then phase 2
@@ -88,7 +91,7 @@ typedef struct {
   uint64_t dma_bytes_per_us;
   uint64_t prefill_ns_per_tok;   /* t_p in ns per token, for TTFT */
   uint32_t debug;                /* 1: check invariants and both TIDE forms every event */
-  uint32_t pad1;
+  uint32_t hazard_online;        /* 1: the hazard table starts empty and grows as sessions complete (R26) */
 } or_params;
 
 typedef struct {
@@ -581,10 +584,13 @@ int or_replay(const or_trace *tr, const or_params *p, or_result *res, or_logrec 
   st.log = log;
   st.log_cap = log_cap;
 
-  /* Offline hazard table fitted on all sessions of the trace (R5). */
+  /* Offline hazard table fitted on all sessions of the trace (R5), or (R26,
+   * Sec. V-F) an online table that starts empty: tps then lists the turn
+   * counts of the sessions completed so far. */
   uint16_t h_q[OR_T_MAX + 1];
+  uint64_t n_done = 0;
   for (uint64_t s = 0; s < S; s++) tps[s] = (uint32_t)(tr->turn_off[s + 1] - tr->turn_off[s]);
-  or_hazard_lut(tps, S, p->hazard_bucket, h_q, st.sigma_q);
+  or_hazard_lut(tps, p->hazard_online ? 0 : S, p->hazard_bucket, h_q, st.sigma_q);
 
   /* Belady next reference: event index of each session's next arrival. */
   {
@@ -684,6 +690,12 @@ int or_replay(const or_trace *tr, const or_params *p, or_result *res, or_logrec 
       int final = (x->turn + 1 == tr->turn_off[s + 1] - tr->turn_off[s]);
       if (final) {
         R->done = 1; /* R12: stays resident with the maximal key */
+        if (p->hazard_online) {
+          /* R26: the session's turn count joins the table; every later key
+           * uses the rebuilt sigma */
+          tps[n_done++] = x->turn + 1;
+          or_hazard_lut(tps, n_done, p->hazard_bucket, h_q, st.sigma_q);
+        }
       } else if (has_tide(p->policy) && !dma_busy) {
         /* gap_start with DMA free: TIDE with budget = Delta * B (R11) */
         uint64_t budget = R->g_q * p->dma_bytes_per_us;

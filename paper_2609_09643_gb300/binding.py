@@ -16,6 +16,7 @@ import numpy as np
 from .native import LIB
 
 POLICY = {"lru": 0, "timeout": 1, "spear": 2, "spear_tide": 3, "belady": 4, "lru_tide": 5}
+FLAG_HAZARD_ONLINE = 1  # unison_replay_params.flags bit 0
 KIND = ["COLD", "HIT_S", "HIT_H", "MISS", "PLACE_S", "PLACE_H", "BYPASS", "DEMOTE", "EVICT",
         "PROMOTE", "TIDE_DEMOTE", "EXPIRE"]
 OK, ERR_ARG, ERR_IO, ERR_FORMAT, ERR_RANGE, ERR_CUDA, ERR_OOM, ERR_LOG_FULL, ERR_TIMEOUT, ERR_CAPACITY = \
@@ -48,7 +49,7 @@ class ReplayParams(C.Structure):
                 ("hazard_bucket", C.c_uint32), ("ttl_us", C.c_uint32), ("penalty_q", C.c_uint64),
                 ("dma_bytes_per_us", C.c_uint64), ("t_s_ps_per_tok", C.c_uint64),
                 ("t_h_ps_per_tok", C.c_uint64), ("t_p_ps_per_tok", C.c_uint64),
-                ("ttft_load", C.c_uint32), ("reserved", C.c_uint32)]
+                ("ttft_load", C.c_uint32), ("flags", C.c_uint32)]
 
 
 RESULT_FIELDS = ["events", "req_warm", "cold", "hit_s", "hit_h", "miss", "bypass", "place_s", "place_h",
@@ -207,7 +208,8 @@ def make_params(p: dict, trace_idx: int = 0) -> ReplayParams:
     return ReplayParams(pol, q.get("trace_idx", trace_idx), q["cap_fast_bytes"], q["cap_hbm_bytes"],
                         q["kv_bytes_per_token"], q["max_sessions"], q["ema_num"], q["ema_den"],
                         q["hazard_bucket"], q["ttl_us"], q["penalty_q"], q["dma_bytes_per_us"],
-                        q["t_s_ps_per_tok"], q["t_h_ps_per_tok"], q["t_p_ps_per_tok"], q["ttft_load"], 0)
+                        q["t_s_ps_per_tok"], q["t_h_ps_per_tok"], q["t_p_ps_per_tok"], q["ttft_load"],
+                        FLAG_HAZARD_ONLINE if q.get("hazard_online") else 0)
 
 
 def result_dict(r: ReplayResult) -> dict:

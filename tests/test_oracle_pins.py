@@ -480,3 +480,81 @@ def test_ase_zero_readings():
     am[1, 1] = 0.0                     # a zero AMAT minimum: the others' factor is 0
     z = oracle.ase(hr, am, tt)
     assert z[0] == 0.0 and z[2] == 0.0 and z[1] > 0.0
+
+
+# ------------------------------------------------- online hazard table --
+MIB, GIB = 1 << 20, 1 << 30
+def _online_logs(tr, p_online, p_offline):
+    from cases import to_oracle
+    cap = 16 * tr.n_events
+    a = oracle.replay(tr, to_oracle(p_online), log=True, log_capacity=cap, debug=True)
+    b = oracle.replay(tr, to_oracle(p_offline), log=True, log_capacity=cap, debug=True)
+    assert a["status"] == 0 and b["status"] == 0
+    return [np.asarray(x) for x in a["log"]], [np.asarray(x) for x in b["log"]], a, b
+
+
+def test_online_hazard_beyond_horizon():
+    """Sessions of more than 51 turns have d(t) = 0 for every table entry
+    t <= 50: the online table never leaves zero hazard, as the offline one,
+    so both make the same decisions.  With turn counts inside the horizon the
+    two differ (the decisions do depend on the table)."""
+    from cases import base
+    long = synth.make_trace(11, np.full(40, 55), 0.5, synth.GAP_MIX_CODING)
+    short = synth.make_trace(11, 2 + (np.arange(40) % 15), 0.5, synth.GAP_MIX_CODING)
+    for pol in ("spear", "spear_tide"):
+        p = base(pol, 48 * MIB, 1 * GIB, 131072)
+        la, lb, _, _ = _online_logs(long, dict(p, online=True), p)
+        assert all(np.array_equal(x, y) for x, y in zip(la, lb)), pol
+        sa, sb, _, _ = _online_logs(short, dict(p, online=True), p)
+        assert not all(np.array_equal(x, y) for x, y in zip(sa, sb)), pol
+
+
+def _two_phase_trace():
+    """Wave 1: three small sessions (3, 4, 4 turns) that finish early.  Wave 2:
+    ten 3-turn and twenty 4-turn sessions (the same turn-count ratios): their
+    turns but the last run within the first minutes, their last turns all
+    arrive in one burst at 1,000 s, and they all complete at 1,500 s, after
+    every decision."""
+    arr, comp, ins, outs = [], [], [], []
+    for i, ts in enumerate((3, 4, 4)):
+        a0 = 1000 + 200_000 * i
+        arr.append([a0 + 100_000 * k for k in range(ts)])
+        comp.append([a0 + 100_000 * k + 1000 for k in range(ts)])
+        ins.append([100 + 50 * k for k in range(ts)])
+        outs.append([120 + 50 * k for k in range(ts)])
+    for j in range(30):
+        ts = 3 if j < 10 else 4
+        t = 5_000_000 + 300_000 * j
+        a, c, i_, o_ = [], [], [], []
+        tok = 3000 + 500 * (j % 5)
+        for k in range(ts):
+            final = k + 1 == ts
+            if final:
+                t = 1_000_000_000 + 1000 * j
+            a.append(t)
+            i_.append(tok)
+            tok += 100 + 40 * ((j + k) % 7)
+            o_.append(tok)
+            c.append(1_500_000_000 + j if final else t + 2000)
+            t = c[-1] + 200_000 * (1 + ((j * 7 + k * 13) % 10) ** 2)
+        arr.append(a), comp.append(c), ins.append(i_), outs.append(o_)
+    return synth.trace_from_turns(arr, comp, ins, outs)
+
+
+def test_online_hazard_two_phase_equals_offline():
+    """After wave 1 completes, the online table holds turn counts {3, 4, 4};
+    the offline table over both waves holds {3 x 11, 4 x 22}: the same d/n
+    in every entry, hence the same table (worked: h(2) = floor((2*1*4095+3)/6)
+    = floor((2*11*4095+33)/66) = 1365, h(3) = 4095, h = 0 elsewhere).  Wave 1 never fills a
+    tier, and no wave-2 session completes before the last decision, so the
+    online and offline replays decide identically.  Pooling turns (bucket 3)
+    changes the table and the decisions."""
+    from cases import base
+    tr = _two_phase_trace()
+    for pol in ("spear", "spear_tide"):
+        p = base(pol, 6000 * 131072, 20000 * 131072, 131072, dma=2000)
+        la, lb, a, b = _online_logs(tr, dict(p, online=True), p)
+        assert all(np.array_equal(x, y) for x, y in zip(la, lb)), pol
+        assert a["evict"] + a["demote"] > 0, pol  # the tiers do fill in wave 2
+        _, lc, _, _ = _online_logs(tr, p, dict(p, bucket=3))
+        assert not all(np.array_equal(x, y) for x, y in zip(lb, lc)), pol
