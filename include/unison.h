@@ -155,8 +155,9 @@ typedef struct {
  * of each session joins it at that session's final completion, which then
  * re-ranks every resident under the rebuilt table before the next event.
  * SPEAR and SPEAR+TIDE only (else UNISON_ERR_ARG); the trace must have at
- * most 32,768 sessions and the replay's resident lists must fit in shared
- * memory (else UNISON_ERR_RANGE). */
+ * most 32,768 sessions and the replay's resident lists, rounded up to powers
+ * of two, plus 7 bytes per session must fit in shared memory (else
+ * UNISON_ERR_RANGE).  Any other bit of `flags` is UNISON_ERR_ARG. */
 #define UNISON_HAZARD_ONLINE 1u
 
 /* Per-replay counters (written by the device). */

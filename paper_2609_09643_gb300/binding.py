@@ -209,7 +209,7 @@ def make_params(p: dict, trace_idx: int = 0) -> ReplayParams:
                         q["kv_bytes_per_token"], q["max_sessions"], q["ema_num"], q["ema_den"],
                         q["hazard_bucket"], q["ttl_us"], q["penalty_q"], q["dma_bytes_per_us"],
                         q["t_s_ps_per_tok"], q["t_h_ps_per_tok"], q["t_p_ps_per_tok"], q["ttft_load"],
-                        FLAG_HAZARD_ONLINE if q.get("hazard_online") else 0)
+                        q.get("flags", FLAG_HAZARD_ONLINE if q.get("hazard_online") else 0))
 
 
 def result_dict(r: ReplayResult) -> dict:

@@ -70,8 +70,9 @@ struct ReplayDesc {
   uint32_t n_events, n_turns, n_sessions, policy;
   uint32_t max_sessions, kvb, ttl, load;
   uint32_t rcap_s, rcap_h;
-  uint32_t tmap;  // 1: a per-session tier byte follows the lists in shared memory
-  uint32_t pad_;
+  uint32_t tmap;    // 1: a per-session tier byte follows the lists in shared memory
+  uint32_t bucket;  // hazard bucket width (online hazard replays)
+  uint64_t penalty;  // P_Z in quantised units (online hazard replays)
 };
 
 // --------------------------------------------------------------------------
@@ -189,6 +190,13 @@ struct Sorted {
   uint4 *e;
   uint32_t n, cap;
 };
+
+// Smallest power of two >= x (x >= 1).
+__host__ __device__ __forceinline__ uint32_t ring_size(uint32_t x) {
+  uint32_t r = 1;
+  while (r < x) r <<= 1;
+  return r;
+}
 
 __device__ __forceinline__ uint64_t ekey(uint4 v) { return ((uint64_t)v.y << 32) | v.x; }
 
@@ -567,7 +575,125 @@ __device__ __forceinline__ bool has_tide(uint32_t policy) {
   return policy == UNISON_SPEAR_TIDE || policy == UNISON_LRU_TIDE;
 }
 
-template <bool kGlobalLists>
+// --------------------------------------------------------------------------
+// Online hazard table (Sec. V-F): counts n(t), d(t) of the sessions completed
+// so far, and the table built from them exactly as the offline one (eqs.
+// (hazard), (hq), (survq), (t2); bucket pooling).  Lives in shared memory
+// after the per-session state of an online replay.
+// --------------------------------------------------------------------------
+struct OnlineTable {
+  uint32_t n[kLutN], d[kLutN], sig[kLutN];
+  unsigned long long t2[kLutN];
+};
+
+__device__ __forceinline__ uint64_t online_key(const OnlineTable &ot, uint32_t g, uint32_t t, uint32_t s) {
+  const uint32_t tt = t < kTMax ? t : kTMax;
+  return pack_key((uint64_t)g * kLambda / ot.sig[tt] + ot.t2[tt], s);
+}
+
+// A session of `turns` turns has completed: add it to the counts and rebuild
+// sigma and T2 for every turn index.
+__device__ bool online_add(OnlineTable &ot, uint32_t turns, uint32_t bucket, uint64_t penalty, int lane) {
+  for (uint32_t t = lane; t < kLutN; t += 32) {
+    ot.n[t] += turns >= t + 1 ? 1u : 0u;
+    ot.d[t] += turns == t + 1 ? 1u : 0u;
+  }
+  __syncwarp();
+  uint32_t sg[2];
+  unsigned long long t2[2];
+#pragma unroll
+  for (int q = 0; q < 2; q++) {
+    const uint32_t t = lane + 32 * q;
+    sg[q] = kLambda;
+    t2[q] = 0;
+    if (t < kLutN) {
+      uint64_t nn = 0, dd = 0;
+      for (uint32_t u = (t / bucket) * bucket; u < kLutN && u / bucket == t / bucket; u++) {
+        nn += ot.n[u];
+        dd += ot.d[u];
+      }
+      uint64_t hq = nn ? (2 * dd * kLambda + nn) / (2 * nn) : 0;
+      if (hq > kLambda) hq = kLambda;
+      const uint32_t sq = (uint32_t)(kLambda - hq) < kEpsQ ? kEpsQ : (uint32_t)(kLambda - hq);
+      sg[q] = sq;
+      t2[q] = ((unsigned long long)(kLambda - sq) * penalty) / kLambda;
+    }
+  }
+  bool changed = false;
+#pragma unroll
+  for (int q = 0; q < 2; q++) changed |= (lane + 32 * q < kLutN) && ot.sig[lane + 32 * q] != sg[q];
+  __syncwarp();
+#pragma unroll
+  for (int q = 0; q < 2; q++) {
+    const uint32_t t = lane + 32 * q;
+    if (t < kLutN) {
+      ot.sig[t] = sg[q];
+      ot.t2[t] = t2[q];
+    }
+  }
+  __syncwarp();
+  return __any_sync(kFull, changed);  // T2 is a function of sigma
+}
+
+// Every resident's key under the rebuilt table, then the tier re-sorted:
+// bitonic network (descending, padded to a power of two with key 0, which no
+// packed key equals since session ids stay below 2^24 - 1), then reversed.
+// The tier's array holds a power of two >= its capacity.
+__device__ void online_rerank(Sorted &T, const OnlineTable &ot, const uint32_t *gs, const uint16_t *ks, int lane) {
+  if (T.n < 2) {
+    if (T.n == 1 && lane == 0) {
+      uint4 v = T.e[0];
+      const uint64_t k = ekey(v);
+      if ((k >> 24) != kKeyMax40) {
+        const uint32_t id = packed_id(k);
+        const uint64_t nk = online_key(ot, gs[id], (uint32_t)ks[id] - 1, id);
+        v.x = (uint32_t)nk;
+        v.y = (uint32_t)(nk >> 32);
+        T.e[0] = v;
+      }
+    }
+    __syncwarp();
+    return;
+  }
+  const uint32_t ring = ring_size(T.n);
+  for (uint32_t i = lane; i < T.n; i += 32) {
+    uint4 v = T.e[i];
+    const uint64_t k = ekey(v);
+    if ((k >> 24) != kKeyMax40) {  // completed sessions keep the maximal key
+      const uint32_t id = packed_id(k);
+      const uint64_t nk = online_key(ot, gs[id], (uint32_t)ks[id] - 1, id);
+      v.x = (uint32_t)nk;
+      v.y = (uint32_t)(nk >> 32);
+      T.e[i] = v;
+    }
+  }
+  for (uint32_t i = T.n + lane; i < ring; i += 32) T.e[i] = make_uint4(0u, 0u, 0u, 0u);
+  __syncwarp();
+  for (uint32_t k = 2; k <= ring; k <<= 1) {
+    for (uint32_t j = k >> 1; j > 0; j >>= 1) {
+      for (uint32_t i = lane; i < ring; i += 32) {
+        const uint32_t ij = i ^ j;
+        if (ij > i) {
+          const uint4 a = T.e[i], b = T.e[ij];
+          const bool desc = (i & k) == 0;
+          if (desc ? ekey(a) < ekey(b) : ekey(a) > ekey(b)) {
+            T.e[i] = b;
+            T.e[ij] = a;
+          }
+        }
+      }
+      __syncwarp();
+    }
+  }
+  for (uint32_t i = lane; i < T.n / 2; i += 32) {
+    const uint4 a = T.e[i], b = T.e[T.n - 1 - i];
+    T.e[i] = b;
+    T.e[T.n - 1 - i] = a;
+  }
+  __syncwarp();
+}
+
+template <bool kGlobalLists, bool kOnline>
 __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, const uint32_t *order) {
   extern __shared__ __align__(16) unsigned char smem[];
   const int lane = threadIdx.x & 31;
@@ -578,12 +704,16 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
   const Hot hot{D.cap_s, D.cap_h, D.kvb, D.dma, D.max_sessions};
 
   ReplayState st;
+  uint32_t *online_gs = nullptr;
+  uint16_t *online_ks = nullptr;
+  OnlineTable *online_tab = nullptr;
   {
     uint4 *p = reinterpret_cast<uint4 *>(kGlobalLists ? reinterpret_cast<unsigned char *>(D.glist) : smem);
+    // online replays keep power-of-two tiers (for the re-sort)
     st.S.e = p;
-    p += D.rcap_s;
+    p += kOnline ? ring_size(D.rcap_s) : D.rcap_s;
     st.H.e = p;
-    p += D.rcap_h;
+    p += kOnline ? ring_size(D.rcap_h) : D.rcap_h;
     st.pin = p;
     p += D.rcap_s + D.rcap_h;
     st.tmp = p;
@@ -593,6 +723,26 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
       st.tmap = reinterpret_cast<uint8_t *>(p);
       uint32_t *m32 = reinterpret_cast<uint32_t *>(p);
       for (uint32_t i = lane; i < (D.n_sessions + 3) / 4; i += 32) m32[i] = 0u;
+      __syncwarp();
+    }
+    if (kOnline) {
+      // after the tier map: gap average (u32) and arrivals so far (u16) per
+      // session, then the table
+      unsigned char *q = reinterpret_cast<unsigned char *>(p) + ((D.n_sessions + 15) & ~15u);
+      online_gs = reinterpret_cast<uint32_t *>(q);
+      q += 4 * ((D.n_sessions + 3) & ~3u);
+      online_ks = reinterpret_cast<uint16_t *>(q);
+      q += 2 * ((D.n_sessions + 7) & ~7u);
+      online_tab = reinterpret_cast<OnlineTable *>(q);
+      for (uint32_t i = lane; i < D.n_sessions; i += 32) {
+        online_gs[i] = 0u;
+        online_ks[i] = 0;
+      }
+      for (uint32_t t = lane; t < kLutN; t += 32) {
+        online_tab->n[t] = online_tab->d[t] = 0u;
+        online_tab->sig[t] = kLambda;  // no session completed: zero hazard
+        online_tab->t2[t] = 0ull;
+      }
       __syncwarp();
     }
     st.S.n = st.H.n = 0;
@@ -639,11 +789,11 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
       cp_async4(&sprev[bi][lane], &D.prev_out[i]);
       cp_async4(&spev[bi][lane], &D.prev_ev[i]);
       if (belady) cp_async4(&snref[bi][lane], &D.nref[i]);
-      if (spear_keys) {
+      if (spear_keys && !kOnline) {
         cp_async8(&spk[bi][lane], &D.pkey[i]);
         cp_async8(&spkb[bi][lane], &D.pkb[i]);
       }
-      if (tide_on) cp_async4(&sgq[bi][lane], &D.gq[i]);
+      if (tide_on || kOnline) cp_async4(&sgq[bi][lane], &D.gq[i]);
     }
     cp_async_commit();
   };
@@ -687,7 +837,9 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
         uint32_t pos = 0;
         if (!edge) {
           uint64_t pkb;
-          if (spear_keys)
+          if (kOnline)
+            pkb = online_key(*online_tab, online_gs[s], (uint32_t)online_ks[s] - 1, s);
+          else if (spear_keys)
             pkb = spkb[bi][j];
           else if (belady)
             pkb = pack_key(e, s);  // the previous arrival's next reference is this event
@@ -760,7 +912,18 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
           set_tier(st, s, kTierNone);
         }
         uint64_t pk;
-        if (spear_keys)
+        if (kOnline) {
+          // turn k = arrivals so far; the session's gap average and turn
+          // index advance (the count saturates far above the last table row)
+          const uint32_t k = online_ks[s];
+          pk = online_key(*online_tab, sgq[bi][j], k, s);
+          __syncwarp();
+          if (lane == 0) {
+            online_gs[s] = sgq[bi][j];
+            online_ks[s] = (uint16_t)(k < 0xFFFFu ? k + 1 : k);
+          }
+          __syncwarp();
+        } else if (spear_keys)
           pk = spk[bi][j];
         else if (belady) {
           const uint32_t nr = snref[bi][j];
@@ -784,7 +947,10 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
           st.npin--;
           const uint32_t tier = pe.w >> 30, sz = pe.z;
           uint64_t pk = ((uint64_t)pe.y << 32) | pe.x;
-          if (spear_keys)
+          if (kOnline)
+            pk = edge ? pack_key(kKeyMax40, s)
+                      : online_key(*online_tab, online_gs[s], (uint32_t)online_ks[s] - 1, s);
+          else if (spear_keys)
             pk = spk[bi][j];
           else if (!belady)
             pk = pack_key(0xFFFFFFFFull - e, s);
@@ -795,6 +961,14 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
           } else {
             st.pinned_h -= sz;
             if (!sorted_insert(st, st.H, v, lane, kTierH)) break;
+          }
+        }
+        if (kOnline && edge) {
+          // Sec. V-F: the finished session's turn count joins the table and
+          // every resident is ranked under the rebuilt one
+          if (online_add(*online_tab, online_ks[s], D.bucket, D.penalty, lane)) {
+            online_rerank(st.S, *online_tab, online_gs, online_ks, lane);
+            online_rerank(st.H, *online_tab, online_gs, online_ks, lane);
           }
         }
         if (!edge && tide_on && !dma_busy) {
@@ -920,6 +1094,9 @@ int check_params(const unison_replay_params &p, int n_traces) {
   if (p.dma_bytes_per_us >= (1ull << 32)) return UNISON_ERR_RANGE;
   if (p.ttl_us != 0xFFFFFFFFu && p.ttl_us >= (1u << 31)) return UNISON_ERR_RANGE;
   if (p.ttft_load == 0) return UNISON_ERR_ARG;
+  if (p.flags & ~UNISON_HAZARD_ONLINE) return UNISON_ERR_ARG;
+  if ((p.flags & UNISON_HAZARD_ONLINE) && p.policy != UNISON_SPEAR && p.policy != UNISON_SPEAR_TIDE)
+    return UNISON_ERR_ARG;
   return UNISON_OK;
 }
 
@@ -942,8 +1119,8 @@ struct ReplayPlan {
   std::vector<int> replay_combo;
   size_t off_desc = 0, off_order = 0, off_combo = 0, bytes = 0;
   std::vector<size_t> off_lut, off_stream, off_ttft, off_glist;
-  std::vector<uint32_t> rcap_s, rcap_h, in_smem, in_global, tmap;
-  size_t max_smem = 0;
+  std::vector<uint32_t> rcap_s, rcap_h, in_smem, in_global, in_online, tmap;
+  size_t max_smem = 0, max_smem_online = 0;
 };
 
 // Resident-list capacity of a tier: at most one entry per session and no more
@@ -960,8 +1137,16 @@ uint32_t list_cap(uint64_t cap_tok, const unison_trace *tr) {
 constexpr uint32_t kTierMapMax = 32768;
 size_t list_bytes(uint32_t cs, uint32_t ch) { return 16ull * (4ull * cs + 2ull * ch); }
 
-void plan_replays(const unison_trace *const *traces, const unison_replay_params *params, int n_replays,
-                  size_t smem_limit, bool results_in_scratch, ReplayPlan &P, size_t &off_res) {
+// An online hazard replay: both tiers rounded up to powers of two, the tier
+// map, the per-session gap average (4 B) and arrival count (2 B), the table.
+size_t online_bytes(uint32_t cs, uint32_t ch, uint32_t n_sessions) {
+  const size_t n = n_sessions;
+  return 16ull * (ring_size(cs) + ring_size(ch) + 3ull * cs + ch) + align_up(n, 16) + 4 * align_up(n, 4) +
+         2 * align_up(n, 8) + align_up(sizeof(OnlineTable), 16);
+}
+
+int plan_replays(const unison_trace *const *traces, const unison_replay_params *params, int n_replays,
+                 size_t smem_limit, bool results_in_scratch, ReplayPlan &P, size_t &off_res) {
   std::map<std::tuple<uint32_t, uint32_t, uint32_t, uint32_t, uint64_t>, int> combo_of;
   P.replay_combo.assign(n_replays, -1);
   for (int r = 0; r < n_replays; r++) {
@@ -1005,7 +1190,14 @@ void plan_replays(const unison_trace *const *traces, const unison_replay_params 
     // the tier map (one byte per session) when it fits beside the lists
     const size_t map = align_up(tr->n_sessions, 16);
     P.tmap[r] = tr->n_sessions <= kTierMapMax && lists + map <= smem_limit;
-    if (lists <= smem_limit) {
+    if (p.flags & UNISON_HAZARD_ONLINE) {
+      // online hazard replays run from shared memory only
+      const size_t ob = online_bytes(P.rcap_s[r], P.rcap_h[r], tr->n_sessions);
+      if (tr->n_sessions > kTierMapMax || ob > smem_limit) return UNISON_ERR_RANGE;
+      P.tmap[r] = 1;
+      P.in_online.push_back((uint32_t)r);
+      P.max_smem_online = std::max(P.max_smem_online, ob);
+    } else if (lists <= smem_limit) {
       P.in_smem.push_back((uint32_t)r);
       P.max_smem = std::max<size_t>(P.max_smem, lists + (P.tmap[r] ? map : 0));
     } else {
@@ -1023,6 +1215,7 @@ void plan_replays(const unison_trace *const *traces, const unison_replay_params 
     off = align_up(off + sizeof(unison_replay_result) * n_replays, 256);
   }
   P.bytes = off;
+  return UNISON_OK;
 }
 
 // Fill the descriptors for a plan placed at `scratch`.
@@ -1083,11 +1276,13 @@ void fill_descs(const unison_trace *const *traces, const unison_replay_params *p
     d.rcap_s = P.rcap_s[r];
     d.rcap_h = P.rcap_h[r];
     d.tmap = P.tmap[r];
-    d.pad_ = 0;
+    d.bucket = p.hazard_bucket;
+    d.penalty = p.penalty_q;
   }
   order.clear();
   order.insert(order.end(), P.in_smem.begin(), P.in_smem.end());
   order.insert(order.end(), P.in_global.begin(), P.in_global.end());
+  order.insert(order.end(), P.in_online.begin(), P.in_online.end());
 }
 
 // Queue the kernels of a planned batch on `stream`.
@@ -1119,13 +1314,23 @@ int launch_replays(const ReplayPlan &P, char *scratch, const std::vector<ComboDe
   {
     ProfSpan span(profile ? "replay" : "", stream);
     if (!P.in_smem.empty()) {
-      ck(cudaFuncSetAttribute(replay_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P.max_smem));
-      replay_kernel<false><<<(unsigned)P.in_smem.size(), 32, P.max_smem, stream>>>(d_desc, d_order);
+      ck(cudaFuncSetAttribute(replay_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)P.max_smem));
+      replay_kernel<false, false><<<(unsigned)P.in_smem.size(), 32, P.max_smem, stream>>>(d_desc, d_order);
       count_launches(1);
       ck(cudaGetLastError());
     }
     if (!P.in_global.empty()) {
-      replay_kernel<true><<<(unsigned)P.in_global.size(), 32, 0, stream>>>(d_desc, d_order + P.in_smem.size());
+      replay_kernel<true, false><<<(unsigned)P.in_global.size(), 32, 0, stream>>>(d_desc,
+                                                                                 d_order + P.in_smem.size());
+      count_launches(1);
+      ck(cudaGetLastError());
+    }
+    if (!P.in_online.empty()) {
+      ck(cudaFuncSetAttribute(replay_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)P.max_smem_online));
+      replay_kernel<false, true><<<(unsigned)P.in_online.size(), 32, P.max_smem_online, stream>>>(
+          d_desc, d_order + P.in_smem.size() + P.in_global.size());
       count_launches(1);
       ck(cudaGetLastError());
     }
@@ -1170,7 +1375,8 @@ extern "C" int unison_replay_batch(const unison_trace *const *traces, int n_trac
   cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
   ReplayPlan P;
   size_t off_res = 0;
-  plan_replays(traces, params, n_replays, smem_limit, results_dev == nullptr, P, off_res);
+  rc = plan_replays(traces, params, n_replays, smem_limit, results_dev == nullptr, P, off_res);
+  if (rc != UNISON_OK) return rc;
   char *scratch = nullptr;
   if (cudaMallocAsync(reinterpret_cast<void **>(&scratch), P.bytes, stream) != cudaSuccess) {
     cudaGetLastError();
@@ -1306,7 +1512,8 @@ extern "C" int unison_replay_batch_noalloc(const unison_trace *const *traces, in
   if (rc != UNISON_OK) return rc;
   ReplayPlan P;
   size_t off_res = 0;
-  plan_replays(traces, params, n_replays, smem_limit, false, P, off_res);
+  rc = plan_replays(traces, params, n_replays, smem_limit, false, P, off_res);
+  if (rc != UNISON_OK) return rc;
   if (P.bytes > UNISON_NOALLOC_SCRATCH_BYTES) return UNISON_ERR_RANGE;  // batch too large for the fixed scratch
   // Every scratch region is written before it is read within one call (the
   // descriptors by the copies in launch_replays, the tables and streams by

@@ -230,3 +230,79 @@ def test_hazard_lut_kernel(B):
             oh, osig = oracle.hazard_lut(tps, w)
             assert (sig.cpu().numpy().astype(np.uint16) == osig).all()
             assert (hq.cpu().numpy().astype(np.uint16) == oh).all()
+
+
+# ---- online hazard table (Sec. V-F) ------------------------------------------
+
+ONLINE_POLS = ("spear", "spear_tide")
+
+
+def test_online_hazard_tiny_full_logs(B):
+    tr, _ = tiny_case()
+    reps = [(0, base(pol, 512 * MIB, 8 * GIB, 28672, online=True, bucket=b)) for pol in ONLINE_POLS for b in (1, 3)]
+    cap = 8 * tr.n_events
+    res, log, _ = run_gpu(B, [tr], reps, log_capacity=cap)
+    for i, (_, p) in enumerate(reps):
+        o = oracle.replay(tr, to_oracle(p), log=True, log_capacity=cap)
+        assert_same(res[i], o, (p["policy"], p["bucket"]))
+        assert_same_log(B, log[i], res[i], o, (p["policy"], p["bucket"]))
+
+
+def test_online_hazard_paper_scale_mixed_batch(B):
+    """Online and offline replays of the same settings in one call (the
+    online ones run as their own launch): both gap mixes x 3 KV sizes x 2
+    policies x buckets 1 and 4.  The online table changes decisions."""
+    from cases import KVB_PAPER
+    trs = [synth.paper_scale_trace(1, "coding"), synth.paper_scale_trace(1, "general")]
+    reps = []
+    for ti in range(2):
+        for kvb in KVB_PAPER:
+            for pol in ONLINE_POLS:
+                for b in (1, 4):
+                    reps.append((ti, base(pol, 4 * GIB, 64 * GIB, kvb, bucket=b, online=True)))
+                    reps.append((ti, base(pol, 4 * GIB, 64 * GIB, kvb, bucket=b)))
+    cap = 4 * trs[0].n_events
+    res, log, _ = run_gpu(B, trs, reps, log_capacity=cap)
+    n_differ = 0
+    for i, (ti, p) in enumerate(reps):
+        o = oracle.replay(trs[ti], to_oracle(p), log=(i % 8 == 0), log_capacity=cap)
+        assert_same(res[i], o, (i, ti, p["policy"], p["kvb"], p["online"]))
+        if i % 8 == 0:
+            assert_same_log(B, log[i], res[i], o, (i, ti, p["policy"], p["kvb"], p["online"]))
+        if p["online"]:
+            n_differ += res[i]["decision_hash"] != res[i + 1]["decision_hash"]
+    assert n_differ >= len(reps) // 4
+
+
+def test_online_hazard_two_phase_trace(B):
+    """The trace whose online and offline tables coincide once wave 1 has
+    completed: full logs against the oracle, online and offline."""
+    from test_oracle_pins import _two_phase_trace
+    tr = _two_phase_trace()
+    reps = [(0, base(pol, 6000 * 131072, 20000 * 131072, 131072, dma=2000, online=on, bucket=b))
+            for pol in ONLINE_POLS for on in (True, False) for b in (1, 3)]
+    cap = 16 * tr.n_events
+    res, log, _ = run_gpu(B, [tr], reps, log_capacity=cap)
+    for i, (_, p) in enumerate(reps):
+        o = oracle.replay(tr, to_oracle(p), log=True, log_capacity=cap)
+        assert_same(res[i], o, i)
+        assert_same_log(B, log[i], res[i], o, i)
+    assert res[0]["decision_hash"] == res[2]["decision_hash"]  # online == offline at bucket 1
+
+
+def test_online_hazard_rejected_cases(B):
+    tr, _ = tiny_case()
+    h = [B.Trace(tr).upload()]
+    for pol, flags, err in (("lru", 1, B.ERR_ARG), ("belady", 1, B.ERR_ARG), ("lru_tide", 1, B.ERR_ARG),
+                            ("spear", 2, B.ERR_ARG), ("spear", 1 << 31, B.ERR_ARG)):
+        q = to_lib(base(pol, 1 * GIB, 8 * GIB, 28672))
+        q["flags"] = flags
+        with pytest.raises(B.UnisonError) as ei:
+            B.replay_batch(h, [q])
+        assert ei.value.code == err, (pol, flags)
+    # more sessions than an online replay keeps in shared memory
+    big = synth.make_trace(5, np.full(40000, 2), 0.005, synth.GAP_MIX_GENERAL)
+    hb = [B.Trace(big).upload()]
+    with pytest.raises(B.UnisonError) as ei:
+        B.replay_batch(hb, [to_lib(base("spear", 1 * GIB, 8 * GIB, 16384, online=True))])
+    assert ei.value.code == B.ERR_RANGE
