@@ -63,6 +63,7 @@ def parse():
     ap.add_argument("--rank-n", type=int, default=1 << 24, help="records per live set")
     ap.add_argument("--rank-sets", type=int, default=7, help="live sets per call (<= 7)")
     ap.add_argument("--no-rank-sizes", action="store_true", help="skip the live-set size sweep")
+    ap.add_argument("--no-online", action="store_true", help="skip the online hazard-table report")
     return ap.parse_args()
 
 
@@ -258,6 +259,60 @@ def sweep_ase(B, results, reps, lib_params):
             "median": sorted(vals)[per // 2], "worst": vals[order[-1]]}
 
 
+def online_hazard_report(B, stream, steps: int = 3, points: int = 8):
+    """Sec. V-F: the paper-scale replays (coding and general gap mixes x 3 KV
+    sizes x SPEAR and SPEAR+TIDE, fast 4 GiB / HBM 64 GiB) with a hazard table
+    that starts empty and grows at every session completion: device time per
+    call, and eq. (attainment) of each against the offline-table and LRU
+    replays of the same setting over `points` windows of observed sessions."""
+    import math
+    import torch
+    import synth
+    from cases import GIB, KVB_PAPER, base, to_lib
+    mixes = ("coding", "general")
+    trs = [synth.paper_scale_trace(1, m) for m in mixes]
+    handles = [B.Trace(t).upload(stream) for t in trs]
+    settings = [(ti, kvb, pol) for ti in range(2) for kvb in KVB_PAPER for pol in ("spear", "spear_tide")]
+    online = [to_lib(base(pol, 4 * GIB, 64 * GIB, kvb, online=True), ti) for ti, kvb, pol in settings]
+    offline = [to_lib(base(pol, 4 * GIB, 64 * GIB, kvb), ti) for ti, kvb, pol in settings]
+    lru = [to_lib(base("lru", 4 * GIB, 64 * GIB, kvb), ti) for ti, kvb, _ in settings]
+    events = sum(2 * trs[ti].n_turns for ti, _, _ in settings)
+    out = torch.zeros(B.result_nbytes(len(online)), dtype=torch.uint8, device="cuda")
+    for _ in range(2):
+        B.replay_batch_async(handles, online, out, stream=stream)
+    torch.cuda.synchronize()
+    B.profile_enable(True)
+    B.profile_read("replay", reset=True)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(steps):
+        B.replay_batch_async(handles, online, out, stream=stream)
+    b.record(stream)
+    torch.cuda.synchronize()
+    call_ms = a.elapsed_time(b) / steps
+    k_ms, k_n = B.profile_read("replay", reset=True)
+    B.profile_enable(False)
+    assert all(r["status"] == 0 for r in B.results_from_tensor(out)), "online replay status"
+
+    n = len(settings)
+    cap = 4 * max(t.n_events for t in trs)
+    res, log = B.replay_batch(handles, online + offline + lru, log_capacity=cap, stream=stream)
+    assert all(r["status"] == 0 for r in res), "attainment replay status"
+    fin = lambda v: None if v is None or math.isnan(v) else round(v, 4)
+    hr = lambda r: (r["hit_s"] + r["hit_h"]) / r["req_warm"] if r["req_warm"] else None
+    curves = []
+    for i, (ti, kvb, pol) in enumerate(settings):
+        logs = [B.decode_log(log[j], res[j]["log_len"]) for j in (i, n + i, 2 * n + i)]
+        pts = B.attainment(handles[ti], logs, points)
+        curves.append({"trace": mixes[ti], "kv_bytes_per_token": kvb, "policy": pol,
+                       "sessions_seen": [p["sessions_seen"] for p in pts],
+                       "attainment": [fin(p["attainment"]) for p in pts],
+                       "hr_online": fin(hr(res[i])), "hr_offline": fin(hr(res[n + i])), "hr_lru": fin(hr(res[2 * n + i]))})
+    return {"replays": n, "events_per_call": events, "call_ms": call_ms,
+            "kernel_ms": k_ms / k_n if k_n else None, "events_per_s": events / (call_ms / 1e3),
+            "windows": points, "curves": curves}
+
+
 def cpu_baseline_replay(trs, reps, budget_s: float = 12.0):
     """The oracle as it stands, single-threaded, on a bounded sample of the
     sweep's replays (spread over the batch) until budget_s of CPU work."""
@@ -441,6 +496,10 @@ def main():
             e["call_frac_of_peak"] = e["call_gbs"] / pk
             e["filter_frac_of_peak"] = e["filter_gbs"] / pk if e["filter_gbs"] else None
 
+    online = None
+    if not (args.no_online or args.rank_only or args.replay_only) and rank == 0:
+        online = online_hazard_report(B, stream)
+
     # end to end through the public API: host trace staging -> device, replay,
     # results back to the host, every step
     e2e = None
@@ -511,7 +570,7 @@ def main():
                                    "paper-scale coding trace, 131072 B/token, SPEAR+TIDE)",
                        "replays": n_rep, "events_per_step": events_per_step,
                        "l2": "flushed before every step (256 MiB write, inside the timed region)"},
-            "roofline": roofline, "rank": rank_leg, "rank_sizes": sizes, "rank_kendall": tau, "sweep_ase": ase, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roofline, "rank": rank_leg, "rank_sizes": sizes, "rank_kendall": tau, "sweep_ase": ase, "online_hazard": online, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches, "clocks": clocks,
             "peaks": {"hbm_gbs": peaks.get("hbm_gbs"), "source": "MEASURED_PEAKS.json"}}
     if cpu is not None:

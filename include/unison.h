@@ -295,6 +295,33 @@ int unison_stats(const unison_replay_result *r, const unison_replay_params *p, u
  * metric gives UNISON_ERR_RANGE. */
 int unison_ase(const unison_stats_t *stats, int n_configs, int n_datasets, double *ase_out);
 
+/* Attainment A(n) (Sec. V-F, eq. attainment) of an online-table replay
+ * (UNISON_HAZARD_ONLINE) against the offline-table and LRU replays of the
+ * same trace:  A = (H_on - H_LRU) / (H_off - H_LRU), H a hit rate.  Reading:
+ * "after n observed sessions" is a window of the trace, the warm requests
+ * (decisions HIT_S, HIT_H, MISS) arriving while n_j <= n < n_{j+1} sessions
+ * have completed, n_j = floor(j N / n_points), j = 0 .. n_points-1, N the
+ * trace's sessions; the last window runs to the end of the trace.  Window j
+ * fills out[j]: n_j, its warm requests, the three hit rates over them, and A
+ * (NaN when the window holds no warm request or H_off = H_LRU).
+ * trace: a handle from unison_trace_create/_load (host data only is read);
+ * logs: host copies of the three replays' complete decision logs (len =
+ * the result's log_len, which must not exceed the capacity used).
+ * Errors: a null pointer -> UNISON_ERR_ARG; n_points = 0 or > N ->
+ * UNISON_ERR_RANGE; an event index outside the trace, or logs that disagree
+ * on which events are warm requests -> UNISON_ERR_FORMAT. */
+typedef struct {
+  uint32_t sessions_seen;  /* n_j */
+  uint32_t reserved;
+  uint64_t warm;           /* warm requests in the window */
+  double hr_online, hr_offline, hr_lru;
+  double attainment;
+} unison_attainment_point;
+
+int unison_attainment(const unison_trace *trace, const unison_decision *log_online, uint64_t len_online,
+                      const unison_decision *log_offline, uint64_t len_offline, const unison_decision *log_lru,
+                      uint64_t len_lru, uint32_t n_points, unison_attainment_point *out);
+
 /* ============================================================ hazard LUT */
 /* The survival table of eqs. (hazard), (hq), (survq) built on the device
  * from turns-per-session counts: n(t) = #{T_s >= t+1}, d(t) = #{T_s = t+1}

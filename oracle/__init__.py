@@ -107,6 +107,8 @@ def lib():
             L.or_kendall_brute.restype = C.c_double
             L.or_ase.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_void_p]
             L.or_ase.restype = None
+            L.or_attainment.argtypes = [C.POINTER(_Trace), C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p]
+            L.or_attainment.restype = C.c_int
             _lib = L
     return _lib
 
@@ -222,3 +224,22 @@ def ase(hit_rate, amat, ttft):
     out = np.zeros(nc, dtype=np.float64)
     lib().or_ase(_ptr(hr), _ptr(am), _ptr(tt), nc, nd, _ptr(out))
     return out
+
+
+def attainment(tr, logs, n_points: int):
+    """Eq. (attainment) over the windows of reading R27: ``logs`` are the
+    (event, kind, session) triples of the online-table, offline-table and LRU
+    replays (``replay(..., log=True)["log"]``).  Returns (status, array
+    [n_points, 6] of n_j, warm requests, H_on, H_off, H_LRU, A_j)."""
+    ts, keep = _trace_struct(tr)
+    packed = []
+    for ev, kind, sess in logs:
+        a = np.empty((len(ev), 2), dtype=np.uint32)
+        a[:, 0] = ev
+        a[:, 1] = (np.asarray(kind, np.uint32) << 24) | np.asarray(sess, np.uint32)
+        packed.append(a)
+    ptrs = (C.c_void_p * 3)(*(_ptr(a) for a in packed))
+    lens = np.array([a.shape[0] for a in packed], dtype=np.uint64)
+    out = np.zeros((max(n_points, 1), 6), dtype=np.float64)
+    rc = lib().or_attainment(C.byref(ts), C.cast(ptrs, C.c_void_p), _ptr(lens), n_points, _ptr(out))
+    return rc, out[:n_points]

@@ -32,6 +32,11 @@
  *   R26 online hazard table (Sec. V-F): starts with no sessions; at the final
  *       completion of a session its turn count T_s is added and the table is
  *       rebuilt with the quantizer of R5; every later key uses it.
+ *   R27 attainment A(n) (eq. attainment): "after n observed sessions" is a
+ *       window of the trace, the warm requests arriving while the online
+ *       table holds n_j <= n < n_{j+1} sessions, n_j = floor(j N / P) for P
+ *       points (the last window includes n = N); H is a replay's hit rate
+ *       over that window.
  *   R12 a completed session stays resident with the maximal key.
  *   R13 DMA busy until now + ceil(moved / dma bytes per us).
  *   R14 TIDE phase 1 (promotion into free fast-tier space) then phase 2
@@ -882,4 +887,69 @@ void or_ase(const double *hr, const double *amat, const double *ttft, int nc, in
     }
     out[c] = pow(prod, 1.0 / (3.0 * nd));
   }
+}
+
+/* Attainment (Sec. V-F, eq. attainment) of an online-table replay against the
+ * offline-table and LRU replays of the same trace, from their decision logs
+ * (kinds HIT_S, HIT_H, MISS mark warm requests).  Windows per reading R27.
+ * out[6j .. 6j+5] = n_j, warm requests in window j, H_on, H_off, H_LRU,
+ * A_j = (H_on - H_LRU) / (H_off - H_LRU); A_j is NaN when the window holds no
+ * warm request or H_off = H_LRU.  The three logs must list the same warm
+ * requests (else OR_ERR_FORMAT). */
+int or_attainment(const or_trace *tr, const or_logrec *const *logs, const uint64_t *lens, uint32_t P,
+                  double *out) {
+  if (!tr || !logs || !lens || !out) return OR_ERR_ARG;
+  const uint64_t N = tr->n_sessions;
+  if (P == 0 || P > N) return OR_ERR_RANGE;
+  or_event *ev = NULL;
+  int rc = or_validate(tr, &ev);
+  if (rc != OR_OK) return rc;
+  const uint64_t E = 2 * tr->n_turns;
+  /* window of every event: sessions completed before it, then the largest
+   * j with floor(j N / P) <= that count */
+  uint32_t *win = (uint32_t *)malloc(sizeof(uint32_t) * (E + 1));
+  uint64_t *warm = (uint64_t *)calloc(3 * (size_t)P, sizeof(uint64_t));
+  uint64_t *hit = (uint64_t *)calloc(3 * (size_t)P, sizeof(uint64_t));
+  if (!win || !warm || !hit) {
+    free(ev), free(win), free(warm), free(hit);
+    return OR_ERR_OOM;
+  }
+  uint64_t done = 0;
+  for (uint64_t e = 0; e < E; e++) {
+    uint32_t j = 0;
+    while (j + 1 < P && (j + 1) * N / P <= done) j++;
+    win[e] = j;
+    const or_event *x = &ev[e];
+    if (x->type == OR_COMPLETION && x->turn + 1 == tr->turn_off[x->session + 1] - tr->turn_off[x->session]) done++;
+  }
+  for (int r = 0; r < 3 && rc == OR_OK; r++) {
+    for (uint64_t i = 0; i < lens[r]; i++) {
+      const uint32_t e = logs[r][i].event, kind = logs[r][i].kind_session >> 24;
+      if (e >= E) {
+        rc = OR_ERR_FORMAT;
+        break;
+      }
+      if (kind == K_HIT_S || kind == K_HIT_H || kind == K_MISS) {
+        warm[r * P + win[e]]++;
+        if (kind != K_MISS) hit[r * P + win[e]]++;
+      }
+    }
+  }
+  for (uint32_t j = 0; j < P && rc == OR_OK; j++) {
+    if (warm[j] != warm[P + j] || warm[j] != warm[2 * P + j]) {
+      rc = OR_ERR_FORMAT;
+      break;
+    }
+    double h[3];
+    for (int r = 0; r < 3; r++) h[r] = warm[j] ? (double)hit[r * P + j] / (double)warm[j] : NAN;
+    double *o = out + 6 * (size_t)j;
+    o[0] = (double)((uint64_t)j * N / P);
+    o[1] = (double)warm[j];
+    o[2] = h[0];
+    o[3] = h[1];
+    o[4] = h[2];
+    o[5] = (warm[j] && h[1] != h[2]) ? (h[0] - h[2]) / (h[1] - h[2]) : NAN;
+  }
+  free(ev), free(win), free(warm), free(hit);
+  return rc;
 }

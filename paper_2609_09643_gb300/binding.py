@@ -92,7 +92,7 @@ EXPORTS = ["unison_strerror", "unison_version", "unison_trace_create", "unison_t
            "unison_trace_upload", "unison_trace_free", "unison_trace_info", "unison_trace_device_bytes",
            "unison_replay_batch", "unison_stats", "unison_hazard_lut", "unison_rank_batch",
            "unison_profile_enable", "unison_profile_read", "unison_launch_count",
-           "unison_replay_batch_noalloc", "unison_ase"]
+           "unison_replay_batch_noalloc", "unison_ase", "unison_attainment"]
 
 
 def lib_path() -> str:
@@ -132,6 +132,8 @@ def lib():
             L.unison_launch_count.restype = C.c_uint64
             L.unison_replay_batch_noalloc.argtypes = L.unison_replay_batch.argtypes
             L.unison_ase.argtypes = [C.POINTER(Stats), C.c_int, C.c_int, C.POINTER(C.c_double)]
+            L.unison_attainment.argtypes = [C.c_void_p, C.c_void_p, C.c_uint64, C.c_void_p, C.c_uint64,
+                                            C.c_void_p, C.c_uint64, C.c_uint32, C.POINTER(AttainmentPoint)]
             _lib = L
     return _lib
 
@@ -292,6 +294,29 @@ def ase(stats_grid) -> List[float]:
     out = (C.c_double * max(nc, 1))()
     _check("unison_ase", lib().unison_ase(arr, nc, nd, out))
     return [out[i] for i in range(nc)]
+
+
+class AttainmentPoint(C.Structure):
+    _fields_ = [("sessions_seen", C.c_uint32), ("reserved", C.c_uint32), ("warm", C.c_uint64),
+                ("hr_online", C.c_double), ("hr_offline", C.c_double), ("hr_lru", C.c_double),
+                ("attainment", C.c_double)]
+
+
+def attainment(trace: Trace, logs, n_points: int) -> List[dict]:
+    """unison_attainment: logs are the (event, kind, session) arrays of the
+    online-table, offline-table and LRU replays (decode_log output)."""
+    packed = []
+    for ev, kind, sess in logs:
+        a = np.empty((len(ev), 2), dtype=np.uint32)
+        a[:, 0] = ev
+        a[:, 1] = (np.asarray(kind, np.uint32) << 24) | np.asarray(sess, np.uint32)
+        packed.append(a)
+    out = (AttainmentPoint * max(n_points, 1))()
+    args = []
+    for a in packed:
+        args += [a.ctypes.data, a.shape[0]]
+    _check("unison_attainment", lib().unison_attainment(trace.handle, *args, n_points, out))
+    return [{f: getattr(out[i], f) for f, _ in AttainmentPoint._fields_ if f != "reserved"} for i in range(n_points)]
 
 
 def hazard_lut(turns_dev, bucket: int = 1, stream=None):

@@ -1455,6 +1455,57 @@ extern "C" int unison_ase(const unison_stats_t *stats, int n_configs, int n_data
   return UNISON_OK;
 }
 
+// Eq. (attainment) over windows of observed sessions.  Every event's window
+// comes from the trace's host event array (a final completion has the edge
+// flag); each log then adds its warm requests, and hits, to their windows.
+extern "C" int unison_attainment(const unison_trace *trace, const unison_decision *log_online, uint64_t len_online,
+                                 const unison_decision *log_offline, uint64_t len_offline,
+                                 const unison_decision *log_lru, uint64_t len_lru, uint32_t n_points,
+                                 unison_attainment_point *out) {
+  if (!trace || !trace->h_block || !out || (len_online && !log_online) || (len_offline && !log_offline) ||
+      (len_lru && !log_lru))
+    return UNISON_ERR_ARG;
+  const uint64_t N = trace->n_sessions, E = trace->n_events;
+  if (n_points == 0 || n_points > N) return UNISON_ERR_RANGE;
+  const uint4 *ev = trace->h<uint4>(trace->off_ev);
+  std::vector<uint32_t> window(E);
+  uint64_t seen = 0;
+  uint32_t j = 0;  // windows only advance: seen grows with the event index
+  for (uint64_t e = 0; e < E; e++) {
+    while (j + 1 < n_points && (uint64_t)(j + 1) * N / n_points <= seen) j++;
+    window[e] = j;
+    const uint32_t w1 = ev[e].y;
+    if (!(w1 & kEvArrival) && (w1 & kEvEdge)) seen++;
+  }
+  const unison_decision *logs[3] = {log_online, log_offline, log_lru};
+  const uint64_t lens[3] = {len_online, len_offline, len_lru};
+  std::vector<uint64_t> warm(3 * (size_t)n_points, 0), hits(3 * (size_t)n_points, 0);
+  for (int r = 0; r < 3; r++)
+    for (uint64_t i = 0; i < lens[r]; i++) {
+      const unison_decision &d = logs[r][i];
+      const uint32_t kind = d.kind_session >> 24;
+      if (d.event >= E) return UNISON_ERR_FORMAT;
+      if (kind == UNISON_KIND_HIT_S || kind == UNISON_KIND_HIT_H || kind == UNISON_KIND_MISS) {
+        const size_t w = (size_t)r * n_points + window[d.event];
+        warm[w]++;
+        hits[w] += kind != UNISON_KIND_MISS;
+      }
+    }
+  for (uint32_t k = 0; k < n_points; k++) {
+    const uint64_t n = warm[k];
+    if (warm[n_points + k] != n || warm[2 * (size_t)n_points + k] != n) return UNISON_ERR_FORMAT;
+    unison_attainment_point &o = out[k];
+    o.sessions_seen = (uint32_t)((uint64_t)k * N / n_points);
+    o.reserved = 0;
+    o.warm = n;
+    o.hr_online = n ? (double)hits[k] / (double)n : NAN;
+    o.hr_offline = n ? (double)hits[n_points + k] / (double)n : NAN;
+    o.hr_lru = n ? (double)hits[2 * (size_t)n_points + k] / (double)n : NAN;
+    o.attainment = (n && o.hr_offline != o.hr_lru) ? (o.hr_online - o.hr_lru) / (o.hr_offline - o.hr_lru) : NAN;
+  }
+  return UNISON_OK;
+}
+
 // ---------------------------------------------------------------------------
 // Replay without device allocation.
 //

@@ -55,7 +55,7 @@ def make_records(seed: int, n: int) -> Records:
     pinned = rng.uniform(seed, _R_PIN, i) < (1.0 / 64.0)
     done = (~pinned) & (t == t_s - 1)
     flags = (pinned.astype(np.uint8) * FLAG_PINNED) | (done.astype(np.uint8) * FLAG_DONE)
-    gap = np.floor(_lognormal_mixture(seed ^ 0x5A5A, i, GAP_MIX_CODING) * 1e6 + 0.5)
+    gap = np.floor(_lognormal_mixture(seed ^ 0x5A5A, i, i, GAP_MIX_CODING, 0.0) * 1e6 + 0.5)
     gap = np.clip(gap, 1, GAP_MAX_US).astype(np.int64)
     gap[t == 0] = 0
     growth = 545.0 * np.exp(0.3 * rng.normal(seed, _R_KV, i))

@@ -18,7 +18,14 @@ Workload model (one reading, stated once, used by every generator here):
   ``decode_k ~ U{64..256}``;
 * the trace is open loop: ``c_{s,k} = a_{s,k} + 20 us * decode_k`` and
   ``a_{s,k+1} = c_{s,k} + gap``, the gap drawn from a lognormal mixture and
-  clamped to [1, 2**31 - 1] microseconds.
+  clamped to [1, 2**31 - 1] microseconds;
+* gaps recur per session (the gap average of Sec. IV-C tracks a session's
+  characteristic return interval): a session draws its mixture component
+  once and a characteristic interval ``med * exp(sig * sqrt(rho) * Z_s)``,
+  and each gap is that interval times ``exp(sig * sqrt(1 - rho) * Z_{s,k})``:
+  each component keeps its marginal LN(med, sig), and log-gaps of one
+  session correlate with coefficient ``rho`` (0.7; 0 draws every gap on its
+  own, component included).
 
 Times are absolute unsigned 64-bit microseconds.
 """
@@ -41,8 +48,12 @@ FIRST_PREFIX_TOKENS = 2048
 DECODE_US_PER_TOKEN = 20
 GAP_MAX_US = (1 << 31) - 1
 
+# Share of a gap's log-variance fixed per session.
+GAP_PERSIST = 0.7
+
 # Stream ids: one counter-addressed stream per kind of draw.
 _ST_START, _ST_TURNS, _ST_DECODE, _ST_INSERT, _ST_GAPC, _ST_GAPN = 1, 2, 4, 6, 8, 10
+_ST_SESSC, _ST_SESSN = 12, 14  # per-session component and interval (by session id)
 
 _UTR_MAGIC = b"UTR1"
 
@@ -106,11 +117,17 @@ def geometric_turns(seed: int, n_sessions: int, mean: float, lo: int, hi: int,
     return t
 
 
-def _lognormal_mixture(seed: int, idx: np.ndarray, mix) -> np.ndarray:
-    """Seconds drawn from a lognormal mixture: component by one uniform,
-    then median * exp(sigma * Z)."""
-    u = rng.uniform(seed, _ST_GAPC, idx)
-    z = rng.normal(seed, _ST_GAPN, idx)
+def _lognormal_mixture(seed: int, sess: np.ndarray, idx: np.ndarray, mix, rho: float) -> np.ndarray:
+    """Seconds drawn from a lognormal mixture (see module doc): the component
+    by one uniform (per session when rho > 0, else per turn), then median *
+    exp(sigma * (sqrt(rho) Z_s + sqrt(1 - rho) Z_{s,k}))."""
+    if not 0.0 <= rho <= 1.0:
+        raise ValueError("gap persistence must be in [0, 1]")
+    su = sess.astype(np.uint64)
+    u = rng.uniform(seed, _ST_SESSC, su) if rho > 0 else rng.uniform(seed, _ST_GAPC, idx)
+    z = np.sqrt(1.0 - rho) * rng.normal(seed, _ST_GAPN, idx)
+    if rho > 0:
+        z = z + np.sqrt(rho) * rng.normal(seed, _ST_SESSN, su)
     out = np.empty(idx.shape[0], dtype=np.float64)
     acc = 0.0
     chosen = np.zeros(idx.shape[0], dtype=bool)
@@ -123,7 +140,8 @@ def _lognormal_mixture(seed: int, idx: np.ndarray, mix) -> np.ndarray:
 
 
 def make_trace(seed: int, turns: Sequence[int] | np.ndarray, start_mean_s: float,
-               gap_mix=GAP_MIX_CODING, first_start_at_zero: bool = False) -> Trace:
+               gap_mix=GAP_MIX_CODING, first_start_at_zero: bool = False,
+               gap_persist: float = GAP_PERSIST) -> Trace:
     """Build a trace with the given turns per session (see module doc)."""
     t_s = np.asarray(turns, dtype=np.int64)
     n = t_s.shape[0]
@@ -160,7 +178,7 @@ def make_trace(seed: int, turns: Sequence[int] | np.ndarray, start_mean_s: float
     if out_tok.max(initial=0) >= (1 << 32):
         raise ValueError("token counts overflow 32 bits")
 
-    gap = np.floor(_lognormal_mixture(seed, addr, gap_mix) * 1e6 + 0.5)
+    gap = np.floor(_lognormal_mixture(seed, sess, addr, gap_mix, gap_persist) * 1e6 + 0.5)
     gap = np.clip(gap, 1, GAP_MAX_US).astype(np.int64)
     gap[k == 0] = 0  # turn 0 has no preceding gap
     # a_k = start + sum_{j<k} (20 us * decode_j) + sum_{j<=k} gap_j

@@ -142,3 +142,44 @@ def test_ase_library_matches_oracle(B):
         B.ase([[dict(hit_rate=-1.0, amat_ps=1.0, ttft_mean_ns=1.0)]])
     with pytest.raises(B.UnisonError):
         B.ase([])
+
+
+def test_attainment_library_matches_oracle(B):
+    """unison_attainment (host function over a trace handle) against the
+    oracle's on the worked hand case and on three replays' logs; errors."""
+    import oracle
+    from cases import base, to_oracle
+    from test_oracle_pins import _attain_hand, _ATTAIN_HAND
+    tr, logs = _attain_hand()
+    h = B.Trace(tr)
+    for P, want in _ATTAIN_HAND.items():
+        got = B.attainment(h, logs, P)
+        arr = np.array([[g["sessions_seen"], g["warm"], g["hr_online"], g["hr_offline"], g["hr_lru"],
+                         g["attainment"]] for g in got])
+        np.testing.assert_array_equal(arr, oracle.attainment(tr, logs, P)[1])
+        np.testing.assert_allclose(arr, np.array(want), rtol=1e-15, atol=0, equal_nan=True)
+    for P in (0, 5):
+        with pytest.raises(B.UnisonError) as ei:
+            B.attainment(h, logs, P)
+        assert ei.value.code == B.ERR_RANGE
+    bad = (logs[0][0], logs[0][1].copy(), logs[0][2])
+    bad[1][2] = 0
+    with pytest.raises(B.UnisonError) as ei:
+        B.attainment(h, [bad, logs[1], logs[2]], 2)
+    assert ei.value.code == B.ERR_FORMAT
+    far = (logs[0][0].copy(), logs[0][1], logs[0][2])
+    far[0][-1] = 16
+    with pytest.raises(B.UnisonError) as ei:
+        B.attainment(h, [far, logs[1], logs[2]], 2)
+    assert ei.value.code == B.ERR_FORMAT
+
+    tr = synth.make_trace(21, 2 + (np.arange(120) % 9), 0.3, synth.GAP_MIX_CODING)
+    cap = 16 * tr.n_events
+    lg = [oracle.replay(tr, to_oracle(base(p, 20000 * 131072, 100000 * 131072, 131072, online=o)), log=True,
+                        log_capacity=cap)["log"] for p, o in (("spear", True), ("spear", False), ("lru", False))]
+    h = B.Trace(tr)
+    for P in (1, 7, 16, 120):
+        got = B.attainment(h, lg, P)
+        arr = np.array([[g["sessions_seen"], g["warm"], g["hr_online"], g["hr_offline"], g["hr_lru"],
+                         g["attainment"]] for g in got])
+        np.testing.assert_array_equal(arr, oracle.attainment(tr, lg, P)[1])

@@ -306,3 +306,21 @@ def test_online_hazard_rejected_cases(B):
     with pytest.raises(B.UnisonError) as ei:
         B.replay_batch(hb, [to_lib(base("spear", 1 * GIB, 8 * GIB, 16384, online=True))])
     assert ei.value.code == B.ERR_RANGE
+
+
+def test_online_attainment_from_device_logs(B):
+    """Eq. (attainment) from the device's decision logs (online SPEAR+TIDE,
+    offline SPEAR+TIDE, LRU on the paper-scale coding trace) equals the
+    oracle's from its own logs."""
+    tr = synth.paper_scale_trace(1, "coding")
+    ps = [base("spear_tide", 4 * GIB, 64 * GIB, 131072, online=True), base("spear_tide", 4 * GIB, 64 * GIB, 131072),
+          base("lru", 4 * GIB, 64 * GIB, 131072)]
+    cap = 4 * tr.n_events
+    res, log, handles = run_gpu(B, [tr], [(0, p) for p in ps], log_capacity=cap)
+    logs = [B.decode_log(log[i], res[i]["log_len"]) for i in range(3)]
+    ologs = [oracle.replay(tr, to_oracle(p), log=True, log_capacity=cap)["log"] for p in ps]
+    for P in (1, 8, 32):
+        got = B.attainment(handles[0], logs, P)
+        arr = np.array([[g["sessions_seen"], g["warm"], g["hr_online"], g["hr_offline"], g["hr_lru"],
+                         g["attainment"]] for g in got])
+        np.testing.assert_array_equal(arr, oracle.attainment(tr, ologs, P)[1])

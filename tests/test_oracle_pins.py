@@ -558,3 +558,82 @@ def test_online_hazard_two_phase_equals_offline():
         assert a["evict"] + a["demote"] > 0, pol  # the tiers do fill in wave 2
         _, lc, _, _ = _online_logs(tr, p, dict(p, bucket=3))
         assert not all(np.array_equal(x, y) for x, y in zip(lb, lc)), pol
+
+
+# ---- attainment A(n) (Sec. V-F, eq. attainment; reading R27) ---------------------
+
+def _attain_hand():
+    """Four sessions of two turns.  Events in time order: the four first turns
+    (e0..e7), then e8 = arrival of s0's second turn, e9 its final completion,
+    e10/e11 the same for s1, e12/e13 for s2, e14/e15 for s3.  So the warm
+    arrivals e8, e10, e12, e14 see 0, 1, 2, 3 completed sessions."""
+    arr = [[0, 100], [20, 200], [40, 300], [60, 400]]
+    comp = [[10, 110], [30, 210], [50, 310], [70, 410]]
+    tr = synth.trace_from_turns(arr, comp, [[100, 200]] * 4, [[150, 250]] * 4)
+    HS, HH, MI, CO, PS, EV = 1, 2, 3, 0, 4, 8
+
+    def lg(kinds):  # warm decisions at e8, e10, e12, e14 plus ignored records
+        ev = [0, 1, 8, 10, 11, 12, 14]
+        kd = [CO, PS, kinds[0], kinds[1], EV, kinds[2], kinds[3]]
+        ss = [0, 0, 0, 1, 2, 2, 3]
+        return np.array(ev, np.uint32), np.array(kd, np.uint8), np.array(ss, np.uint32)
+
+    return tr, [lg((HS, MI, HH, HS)), lg((HS, HS, HS, HH)), lg((MI, MI, HS, MI))]
+
+
+# expected (n_j, warm, H_on, H_off, H_lru, A) per point count, worked by hand:
+# P=1: H = 3/4, 4/4, 1/4 -> A = (3/4 - 1/4) / (1 - 1/4) = 2/3
+# P=2 (n_j = 0, 2): {e8, e10} -> 1/2, 1, 0 -> 1/2;  {e12, e14} -> 1, 1, 1/2 -> 1
+# P=3 (n_j = 0, 1, 2): {e8} -> 1;  {e10} -> 0, 1, 0 -> 0;  {e12, e14} -> 1
+# P=4: {e8} -> 1;  {e10} -> 0;  {e12} -> 1, 1, 1 -> undefined;  {e14} -> 1, 1, 0 -> 1
+_ATTAIN_HAND = {
+    1: [(0, 4, 0.75, 1.0, 0.25, 2 / 3)],
+    2: [(0, 2, 0.5, 1.0, 0.0, 0.5), (2, 2, 1.0, 1.0, 0.5, 1.0)],
+    3: [(0, 1, 1.0, 1.0, 0.0, 1.0), (1, 1, 0.0, 1.0, 0.0, 0.0), (2, 2, 1.0, 1.0, 0.5, 1.0)],
+    4: [(0, 1, 1.0, 1.0, 0.0, 1.0), (1, 1, 0.0, 1.0, 0.0, 0.0), (2, 1, 1.0, 1.0, 1.0, float("nan")),
+        (3, 1, 1.0, 1.0, 0.0, 1.0)],
+}
+
+
+def test_attainment_hand_case():
+    tr, logs = _attain_hand()
+    for P, want in _ATTAIN_HAND.items():
+        rc, got = oracle.attainment(tr, logs, P)
+        assert rc == 0
+        np.testing.assert_allclose(got, np.array(want), rtol=1e-15, atol=0, equal_nan=True, err_msg=str(P))
+
+
+def test_attainment_errors():
+    tr, logs = _attain_hand()
+    assert oracle.attainment(tr, logs, 0)[0] == -4  # OR_ERR_RANGE
+    assert oracle.attainment(tr, logs, 5)[0] == -4  # more points than sessions
+    bad = (logs[0][0], logs[0][1].copy(), logs[0][2])
+    bad[1][2] = 0  # e8 no longer a warm request in one log
+    assert oracle.attainment(tr, [bad, logs[1], logs[2]], 2)[0] == -3  # OR_ERR_FORMAT
+    far = (logs[0][0].copy(), logs[0][1], logs[0][2])
+    far[0][-1] = 16  # past the last event
+    assert oracle.attainment(tr, [far, logs[1], logs[2]], 2)[0] == -3
+
+
+def test_attainment_identities_on_replays():
+    """On real replay logs: the offline replay against itself attains 1 and
+    LRU attains 0 in every window where they differ; the windows partition
+    the warm requests; n_j = floor(j N / P)."""
+    from cases import base, to_oracle
+    tr = synth.make_trace(21, 2 + (np.arange(120) % 9), 0.3, synth.GAP_MIX_CODING)
+    cap = 16 * tr.n_events
+    r_on, r_off, r_lru = (oracle.replay(tr, to_oracle(base(p, 20000 * 131072, 100000 * 131072, 131072, online=o)),
+                                        log=True, log_capacity=cap)
+                          for p, o in (("spear", True), ("spear", False), ("lru", False)))
+    for P in (1, 7, 16, 120):
+        rc, a = oracle.attainment(tr, [r_off["log"], r_off["log"], r_lru["log"]], P)
+        assert rc == 0
+        d = (a[:, 1] > 0) & (a[:, 3] != a[:, 4])
+        assert d.any()
+        assert np.all(a[d, 5] == 1.0) and np.all(np.isnan(a[~d, 5]))
+        rc, z = oracle.attainment(tr, [r_lru["log"], r_off["log"], r_lru["log"]], P)
+        assert np.all(z[d, 5] == 0.0)
+        rc, b = oracle.attainment(tr, [r_on["log"], r_off["log"], r_lru["log"]], P)
+        assert rc == 0
+        assert int(b[:, 1].sum()) == r_on["req_warm"]
+        assert list(b[:, 0]) == [j * 120 // P for j in range(P)]
