@@ -667,19 +667,23 @@ __device__ void online_rerank(Sorted &T, const OnlineTable &ot, const uint32_t *
       T.e[i] = v;
     }
   }
+  __syncwarp();
+  // a small change of the table often keeps the order: then nothing moves
+  bool out_of_order = false;
+  for (uint32_t i = lane + 1; i < T.n; i += 32) out_of_order |= ekey(T.e[i - 1]) > ekey(T.e[i]);
+  if (!__any_sync(kFull, out_of_order)) return;
   for (uint32_t i = T.n + lane; i < ring; i += 32) T.e[i] = make_uint4(0u, 0u, 0u, 0u);
   __syncwarp();
   for (uint32_t k = 2; k <= ring; k <<= 1) {
     for (uint32_t j = k >> 1; j > 0; j >>= 1) {
-      for (uint32_t i = lane; i < ring; i += 32) {
-        const uint32_t ij = i ^ j;
-        if (ij > i) {
-          const uint4 a = T.e[i], b = T.e[ij];
-          const bool desc = (i & k) == 0;
-          if (desc ? ekey(a) < ekey(b) : ekey(a) > ekey(b)) {
-            T.e[i] = b;
-            T.e[ij] = a;
-          }
+      for (uint32_t q = lane; q < ring / 2; q += 32) {
+        // q-th pair (i, i + j): i has a zero at bit j
+        const uint32_t i = ((q & ~(j - 1)) << 1) | (q & (j - 1)), ij = i | j;
+        const uint4 a = T.e[i], b = T.e[ij];
+        const bool desc = (i & k) == 0;
+        if (desc ? ekey(a) < ekey(b) : ekey(a) > ekey(b)) {
+          T.e[i] = b;
+          T.e[ij] = a;
         }
       }
       __syncwarp();
