@@ -26,6 +26,8 @@ _BUILD = os.path.join(_HERE, "_build")
 _LIB = os.path.join(_BUILD, "libunison_oracle.so")
 
 POLICIES = {"lru": 0, "timeout": 1, "spear": 2, "spear_tide": 3, "belady": 4, "lru_tide": 5}
+# R28 sync points of the stale-snapshot (dual design) replays
+STALE_SYNC = {"live": 0, "event": 1, "arrivals": 2, "gap_start": 3}
 KINDS = ["COLD", "HIT_S", "HIT_H", "MISS", "PLACE_S", "PLACE_H", "BYPASS", "DEMOTE", "EVICT",
          "PROMOTE", "TIDE_DEMOTE", "EXPIRE"]
 
@@ -50,14 +52,15 @@ class _Params(C.Structure):
                 ("ema_num", C.c_uint32), ("ema_den", C.c_uint32), ("penalty_q", C.c_uint64),
                 ("ttl_us", C.c_uint32), ("ttft_load", C.c_uint32),
                 ("dma_bytes_per_us", C.c_uint64), ("prefill_ns_per_tok", C.c_uint64),
-                ("debug", C.c_uint32), ("hazard_online", C.c_uint32)]
+                ("debug", C.c_uint32), ("hazard_online", C.c_uint32), ("stale_sync", C.c_uint32),
+                ("stale_m", C.c_uint32)]
 
 
 RESULT_FIELDS = ["events", "req_warm", "cold", "hit_s", "hit_h", "miss", "bypass", "place_s",
                  "place_h", "evict", "demote", "promote", "tide_demote", "expire", "tok_hit_s",
                  "tok_hit_h", "tok_miss", "tok_computed", "tok_needed", "dma_bytes", "tide_calls",
                  "promoted_then_hit_s", "ttft_sum_lo", "ttft_sum_hi", "ttft_p50_ns", "ttft_n",
-                 "decision_hash", "log_len"]
+                 "decision_hash", "log_len", "vict_n", "vict_diff", "prom_n", "prom_diff"]
 
 
 class _Result(C.Structure):
@@ -133,7 +136,8 @@ def _params_struct(p: dict, debug: bool):
     return _Params(pol, q["hazard_bucket"], q["cap_s_bytes"], q["cap_h_bytes"],
                    q["kv_bytes_per_token"], q["max_sessions"], q["ema_num"], q["ema_den"],
                    q["penalty_q"], q["ttl_us"], q["ttft_load"], q["dma_bytes_per_us"],
-                   q["t_p_ps_per_tok"] // 1000, 1 if debug else 0, 1 if q.get("hazard_online") else 0)
+                   q["t_p_ps_per_tok"] // 1000, 1 if debug else 0, 1 if q.get("hazard_online") else 0,
+                   STALE_SYNC[q.get("stale_sync", "live")], q.get("stale_m", 0))
 
 
 def replay(tr, params: dict, log: bool = False, ttft: bool = False, debug: bool = False,

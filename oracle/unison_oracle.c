@@ -32,6 +32,15 @@
  *   R26 online hazard table (Sec. V-F): starts with no sessions; at the final
  *       completion of a session its turn count T_s is added and the table is
  *       rebuilt with the quantizer of R5; every later key uses it.
+ *   R28 stale snapshot of a dual design (Sec. IV-B eq. stale, Tab. org): the
+ *       ranking decisions (make-room victims, slot-limit evictions, TIDE's
+ *       promotions and demotions) score every session from a copy of its
+ *       register row (g_q, turn, done) taken at the last sync point, after
+ *       that event's own decisions; residency, sizes and pins stay live.  Rows
+ *       start at zero.  Sync points: every event, every m-th arrival, or
+ *       every gap_start.  Vict!= (Prom!=) counts the acted-upon victim
+ *       (promotion) choices whose session differs from the choice by the
+ *       live rows over the same candidates.
  *   R27 attainment A(n) (eq. attainment): "after n observed sessions" is a
  *       window of the trace, the warm requests arriving while the online
  *       table holds n_j <= n < n_{j+1} sessions, n_j = floor(j N / P) for P
@@ -97,7 +106,11 @@ typedef struct {
   uint64_t prefill_ns_per_tok;   /* t_p in ns per token, for TTFT */
   uint32_t debug;                /* 1: check invariants and both TIDE forms every event */
   uint32_t hazard_online;        /* 1: the hazard table starts empty and grows as sessions complete (R26) */
+  uint32_t stale_sync;           /* R28: 0 live; 1 every event; 2 every stale_m arrivals; 3 every gap_start */
+  uint32_t stale_m;
 } or_params;
+
+enum { OR_SYNC_LIVE = 0, OR_SYNC_EVENT = 1, OR_SYNC_ARRIVALS = 2, OR_SYNC_GAP_START = 3 };
 
 typedef struct {
   uint64_t events, req_warm, cold, hit_s, hit_h, miss, bypass, place_s, place_h;
@@ -106,6 +119,7 @@ typedef struct {
   uint64_t dma_bytes, tide_calls, promoted_then_hit_s;
   uint64_t ttft_sum_lo, ttft_sum_hi, ttft_p50_ns, ttft_n;
   uint64_t decision_hash, log_len;
+  uint64_t vict_n, vict_diff, prom_n, prom_diff; /* R28 */
   int32_t status;
   uint32_t pad2;
 } or_result;
@@ -191,6 +205,9 @@ typedef struct {
   or_result *res;
   or_sess *S;
   uint16_t sigma_q[OR_T_MAX + 1];
+  int stale;           /* R28: rank from the snapshot rows below */
+  uint64_t *snap_g;
+  uint32_t *snap_turn, *snap_done;
   uint32_t *resident;  /* ids of sessions in a tier, unordered */
   uint64_t n_resident;
   uint64_t cap_s, cap_h;  /* tokens */
@@ -209,8 +226,9 @@ static int cmp_event(const void *a, const void *b) {
   return 0;
 }
 
-/* Policy key of session s (R8); larger = more evictable. */
-static uint64_t key_of(const or_state *st, uint32_t s) {
+/* Policy key of session s from its live register row (R8); larger = more
+ * evictable. */
+static uint64_t live_key_of(const or_state *st, uint32_t s) {
   const or_sess *x = &st->S[s];
   switch (st->p->policy) {
     case OR_SPEAR:
@@ -225,9 +243,22 @@ static uint64_t key_of(const or_state *st, uint32_t s) {
   }
 }
 
+/* The key decisions rank by: the live row, or the snapshot row (R28). */
+static uint64_t key_of(const or_state *st, uint32_t s) {
+  if (!st->stale) return live_key_of(st, s);
+  uint32_t t = st->snap_turn[s] < OR_T_MAX ? st->snap_turn[s] : OR_T_MAX;
+  return or_spear_score(st->snap_g[s], st->sigma_q[t], st->p->penalty_q, (int)st->snap_done[s]);
+}
+
 /* a more evictable than b: larger key, then smaller id. */
 static int more_evictable(const or_state *st, uint32_t a, uint32_t b) {
   uint64_t ka = key_of(st, a), kb = key_of(st, b);
+  if (ka != kb) return ka > kb;
+  return a < b;
+}
+
+static int more_evictable_live(const or_state *st, uint32_t a, uint32_t b) {
+  uint64_t ka = live_key_of(st, a), kb = live_key_of(st, b);
   if (ka != kb) return ka > kb;
   return a < b;
 }
@@ -306,6 +337,42 @@ static int64_t argmin_unpinned(const or_state *st, uint32_t tier) {
   return best;
 }
 
+/* Most / least evictable unpinned resident of a tier by the live rows. */
+static int64_t argmax_unpinned_live(const or_state *st, uint32_t tier) {
+  int64_t best = -1;
+  for (uint64_t i = 0; i < st->n_resident; i++) {
+    uint32_t s = st->resident[i];
+    const or_sess *x = &st->S[s];
+    if (x->pinned || (tier != 0 && x->tier != tier)) continue;
+    if (best < 0 || more_evictable_live(st, s, (uint32_t)best)) best = s;
+  }
+  return best;
+}
+
+static int64_t argmin_unpinned_live(const or_state *st, uint32_t tier) {
+  int64_t best = -1;
+  for (uint64_t i = 0; i < st->n_resident; i++) {
+    uint32_t s = st->resident[i];
+    const or_sess *x = &st->S[s];
+    if (x->pinned || x->tier != tier) continue;
+    if (best < 0 || more_evictable_live(st, (uint32_t)best, s)) best = s;
+  }
+  return best;
+}
+
+/* R28: one acted-upon victim (promotion) choice against the live choice. */
+static void count_victim(or_state *st, uint32_t chosen, int64_t live) {
+  if (!st->stale) return;
+  st->res->vict_n++;
+  st->res->vict_diff += live != (int64_t)chosen;
+}
+
+static void count_promotion(or_state *st, uint32_t chosen, int64_t live) {
+  if (!st->stale) return;
+  st->res->prom_n++;
+  st->res->prom_diff += live != (int64_t)chosen;
+}
+
 /* R9: admit a session demoted from the fast tier into the HBM tier. */
 static void admit_demoted(or_state *st, uint32_t d, uint64_t size) {
   uint64_t pinned_h = used_of(st, OR_H, 1);
@@ -317,6 +384,11 @@ static void admit_demoted(or_state *st, uint32_t d, uint64_t size) {
   while (st->used_h + size > st->cap_h) {
     int64_t v = argmax_unpinned(st, OR_H);
     /* v = most evictable of (unpinned H) u {d}; if that is d, drop d. */
+    if (st->stale) {
+      int64_t lv = argmax_unpinned_live(st, OR_H);
+      int64_t live = (lv < 0 || more_evictable_live(st, d, (uint32_t)lv)) ? (int64_t)d : lv;
+      count_victim(st, (v < 0 || more_evictable(st, d, (uint32_t)v)) ? d : (uint32_t)v, live);
+    }
     if (v < 0 || more_evictable(st, d, (uint32_t)v)) {
       log_decision(st, K_EVICT, d);
       st->res->evict++;
@@ -347,6 +419,7 @@ static void place(or_state *st, uint32_t s, uint64_t n) {
     while (st->used_s + n > st->cap_s) {
       int64_t d = argmax_unpinned(st, OR_S);
       if (d < 0) { st->res->status = OR_ERR_INVARIANT; return; }
+      if (st->stale) count_victim(st, (uint32_t)d, argmax_unpinned_live(st, OR_S));
       uint64_t sz = st->S[d].size;
       res_remove(st, (uint32_t)d);
       admit_demoted(st, (uint32_t)d, sz);
@@ -359,6 +432,7 @@ static void place(or_state *st, uint32_t s, uint64_t n) {
     while (st->used_h + n > st->cap_h) {
       int64_t v = argmax_unpinned(st, OR_H);
       if (v < 0) { st->res->status = OR_ERR_INVARIANT; return; }
+      if (st->stale) count_victim(st, (uint32_t)v, argmax_unpinned_live(st, OR_H));
       evict(st, (uint32_t)v, K_EVICT);
     }
     res_add(st, s, OR_H, n);
@@ -374,6 +448,7 @@ static void place(or_state *st, uint32_t s, uint64_t n) {
     while (st->n_resident > p->max_sessions) {
       int64_t v = argmax_unpinned(st, 0);
       if (v < 0) { st->res->status = OR_ERR_INVARIANT; return; }
+      if (st->stale) count_victim(st, (uint32_t)v, argmax_unpinned_live(st, 0));
       evict(st, (uint32_t)v, K_EVICT);
     }
   }
@@ -454,6 +529,7 @@ static uint64_t tide_loop_form(or_state *st, uint64_t budget, or_tide_moves *rec
     if (p < 0) break;
     uint64_t sz = st->S[p].size, by = sz * kvB;
     if (by > rem || st->used_s + sz > st->cap_s) break;
+    if (st->stale) count_promotion(st, (uint32_t)p, argmin_unpinned_live(st, OR_H));
     rem -= by;
     res_remove(st, (uint32_t)p);
     res_add(st, (uint32_t)p, OR_S, sz);
@@ -471,6 +547,10 @@ static uint64_t tide_loop_form(or_state *st, uint64_t budget, or_tide_moves *rec
     if (by > rem) break;
     if (st->used_s - sd + sp > st->cap_s) break;
     if (st->used_h - sp + sd > st->cap_h) break;
+    if (st->stale) {
+      count_promotion(st, (uint32_t)p, argmin_unpinned_live(st, OR_H));
+      count_victim(st, (uint32_t)d, argmax_unpinned_live(st, OR_S));
+    }
     rem -= by;
     res_remove(st, (uint32_t)p);
     res_remove(st, (uint32_t)d);
@@ -553,7 +633,10 @@ int or_replay(const or_trace *tr, const or_params *p, or_result *res, or_logrec 
   if (!tr || !p || p->hazard_bucket == 0 || p->ema_den == 0 || p->ema_num > p->ema_den ||
       p->kv_bytes_per_token == 0 || p->kv_bytes_per_token > (1u << 24) || p->ttft_load == 0 ||
       p->policy > OR_LRU_TIDE || p->penalty_q >= (1ull << 32) ||
-      (p->ttl_us != UINT32_MAX && p->ttl_us >= (1u << 31)) || p->dma_bytes_per_us >= (1ull << 32))
+      (p->ttl_us != UINT32_MAX && p->ttl_us >= (1u << 31)) || p->dma_bytes_per_us >= (1ull << 32) ||
+      p->stale_sync > OR_SYNC_GAP_START || (p->stale_sync == OR_SYNC_ARRIVALS && p->stale_m == 0) ||
+      (p->stale_sync != OR_SYNC_LIVE &&
+       (p->hazard_online || (p->policy != OR_SPEAR && p->policy != OR_SPEAR_TIDE))))
     return res->status = OR_ERR_ARG;
   or_event *ev = NULL;
   int rc = or_validate(tr, &ev);
@@ -566,6 +649,10 @@ int or_replay(const or_trace *tr, const or_params *p, or_result *res, or_logrec 
   st.p = p;
   st.res = res;
   st.S = (or_sess *)calloc(S + 1, sizeof(or_sess));
+  st.stale = p->stale_sync != OR_SYNC_LIVE;
+  st.snap_g = (uint64_t *)calloc(S + 1, sizeof(uint64_t)); /* R28: rows start at zero */
+  st.snap_turn = (uint32_t *)calloc(S + 1, sizeof(uint32_t));
+  st.snap_done = (uint32_t *)calloc(S + 1, sizeof(uint32_t));
   st.resident = (uint32_t *)malloc(sizeof(uint32_t) * (S + 1));
   uint64_t *ttft = (uint64_t *)malloc(sizeof(uint64_t) * (T + 1));
   uint64_t *next_arr = (uint64_t *)malloc(sizeof(uint64_t) * (E + 1));
@@ -579,7 +666,7 @@ int or_replay(const or_trace *tr, const or_params *p, or_result *res, or_logrec 
   m2.p1 = (uint32_t *)malloc(sizeof(uint32_t) * (S + 1));
   m2.p2 = (uint32_t *)malloc(sizeof(uint32_t) * (S + 1));
   m2.d2 = (uint32_t *)malloc(sizeof(uint32_t) * (S + 1));
-  if (!st.S || !st.resident || !ttft || !next_arr || !tps || !m1.p1 || !m1.p2 || !m1.d2 ||
+  if (!st.S || !st.snap_g || !st.snap_turn || !st.snap_done || !st.resident || !ttft || !next_arr || !tps || !m1.p1 || !m1.p2 || !m1.d2 ||
       !m2.p1 || !m2.p2 || !m2.d2) {
     rc = OR_ERR_OOM;
     goto done;
@@ -611,7 +698,7 @@ int or_replay(const or_trace *tr, const or_params *p, or_result *res, or_logrec 
     free(last_arr_of);
   }
 
-  uint64_t t0 = E ? ev[0].time : 0, q_free = 0, n_ttft = 0;
+  uint64_t t0 = E ? ev[0].time : 0, q_free = 0, n_ttft = 0, n_arrivals = 0;
   unsigned __int128 ttft_sum = 0;
   uint64_t dma_busy_until = 0;
   int dma_busy = 0;
@@ -720,6 +807,20 @@ int or_replay(const or_trace *tr, const or_params *p, or_result *res, or_logrec 
         }
       }
     }
+    /* R28: a sync point copies every live row into the snapshot, after the
+     * event's own decisions */
+    if (st.stale) {
+      int sync = p->stale_sync == OR_SYNC_EVENT;
+      if (x->type == OR_ARRIVAL && p->stale_sync == OR_SYNC_ARRIVALS) sync = ++n_arrivals % p->stale_m == 0;
+      if (x->type == OR_COMPLETION && p->stale_sync == OR_SYNC_GAP_START)
+        sync = x->turn + 1 != tr->turn_off[s + 1] - tr->turn_off[s];
+      if (sync)
+        for (uint64_t v = 0; v < S; v++) {
+          st.snap_g[v] = st.S[v].g_q;
+          st.snap_turn[v] = st.S[v].turn;
+          st.snap_done[v] = st.S[v].done;
+        }
+    }
     if (p->debug) check_invariants(&st);
   }
 
@@ -736,6 +837,9 @@ int or_replay(const or_trace *tr, const or_params *p, or_result *res, or_logrec 
 done:
   free(ev);
   free(st.S);
+  free(st.snap_g);
+  free(st.snap_turn);
+  free(st.snap_done);
   free(st.resident);
   free(ttft);
   free(next_arr);

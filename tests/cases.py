@@ -16,7 +16,8 @@ MIB = 1 << 20
 
 def base(policy, cap_s, cap_h, kvb, **kw):
     p = dict(policy=policy, cap_s=cap_s, cap_h=cap_h, kvb=kvb, max_sessions=0, ema_num=3, ema_den=10,
-             bucket=1, penalty=500_000_000, ttl=10_000_000, dma=64_000, load=4, t_p=20_000_000, online=False)
+             bucket=1, penalty=500_000_000, ttl=10_000_000, dma=64_000, load=4, t_p=20_000_000, online=False,
+             stale="live", stale_m=0)
     p.update(kw)
     return p
 
@@ -25,7 +26,8 @@ def to_oracle(p: dict) -> dict:
     return dict(policy=p["policy"], cap_s_bytes=p["cap_s"], cap_h_bytes=p["cap_h"], kv_bytes_per_token=p["kvb"],
                 max_sessions=p["max_sessions"], ema_num=p["ema_num"], ema_den=p["ema_den"],
                 hazard_bucket=p["bucket"], penalty_q=p["penalty"], ttl_us=p["ttl"], dma_bytes_per_us=p["dma"],
-                ttft_load=p["load"], t_p_ps_per_tok=p["t_p"], hazard_online=bool(p.get("online")))
+                ttft_load=p["load"], t_p_ps_per_tok=p["t_p"], hazard_online=bool(p.get("online")),
+                stale_sync=p.get("stale", "live"), stale_m=p.get("stale_m", 0))
 
 
 def to_lib(p: dict, trace_idx: int = 0) -> dict:
@@ -34,7 +36,8 @@ def to_lib(p: dict, trace_idx: int = 0) -> dict:
                 kv_bytes_per_token=kvb, max_sessions=p["max_sessions"], ema_num=p["ema_num"],
                 ema_den=p["ema_den"], hazard_bucket=p["bucket"], penalty_q=p["penalty"], ttl_us=p["ttl"],
                 dma_bytes_per_us=p["dma"], ttft_load=p["load"], t_p_ps_per_tok=p["t_p"],
-                t_s_ps_per_tok=kvb // 16, t_h_ps_per_tok=kvb // 4, hazard_online=bool(p.get("online")))
+                t_s_ps_per_tok=kvb // 16, t_h_ps_per_tok=kvb // 4, hazard_online=bool(p.get("online")),
+                stale_sync=p.get("stale", "live"), stale_m=p.get("stale_m", 0))
 
 
 # ---- the five workloads --------------------------------------------------------

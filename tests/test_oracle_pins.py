@@ -637,3 +637,51 @@ def test_attainment_identities_on_replays():
         assert rc == 0
         assert int(b[:, 1].sum()) == r_on["req_warm"]
         assert list(b[:, 0]) == [j * 120 // P for j in range(P)]
+
+
+# ---- stale snapshot of a dual design (Sec. IV-B eq. stale; reading R28) -------------
+
+STALE_HAND = dict(policy="spear", kv_bytes_per_token=1, cap_s_bytes=300, cap_h_bytes=0,
+                  t_p_ps_per_tok=20_000_000, ttft_load=4)
+
+
+def test_hand_replay_stale_snapshot():
+    tr, log, counts = _hand_trace("replay_hand_stale.txt")
+    for sync, m in (("arrivals", 100), ("gap_start", 0)):  # e5 is final: no gap_start sync after e3
+        r = oracle.replay(tr, dict(STALE_HAND, stale_sync=sync, stale_m=m), log=True, debug=True)
+        assert r["status"] == 0
+        assert list(zip(*(map(int, a) for a in r["log"]))) == log, sync
+        for k, v in counts.items():
+            assert r[k] == v, (sync, k)
+    # synced after every event, the snapshot is the live state: s1 is dropped at e6, s0 hits at e8
+    live = oracle.replay(tr, STALE_HAND, log=True)
+    r = oracle.replay(tr, dict(STALE_HAND, stale_sync="event"), log=True, debug=True)
+    assert r["decision_hash"] == live["decision_hash"] and r["vict_diff"] == 0 and r["vict_n"] == 1
+    got = list(zip(*(map(int, a) for a in live["log"])))
+    assert (6, oracle.KINDS.index("EVICT"), 1) in got and (8, oracle.KINDS.index("HIT_S"), 0) in got
+
+
+@pytest.mark.parametrize("mix", ["coding", "general"])
+def test_stale_every_event_is_live(mix):
+    """A snapshot copied after every event holds, at each decision, the rows
+    of the candidates as they are live (their rows change only at their own
+    events, and a session is pinned through its arrival's decisions), so the
+    dual design decides exactly as the live one."""
+    from cases import base, to_oracle
+    tr = synth.paper_scale_trace(2, mix)
+    for pol in ("spear", "spear_tide"):
+        p = base(pol, 2 * GIB, 16 * GIB, 131072)
+        live = oracle.replay(tr, to_oracle(p))
+        st = oracle.replay(tr, to_oracle(dict(p, stale="event")))
+        assert st["status"] == 0 and st["decision_hash"] == live["decision_hash"]
+        assert st["vict_n"] > 1000 and st["vict_diff"] == 0 and st["prom_diff"] == 0
+        assert (st["prom_n"] > 0) == (pol == "spear_tide")
+        lag = oracle.replay(tr, to_oracle(dict(p, stale="arrivals", stale_m=8)))
+        assert lag["decision_hash"] != live["decision_hash"] and lag["vict_diff"] > 0
+
+
+def test_stale_snapshot_rejected_params():
+    tr, _, _ = _hand_trace("replay_hand_stale.txt")
+    for bad in (dict(policy="lru", stale_sync="event"), dict(policy="belady", stale_sync="gap_start"),
+                dict(stale_sync="arrivals", stale_m=0), dict(stale_sync="event", hazard_online=True)):
+        assert oracle.replay(tr, dict(STALE_HAND, **bad))["status"] == -1
