@@ -148,7 +148,27 @@ typedef struct {
   uint64_t t_p_ps_per_tok;     /* prefill cost; TTFT uses t_p / 1000 ns per token */
   uint32_t ttft_load;          /* arrival compression factor of the TTFT queue    */
   uint32_t flags;              /* UNISON_HAZARD_ONLINE, or 0                      */
+  uint32_t stale_sync;         /* UNISON_SYNC_*: dual-design ablation, or 0       */
+  uint32_t stale_m;            /* arrivals per sync for UNISON_SYNC_ARRIVALS      */
 } unison_replay_params;
+
+/* Stale-snapshot replays (Sec. IV-B eq. stale, Tab. org): the ranking of a
+ * dual design whose engines copy the register file only at sync points.
+ * Every ranking decision (make-room victims, slot-limit evictions, TIDE's
+ * promotions and demotions) scores each session from its register row
+ * (gap average, turn, done) as of the last sync; rows start at zero; a sync
+ * copies every row after that event's own decisions; residency, sizes and
+ * pins stay live.  Each acted-upon victim (promotion) choice is compared
+ * with the choice by the live rows over the same candidates: the result's
+ * vict_n / vict_diff (prom_n / prom_diff) count them.  UNISON_SYNC_EVENT
+ * decides exactly as the live replay.  SPEAR and SPEAR+TIDE only, not with
+ * UNISON_HAZARD_ONLINE, stale_m >= 1 for UNISON_SYNC_ARRIVALS (else
+ * UNISON_ERR_ARG); the same shared-memory and session limits as the online
+ * table apply, with 16 bytes per session (else UNISON_ERR_RANGE). */
+#define UNISON_SYNC_LIVE 0u      /* no snapshot: the live ranking          */
+#define UNISON_SYNC_EVENT 1u     /* copy after every event                 */
+#define UNISON_SYNC_ARRIVALS 2u  /* copy after every stale_m-th arrival    */
+#define UNISON_SYNC_GAP_START 3u /* copy after every non-final completion  */
 
 /* Online hazard table (Sec. V-F, eq. attainment): instead of the table fitted
  * on the whole trace, the table starts with no sessions, and the turn count
@@ -171,6 +191,8 @@ typedef struct {
   uint64_t ttft_p50_ns, ttft_n;            /* lower median over all requests       */
   uint64_t decision_hash;                  /* see UNISON_KIND_* below              */
   uint64_t log_len;                        /* decisions made (logged or not)       */
+  uint64_t vict_n, vict_diff;              /* stale snapshot: victim choices, and  */
+  uint64_t prom_n, prom_diff;              /* promotions, unlike the live choice   */
   int32_t status;
   uint32_t reserved;
 } unison_replay_result;

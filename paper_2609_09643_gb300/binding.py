@@ -17,6 +17,7 @@ from .native import LIB
 
 POLICY = {"lru": 0, "timeout": 1, "spear": 2, "spear_tide": 3, "belady": 4, "lru_tide": 5}
 FLAG_HAZARD_ONLINE = 1  # unison_replay_params.flags bit 0
+STALE_SYNC = {"live": 0, "event": 1, "arrivals": 2, "gap_start": 3}  # UNISON_SYNC_*
 KIND = ["COLD", "HIT_S", "HIT_H", "MISS", "PLACE_S", "PLACE_H", "BYPASS", "DEMOTE", "EVICT",
         "PROMOTE", "TIDE_DEMOTE", "EXPIRE"]
 OK, ERR_ARG, ERR_IO, ERR_FORMAT, ERR_RANGE, ERR_CUDA, ERR_OOM, ERR_LOG_FULL, ERR_TIMEOUT, ERR_CAPACITY = \
@@ -49,14 +50,15 @@ class ReplayParams(C.Structure):
                 ("hazard_bucket", C.c_uint32), ("ttl_us", C.c_uint32), ("penalty_q", C.c_uint64),
                 ("dma_bytes_per_us", C.c_uint64), ("t_s_ps_per_tok", C.c_uint64),
                 ("t_h_ps_per_tok", C.c_uint64), ("t_p_ps_per_tok", C.c_uint64),
-                ("ttft_load", C.c_uint32), ("flags", C.c_uint32)]
+                ("ttft_load", C.c_uint32), ("flags", C.c_uint32), ("stale_sync", C.c_uint32),
+                ("stale_m", C.c_uint32)]
 
 
 RESULT_FIELDS = ["events", "req_warm", "cold", "hit_s", "hit_h", "miss", "bypass", "place_s", "place_h",
                  "evict", "demote", "promote", "tide_demote", "expire", "tok_hit_s", "tok_hit_h",
                  "tok_miss", "tok_computed", "tok_needed", "dma_bytes", "tide_calls",
                  "promoted_then_hit_s", "ttft_sum_lo", "ttft_sum_hi", "ttft_p50_ns", "ttft_n",
-                 "decision_hash", "log_len"]
+                 "decision_hash", "log_len", "vict_n", "vict_diff", "prom_n", "prom_diff"]
 
 
 class ReplayResult(C.Structure):
@@ -211,7 +213,9 @@ def make_params(p: dict, trace_idx: int = 0) -> ReplayParams:
                         q["kv_bytes_per_token"], q["max_sessions"], q["ema_num"], q["ema_den"],
                         q["hazard_bucket"], q["ttl_us"], q["penalty_q"], q["dma_bytes_per_us"],
                         q["t_s_ps_per_tok"], q["t_h_ps_per_tok"], q["t_p_ps_per_tok"], q["ttft_load"],
-                        q.get("flags", FLAG_HAZARD_ONLINE if q.get("hazard_online") else 0))
+                        q.get("flags", FLAG_HAZARD_ONLINE if q.get("hazard_online") else 0),
+                        STALE_SYNC[q.get("stale_sync", "live")] if isinstance(q.get("stale_sync", "live"), str)
+                        else int(q["stale_sync"]), q.get("stale_m", 0))
 
 
 def result_dict(r: ReplayResult) -> dict:

@@ -73,6 +73,8 @@ struct ReplayDesc {
   uint32_t tmap;    // 1: a per-session tier byte follows the lists in shared memory
   uint32_t bucket;  // hazard bucket width (online hazard replays)
   uint64_t penalty;  // P_Z in quantised units (online hazard replays)
+  const uint64_t *t2;  // eq. (t2) per turn index of the offline table (stale-snapshot replays)
+  uint32_t stale_sync, stale_m;  // UNISON_SYNC_* and arrivals per sync
 };
 
 // --------------------------------------------------------------------------
@@ -287,6 +289,10 @@ struct ReplayState {
   uint32_t n_warm, n_cold, n_hit_s, n_hit_h, n_miss, n_bypass, n_place_s, n_place_h;
   uint32_t n_evict, n_demote, n_promote, n_tide_demote, n_expire, n_tide_calls, n_pth;
   uint64_t tok_hit_s, tok_hit_h, tok_miss, tok_computed, tok_needed, dma_bytes;
+  // stale-snapshot replays: every session's live key, and the choices made
+  // against it
+  const uint64_t *live;
+  uint32_t vict_n, vict_diff, prom_n, prom_diff;
 };
 
 #define CNT(st, field, v) ((st).field += (v))
@@ -344,9 +350,45 @@ __device__ __forceinline__ uint4 sorted_pop_back(ReplayState &st, Sorted &T) {
 
 __device__ __forceinline__ uint32_t esize(uint4 v) { return v.z & kSizeMask; }
 
+// Stale-snapshot replays (eq. stale): the arrays are ordered by snapshot
+// keys; a choice made on them is compared with the most (least) evictable
+// candidate by live keys.  Live keys are packed with the session id, so the
+// extreme key names one session.
+__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = max(v, (uint64_t)__shfl_xor_sync(kFull, (unsigned long long)v, o));
+  return v;
+}
+__device__ __forceinline__ uint64_t warp_min_u64(uint64_t v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = min(v, (uint64_t)__shfl_xor_sync(kFull, (unsigned long long)v, o));
+  return v;
+}
+__device__ __forceinline__ uint64_t live_max(const ReplayState &st, const Sorted &T, uint32_t lo, uint32_t hi,
+                                             int lane) {
+  uint64_t m = 0;
+  for (uint32_t i = lo + lane; i < hi; i += 32) m = max(m, st.live[packed_id(ekey(T.e[i]))]);
+  return warp_max_u64(m);
+}
+__device__ __forceinline__ uint64_t live_min(const ReplayState &st, const Sorted &T, uint32_t lo, uint32_t hi,
+                                             int lane) {
+  uint64_t m = ~0ull;
+  for (uint32_t i = lo + lane; i < hi; i += 32) m = min(m, st.live[packed_id(ekey(T.e[i]))]);
+  return warp_min_u64(m);
+}
+__device__ __forceinline__ void count_victim(ReplayState &st, uint32_t chosen, uint64_t live_best) {
+  st.vict_n++;
+  st.vict_diff += packed_id(live_best) != chosen;
+}
+__device__ __forceinline__ void count_promotion(ReplayState &st, uint32_t chosen, uint64_t live_best) {
+  st.prom_n++;
+  st.prom_diff += packed_id(live_best) != chosen;
+}
+
 // A session demoted out of the fast tier enters HBM, displacing the most
 // evictable unpinned HBM sessions, or is dropped when it is itself the most
 // evictable of (unpinned HBM) + {itself}.
+template <bool kStale>
 __device__ __forceinline__ bool admit_demoted(ReplayState &st, const Hot &D, uint4 d, int lane) {
   const uint32_t id = packed_id(ekey(d));
   const uint32_t size = esize(d);
@@ -356,6 +398,11 @@ __device__ __forceinline__ bool admit_demoted(ReplayState &st, const Hot &D, uin
     return true;
   }
   while (st.used_h + size > D.cap_h) {
+    if (kStale) {
+      const bool drop = st.H.n == 0 || ekey(d) > ekey(st.H.e[st.H.n - 1]);
+      count_victim(st, drop ? id : packed_id(ekey(st.H.e[st.H.n - 1])),
+                   max(live_max(st, st.H, 0, st.H.n, lane), st.live[id]));
+    }
     if (st.H.n == 0 || ekey(d) > ekey(st.H.e[st.H.n - 1])) {
       log_dec(st, UNISON_KIND_EVICT, id, lane);
       CNT(st, n_evict, 1);
@@ -386,6 +433,7 @@ __device__ __forceinline__ bool pin_append(ReplayState &st, uint64_t pk, uint32_
 }
 
 // Placement of the arriving (pinned) session s with n tokens.
+template <bool kStale>
 __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s, uint64_t pk, uint32_t n,
                                       int lane) {
   if (D.max_sessions && st.npin >= D.max_sessions) {
@@ -399,9 +447,10 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
         st.status = UNISON_ERR_CAPACITY;
         return false;
       }
+      if (kStale) count_victim(st, packed_id(ekey(st.S.e[st.S.n - 1])), live_max(st, st.S, 0, st.S.n, lane));
       const uint4 d = sorted_pop_back(st, st.S);  // most evictable unpinned fast-tier session
       st.used_s -= esize(d);
-      if (!admit_demoted(st, D, d, lane)) return false;
+      if (!admit_demoted<kStale>(st, D, d, lane)) return false;
     }
     if (!pin_append(st, pk, n, s, kTierS, lane)) return false;
     st.used_s += n;
@@ -414,6 +463,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
         st.status = UNISON_ERR_CAPACITY;
         return false;
       }
+      if (kStale) count_victim(st, packed_id(ekey(st.H.e[st.H.n - 1])), live_max(st, st.H, 0, st.H.n, lane));
       const uint4 v = sorted_pop_back(st, st.H);
       st.used_h -= esize(v);
       log_dec(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
@@ -437,6 +487,9 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
       }
       const bool from_s =
           st.H.n == 0 || (st.S.n > 0 && ekey(st.S.e[st.S.n - 1]) > ekey(st.H.e[st.H.n - 1]));
+      if (kStale)
+        count_victim(st, packed_id(ekey(from_s ? st.S.e[st.S.n - 1] : st.H.e[st.H.n - 1])),
+                     max(live_max(st, st.S, 0, st.S.n, lane), live_max(st, st.H, 0, st.H.n, lane)));
       const uint4 v = sorted_pop_back(st, from_s ? st.S : st.H);
       if (from_s)
         st.used_s -= esize(v);
@@ -454,6 +507,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
 // free fast-tier space; phase 2: pair the next least evictable HBM session
 // with the most evictable fast-tier one), which makes the same moves as the
 // pair loop of Algorithm 1, and are then applied in bulk.
+template <bool kStale>
 __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t budget, uint32_t rcap_s,
                                          int lane) {
   uint64_t rem = budget;
@@ -463,6 +517,8 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     const uint4 p = st.H.e[n1];
     const uint64_t sz = esize(p), by = sz * kvb;
     if (by > rem || st.used_s + sz > D.cap_s) break;
+    // (the loop form's candidates: HBM less the sessions promoted so far)
+    if (kStale) count_promotion(st, packed_id(ekey(p)), live_min(st, st.H, n1, st.H.n, lane));
     rem -= by;
     st.used_s += sz;
     st.used_h -= sz;
@@ -482,6 +538,15 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     if (by > rem) break;
     if (st.used_s - sd + sp > D.cap_s) break;
     if (st.used_h - sp + sd > D.cap_h) break;
+    if (kStale) {
+      // at this step HBM holds its entries from n1 + pairs on plus the pairs
+      // demoted so far (the top `pairs` fast-tier entries); the fast tier
+      // its first S.n - pairs entries plus the n1 + pairs promoted so far
+      count_promotion(st, packed_id(ekey(p)),
+                      min(live_min(st, st.H, n1 + pairs, st.H.n, lane), live_min(st, st.S, st.S.n - pairs, st.S.n, lane)));
+      count_victim(st, packed_id(ekey(d)),
+                   max(live_max(st, st.S, 0, st.S.n - pairs, lane), live_max(st, st.H, 0, n1 + pairs, lane)));
+    }
     rem -= by;
     st.used_s = st.used_s - sd + sp;
     st.used_h = st.used_h - sp + sd;
@@ -635,43 +700,26 @@ __device__ bool online_add(OnlineTable &ot, uint32_t turns, uint32_t bucket, uin
   return __any_sync(kFull, changed);  // T2 is a function of sigma
 }
 
-// Every resident's key under the rebuilt table, then the tier re-sorted:
-// bitonic network (descending, padded to a power of two with key 0, which no
-// packed key equals since session ids stay below 2^24 - 1), then reversed.
-// The tier's array holds a power of two >= its capacity.
-__device__ void online_rerank(Sorted &T, const OnlineTable &ot, const uint32_t *gs, const uint16_t *ks, int lane) {
-  if (T.n < 2) {
-    if (T.n == 1 && lane == 0) {
-      uint4 v = T.e[0];
-      const uint64_t k = ekey(v);
-      if ((k >> 24) != kKeyMax40) {
-        const uint32_t id = packed_id(k);
-        const uint64_t nk = online_key(ot, gs[id], (uint32_t)ks[id] - 1, id);
-        v.x = (uint32_t)nk;
-        v.y = (uint32_t)(nk >> 32);
-        T.e[0] = v;
-      }
-    }
-    __syncwarp();
-    return;
-  }
-  const uint32_t ring = ring_size(T.n);
+// Every resident takes a new key (new_key maps an entry's key to it), then the
+// tier is re-sorted if that broke its order: bitonic network (descending,
+// padded to a power of two with key 0, which no packed key equals since
+// session ids stay below 2^24 - 1), then reversed.  The tier's array holds a
+// power of two >= its capacity.
+template <class KeyFn>
+__device__ void rerank(Sorted &T, KeyFn new_key, int lane) {
   for (uint32_t i = lane; i < T.n; i += 32) {
     uint4 v = T.e[i];
-    const uint64_t k = ekey(v);
-    if ((k >> 24) != kKeyMax40) {  // completed sessions keep the maximal key
-      const uint32_t id = packed_id(k);
-      const uint64_t nk = online_key(ot, gs[id], (uint32_t)ks[id] - 1, id);
-      v.x = (uint32_t)nk;
-      v.y = (uint32_t)(nk >> 32);
-      T.e[i] = v;
-    }
+    const uint64_t nk = new_key(ekey(v));
+    v.x = (uint32_t)nk;
+    v.y = (uint32_t)(nk >> 32);
+    T.e[i] = v;
   }
   __syncwarp();
-  // a small change of the table often keeps the order: then nothing moves
+  // a small change of the keys often keeps the order: then nothing moves
   bool out_of_order = false;
   for (uint32_t i = lane + 1; i < T.n; i += 32) out_of_order |= ekey(T.e[i - 1]) > ekey(T.e[i]);
   if (!__any_sync(kFull, out_of_order)) return;
+  const uint32_t ring = ring_size(T.n);
   for (uint32_t i = T.n + lane; i < ring; i += 32) T.e[i] = make_uint4(0u, 0u, 0u, 0u);
   __syncwarp();
   for (uint32_t k = 2; k <= ring; k <<= 1) {
@@ -697,8 +745,23 @@ __device__ void online_rerank(Sorted &T, const OnlineTable &ot, const uint32_t *
   __syncwarp();
 }
 
-template <bool kGlobalLists, bool kOnline>
+// Keys of every resident under a rebuilt online table; completed sessions
+// keep the maximal key.
+__device__ void online_rerank(Sorted &T, const OnlineTable &ot, const uint32_t *gs, const uint16_t *ks, int lane) {
+  rerank(T, [&](uint64_t k) {
+    if ((k >> 24) == kKeyMax40) return k;
+    const uint32_t id = packed_id(k);
+    return online_key(ot, gs[id], (uint32_t)ks[id] - 1, id);
+  }, lane);
+}
+
+constexpr int kKeyStream = 0;  // keys from the per-session key stream
+constexpr int kKeyOnline = 1;  // keys under the online hazard table
+constexpr int kKeyStale = 2;   // snapshot keys of a dual design
+
+template <bool kGlobalLists, int kKeys>
 __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, const uint32_t *order) {
+  constexpr bool kOnline = kKeys == kKeyOnline, kStale = kKeys == kKeyStale;
   extern __shared__ __align__(16) unsigned char smem[];
   const int lane = threadIdx.x & 31;
   __shared__ ReplayDesc Dsh;
@@ -711,13 +774,14 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
   uint32_t *online_gs = nullptr;
   uint16_t *online_ks = nullptr;
   OnlineTable *online_tab = nullptr;
+  uint64_t *stale_live = nullptr, *stale_snap = nullptr;
   {
     uint4 *p = reinterpret_cast<uint4 *>(kGlobalLists ? reinterpret_cast<unsigned char *>(D.glist) : smem);
-    // online replays keep power-of-two tiers (for the re-sort)
+    // online and stale-snapshot replays keep power-of-two tiers (for re-sorts)
     st.S.e = p;
-    p += kOnline ? ring_size(D.rcap_s) : D.rcap_s;
+    p += (kOnline || kStale) ? ring_size(D.rcap_s) : D.rcap_s;
     st.H.e = p;
-    p += kOnline ? ring_size(D.rcap_h) : D.rcap_h;
+    p += (kOnline || kStale) ? ring_size(D.rcap_h) : D.rcap_h;
     st.pin = p;
     p += D.rcap_s + D.rcap_h;
     st.tmp = p;
@@ -749,6 +813,18 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
       }
       __syncwarp();
     }
+    if (kStale) {
+      // after the tier map: each session's live key and snapshot key; a zero
+      // register row (gap average 0, turn 0, not done) scores T2 of turn 0
+      unsigned char *q = reinterpret_cast<unsigned char *>(p) + ((D.n_sessions + 15) & ~15u);
+      stale_live = reinterpret_cast<uint64_t *>(q);
+      stale_snap = stale_live + ((D.n_sessions + 1) & ~1u);
+      const uint64_t k0 = D.t2[0];
+      for (uint32_t i = lane; i < D.n_sessions; i += 32) stale_live[i] = stale_snap[i] = pack_key(k0, i);
+      __syncwarp();
+    }
+    st.live = stale_live;
+    st.vict_n = st.vict_diff = st.prom_n = st.prom_diff = 0;
     st.S.n = st.H.n = 0;
     st.S.cap = D.rcap_s;
     st.H.cap = D.rcap_h;
@@ -777,6 +853,7 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
   const uint32_t load = D.load;
   const uint64_t ns_per_us = (1000u % load == 0) ? 1000u / load : 0u;  // 0: divide exactly
   unsigned long long s_lo = 0, s_hi = 0;
+  uint32_t stale_arrivals = 0;
   bool dma_busy = false;
   uint32_t busy_until = 0;
 
@@ -843,6 +920,8 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
           uint64_t pkb;
           if (kOnline)
             pkb = online_key(*online_tab, online_gs[s], (uint32_t)online_ks[s] - 1, s);
+          else if (kStale)
+            pkb = stale_snap[s];  // residents carry their snapshot keys
           else if (spear_keys)
             pkb = spkb[bi][j];
           else if (belady)
@@ -927,6 +1006,9 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
             online_ks[s] = (uint16_t)(k < 0xFFFFu ? k + 1 : k);
           }
           __syncwarp();
+        } else if (kStale) {
+          pk = stale_snap[s];
+          stale_live[s] = spk[bi][j];  // every lane stores the same key
         } else if (spear_keys)
           pk = spk[bi][j];
         else if (belady) {
@@ -934,9 +1016,10 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
           pk = pack_key(nr == kNoRef ? kKeyMax40 : (uint64_t)nr, s);
         } else
           pk = pack_key(0xFFFFFFFFull - e, s);
-        if (!place(st, hot, s, pk, out, lane)) break;
+        if (!place<kStale>(st, hot, s, pk, out, lane)) break;
       } else {
         // completion: unpin (if resident) and rank the session with its new key
+        if (kStale) stale_live[s] = spk[bi][j];
         int mine = -1;
         for (uint32_t i = lane; i < st.npin; i += 32)
           if ((st.pin[i].w & kIdMask) == s) mine = (int)i;
@@ -954,6 +1037,8 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
           if (kOnline)
             pk = edge ? pack_key(kKeyMax40, s)
                       : online_key(*online_tab, online_gs[s], (uint32_t)online_ks[s] - 1, s);
+          else if (kStale)
+            pk = stale_snap[s];
           else if (spear_keys)
             pk = spk[bi][j];
           else if (!belady)
@@ -979,13 +1064,27 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
           const uint64_t g = sgq[bi][j];
           const uint64_t budget = g * D.dma;
           CNT(st, n_tide_calls, 1);
-          const uint64_t moved = tide(st, hot, budget, D.rcap_s, lane);
+          const uint64_t moved = tide<kStale>(st, hot, budget, D.rcap_s, lane);
           CNT(st, dma_bytes, moved);
           if (moved > 0 && D.dma > 0) {
             dma_busy = true;
             busy_until = now + (uint32_t)((moved + D.dma - 1) / D.dma);
           }
           if (st.status == UNISON_ERR_CAPACITY) break;
+        }
+      }
+      if (kStale) {
+        // a sync point copies every live row into the snapshot, after the
+        // event's own decisions; residents then carry their live keys
+        bool sync = D.stale_sync == UNISON_SYNC_EVENT;
+        if (arrival && D.stale_sync == UNISON_SYNC_ARRIVALS) sync = ++stale_arrivals % D.stale_m == 0;
+        if (!arrival && D.stale_sync == UNISON_SYNC_GAP_START) sync = !edge;
+        if (sync) {
+          for (uint32_t i = lane; i < D.n_sessions; i += 32) stale_snap[i] = stale_live[i];
+          __syncwarp();
+          const auto snap_key = [&](uint64_t k) { return stale_snap[packed_id(k)]; };
+          rerank(st.S, snap_key, lane);
+          rerank(st.H, snap_key, lane);
         }
       }
     }
@@ -1020,6 +1119,10 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
     r.ttft_n = n_arr;
     r.decision_hash = st.hash;
     r.log_len = st.log_len;
+    r.vict_n = st.vict_n;
+    r.vict_diff = st.vict_diff;
+    r.prom_n = st.prom_n;
+    r.prom_diff = st.prom_diff;
     r.status = st.status;
     *D.result = r;
   }
@@ -1101,6 +1204,11 @@ int check_params(const unison_replay_params &p, int n_traces) {
   if (p.flags & ~UNISON_HAZARD_ONLINE) return UNISON_ERR_ARG;
   if ((p.flags & UNISON_HAZARD_ONLINE) && p.policy != UNISON_SPEAR && p.policy != UNISON_SPEAR_TIDE)
     return UNISON_ERR_ARG;
+  if (p.stale_sync > UNISON_SYNC_GAP_START || (p.stale_sync == UNISON_SYNC_ARRIVALS && p.stale_m == 0))
+    return UNISON_ERR_ARG;
+  if (p.stale_sync != UNISON_SYNC_LIVE &&
+      ((p.flags & UNISON_HAZARD_ONLINE) || (p.policy != UNISON_SPEAR && p.policy != UNISON_SPEAR_TIDE)))
+    return UNISON_ERR_ARG;
   return UNISON_OK;
 }
 
@@ -1123,8 +1231,8 @@ struct ReplayPlan {
   std::vector<int> replay_combo;
   size_t off_desc = 0, off_order = 0, off_combo = 0, bytes = 0;
   std::vector<size_t> off_lut, off_stream, off_ttft, off_glist;
-  std::vector<uint32_t> rcap_s, rcap_h, in_smem, in_global, in_online, tmap;
-  size_t max_smem = 0, max_smem_online = 0;
+  std::vector<uint32_t> rcap_s, rcap_h, in_smem, in_global, in_online, in_stale, tmap;
+  size_t max_smem = 0, max_smem_online = 0, max_smem_stale = 0;
 };
 
 // Resident-list capacity of a tier: at most one entry per session and no more
@@ -1143,6 +1251,13 @@ size_t list_bytes(uint32_t cs, uint32_t ch) { return 16ull * (4ull * cs + 2ull *
 
 // An online hazard replay: both tiers rounded up to powers of two, the tier
 // map, the per-session gap average (4 B) and arrival count (2 B), the table.
+// A stale-snapshot replay: power-of-two tiers, the tier map, then the live
+// and snapshot key of every session.
+size_t stale_bytes(uint32_t cs, uint32_t ch, uint32_t n_sessions) {
+  const size_t n = n_sessions;
+  return 16ull * (ring_size(cs) + ring_size(ch) + 3ull * cs + ch) + align_up(n, 16) + 16 * align_up(n, 2);
+}
+
 size_t online_bytes(uint32_t cs, uint32_t ch, uint32_t n_sessions) {
   const size_t n = n_sessions;
   return 16ull * (ring_size(cs) + ring_size(ch) + 3ull * cs + ch) + align_up(n, 16) + 4 * align_up(n, 4) +
@@ -1201,6 +1316,13 @@ int plan_replays(const unison_trace *const *traces, const unison_replay_params *
       P.tmap[r] = 1;
       P.in_online.push_back((uint32_t)r);
       P.max_smem_online = std::max(P.max_smem_online, ob);
+    } else if (p.stale_sync != UNISON_SYNC_LIVE) {
+      // stale-snapshot replays too
+      const size_t sb = stale_bytes(P.rcap_s[r], P.rcap_h[r], tr->n_sessions);
+      if (tr->n_sessions > kTierMapMax || sb > smem_limit) return UNISON_ERR_RANGE;
+      P.tmap[r] = 1;
+      P.in_stale.push_back((uint32_t)r);
+      P.max_smem_stale = std::max(P.max_smem_stale, sb);
     } else if (lists <= smem_limit) {
       P.in_smem.push_back((uint32_t)r);
       P.max_smem = std::max<size_t>(P.max_smem, lists + (P.tmap[r] ? map : 0));
@@ -1282,11 +1404,15 @@ void fill_descs(const unison_trace *const *traces, const unison_replay_params *p
     d.tmap = P.tmap[r];
     d.bucket = p.hazard_bucket;
     d.penalty = p.penalty_q;
+    d.t2 = P.replay_combo[r] >= 0 ? hc[P.replay_combo[r]].t2 : nullptr;
+    d.stale_sync = p.stale_sync;
+    d.stale_m = p.stale_m;
   }
   order.clear();
   order.insert(order.end(), P.in_smem.begin(), P.in_smem.end());
   order.insert(order.end(), P.in_global.begin(), P.in_global.end());
   order.insert(order.end(), P.in_online.begin(), P.in_online.end());
+  order.insert(order.end(), P.in_stale.begin(), P.in_stale.end());
 }
 
 // Queue the kernels of a planned batch on `stream`.
@@ -1318,23 +1444,31 @@ int launch_replays(const ReplayPlan &P, char *scratch, const std::vector<ComboDe
   {
     ProfSpan span(profile ? "replay" : "", stream);
     if (!P.in_smem.empty()) {
-      ck(cudaFuncSetAttribute(replay_kernel<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyStream>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)P.max_smem));
-      replay_kernel<false, false><<<(unsigned)P.in_smem.size(), 32, P.max_smem, stream>>>(d_desc, d_order);
+      replay_kernel<false, kKeyStream><<<(unsigned)P.in_smem.size(), 32, P.max_smem, stream>>>(d_desc, d_order);
       count_launches(1);
       ck(cudaGetLastError());
     }
     if (!P.in_global.empty()) {
-      replay_kernel<true, false><<<(unsigned)P.in_global.size(), 32, 0, stream>>>(d_desc,
-                                                                                 d_order + P.in_smem.size());
+      replay_kernel<true, kKeyStream><<<(unsigned)P.in_global.size(), 32, 0, stream>>>(d_desc,
+                                                                                      d_order + P.in_smem.size());
       count_launches(1);
       ck(cudaGetLastError());
     }
     if (!P.in_online.empty()) {
-      ck(cudaFuncSetAttribute(replay_kernel<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyOnline>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)P.max_smem_online));
-      replay_kernel<false, true><<<(unsigned)P.in_online.size(), 32, P.max_smem_online, stream>>>(
+      replay_kernel<false, kKeyOnline><<<(unsigned)P.in_online.size(), 32, P.max_smem_online, stream>>>(
           d_desc, d_order + P.in_smem.size() + P.in_global.size());
+      count_launches(1);
+      ck(cudaGetLastError());
+    }
+    if (!P.in_stale.empty()) {
+      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyStale>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)P.max_smem_stale));
+      replay_kernel<false, kKeyStale><<<(unsigned)P.in_stale.size(), 32, P.max_smem_stale, stream>>>(
+          d_desc, d_order + P.in_smem.size() + P.in_global.size() + P.in_online.size());
       count_launches(1);
       ck(cudaGetLastError());
     }

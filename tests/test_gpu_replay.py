@@ -15,7 +15,7 @@ pytestmark = pytest.mark.gpu
 FIELDS = ["events", "req_warm", "cold", "hit_s", "hit_h", "miss", "bypass", "place_s", "place_h", "evict",
           "demote", "promote", "tide_demote", "expire", "tok_hit_s", "tok_hit_h", "tok_miss", "tok_computed",
           "tok_needed", "dma_bytes", "tide_calls", "promoted_then_hit_s", "ttft_sum", "ttft_p50_ns", "ttft_n",
-          "decision_hash", "log_len", "status"]
+          "decision_hash", "log_len", "vict_n", "vict_diff", "prom_n", "prom_diff", "status"]
 
 
 @pytest.fixture(scope="module")
@@ -324,3 +324,65 @@ def test_online_attainment_from_device_logs(B):
         arr = np.array([[g["sessions_seen"], g["warm"], g["hr_online"], g["hr_offline"], g["hr_lru"],
                          g["attainment"]] for g in got])
         np.testing.assert_array_equal(arr, oracle.attainment(tr, ologs, P)[1])
+
+
+# ---- stale snapshot of a dual design (Sec. IV-B eq. stale) ---------------------
+
+STALE_MODES = (("event", 0), ("arrivals", 3), ("arrivals", 8), ("gap_start", 0))
+
+
+def test_stale_snapshot_tiny_full_logs(B):
+    tr, _ = tiny_case()
+    reps = [(0, base(pol, 512 * MIB, 8 * GIB, 28672, stale=sy, stale_m=m)) for pol in ONLINE_POLS
+            for sy, m in STALE_MODES]
+    cap = 8 * tr.n_events
+    res, log, _ = run_gpu(B, [tr], reps, log_capacity=cap)
+    for i, (_, p) in enumerate(reps):
+        o = oracle.replay(tr, to_oracle(p), log=True, log_capacity=cap)
+        assert_same(res[i], o, (p["policy"], p["stale"], p["stale_m"]))
+        assert_same_log(B, log[i], res[i], o, (p["policy"], p["stale"], p["stale_m"]))
+
+
+def test_stale_snapshot_hand_trace_on_device(B):
+    from test_oracle_pins import _hand_trace
+    tr, lg, counts = _hand_trace("replay_hand_stale.txt")
+    p = base("spear", 300, 0, 1, t_p=20_000_000, stale="arrivals", stale_m=100)
+    res, log, _ = run_gpu(B, [tr], [(0, p)], log_capacity=64)
+    r = res[0]
+    assert list(zip(*(map(int, a) for a in B.decode_log(log[0], r["log_len"])))) == lg
+    for k, v in counts.items():
+        assert r[k] == v, k
+
+
+def test_stale_snapshot_paper_scale(B):
+    """Both gap mixes x 2 KV sizes x SPEAR / SPEAR+TIDE x the sync modes, in
+    one call with the live replays; every-event sync decides as the live
+    replay."""
+    trs = [synth.paper_scale_trace(1, "coding"), synth.paper_scale_trace(1, "general")]
+    reps = []
+    for ti in range(2):
+        for kvb in (131072, 163840):
+            for pol in ONLINE_POLS:
+                reps.append((ti, base(pol, 4 * GIB, 64 * GIB, kvb)))
+                reps += [(ti, base(pol, 4 * GIB, 64 * GIB, kvb, stale=sy, stale_m=m)) for sy, m in STALE_MODES]
+    cap = 4 * trs[0].n_events
+    res, log, _ = run_gpu(B, trs, reps, log_capacity=cap)
+    for i, (ti, p) in enumerate(reps):
+        o = oracle.replay(trs[ti], to_oracle(p), log=(i % 5 == 2), log_capacity=cap)
+        assert_same(res[i], o, (i, p["policy"], p["kvb"], p["stale"], p["stale_m"]))
+        if i % 5 == 2:
+            assert_same_log(B, log[i], res[i], o, (i, p["policy"], p["stale"]))
+        if p["stale"] == "event":
+            assert res[i]["decision_hash"] == res[i - 1]["decision_hash"] and res[i]["vict_diff"] == 0
+
+
+def test_stale_snapshot_rejected(B):
+    tr, _ = tiny_case()
+    h = [B.Trace(tr).upload()]
+    for pol, sy, m, online in (("lru", 1, 0, False), ("belady", 3, 0, False), ("spear", 2, 0, False),
+                               ("spear", 4, 0, False), ("spear_tide", 1, 0, True)):
+        q = to_lib(base(pol, 1 * GIB, 8 * GIB, 28672, online=online))
+        q.update(stale_sync=sy, stale_m=m)
+        with pytest.raises(B.UnisonError) as ei:
+            B.replay_batch(h, [q])
+        assert ei.value.code == B.ERR_ARG, (pol, sy, m, online)
