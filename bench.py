@@ -64,6 +64,8 @@ def parse():
     ap.add_argument("--rank-sets", type=int, default=7, help="live sets per call (<= 7)")
     ap.add_argument("--no-rank-sizes", action="store_true", help="skip the live-set size sweep")
     ap.add_argument("--no-online", action="store_true", help="skip the online hazard-table report")
+    ap.add_argument("--no-stale", action="store_true", help="skip the stale-snapshot (dual design) report")
+    ap.add_argument("--no-ablation", action="store_true", help="skip the component/signal/capacity ablations")
     return ap.parse_args()
 
 
@@ -313,6 +315,124 @@ def online_hazard_report(B, stream, steps: int = 3, points: int = 8):
             "windows": points, "curves": curves}
 
 
+def stale_snapshot_report(B, stream, steps: int = 3):
+    """Sec. IV-B eq. (stale), Tab. org: SPEAR+TIDE on the paper-scale traces
+    (coding and general gap mixes x 131,072 and 163,840 B/token, fast 4 GiB /
+    HBM 64 GiB) ranked from a register-file copy synced after every event,
+    every 8 arrivals, or at every gap_start, against the live ranking: the
+    shares of victim and promotion choices that differ, and the shifts of hit
+    rate, fast-tier hit share, prefill reduction (points) and AMAT (percent)."""
+    import torch
+    import synth
+    from cases import GIB, base, to_lib
+    mixes = ("coding", "general")
+    trs = [synth.paper_scale_trace(1, m) for m in mixes]
+    handles = [B.Trace(t).upload(stream) for t in trs]
+    modes = (("event", 0), ("arrivals", 8), ("gap_start", 0))
+    settings = [(ti, kvb) for ti in range(2) for kvb in (131072, 163840)]
+    live = [to_lib(base("spear_tide", 4 * GIB, 64 * GIB, kvb), ti) for ti, kvb in settings]
+    stale = [to_lib(base("spear_tide", 4 * GIB, 64 * GIB, kvb, stale=sy, stale_m=m), ti)
+             for ti, kvb in settings for sy, m in modes]
+    events = sum(2 * trs[ti].n_turns for ti, _ in settings) * len(modes)
+    out = torch.zeros(B.result_nbytes(len(stale)), dtype=torch.uint8, device="cuda")
+    for _ in range(2):
+        B.replay_batch_async(handles, stale, out, stream=stream)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(steps):
+        B.replay_batch_async(handles, stale, out, stream=stream)
+    b.record(stream)
+    torch.cuda.synchronize()
+    call_ms = a.elapsed_time(b) / steps
+    rs = B.results_from_tensor(out)
+    rl, _ = B.replay_batch(handles, live, stream=stream)
+    assert all(r["status"] == 0 for r in rs + rl), "stale-snapshot replay status"
+    rows = []
+    for i, (ti, kvb) in enumerate(settings):
+        sl = B.stats(rl[i], live[i])
+        hs = lambda r: r["hit_s"] / r["req_warm"] if r["req_warm"] else 0.0
+        for j, (sy, m) in enumerate(modes):
+            r, q = rs[i * len(modes) + j], stale[i * len(modes) + j]
+            st = B.stats(r, q)
+            rows.append({"trace": mixes[ti], "kv_bytes_per_token": kvb, "sync": sy if not m else f"every {m} arrivals",
+                         "vict_diff_pct": 100.0 * r["vict_diff"] / r["vict_n"] if r["vict_n"] else None,
+                         "prom_diff_pct": 100.0 * r["prom_diff"] / r["prom_n"] if r["prom_n"] else None,
+                         "d_hr_pp": 100.0 * (st["hit_rate"] - sl["hit_rate"]),
+                         "d_fast_pp": 100.0 * (hs(r) - hs(rl[i])),
+                         "d_prered_pp": 100.0 * (st["prered"] - sl["prered"]),
+                         "d_amat_pct": 100.0 * (st["amat_ps"] / sl["amat_ps"] - 1.0) if sl["amat_ps"] else None,
+                         "same_decisions_as_live": r["decision_hash"] == rl[i]["decision_hash"]})
+    return {"policy": "spear_tide", "replays": len(stale), "events_per_call": events, "call_ms": call_ms,
+            "events_per_s": events / (call_ms / 1e3), "rows": rows}
+
+
+def ablation_report(B, stream):
+    """Sec. V-C..V-E on the paper-scale traces (coding and general mixes,
+    131,072 B/token), one batched call for all of it:
+    - components (Fig. ablation): LRU, LRU+TIDE, SPEAR, SPEAR+TIDE at fast
+      4 GiB / HBM 64 GiB: hit rate, AMAT over LRU's, prefill reduction,
+      prefetch accuracy;
+    - signals (Fig. signal): SPEAR+TIDE without the gap signal or without the
+      hazard signal, shifts of hit rate (points) and AMAT (percent);
+    - capacity axes (Tab. robust): SPEAR+TIDE against LRU with HBM swept at
+      fast 32K tokens, the fast tier swept at HBM 512K tokens, and the fast
+      share of a 256K-token total swept: mean gains over the two traces."""
+    import synth
+    from cases import base, to_lib
+    kvb, tok = 131072, lambda n: n * 131072
+    mixes = ("coding", "general")
+    trs = [synth.paper_scale_trace(1, m) for m in mixes]
+    handles = [B.Trace(t).upload(stream) for t in trs]
+    jobs = []  # (section, label, trace index, params)
+    for ti in range(2):
+        for pol in ("lru", "lru_tide", "spear", "spear_tide"):
+            jobs.append(("component", pol, ti, base(pol, tok(32768), tok(524288), kvb)))
+        for lab, ng, nh in (("full", False, False), ("no gap signal", True, False), ("no hazard signal", False, True)):
+            jobs.append(("signal", lab, ti, base("spear_tide", tok(32768), tok(524288), kvb, no_gap=ng, no_hazard=nh)))
+    axes = [("hbm", f"hbm {h // 1024}K, fast 32K", 32768, h) for h in (131072, 262144, 524288, 1048576)]
+    axes += [("fast", f"fast {f // 1024}K, hbm 512K", f, 524288) for f in (8192, 16384, 32768, 65536)]
+    axes += [("partition", f"fast share {sh}%", 262144 * sh // 100, 262144 - 262144 * sh // 100)
+             for sh in (10, 25, 50, 75)]
+    for ax, lab, fs, hb in axes:
+        for ti in range(2):
+            for pol in ("lru", "spear_tide"):
+                jobs.append(("capacity", (ax, lab, pol), ti, base(pol, tok(fs), tok(hb), kvb)))
+    params = [to_lib(p, ti) for _, _, ti, p in jobs]
+    res, _ = B.replay_batch(handles, params, stream=stream)
+    assert all(r["status"] == 0 for r in res), "ablation replay status"
+    st = [B.stats(r, q) for r, q in zip(res, params)]
+    by = {(j[0], j[1], j[2]): i for i, j in enumerate(jobs)}
+    comp = []
+    for ti in range(2):
+        lru_amat = st[by[("component", "lru", ti)]]["amat_ps"]
+        for pol in ("lru", "lru_tide", "spear", "spear_tide"):
+            x = st[by[("component", pol, ti)]]
+            comp.append({"trace": mixes[ti], "policy": pol, "hit_rate": x["hit_rate"],
+                         "amat_over_lru": x["amat_ps"] / lru_amat if lru_amat else None, "prered": x["prered"],
+                         "prefetch_acc": x["prefetch_acc"] if pol.endswith("tide") else None})
+    sig = []
+    for ti in range(2):
+        f = st[by[("signal", "full", ti)]]
+        for lab in ("no gap signal", "no hazard signal"):
+            x = st[by[("signal", lab, ti)]]
+            sig.append({"trace": mixes[ti], "variant": lab, "d_hr_pp": 100 * (x["hit_rate"] - f["hit_rate"]),
+                        "d_amat_pct": 100 * (x["amat_ps"] / f["amat_ps"] - 1) if f["amat_ps"] else None})
+    cap = []
+    for ax, lab, fs, hb in axes:
+        g_hr, g_amat, g_pre = [], [], []
+        for ti in range(2):
+            l, u = st[by[("capacity", (ax, lab, "lru"), ti)]], st[by[("capacity", (ax, lab, "spear_tide"), ti)]]
+            g_hr.append(100 * (u["hit_rate"] - l["hit_rate"]))
+            g_amat.append(100 * (1 - u["amat_ps"] / l["amat_ps"]) if l["amat_ps"] else 0.0)
+            g_pre.append(100 * (u["prered"] - l["prered"]))
+        cap.append({"axis": ax, "point": lab, "fast_tokens": fs, "hbm_tokens": hb,
+                    "mean_hr_gain_pp": sum(g_hr) / 2, "mean_amat_gain_pct": sum(g_amat) / 2,
+                    "mean_prered_gain_pp": sum(g_pre) / 2})
+    return {"kv_bytes_per_token": kvb, "replays": len(jobs), "components": comp, "signals": sig,
+            "capacity_axes": cap, "elapsed_idle_signal": "not built: the hardware scoring contract drops it"}
+
+
 def cpu_baseline_replay(trs, reps, budget_s: float = 12.0):
     """The oracle as it stands, single-threaded, on a bounded sample of the
     sweep's replays (spread over the batch) until budget_s of CPU work."""
@@ -499,6 +619,12 @@ def main():
     online = None
     if not (args.no_online or args.rank_only or args.replay_only) and rank == 0:
         online = online_hazard_report(B, stream)
+    stale = None
+    if not (args.no_stale or args.rank_only or args.replay_only) and rank == 0:
+        stale = stale_snapshot_report(B, stream)
+    ablation = None
+    if not (args.no_ablation or args.rank_only or args.replay_only) and rank == 0:
+        ablation = ablation_report(B, stream)
 
     # end to end through the public API: host trace staging -> device, replay,
     # results back to the host, every step
@@ -570,7 +696,7 @@ def main():
                                    "paper-scale coding trace, 131072 B/token, SPEAR+TIDE)",
                        "replays": n_rep, "events_per_step": events_per_step,
                        "l2": "flushed before every step (256 MiB write, inside the timed region)"},
-            "roofline": roofline, "rank": rank_leg, "rank_sizes": sizes, "rank_kendall": tau, "sweep_ase": ase, "online_hazard": online, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roofline, "rank": rank_leg, "rank_sizes": sizes, "rank_kendall": tau, "sweep_ase": ase, "online_hazard": online, "stale_snapshot": stale, "ablation": ablation, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": launches, "clocks": clocks,
             "peaks": {"hbm_gbs": peaks.get("hbm_gbs"), "source": "MEASURED_PEAKS.json"}}
     if cpu is not None:

@@ -147,7 +147,7 @@ typedef struct {
   uint64_t t_h_ps_per_tok;
   uint64_t t_p_ps_per_tok;     /* prefill cost; TTFT uses t_p / 1000 ns per token */
   uint32_t ttft_load;          /* arrival compression factor of the TTFT queue    */
-  uint32_t flags;              /* UNISON_HAZARD_ONLINE, or 0                      */
+  uint32_t flags;              /* UNISON_HAZARD_ONLINE, UNISON_SIGNAL_*, or 0     */
   uint32_t stale_sync;         /* UNISON_SYNC_*: dual-design ablation, or 0       */
   uint32_t stale_m;            /* arrivals per sync for UNISON_SYNC_ARRIVALS      */
 } unison_replay_params;
@@ -177,8 +177,16 @@ typedef struct {
  * SPEAR and SPEAR+TIDE only (else UNISON_ERR_ARG); the trace must have at
  * most 32,768 sessions and the replay's resident lists, rounded up to powers
  * of two, plus 7 bytes per session must fit in shared memory (else
- * UNISON_ERR_RANGE).  Any other bit of `flags` is UNISON_ERR_ARG. */
+ * UNISON_ERR_RANGE).  A bit of `flags` not defined here is UNISON_ERR_ARG. */
 #define UNISON_HAZARD_ONLINE 1u
+
+/* Signal leave-one-out (Sec. V-D, Fig. signal), SPEAR and SPEAR+TIDE only,
+ * not with UNISON_HAZARD_ONLINE (else UNISON_ERR_ARG): the score drops one
+ * of its two signals.  Without the gap recurrence it sees a gap average of 0
+ * (score = T2 of the turn); without the hazard it sees sigma_q = Lambda, a
+ * zero hazard (score = g_q).  TIDE's budget keeps the true gap average. */
+#define UNISON_SIGNAL_NO_GAP 2u
+#define UNISON_SIGNAL_NO_HAZARD 4u
 
 /* Per-replay counters (written by the device). */
 typedef struct {

@@ -53,7 +53,7 @@ class _Params(C.Structure):
                 ("ttl_us", C.c_uint32), ("ttft_load", C.c_uint32),
                 ("dma_bytes_per_us", C.c_uint64), ("prefill_ns_per_tok", C.c_uint64),
                 ("debug", C.c_uint32), ("hazard_online", C.c_uint32), ("stale_sync", C.c_uint32),
-                ("stale_m", C.c_uint32)]
+                ("stale_m", C.c_uint32), ("signals", C.c_uint32), ("pad3", C.c_uint32)]
 
 
 RESULT_FIELDS = ["events", "req_warm", "cold", "hit_s", "hit_h", "miss", "bypass", "place_s",
@@ -137,7 +137,8 @@ def _params_struct(p: dict, debug: bool):
                    q["kv_bytes_per_token"], q["max_sessions"], q["ema_num"], q["ema_den"],
                    q["penalty_q"], q["ttl_us"], q["ttft_load"], q["dma_bytes_per_us"],
                    q["t_p_ps_per_tok"] // 1000, 1 if debug else 0, 1 if q.get("hazard_online") else 0,
-                   STALE_SYNC[q.get("stale_sync", "live")], q.get("stale_m", 0))
+                   STALE_SYNC[q.get("stale_sync", "live")], q.get("stale_m", 0),
+                   (2 if q.get("no_gap") else 0) | (4 if q.get("no_hazard") else 0), 0)
 
 
 def replay(tr, params: dict, log: bool = False, ttft: bool = False, debug: bool = False,

@@ -41,6 +41,9 @@
  *       every gap_start.  Vict!= (Prom!=) counts the acted-upon victim
  *       (promotion) choices whose session differs from the choice by the
  *       live rows over the same candidates.
+ *   R29 signal leave-one-out (Sec. V-D, Fig. signal): without the gap
+ *       recurrence signal the score sees g_q = 0; without the hazard signal
+ *       it sees sigma_q = Lambda (zero hazard, so T2 = 0 as well).
  *   R27 attainment A(n) (eq. attainment): "after n observed sessions" is a
  *       window of the trace, the warm requests arriving while the online
  *       table holds n_j <= n < n_{j+1} sessions, n_j = floor(j N / P) for P
@@ -108,7 +111,11 @@ typedef struct {
   uint32_t hazard_online;        /* 1: the hazard table starts empty and grows as sessions complete (R26) */
   uint32_t stale_sync;           /* R28: 0 live; 1 every event; 2 every stale_m arrivals; 3 every gap_start */
   uint32_t stale_m;
+  uint32_t signals;              /* R29: bit 1 drops the gap signal, bit 2 the hazard signal */
+  uint32_t pad3;
 } or_params;
+
+enum { OR_NO_GAP = 2, OR_NO_HAZARD = 4 };
 
 enum { OR_SYNC_LIVE = 0, OR_SYNC_EVENT = 1, OR_SYNC_ARRIVALS = 2, OR_SYNC_GAP_START = 3 };
 
@@ -226,16 +233,22 @@ static int cmp_event(const void *a, const void *b) {
   return 0;
 }
 
+/* SPEAR key of a register row (g_q, turn, done), with the signals of R29. */
+static uint64_t spear_key(const or_state *st, uint64_t g_q, uint32_t turn, uint32_t done) {
+  uint32_t t = turn < OR_T_MAX ? turn : OR_T_MAX;
+  uint64_t g = (st->p->signals & OR_NO_GAP) ? 0 : g_q;
+  uint32_t sigma = (st->p->signals & OR_NO_HAZARD) ? OR_LAMBDA : st->sigma_q[t];
+  return or_spear_score(g, sigma, st->p->penalty_q, (int)done);
+}
+
 /* Policy key of session s from its live register row (R8); larger = more
  * evictable. */
 static uint64_t live_key_of(const or_state *st, uint32_t s) {
   const or_sess *x = &st->S[s];
   switch (st->p->policy) {
     case OR_SPEAR:
-    case OR_SPEAR_TIDE: {
-      uint32_t t = x->turn < OR_T_MAX ? x->turn : OR_T_MAX;
-      return or_spear_score(x->g_q, st->sigma_q[t], st->p->penalty_q, (int)x->done);
-    }
+    case OR_SPEAR_TIDE:
+      return spear_key(st, x->g_q, x->turn, x->done);
     case OR_BELADY:
       return x->next_ref;
     default: /* LRU, Timeout, LRU+TIDE: older last touch = more evictable */
@@ -246,8 +259,7 @@ static uint64_t live_key_of(const or_state *st, uint32_t s) {
 /* The key decisions rank by: the live row, or the snapshot row (R28). */
 static uint64_t key_of(const or_state *st, uint32_t s) {
   if (!st->stale) return live_key_of(st, s);
-  uint32_t t = st->snap_turn[s] < OR_T_MAX ? st->snap_turn[s] : OR_T_MAX;
-  return or_spear_score(st->snap_g[s], st->sigma_q[t], st->p->penalty_q, (int)st->snap_done[s]);
+  return spear_key(st, st->snap_g[s], st->snap_turn[s], st->snap_done[s]);
 }
 
 /* a more evictable than b: larger key, then smaller id. */
@@ -636,7 +648,9 @@ int or_replay(const or_trace *tr, const or_params *p, or_result *res, or_logrec 
       (p->ttl_us != UINT32_MAX && p->ttl_us >= (1u << 31)) || p->dma_bytes_per_us >= (1ull << 32) ||
       p->stale_sync > OR_SYNC_GAP_START || (p->stale_sync == OR_SYNC_ARRIVALS && p->stale_m == 0) ||
       (p->stale_sync != OR_SYNC_LIVE &&
-       (p->hazard_online || (p->policy != OR_SPEAR && p->policy != OR_SPEAR_TIDE))))
+       (p->hazard_online || (p->policy != OR_SPEAR && p->policy != OR_SPEAR_TIDE))) ||
+      (p->signals & ~(uint32_t)(OR_NO_GAP | OR_NO_HAZARD)) ||
+      (p->signals && (p->hazard_online || (p->policy != OR_SPEAR && p->policy != OR_SPEAR_TIDE))))
     return res->status = OR_ERR_ARG;
   or_event *ev = NULL;
   int rc = or_validate(tr, &ev);

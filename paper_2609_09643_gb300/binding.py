@@ -17,6 +17,7 @@ from .native import LIB
 
 POLICY = {"lru": 0, "timeout": 1, "spear": 2, "spear_tide": 3, "belady": 4, "lru_tide": 5}
 FLAG_HAZARD_ONLINE = 1  # unison_replay_params.flags bit 0
+FLAG_NO_GAP, FLAG_NO_HAZARD = 2, 4  # signal leave-one-out bits
 STALE_SYNC = {"live": 0, "event": 1, "arrivals": 2, "gap_start": 3}  # UNISON_SYNC_*
 KIND = ["COLD", "HIT_S", "HIT_H", "MISS", "PLACE_S", "PLACE_H", "BYPASS", "DEMOTE", "EVICT",
         "PROMOTE", "TIDE_DEMOTE", "EXPIRE"]
@@ -213,7 +214,8 @@ def make_params(p: dict, trace_idx: int = 0) -> ReplayParams:
                         q["kv_bytes_per_token"], q["max_sessions"], q["ema_num"], q["ema_den"],
                         q["hazard_bucket"], q["ttl_us"], q["penalty_q"], q["dma_bytes_per_us"],
                         q["t_s_ps_per_tok"], q["t_h_ps_per_tok"], q["t_p_ps_per_tok"], q["ttft_load"],
-                        q.get("flags", FLAG_HAZARD_ONLINE if q.get("hazard_online") else 0),
+                        q.get("flags", (FLAG_HAZARD_ONLINE if q.get("hazard_online") else 0) |
+                              (FLAG_NO_GAP if q.get("no_gap") else 0) | (FLAG_NO_HAZARD if q.get("no_hazard") else 0)),
                         STALE_SYNC[q.get("stale_sync", "live")] if isinstance(q.get("stale_sync", "live"), str)
                         else int(q["stale_sync"]), q.get("stale_m", 0))
 

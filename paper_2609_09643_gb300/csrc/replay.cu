@@ -42,7 +42,7 @@ struct ComboDesc {
   const uint32_t *turn_off;  // [S+1]
   const uint32_t *tps;       // [S]
   uint32_t n_sessions, n_events;
-  uint32_t ema_num, ema_den, bucket, pad;
+  uint32_t ema_num, ema_den, bucket, signals;  // signals: UNISON_SIGNAL_* bits of the flags
   uint64_t penalty_q;
   uint16_t *sigma;  // [51]
   uint64_t *t2;     // [51]
@@ -124,6 +124,12 @@ __device__ void build_lut(const uint32_t *tps, uint32_t n_sessions, uint32_t buc
 __global__ void hazard_lut_kernel(const ComboDesc *combos) {
   const ComboDesc &c = combos[blockIdx.x];
   build_lut(c.tps, c.n_sessions, c.bucket, c.penalty_q, c.sigma, nullptr, c.t2);
+  // without the hazard signal (Sec. V-D) the score sees zero hazard: sigma =
+  // Lambda and T2 = 0 (each entry is rewritten by the thread that wrote it)
+  if ((c.signals & UNISON_SIGNAL_NO_HAZARD) && threadIdx.x < kLutN) {
+    c.sigma[threadIdx.x] = (uint16_t)kLambda;
+    c.t2[threadIdx.x] = 0;
+  }
 }
 
 __global__ void hazard_lut_single_kernel(const uint32_t *tps, uint32_t n, uint32_t bucket, uint16_t *sigma,
@@ -149,6 +155,7 @@ __global__ void key_stream_kernel(const ComboDesc *combos) {
   if (s >= c.n_sessions) return;
   const uint32_t b = c.turn_off[s], ts = c.tps[s];
   const uint64_t a_num = c.ema_num, a_rest = c.ema_den - c.ema_num, a_den = c.ema_den;
+  const bool no_gap = (c.signals & UNISON_SIGNAL_NO_GAP) != 0;
   uint64_t g = 0, prev_pk = 0;
   uint32_t prev_c = 0;
   for (uint32_t k = 0; k < ts; k++) {
@@ -160,7 +167,8 @@ __global__ void key_stream_kernel(const ComboDesc *combos) {
     }
     prev_c = tc;
     const uint32_t t = k < kTMax ? k : kTMax;
-    const uint64_t key = (g * kLambda) / sig[t] + t2[t];
+    // without the gap signal (Sec. V-D) the score sees a zero gap average
+    const uint64_t key = ((no_gap ? 0 : g) * kLambda) / sig[t] + t2[t];
     const uint64_t pk = pack_key(key, s);
     const uint32_t ea = c.turn_ev[2 * ti], ec = c.turn_ev[2 * ti + 1];
     c.pkey[ea] = pk;
@@ -1201,7 +1209,11 @@ int check_params(const unison_replay_params &p, int n_traces) {
   if (p.dma_bytes_per_us >= (1ull << 32)) return UNISON_ERR_RANGE;
   if (p.ttl_us != 0xFFFFFFFFu && p.ttl_us >= (1u << 31)) return UNISON_ERR_RANGE;
   if (p.ttft_load == 0) return UNISON_ERR_ARG;
-  if (p.flags & ~UNISON_HAZARD_ONLINE) return UNISON_ERR_ARG;
+  constexpr uint32_t kSignals = UNISON_SIGNAL_NO_GAP | UNISON_SIGNAL_NO_HAZARD;
+  if (p.flags & ~(UNISON_HAZARD_ONLINE | kSignals)) return UNISON_ERR_ARG;
+  if ((p.flags & kSignals) &&
+      ((p.flags & UNISON_HAZARD_ONLINE) || (p.policy != UNISON_SPEAR && p.policy != UNISON_SPEAR_TIDE)))
+    return UNISON_ERR_ARG;
   if ((p.flags & UNISON_HAZARD_ONLINE) && p.policy != UNISON_SPEAR && p.policy != UNISON_SPEAR_TIDE)
     return UNISON_ERR_ARG;
   if (p.stale_sync > UNISON_SYNC_GAP_START || (p.stale_sync == UNISON_SYNC_ARRIVALS && p.stale_m == 0))
@@ -1227,7 +1239,7 @@ namespace {
 
 // Scratch layout and launch plan of one batch (shared by both entry points).
 struct ReplayPlan {
-  std::vector<std::tuple<uint32_t, uint32_t, uint32_t, uint32_t, uint64_t>> combos;
+  std::vector<std::tuple<uint32_t, uint32_t, uint32_t, uint32_t, uint64_t, uint32_t>> combos;
   std::vector<int> replay_combo;
   size_t off_desc = 0, off_order = 0, off_combo = 0, bytes = 0;
   std::vector<size_t> off_lut, off_stream, off_ttft, off_glist;
@@ -1266,12 +1278,13 @@ size_t online_bytes(uint32_t cs, uint32_t ch, uint32_t n_sessions) {
 
 int plan_replays(const unison_trace *const *traces, const unison_replay_params *params, int n_replays,
                  size_t smem_limit, bool results_in_scratch, ReplayPlan &P, size_t &off_res) {
-  std::map<std::tuple<uint32_t, uint32_t, uint32_t, uint32_t, uint64_t>, int> combo_of;
+  std::map<std::tuple<uint32_t, uint32_t, uint32_t, uint32_t, uint64_t, uint32_t>, int> combo_of;
   P.replay_combo.assign(n_replays, -1);
   for (int r = 0; r < n_replays; r++) {
     const unison_replay_params &p = params[r];
     if (!needs_stream(p.policy)) continue;
-    auto key = std::make_tuple(p.trace_idx, p.ema_num, p.ema_den, p.hazard_bucket, p.penalty_q);
+    auto key = std::make_tuple(p.trace_idx, p.ema_num, p.ema_den, p.hazard_bucket, p.penalty_q,
+                               p.flags & (UNISON_SIGNAL_NO_GAP | UNISON_SIGNAL_NO_HAZARD));
     auto it = combo_of.find(key);
     if (it == combo_of.end()) {
       it = combo_of.emplace(key, (int)P.combos.size()).first;
@@ -1362,7 +1375,7 @@ void fill_descs(const unison_trace *const *traces, const unison_replay_params *p
     d.ema_num = std::get<1>(P.combos[c]);
     d.ema_den = std::get<2>(P.combos[c]);
     d.bucket = std::get<3>(P.combos[c]);
-    d.pad = 0;
+    d.signals = std::get<5>(P.combos[c]);
     d.penalty_q = std::get<4>(P.combos[c]);
     d.sigma = reinterpret_cast<uint16_t *>(scratch + P.off_lut[c]);
     d.t2 = reinterpret_cast<uint64_t *>(scratch + P.off_lut[c] + 128);

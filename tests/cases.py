@@ -17,7 +17,7 @@ MIB = 1 << 20
 def base(policy, cap_s, cap_h, kvb, **kw):
     p = dict(policy=policy, cap_s=cap_s, cap_h=cap_h, kvb=kvb, max_sessions=0, ema_num=3, ema_den=10,
              bucket=1, penalty=500_000_000, ttl=10_000_000, dma=64_000, load=4, t_p=20_000_000, online=False,
-             stale="live", stale_m=0)
+             stale="live", stale_m=0, no_gap=False, no_hazard=False)
     p.update(kw)
     return p
 
@@ -27,7 +27,8 @@ def to_oracle(p: dict) -> dict:
                 max_sessions=p["max_sessions"], ema_num=p["ema_num"], ema_den=p["ema_den"],
                 hazard_bucket=p["bucket"], penalty_q=p["penalty"], ttl_us=p["ttl"], dma_bytes_per_us=p["dma"],
                 ttft_load=p["load"], t_p_ps_per_tok=p["t_p"], hazard_online=bool(p.get("online")),
-                stale_sync=p.get("stale", "live"), stale_m=p.get("stale_m", 0))
+                stale_sync=p.get("stale", "live"), stale_m=p.get("stale_m", 0), no_gap=p.get("no_gap", False),
+                no_hazard=p.get("no_hazard", False))
 
 
 def to_lib(p: dict, trace_idx: int = 0) -> dict:
@@ -37,7 +38,8 @@ def to_lib(p: dict, trace_idx: int = 0) -> dict:
                 ema_den=p["ema_den"], hazard_bucket=p["bucket"], penalty_q=p["penalty"], ttl_us=p["ttl"],
                 dma_bytes_per_us=p["dma"], ttft_load=p["load"], t_p_ps_per_tok=p["t_p"],
                 t_s_ps_per_tok=kvb // 16, t_h_ps_per_tok=kvb // 4, hazard_online=bool(p.get("online")),
-                stale_sync=p.get("stale", "live"), stale_m=p.get("stale_m", 0))
+                stale_sync=p.get("stale", "live"), stale_m=p.get("stale_m", 0), no_gap=p.get("no_gap", False),
+                no_hazard=p.get("no_hazard", False))
 
 
 # ---- the five workloads --------------------------------------------------------

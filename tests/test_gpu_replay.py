@@ -294,7 +294,7 @@ def test_online_hazard_rejected_cases(B):
     tr, _ = tiny_case()
     h = [B.Trace(tr).upload()]
     for pol, flags, err in (("lru", 1, B.ERR_ARG), ("belady", 1, B.ERR_ARG), ("lru_tide", 1, B.ERR_ARG),
-                            ("spear", 2, B.ERR_ARG), ("spear", 1 << 31, B.ERR_ARG)):
+                            ("spear", 8, B.ERR_ARG), ("spear", 1 << 31, B.ERR_ARG), ("spear", 3, B.ERR_ARG)):
         q = to_lib(base(pol, 1 * GIB, 8 * GIB, 28672))
         q["flags"] = flags
         with pytest.raises(B.UnisonError) as ei:
@@ -386,3 +386,50 @@ def test_stale_snapshot_rejected(B):
         with pytest.raises(B.UnisonError) as ei:
             B.replay_batch(h, [q])
         assert ei.value.code == B.ERR_ARG, (pol, sy, m, online)
+
+
+# ---- signal leave-one-out (Sec. V-D) ----------------------------------------------
+
+def test_signal_leave_one_out_paper_scale(B):
+    """Both gap mixes x SPEAR / SPEAR+TIDE x {full, no gap, no hazard, neither},
+    in one call (each signal set its own key stream)."""
+    trs = [synth.paper_scale_trace(1, "coding"), synth.paper_scale_trace(1, "general")]
+    reps = [(ti, base(pol, 4 * GIB, 64 * GIB, 131072, no_gap=ng, no_hazard=nh)) for ti in range(2)
+            for pol in ONLINE_POLS for ng in (False, True) for nh in (False, True)]
+    cap = 4 * trs[0].n_events
+    res, log, _ = run_gpu(B, trs, reps, log_capacity=cap)
+    for i, (ti, p) in enumerate(reps):
+        o = oracle.replay(trs[ti], to_oracle(p), log=(i % 3 == 1), log_capacity=cap)
+        assert_same(res[i], o, (i, p["policy"], p["no_gap"], p["no_hazard"]))
+        if i % 3 == 1:
+            assert_same_log(B, log[i], res[i], o, (i, p["policy"], p["no_gap"], p["no_hazard"]))
+    assert len({r["decision_hash"] for r in res}) == len(res)
+
+
+def test_signal_special_traces_on_device(B):
+    """The pins' traces: gaps of 1 us (no gap signal changes nothing) and
+    sessions beyond the table horizon (no hazard signal changes nothing)."""
+    from test_oracle_pins import _unit_gap_trace
+    tu = _unit_gap_trace()
+    th = synth.make_trace(13, 52 + np.arange(30) % 5, 0.4, synth.GAP_MIX_CODING)
+    reps = []
+    for pol in ONLINE_POLS:
+        reps += [(0, base(pol, 3000, 20000, 1)), (0, base(pol, 3000, 20000, 1, no_gap=True))]
+        reps += [(1, base(pol, 40000 * 131072, 200000 * 131072, 131072)),
+                 (1, base(pol, 40000 * 131072, 200000 * 131072, 131072, no_hazard=True))]
+    res, _, _ = run_gpu(B, [tu, th], reps)
+    for i, (ti, p) in enumerate(reps):
+        assert_same(res[i], oracle.replay([tu, th][ti], to_oracle(p)), i)
+        if i % 2:
+            assert res[i]["decision_hash"] == res[i - 1]["decision_hash"], i
+
+
+def test_signal_flags_rejected(B):
+    tr, _ = tiny_case()
+    h = [B.Trace(tr).upload()]
+    for pol, flags in (("lru", 2), ("belady", 4), ("lru_tide", 6), ("spear", 3), ("spear", 8)):
+        q = to_lib(base(pol, 1 * GIB, 8 * GIB, 28672))
+        q["flags"] = flags
+        with pytest.raises(B.UnisonError) as ei:
+            B.replay_batch(h, [q])
+        assert ei.value.code == B.ERR_ARG, (pol, flags)

@@ -685,3 +685,66 @@ def test_stale_snapshot_rejected_params():
     for bad in (dict(policy="lru", stale_sync="event"), dict(policy="belady", stale_sync="gap_start"),
                 dict(stale_sync="arrivals", stale_m=0), dict(stale_sync="event", hazard_online=True)):
         assert oracle.replay(tr, dict(STALE_HAND, **bad))["status"] == -1
+
+
+# ---- signal leave-one-out (Sec. V-D, Fig. signal; reading R29) -----------------------
+
+def _unit_gap_trace(n=60, turns=5):
+    """Every tool gap lasts 1 us: the gap average (3,10) stays at
+    floor(3*1/10) = 0 from the first gap on."""
+    arr, comp, ins, outs = [], [], [], []
+    for s in range(n):
+        a, c, i_, o_ = [], [], [], []
+        t = s * 1500
+        tok = 500 + 37 * (s % 11)
+        for k in range(turns):
+            a.append(t)
+            i_.append(tok)
+            tok += 64 + (s * 7 + k * 13) % 150
+            o_.append(tok)
+            t += 20 * (64 + (s + k) % 150)
+            c.append(t)
+            t += 1
+        arr.append(a), comp.append(c), ins.append(i_), outs.append(o_)
+    return synth.trace_from_turns(arr, comp, ins, outs)
+
+
+def test_signal_no_gap_equals_spear_when_gaps_vanish():
+    from cases import base, to_oracle
+    tr = _unit_gap_trace()
+    for pol in ("spear", "spear_tide"):
+        p = base(pol, 3000, 20000, 1)
+        a = oracle.replay(tr, to_oracle(p), debug=True)
+        b = oracle.replay(tr, to_oracle(dict(p, no_gap=True)), debug=True)
+        assert a["status"] == b["status"] == 0 and a["evict"] + a["demote"] > 10
+        assert a["decision_hash"] == b["decision_hash"], pol
+    tr = synth.paper_scale_trace(2, "coding")
+    p = base("spear", 2 * GIB, 16 * GIB, 131072)
+    assert (oracle.replay(tr, to_oracle(p))["decision_hash"] !=
+            oracle.replay(tr, to_oracle(dict(p, no_gap=True)))["decision_hash"])
+
+
+def test_signal_no_hazard_equals_spear_beyond_horizon():
+    """With every session longer than 51 turns, d(t) = 0 for every table
+    entry: zero hazard, sigma = Lambda, T2 = 0, as without the signal."""
+    from cases import base, to_oracle
+    tr = synth.make_trace(13, 52 + np.arange(30) % 5, 0.4, synth.GAP_MIX_CODING)
+    h, sig = oracle.hazard_lut(52 + np.arange(30) % 5)
+    assert np.all(h == 0) and np.all(sig == 4095)
+    for pol in ("spear", "spear_tide"):
+        p = base(pol, 40000 * 131072, 200000 * 131072, 131072)
+        a = oracle.replay(tr, to_oracle(p), debug=True)
+        b = oracle.replay(tr, to_oracle(dict(p, no_hazard=True)), debug=True)
+        assert a["status"] == b["status"] == 0 and a["evict"] + a["demote"] > 10
+        assert a["decision_hash"] == b["decision_hash"], pol
+    tr = synth.paper_scale_trace(2, "coding")
+    p = base("spear", 2 * GIB, 16 * GIB, 131072)
+    assert (oracle.replay(tr, to_oracle(p))["decision_hash"] !=
+            oracle.replay(tr, to_oracle(dict(p, no_hazard=True)))["decision_hash"])
+
+
+def test_signal_flags_rejected():
+    tr = _unit_gap_trace(4, 2)
+    for bad in (dict(policy="lru", no_gap=True), dict(policy="belady", no_hazard=True),
+                dict(policy="spear", no_gap=True, hazard_online=True)):
+        assert oracle.replay(tr, dict(STALE_HAND, **bad))["status"] == -1
