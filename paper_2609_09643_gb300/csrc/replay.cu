@@ -287,6 +287,7 @@ struct ReplayState {
   uint32_t npin, pin_cap;
   uint4 *tmp;       // TIDE staging: [0, cap_s) promoted, [cap_s, 2 cap_s) demoted
   uint8_t *tmap;    // tier of each unpinned resident session (kTierNone otherwise), or null
+  uint16_t *pslot;  // slot of each pinned session in `pin` (kNoSlot otherwise), or null
   uint64_t used_s, used_h, pinned_s, pinned_h;  // tokens
   unison_decision *log;
   uint64_t log_cap;
@@ -304,6 +305,8 @@ struct ReplayState {
 };
 
 #define CNT(st, field, v) ((st).field += (v))
+
+constexpr uint16_t kNoSlot = 0xFFFF;
 
 __device__ __forceinline__ void log_dec(ReplayState &st, uint32_t kind, uint32_t s, int lane) {
   const uint64_t w = ((uint64_t)st.e << 32) | ((uint64_t)kind << 24) | s;
@@ -435,6 +438,7 @@ __device__ __forceinline__ bool pin_append(ReplayState &st, uint64_t pk, uint32_
     return false;
   }
   if (lane == 0) st.pin[st.npin] = make_uint4((uint32_t)pk, (uint32_t)(pk >> 32), size, s | (tier << 30));
+  if (st.pslot) st.pslot[s] = (uint16_t)st.npin;  // every lane stores the same slot
   __syncwarp();
   st.npin++;
   return true;
@@ -795,16 +799,22 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
     st.tmp = p;
     p += 2 * D.rcap_s;
     st.tmap = nullptr;
+    st.pslot = nullptr;
     if (!kGlobalLists && D.tmap) {
+      // tier map (1 B per session), then pin slots (2 B per session)
       st.tmap = reinterpret_cast<uint8_t *>(p);
       uint32_t *m32 = reinterpret_cast<uint32_t *>(p);
       for (uint32_t i = lane; i < (D.n_sessions + 3) / 4; i += 32) m32[i] = 0u;
+      st.pslot = reinterpret_cast<uint16_t *>(reinterpret_cast<unsigned char *>(p) + ((D.n_sessions + 15) & ~15u));
+      uint32_t *s32 = reinterpret_cast<uint32_t *>(st.pslot);
+      for (uint32_t i = lane; i < (D.n_sessions + 1) / 2; i += 32) s32[i] = 0xFFFFFFFFu;
       __syncwarp();
     }
     if (kOnline) {
       // after the tier map: gap average (u32) and arrivals so far (u16) per
       // session, then the table
-      unsigned char *q = reinterpret_cast<unsigned char *>(p) + ((D.n_sessions + 15) & ~15u);
+      unsigned char *q = reinterpret_cast<unsigned char *>(p) + ((D.n_sessions + 15) & ~15u) +
+                         2 * ((D.n_sessions + 7) & ~7u);
       online_gs = reinterpret_cast<uint32_t *>(q);
       q += 4 * ((D.n_sessions + 3) & ~3u);
       online_ks = reinterpret_cast<uint16_t *>(q);
@@ -824,7 +834,8 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
     if (kStale) {
       // after the tier map: each session's live key and snapshot key; a zero
       // register row (gap average 0, turn 0, not done) scores T2 of turn 0
-      unsigned char *q = reinterpret_cast<unsigned char *>(p) + ((D.n_sessions + 15) & ~15u);
+      unsigned char *q = reinterpret_cast<unsigned char *>(p) + ((D.n_sessions + 15) & ~15u) +
+                         2 * ((D.n_sessions + 7) & ~7u);
       stale_live = reinterpret_cast<uint64_t *>(q);
       stale_snap = stale_live + ((D.n_sessions + 1) & ~1u);
       const uint64_t k0 = D.t2[0];
@@ -1028,16 +1039,25 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
       } else {
         // completion: unpin (if resident) and rank the session with its new key
         if (kStale) stale_live[s] = spk[bi][j];
-        int mine = -1;
-        for (uint32_t i = lane; i < st.npin; i += 32)
-          if ((st.pin[i].w & kIdMask) == s) mine = (int)i;
-        const uint32_t who = __ballot_sync(kFull, mine >= 0);
-        if (who) {
-          const uint32_t pi = (uint32_t)__shfl_sync(kFull, mine, __ffs(who) - 1);
+        uint32_t pi = kNoSlot;
+        if (st.pslot) {
+          pi = st.pslot[s];
+        } else {
+          int mine = -1;
+          for (uint32_t i = lane; i < st.npin; i += 32)
+            if ((st.pin[i].w & kIdMask) == s) mine = (int)i;
+          const uint32_t who = __ballot_sync(kFull, mine >= 0);
+          if (who) pi = (uint32_t)__shfl_sync(kFull, mine, __ffs(who) - 1);
+        }
+        if (pi != kNoSlot) {
           const uint4 pe = st.pin[pi];
           const uint4 last = st.pin[st.npin - 1];
           __syncwarp();
           if (lane == 0) st.pin[pi] = last;
+          if (st.pslot) {  // the last entry moves into the freed slot
+            st.pslot[last.w & kIdMask] = (uint16_t)pi;
+            st.pslot[s] = kNoSlot;
+          }
           __syncwarp();
           st.npin--;
           const uint32_t tier = pe.w >> 30, sz = pe.z;
@@ -1267,12 +1287,14 @@ size_t list_bytes(uint32_t cs, uint32_t ch) { return 16ull * (4ull * cs + 2ull *
 // and snapshot key of every session.
 size_t stale_bytes(uint32_t cs, uint32_t ch, uint32_t n_sessions) {
   const size_t n = n_sessions;
-  return 16ull * (ring_size(cs) + ring_size(ch) + 3ull * cs + ch) + align_up(n, 16) + 16 * align_up(n, 2);
+  return 16ull * (ring_size(cs) + ring_size(ch) + 3ull * cs + ch) + align_up(n, 16) + 2 * align_up(n, 8) +
+         16 * align_up(n, 2);
 }
 
 size_t online_bytes(uint32_t cs, uint32_t ch, uint32_t n_sessions) {
   const size_t n = n_sessions;
-  return 16ull * (ring_size(cs) + ring_size(ch) + 3ull * cs + ch) + align_up(n, 16) + 4 * align_up(n, 4) +
+  return 16ull * (ring_size(cs) + ring_size(ch) + 3ull * cs + ch) + align_up(n, 16) + 2 * align_up(n, 8) +
+         4 * align_up(n, 4) +
          2 * align_up(n, 8) + align_up(sizeof(OnlineTable), 16);
 }
 
@@ -1319,8 +1341,8 @@ int plan_replays(const unison_trace *const *traces, const unison_replay_params *
     P.rcap_s[r] = list_cap(p.cap_fast_bytes / p.kv_bytes_per_token, tr);
     P.rcap_h[r] = list_cap(p.cap_hbm_bytes / p.kv_bytes_per_token, tr);
     const size_t lists = list_bytes(P.rcap_s[r], P.rcap_h[r]);
-    // the tier map (one byte per session) when it fits beside the lists
-    const size_t map = align_up(tr->n_sessions, 16);
+    // the tier map and pin slots (3 bytes per session) when they fit beside the lists
+    const size_t map = align_up(tr->n_sessions, 16) + 2 * align_up(tr->n_sessions, 8);
     P.tmap[r] = tr->n_sessions <= kTierMapMax && lists + map <= smem_limit;
     if (p.flags & UNISON_HAZARD_ONLINE) {
       // online hazard replays run from shared memory only
