@@ -444,8 +444,18 @@ __device__ void joint_select32(const uint32_t (&v)[kLists][Q], uint32_t has, uin
 // into the list's threshold: the smallest list value with that summary (at
 // least r_L samples reach it), plus, per turn index, the smallest gap whose
 // key reaches the threshold's key (gA) or exceeds it (gB).
+// Programmatic dependent launch: the filter is launched while the sample
+// runs, and the finish while the filter runs.  A kernel lets its dependent
+// start once all its CTAs are running (launch_dependents), and a dependent
+// waits for its prerequisite grid to complete, with that grid's memory
+// visible, before it reads what that grid wrote (wait).  Without the launch
+// attribute both are no-ops.
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 template <int Q>
 __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankSet *sets) {
+  pdl_launch_dependents();
   const RankSet &S = sets[blockIdx.y];
   const uint32_t c = blockIdx.x;  // this CTA's share of the sample
   const uint32_t nct = S.sctas;
@@ -756,6 +766,7 @@ __device__ void load_set(const RankSet &S, uint4 *vd, uint2 *pp, uint64_t *t2s, 
 // UNISON_ERR_TIMEOUT, lets its own copies land (bounded) and returns.
 __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) rank_filter_kernel(const RankSet *sets, int n_sets,
                                                                         uint32_t total_tiles, int grouped) {
+  pdl_launch_dependents();
   extern __shared__ __align__(128) unsigned char fsm[];
   FilterStage *stage = reinterpret_cast<FilterStage *>(fsm);
   __shared__ __align__(8) uint64_t full[kStages], empty[kStages];
@@ -845,6 +856,9 @@ __global__ void __launch_bounds__(kFilterCtaThreads, UNISON_FILTER_MINBLOCKS) ra
   }
 
   // ---------------- consumer warps
+  // The producer streams records (inputs) at once; the consumers first wait
+  // for the sample's thresholds.
+  pdl_wait();
   // Consumer thread ct owns, in each tile, kGroups groups of four consecutive
   // records, group gi starting at record gi * kGroupStride + 4 * ct: every
   // shared-memory read of the stage is lane-contiguous (no bank conflicts).
@@ -1234,6 +1248,7 @@ __device__ uint32_t stream_topM(const RankSet &S, int L, uint32_t M, uint64_t *p
 }
 
 __global__ void __launch_bounds__(kFinishThreads) rank_finish_kernel(const RankSet *sets) {
+  pdl_wait();  // candidates and counts come from the filter
   const RankSet &S = sets[blockIdx.y];
   const int L = blockIdx.x;  // this CTA's list
   extern __shared__ __align__(16) unsigned char smem[];
@@ -1750,13 +1765,30 @@ extern "C" int unison_rank_batch(const unison_records *sets, const unison_rank_p
     else
       rank_sample_kernel<4><<<dim3(max_sctas, n_sets), kSampleThreads, 0, stream>>>(d_sets);
   }
+  cudaLaunchAttribute pdl[1];
+  pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  pdl[0].val.programmaticStreamSerializationAllowed = 1;
   {
     ProfSpan span("rank_filter", stream);
-    rank_filter_kernel<<<grid_filter, kFilterCtaThreads, kFilterSmem, stream>>>(d_sets, n_sets, tiles, grouped);
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(grid_filter);
+    lc.blockDim = dim3(kFilterCtaThreads);
+    lc.dynamicSmemBytes = kFilterSmem;
+    lc.stream = stream;
+    lc.attrs = pdl;
+    lc.numAttrs = 1;
+    ck(cudaLaunchKernelEx(&lc, rank_filter_kernel, (const RankSet *)d_sets, n_sets, tiles, grouped));
   }
   {
     ProfSpan span("rank_finish", stream);
-    rank_finish_kernel<<<dim3(kLists, n_sets), kFinishThreads, smem_finish, stream>>>(d_sets);
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = dim3(kLists, n_sets);
+    lc.blockDim = dim3(kFinishThreads);
+    lc.dynamicSmemBytes = smem_finish;
+    lc.stream = stream;
+    lc.attrs = pdl;
+    lc.numAttrs = 1;
+    ck(cudaLaunchKernelEx(&lc, rank_finish_kernel, (const RankSet *)d_sets));
   }
   count_launches(3);
   ck(cudaGetLastError());
