@@ -574,6 +574,15 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     st.status = UNISON_ERR_CAPACITY;
     return budget - rem;
   }
+  if (m == 1 && pairs == 0) {  // one promotion (the common case): move it directly
+    uint4 v = st.H.e[0];
+    v.z |= kPromotedBit;
+    __syncwarp();
+    shift_block(st.H.e, 1, st.H.n, -1, lane);
+    st.H.n -= 1;
+    sorted_insert(st, st.S, v, lane, kTierS);
+    return budget - rem;
+  }
   // stage the moved entries, then fix both arrays
   uint4 *pro = st.tmp, *dem = st.tmp + rcap_s;
   for (uint32_t i = lane; i < m; i += 32) {
