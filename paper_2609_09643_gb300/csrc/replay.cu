@@ -780,15 +780,21 @@ constexpr int kKeyStream = 0;  // keys from the per-session key stream
 constexpr int kKeyOnline = 1;  // keys under the online hazard table
 constexpr int kKeyStale = 2;   // snapshot keys of a dual design
 
-template <bool kGlobalLists, int kKeys>
-__global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, const uint32_t *order) {
+// Event prefetch: the next batch of 32 events and their side streams are
+// copied into this shared-memory double buffer with cp.async while the
+// current batch is processed.
+struct EventBufs {
+  uint4 sev[2][32];
+  uint32_t sprev[2][32], spev[2][32], snref[2][32], sgq[2][32];
+  unsigned long long spk[2][32], spkb[2][32];
+};
+
+// One replay: Algorithm 1 over the trace's events.  kPol is the replay's
+// policy when the body is specialised for it (its policy tests then fold
+// away), or -1 for the body that reads the policy from the descriptor.
+template <bool kGlobalLists, int kKeys, int kPol>
+__device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs, unsigned char *smem, int lane) {
   constexpr bool kOnline = kKeys == kKeyOnline, kStale = kKeys == kKeyStale;
-  extern __shared__ __align__(16) unsigned char smem[];
-  const int lane = threadIdx.x & 31;
-  __shared__ ReplayDesc Dsh;
-  if (lane == 0) Dsh = descs[order[blockIdx.x]];
-  __syncwarp();
-  const ReplayDesc &D = Dsh;
   const Hot hot{D.cap_s, D.cap_h, D.kvb, D.dma, D.max_sessions};
 
   ReplayState st;
@@ -869,7 +875,7 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
   st.n_evict = st.n_demote = st.n_promote = st.n_tide_demote = st.n_expire = st.n_tide_calls = st.n_pth = 0;
   st.tok_hit_s = st.tok_hit_h = st.tok_miss = st.tok_computed = st.tok_needed = st.dma_bytes = 0;
 
-  const uint32_t policy = D.policy;
+  const uint32_t policy = kPol >= 0 ? (uint32_t)kPol : D.policy;
   const bool spear_keys = policy == UNISON_SPEAR || policy == UNISON_SPEAR_TIDE;
   const bool tide_on = has_tide(policy);
   const bool belady = policy == UNISON_BELADY;
@@ -885,11 +891,9 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
   bool dma_busy = false;
   uint32_t busy_until = 0;
 
-  // Event prefetch: the next batch of 32 events is copied into a shared-memory
-  // double buffer with cp.async while the current batch is processed.
-  __shared__ __align__(16) uint4 sev[2][32];
-  __shared__ __align__(16) uint32_t sprev[2][32], spev[2][32], snref[2][32], sgq[2][32];
-  __shared__ __align__(16) unsigned long long spk[2][32], spkb[2][32];
+  auto &sev = bufs.sev;
+  auto &sprev = bufs.sprev, &spev = bufs.spev, &snref = bufs.snref, &sgq = bufs.sgq;
+  auto &spk = bufs.spk, &spkb = bufs.spkb;
   const uint32_t E = D.n_events;
   auto fetch = [&](uint32_t b, int bi) {
     const uint32_t i = b + lane;
@@ -1165,6 +1169,26 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
   }
 }
 
+// One warp per replay.  SPEAR+TIDE replays (the sweep's policy) run a body
+// specialised for it: a smaller, branch-free event loop.  kOnly >= 0: every
+// replay of the launch has that policy, and the kernel holds only its body
+// (and is sized for it alone).
+template <bool kGlobalLists, int kKeys, int kOnly>
+__global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, const uint32_t *order) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  __shared__ ReplayDesc Dsh;
+  __shared__ __align__(16) EventBufs bufs;
+  const int lane = threadIdx.x & 31;
+  if (lane == 0) Dsh = descs[order[blockIdx.x]];
+  __syncwarp();
+  if (kOnly >= 0)
+    replay_body<kGlobalLists, kKeys, kOnly>(Dsh, bufs, smem, lane);
+  else if (kKeys == kKeyStream && Dsh.policy == UNISON_SPEAR_TIDE)
+    replay_body<kGlobalLists, kKeys, UNISON_SPEAR_TIDE>(Dsh, bufs, smem, lane);
+  else
+    replay_body<kGlobalLists, kKeys, -1>(Dsh, bufs, smem, lane);
+}
+
 // Lower median (element floor((n-1)/2) in sorted order) by MSB-first radix select.
 __global__ void __launch_bounds__(256) ttft_median_kernel(const ReplayDesc *descs, uint32_t n_replays) {
   const ReplayDesc &D = descs[blockIdx.x];
@@ -1274,6 +1298,7 @@ struct ReplayPlan {
   std::vector<size_t> off_lut, off_stream, off_ttft, off_glist;
   std::vector<uint32_t> rcap_s, rcap_h, in_smem, in_global, in_online, in_stale, tmap;
   size_t max_smem = 0, max_smem_online = 0, max_smem_stale = 0;
+  bool smem_all_st = true, global_all_st = true;  // every replay of the group is SPEAR+TIDE
 };
 
 // Resident-list capacity of a tier: at most one entry per session and no more
@@ -1379,6 +1404,8 @@ int plan_replays(const unison_trace *const *traces, const unison_replay_params *
     P.off_ttft[r] = off;
     off = align_up(off + 8 * (tr->n_turns + 1), 256);
   }
+  for (uint32_t r : P.in_smem) P.smem_all_st &= params[r].policy == UNISON_SPEAR_TIDE;
+  for (uint32_t r : P.in_global) P.global_all_st &= params[r].policy == UNISON_SPEAR_TIDE;
   off_res = 0;
   if (results_in_scratch) {
     off_res = off;
@@ -1488,30 +1515,32 @@ int launch_replays(const ReplayPlan &P, char *scratch, const std::vector<ComboDe
   {
     ProfSpan span(profile ? "replay" : "", stream);
     if (!P.in_smem.empty()) {
-      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyStream>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)P.max_smem));
-      replay_kernel<false, kKeyStream><<<(unsigned)P.in_smem.size(), 32, P.max_smem, stream>>>(d_desc, d_order);
+      const auto k = P.smem_all_st ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE>
+                                   : replay_kernel<false, kKeyStream, -1>;
+      ck(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P.max_smem));
+      k<<<(unsigned)P.in_smem.size(), 32, P.max_smem, stream>>>(d_desc, d_order);
       count_launches(1);
       ck(cudaGetLastError());
     }
     if (!P.in_global.empty()) {
-      replay_kernel<true, kKeyStream><<<(unsigned)P.in_global.size(), 32, 0, stream>>>(d_desc,
-                                                                                      d_order + P.in_smem.size());
+      const auto k = P.global_all_st ? replay_kernel<true, kKeyStream, UNISON_SPEAR_TIDE>
+                                     : replay_kernel<true, kKeyStream, -1>;
+      k<<<(unsigned)P.in_global.size(), 32, 0, stream>>>(d_desc, d_order + P.in_smem.size());
       count_launches(1);
       ck(cudaGetLastError());
     }
     if (!P.in_online.empty()) {
-      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyOnline>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyOnline, -1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)P.max_smem_online));
-      replay_kernel<false, kKeyOnline><<<(unsigned)P.in_online.size(), 32, P.max_smem_online, stream>>>(
+      replay_kernel<false, kKeyOnline, -1><<<(unsigned)P.in_online.size(), 32, P.max_smem_online, stream>>>(
           d_desc, d_order + P.in_smem.size() + P.in_global.size());
       count_launches(1);
       ck(cudaGetLastError());
     }
     if (!P.in_stale.empty()) {
-      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyStale>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyStale, -1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)P.max_smem_stale));
-      replay_kernel<false, kKeyStale><<<(unsigned)P.in_stale.size(), 32, P.max_smem_stale, stream>>>(
+      replay_kernel<false, kKeyStale, -1><<<(unsigned)P.in_stale.size(), 32, P.max_smem_stale, stream>>>(
           d_desc, d_order + P.in_smem.size() + P.in_global.size() + P.in_online.size());
       count_launches(1);
       ck(cudaGetLastError());
