@@ -308,10 +308,13 @@ struct ReplayState {
 
 constexpr uint16_t kNoSlot = 0xFFFF;
 
+// kLean (here and below): the replay keeps no decision log, has the tier map
+// and pin slots, and no slot limit -- known at compile time.
+template <bool kLean>
 __device__ __forceinline__ void log_dec(ReplayState &st, uint32_t kind, uint32_t s, int lane) {
   const uint64_t w = ((uint64_t)st.e << 32) | ((uint64_t)kind << 24) | s;
   st.hash = (st.hash ^ w) * kFnvPrime;
-  if (st.log) {
+  if (!kLean && st.log) {
     if (st.log_len < st.log_cap) {
       if (lane == 0) {
         unison_decision d;
@@ -328,10 +331,12 @@ __device__ __forceinline__ void log_dec(ReplayState &st, uint32_t kind, uint32_t
 
 // Tier-map update: every lane stores the same byte, so each lane's later
 // reads see it without a warp barrier.
+template <bool kLean>
 __device__ __forceinline__ void set_tier(ReplayState &st, uint32_t id, uint32_t tier) {
-  if (st.tmap) st.tmap[id] = (uint8_t)tier;
+  if (kLean || st.tmap) st.tmap[id] = (uint8_t)tier;
 }
 
+template <bool kLean>
 __device__ __forceinline__ bool sorted_insert(ReplayState &st, Sorted &T, uint4 v, int lane, uint32_t tier) {
   if (T.n >= T.cap) {
     st.status = UNISON_ERR_CAPACITY;
@@ -342,7 +347,7 @@ __device__ __forceinline__ bool sorted_insert(ReplayState &st, Sorted &T, uint4 
   if (lane == 0) T.e[p] = v;
   __syncwarp();
   T.n++;
-  set_tier(st, packed_id(ekey(v)), tier);
+  set_tier<kLean>(st, packed_id(ekey(v)), tier);
   return true;
 }
 
@@ -351,11 +356,12 @@ __device__ __forceinline__ void sorted_erase(Sorted &T, uint32_t p, int lane) {
   T.n--;
 }
 
+template <bool kLean>
 __device__ __forceinline__ uint4 sorted_pop_back(ReplayState &st, Sorted &T) {
   const uint4 v = T.e[T.n - 1];
   __syncwarp();
   T.n--;
-  set_tier(st, packed_id(ekey(v)), kTierNone);
+  set_tier<kLean>(st, packed_id(ekey(v)), kTierNone);
   return v;
 }
 
@@ -399,12 +405,12 @@ __device__ __forceinline__ void count_promotion(ReplayState &st, uint32_t chosen
 // A session demoted out of the fast tier enters HBM, displacing the most
 // evictable unpinned HBM sessions, or is dropped when it is itself the most
 // evictable of (unpinned HBM) + {itself}.
-template <bool kStale>
+template <bool kStale, bool kLean>
 __device__ __forceinline__ bool admit_demoted(ReplayState &st, const Hot &D, uint4 d, int lane) {
   const uint32_t id = packed_id(ekey(d));
   const uint32_t size = esize(d);
   if (st.pinned_h > D.cap_h || size > D.cap_h - st.pinned_h) {
-    log_dec(st, UNISON_KIND_EVICT, id, lane);
+    log_dec<kLean>(st, UNISON_KIND_EVICT, id, lane);
     CNT(st, n_evict, 1);
     return true;
   }
@@ -415,18 +421,18 @@ __device__ __forceinline__ bool admit_demoted(ReplayState &st, const Hot &D, uin
                    max(live_max(st, st.H, 0, st.H.n, lane), st.live[id]));
     }
     if (st.H.n == 0 || ekey(d) > ekey(st.H.e[st.H.n - 1])) {
-      log_dec(st, UNISON_KIND_EVICT, id, lane);
+      log_dec<kLean>(st, UNISON_KIND_EVICT, id, lane);
       CNT(st, n_evict, 1);
       return true;
     }
-    const uint4 v = sorted_pop_back(st, st.H);
+    const uint4 v = sorted_pop_back<kLean>(st, st.H);
     st.used_h -= esize(v);
-    log_dec(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
+    log_dec<kLean>(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
     CNT(st, n_evict, 1);
   }
-  if (!sorted_insert(st, st.H, d, lane, kTierH)) return false;
+  if (!sorted_insert<kLean>(st, st.H, d, lane, kTierH)) return false;
   st.used_h += size;
-  log_dec(st, UNISON_KIND_DEMOTE, id, lane);
+  log_dec<kLean>(st, UNISON_KIND_DEMOTE, id, lane);
   CNT(st, n_demote, 1);
   return true;
 }
@@ -445,11 +451,11 @@ __device__ __forceinline__ bool pin_append(ReplayState &st, uint64_t pk, uint32_
 }
 
 // Placement of the arriving (pinned) session s with n tokens.
-template <bool kStale>
+template <bool kStale, bool kLean>
 __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s, uint64_t pk, uint32_t n,
                                       int lane) {
-  if (D.max_sessions && st.npin >= D.max_sessions) {
-    log_dec(st, UNISON_KIND_BYPASS, s, lane);
+  if (!kLean && D.max_sessions && st.npin >= D.max_sessions) {
+    log_dec<kLean>(st, UNISON_KIND_BYPASS, s, lane);
     CNT(st, n_bypass, 1);
     return true;
   }
@@ -460,14 +466,14 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
         return false;
       }
       if (kStale) count_victim(st, packed_id(ekey(st.S.e[st.S.n - 1])), live_max(st, st.S, 0, st.S.n, lane));
-      const uint4 d = sorted_pop_back(st, st.S);  // most evictable unpinned fast-tier session
+      const uint4 d = sorted_pop_back<kLean>(st, st.S);  // most evictable unpinned fast-tier session
       st.used_s -= esize(d);
-      if (!admit_demoted<kStale>(st, D, d, lane)) return false;
+      if (!admit_demoted<kStale, kLean>(st, D, d, lane)) return false;
     }
     if (!pin_append(st, pk, n, s, kTierS, lane)) return false;
     st.used_s += n;
     st.pinned_s += n;
-    log_dec(st, UNISON_KIND_PLACE_S, s, lane);
+    log_dec<kLean>(st, UNISON_KIND_PLACE_S, s, lane);
     CNT(st, n_place_s, 1);
   } else if (st.pinned_h <= D.cap_h && n <= D.cap_h - st.pinned_h) {
     while (st.used_h + n > D.cap_h) {
@@ -476,22 +482,22 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
         return false;
       }
       if (kStale) count_victim(st, packed_id(ekey(st.H.e[st.H.n - 1])), live_max(st, st.H, 0, st.H.n, lane));
-      const uint4 v = sorted_pop_back(st, st.H);
+      const uint4 v = sorted_pop_back<kLean>(st, st.H);
       st.used_h -= esize(v);
-      log_dec(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
+      log_dec<kLean>(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
       CNT(st, n_evict, 1);
     }
     if (!pin_append(st, pk, n, s, kTierH, lane)) return false;
     st.used_h += n;
     st.pinned_h += n;
-    log_dec(st, UNISON_KIND_PLACE_H, s, lane);
+    log_dec<kLean>(st, UNISON_KIND_PLACE_H, s, lane);
     CNT(st, n_place_h, 1);
   } else {
-    log_dec(st, UNISON_KIND_BYPASS, s, lane);
+    log_dec<kLean>(st, UNISON_KIND_BYPASS, s, lane);
     CNT(st, n_bypass, 1);
     return true;
   }
-  if (D.max_sessions) {
+  if (!kLean && D.max_sessions) {
     while (st.S.n + st.H.n + st.npin > D.max_sessions) {
       if (st.S.n == 0 && st.H.n == 0) {
         st.status = UNISON_ERR_CAPACITY;
@@ -502,12 +508,12 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
       if (kStale)
         count_victim(st, packed_id(ekey(from_s ? st.S.e[st.S.n - 1] : st.H.e[st.H.n - 1])),
                      max(live_max(st, st.S, 0, st.S.n, lane), live_max(st, st.H, 0, st.H.n, lane)));
-      const uint4 v = sorted_pop_back(st, from_s ? st.S : st.H);
+      const uint4 v = sorted_pop_back<kLean>(st, from_s ? st.S : st.H);
       if (from_s)
         st.used_s -= esize(v);
       else
         st.used_h -= esize(v);
-      log_dec(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
+      log_dec<kLean>(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
       CNT(st, n_evict, 1);
     }
   }
@@ -519,7 +525,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
 // free fast-tier space; phase 2: pair the next least evictable HBM session
 // with the most evictable fast-tier one), which makes the same moves as the
 // pair loop of Algorithm 1, and are then applied in bulk.
-template <bool kStale>
+template <bool kStale, bool kLean>
 __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t budget, uint32_t rcap_s,
                                          int lane) {
   uint64_t rem = budget;
@@ -534,7 +540,7 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     rem -= by;
     st.used_s += sz;
     st.used_h -= sz;
-    log_dec(st, UNISON_KIND_PROMOTE, packed_id(ekey(p)), lane);
+    log_dec<kLean>(st, UNISON_KIND_PROMOTE, packed_id(ekey(p)), lane);
     n1++;
   }
   uint32_t pairs = 0;
@@ -562,8 +568,8 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     rem -= by;
     st.used_s = st.used_s - sd + sp;
     st.used_h = st.used_h - sp + sd;
-    log_dec(st, UNISON_KIND_PROMOTE, packed_id(ekey(p)), lane);
-    log_dec(st, UNISON_KIND_TIDE_DEMOTE, packed_id(ekey(d)), lane);
+    log_dec<kLean>(st, UNISON_KIND_PROMOTE, packed_id(ekey(p)), lane);
+    log_dec<kLean>(st, UNISON_KIND_TIDE_DEMOTE, packed_id(ekey(d)), lane);
     pairs++;
   }
   const uint32_t m = n1 + pairs;
@@ -580,7 +586,7 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     __syncwarp();
     shift_block(st.H.e, 1, st.H.n, -1, lane);
     st.H.n -= 1;
-    sorted_insert(st, st.S, v, lane, kTierS);
+    sorted_insert<kLean>(st, st.S, v, lane, kTierS);
     return budget - rem;
   }
   // stage the moved entries, then fix both arrays
@@ -596,15 +602,16 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
   st.H.n -= m;
   st.S.n -= pairs;
   for (uint32_t i = 0; i < m; i++)
-    if (!sorted_insert(st, st.S, pro[i], lane, kTierS)) return budget - rem;
+    if (!sorted_insert<kLean>(st, st.S, pro[i], lane, kTierS)) return budget - rem;
   for (uint32_t i = 0; i < pairs; i++)
-    if (!sorted_insert(st, st.H, dem[i], lane, kTierH)) return budget - rem;
+    if (!sorted_insert<kLean>(st, st.H, dem[i], lane, kTierH)) return budget - rem;
   return budget - rem;
 }
 
 // Timeout: expire unpinned residents idle >= ttl, smallest session id first.
 // Under recency keys the last return time falls as the key grows, so the
 // expired sessions of a tier are a top suffix of its array.
+template <bool kLean>
 __device__ __forceinline__ void expire_idle(ReplayState &st, uint32_t now, uint32_t ttl, int lane) {
   for (;;) {
     // expired suffix lengths
@@ -635,8 +642,8 @@ __device__ __forceinline__ void expire_idle(ReplayState &st, uint32_t now, uint3
     else
       st.used_h -= sz;
     sorted_erase(T, pos, lane);
-    set_tier(st, mid, kTierNone);
-    log_dec(st, UNISON_KIND_EXPIRE, mid, lane);
+    set_tier<kLean>(st, mid, kTierNone);
+    log_dec<kLean>(st, UNISON_KIND_EXPIRE, mid, lane);
     CNT(st, n_expire, 1);
   }
 }
@@ -792,7 +799,7 @@ struct EventBufs {
 // One replay: Algorithm 1 over the trace's events.  kPol is the replay's
 // policy when the body is specialised for it (its policy tests then fold
 // away), or -1 for the body that reads the policy from the descriptor.
-template <bool kGlobalLists, int kKeys, int kPol>
+template <bool kGlobalLists, int kKeys, int kPol, bool kLean>
 __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs, unsigned char *smem, int lane) {
   constexpr bool kOnline = kKeys == kKeyOnline, kStale = kKeys == kKeyStale;
   const Hot hot{D.cap_s, D.cap_h, D.kvb, D.dma, D.max_sessions};
@@ -937,7 +944,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
       n_ev++;
       rel_us += (uint32_t)(now - prev_now);
       prev_now = now;
-      if (timeout) expire_idle(st, now, D.ttl, lane);
+      if (timeout) expire_idle<kLean>(st, now, D.ttl, lane);
       if (dma_busy && (int32_t)(now - busy_until) >= 0) dma_busy = false;
 
       if (arrival) {
@@ -962,7 +969,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
             pkb = pack_key(0xFFFFFFFFull - spev[bi][j], s);
           // with the tier map only the session's own tier is searched (and
           // nothing for a session that is not resident)
-          const uint32_t mt = st.tmap ? st.tmap[s] : (kTierS | kTierH);
+          const uint32_t mt = (kLean || st.tmap) ? st.tmap[s] : (kTierS | kTierH);
           if (mt & kTierS) {
             pos = lower_bound(st.S, pkb, lane);
             if (pos < st.S.n && ekey(st.S.e[pos]) == pkb) {
@@ -981,25 +988,25 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
         }
         uint64_t prefill;
         if (edge) {
-          log_dec(st, UNISON_KIND_COLD, s, lane);
+          log_dec<kLean>(st, UNISON_KIND_COLD, s, lane);
           CNT(st, n_cold, 1);
           prefill = in;
         } else {
           CNT(st, n_warm, 1);
           CNT(st, tok_needed, in);
           if (tier == kTierS) {
-            log_dec(st, UNISON_KIND_HIT_S, s, lane);
+            log_dec<kLean>(st, UNISON_KIND_HIT_S, s, lane);
             CNT(st, n_hit_s, 1);
             CNT(st, tok_hit_s, prev);
             prefill = in - prev;
             if (ent.z & kPromotedBit) CNT(st, n_pth, 1);
           } else if (tier == kTierH) {
-            log_dec(st, UNISON_KIND_HIT_H, s, lane);
+            log_dec<kLean>(st, UNISON_KIND_HIT_H, s, lane);
             CNT(st, n_hit_h, 1);
             CNT(st, tok_hit_h, prev);
             prefill = in - prev;
           } else {
-            log_dec(st, UNISON_KIND_MISS, s, lane);
+            log_dec<kLean>(st, UNISON_KIND_MISS, s, lane);
             CNT(st, n_miss, 1);
             CNT(st, tok_miss, prev);
             prefill = in;
@@ -1020,11 +1027,11 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
         if (tier == kTierS) {
           st.used_s -= esize(ent);
           sorted_erase(st.S, pos, lane);
-          set_tier(st, s, kTierNone);
+          set_tier<kLean>(st, s, kTierNone);
         } else if (tier == kTierH) {
           st.used_h -= esize(ent);
           sorted_erase(st.H, pos, lane);
-          set_tier(st, s, kTierNone);
+          set_tier<kLean>(st, s, kTierNone);
         }
         uint64_t pk;
         if (kOnline) {
@@ -1048,12 +1055,12 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
           pk = pack_key(nr == kNoRef ? kKeyMax40 : (uint64_t)nr, s);
         } else
           pk = pack_key(0xFFFFFFFFull - e, s);
-        if (!place<kStale>(st, hot, s, pk, out, lane)) break;
+        if (!place<kStale, kLean>(st, hot, s, pk, out, lane)) break;
       } else {
         // completion: unpin (if resident) and rank the session with its new key
         if (kStale) stale_live[s] = spk[bi][j];
         uint32_t pi = kNoSlot;
-        if (st.pslot) {
+        if (kLean || st.pslot) {
           pi = st.pslot[s];
         } else {
           int mine = -1;
@@ -1067,7 +1074,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
           const uint4 last = st.pin[st.npin - 1];
           __syncwarp();
           if (lane == 0) st.pin[pi] = last;
-          if (st.pslot) {  // the last entry moves into the freed slot
+          if (kLean || st.pslot) {  // the last entry moves into the freed slot
             st.pslot[last.w & kIdMask] = (uint16_t)pi;
             st.pslot[s] = kNoSlot;
           }
@@ -1087,10 +1094,10 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
           const uint4 v = make_uint4((uint32_t)pk, (uint32_t)(pk >> 32), sz, now);
           if (tier == kTierS) {
             st.pinned_s -= sz;
-            if (!sorted_insert(st, st.S, v, lane, kTierS)) break;
+            if (!sorted_insert<kLean>(st, st.S, v, lane, kTierS)) break;
           } else {
             st.pinned_h -= sz;
-            if (!sorted_insert(st, st.H, v, lane, kTierH)) break;
+            if (!sorted_insert<kLean>(st, st.H, v, lane, kTierH)) break;
           }
         }
         if (kOnline && edge) {
@@ -1105,7 +1112,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
           const uint64_t g = sgq[bi][j];
           const uint64_t budget = g * D.dma;
           CNT(st, n_tide_calls, 1);
-          const uint64_t moved = tide<kStale>(st, hot, budget, D.rcap_s, lane);
+          const uint64_t moved = tide<kStale, kLean>(st, hot, budget, D.rcap_s, lane);
           CNT(st, dma_bytes, moved);
           if (moved > 0 && D.dma > 0) {
             dma_busy = true;
@@ -1172,8 +1179,9 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
 // One warp per replay.  SPEAR+TIDE replays (the sweep's policy) run a body
 // specialised for it: a smaller, branch-free event loop.  kOnly >= 0: every
 // replay of the launch has that policy, and the kernel holds only its body
-// (and is sized for it alone).
-template <bool kGlobalLists, int kKeys, int kOnly>
+// (and is sized for it alone); kLean: every replay of the launch is lean
+// (see log_dec).
+template <bool kGlobalLists, int kKeys, int kOnly, bool kLean>
 __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, const uint32_t *order) {
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ ReplayDesc Dsh;
@@ -1182,11 +1190,11 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
   if (lane == 0) Dsh = descs[order[blockIdx.x]];
   __syncwarp();
   if (kOnly >= 0)
-    replay_body<kGlobalLists, kKeys, kOnly>(Dsh, bufs, smem, lane);
+    replay_body<kGlobalLists, kKeys, kOnly, kLean>(Dsh, bufs, smem, lane);
   else if (kKeys == kKeyStream && Dsh.policy == UNISON_SPEAR_TIDE)
-    replay_body<kGlobalLists, kKeys, UNISON_SPEAR_TIDE>(Dsh, bufs, smem, lane);
+    replay_body<kGlobalLists, kKeys, UNISON_SPEAR_TIDE, false>(Dsh, bufs, smem, lane);
   else
-    replay_body<kGlobalLists, kKeys, -1>(Dsh, bufs, smem, lane);
+    replay_body<kGlobalLists, kKeys, -1, false>(Dsh, bufs, smem, lane);
 }
 
 // Lower median (element floor((n-1)/2) in sorted order) by MSB-first radix select.
@@ -1299,6 +1307,7 @@ struct ReplayPlan {
   std::vector<uint32_t> rcap_s, rcap_h, in_smem, in_global, in_online, in_stale, tmap;
   size_t max_smem = 0, max_smem_online = 0, max_smem_stale = 0;
   bool smem_all_st = true, global_all_st = true;  // every replay of the group is SPEAR+TIDE
+  bool smem_lean = true;  // ... and has the tier map and no slot limit (the log is per call)
 };
 
 // Resident-list capacity of a tier: at most one entry per session and no more
@@ -1404,7 +1413,10 @@ int plan_replays(const unison_trace *const *traces, const unison_replay_params *
     P.off_ttft[r] = off;
     off = align_up(off + 8 * (tr->n_turns + 1), 256);
   }
-  for (uint32_t r : P.in_smem) P.smem_all_st &= params[r].policy == UNISON_SPEAR_TIDE;
+  for (uint32_t r : P.in_smem) {
+    P.smem_all_st &= params[r].policy == UNISON_SPEAR_TIDE;
+    P.smem_lean &= P.tmap[r] && params[r].max_sessions == 0;
+  }
   for (uint32_t r : P.in_global) P.global_all_st &= params[r].policy == UNISON_SPEAR_TIDE;
   off_res = 0;
   if (results_in_scratch) {
@@ -1489,7 +1501,7 @@ void fill_descs(const unison_trace *const *traces, const unison_replay_params *p
 // Queue the kernels of a planned batch on `stream`.
 int launch_replays(const ReplayPlan &P, char *scratch, const std::vector<ComboDesc> &hc,
                    const std::vector<ReplayDesc> &hd, const std::vector<uint32_t> &order, int n_replays,
-                   cudaStream_t stream, bool profile) {
+                   cudaStream_t stream, bool profile, bool logged) {
   int rc = UNISON_OK;
   auto ck = [&](cudaError_t e) {
     if (e != cudaSuccess && rc == UNISON_OK) rc = UNISON_ERR_CUDA;
@@ -1515,32 +1527,33 @@ int launch_replays(const ReplayPlan &P, char *scratch, const std::vector<ComboDe
   {
     ProfSpan span(profile ? "replay" : "", stream);
     if (!P.in_smem.empty()) {
-      const auto k = P.smem_all_st ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE>
-                                   : replay_kernel<false, kKeyStream, -1>;
+      const auto k = !P.smem_all_st ? replay_kernel<false, kKeyStream, -1, false>
+                     : (P.smem_lean && !logged) ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true>
+                                                : replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, false>;
       ck(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P.max_smem));
       k<<<(unsigned)P.in_smem.size(), 32, P.max_smem, stream>>>(d_desc, d_order);
       count_launches(1);
       ck(cudaGetLastError());
     }
     if (!P.in_global.empty()) {
-      const auto k = P.global_all_st ? replay_kernel<true, kKeyStream, UNISON_SPEAR_TIDE>
-                                     : replay_kernel<true, kKeyStream, -1>;
+      const auto k = P.global_all_st ? replay_kernel<true, kKeyStream, UNISON_SPEAR_TIDE, false>
+                                     : replay_kernel<true, kKeyStream, -1, false>;
       k<<<(unsigned)P.in_global.size(), 32, 0, stream>>>(d_desc, d_order + P.in_smem.size());
       count_launches(1);
       ck(cudaGetLastError());
     }
     if (!P.in_online.empty()) {
-      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyOnline, -1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyOnline, -1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)P.max_smem_online));
-      replay_kernel<false, kKeyOnline, -1><<<(unsigned)P.in_online.size(), 32, P.max_smem_online, stream>>>(
+      replay_kernel<false, kKeyOnline, -1, false><<<(unsigned)P.in_online.size(), 32, P.max_smem_online, stream>>>(
           d_desc, d_order + P.in_smem.size() + P.in_global.size());
       count_launches(1);
       ck(cudaGetLastError());
     }
     if (!P.in_stale.empty()) {
-      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyStale, -1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyStale, -1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               (int)P.max_smem_stale));
-      replay_kernel<false, kKeyStale, -1><<<(unsigned)P.in_stale.size(), 32, P.max_smem_stale, stream>>>(
+      replay_kernel<false, kKeyStale, -1, false><<<(unsigned)P.in_stale.size(), 32, P.max_smem_stale, stream>>>(
           d_desc, d_order + P.in_smem.size() + P.in_global.size() + P.in_online.size());
       count_launches(1);
       ck(cudaGetLastError());
@@ -1598,7 +1611,7 @@ extern "C" int unison_replay_batch(const unison_trace *const *traces, int n_trac
   std::vector<ReplayDesc> hd;
   std::vector<uint32_t> order;
   fill_descs(traces, params, n_replays, P, scratch, res, log_dev, log_capacity_per_replay, hc, hd, order);
-  rc = launch_replays(P, scratch, hc, hd, order, n_replays, stream, true);
+  rc = launch_replays(P, scratch, hc, hd, order, n_replays, stream, true, log_dev != nullptr);
   if (results_host &&
       cudaMemcpyAsync(results_host, res, sizeof(unison_replay_result) * n_replays, cudaMemcpyDeviceToHost, stream) !=
           cudaSuccess &&
@@ -1785,7 +1798,7 @@ extern "C" int unison_replay_batch_noalloc(const unison_trace *const *traces, in
   std::vector<ReplayDesc> hd;
   std::vector<uint32_t> order;
   fill_descs(traces, params, n_replays, P, scratch, results_dev, log_dev, log_capacity_per_replay, hc, hd, order);
-  rc = launch_replays(P, scratch, hc, hd, order, n_replays, stream, false);
+  rc = launch_replays(P, scratch, hc, hd, order, n_replays, stream, false, log_dev != nullptr);
   if (results_host) {
     if (cudaMemcpyAsync(results_host, results_dev, sizeof(unison_replay_result) * n_replays, cudaMemcpyDeviceToHost,
                         stream) != cudaSuccess &&
