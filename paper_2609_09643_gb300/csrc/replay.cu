@@ -892,6 +892,9 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
   uint64_t rel_us = 0, q_free = 0;
   uint32_t prev_now = 0, n_arr = 0, n_ev = 0;
   const uint32_t load = D.load;
+  const uint64_t prefill_ns = D.prefill_ns;
+  const uint32_t n_turns = D.n_turns;
+  uint64_t *const ttft_out = D.ttft;
   const uint64_t ns_per_us = (1000u % load == 0) ? 1000u / load : 0u;  // 0: divide exactly
   unsigned long long s_lo = 0, s_hi = 0;
   uint32_t stale_arrivals = 0;
@@ -907,7 +910,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
     if (i < E) {
       cp_async16(&sev[bi][lane], &D.ev[i]);
       cp_async4(&sprev[bi][lane], &D.prev_out[i]);
-      cp_async4(&spev[bi][lane], &D.prev_ev[i]);
+      if (!spear_keys) cp_async4(&spev[bi][lane], &D.prev_ev[i]);  // recency keys only
       if (belady) cp_async4(&snref[bi][lane], &D.nref[i]);
       if (spear_keys && !kOnline) {
         cp_async8(&spk[bi][lane], &D.pkey[i]);
@@ -1016,9 +1019,9 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
         {
           const uint64_t arr = ns_per_us ? rel_us * ns_per_us : rel_us * 1000ull / load;
           if (q_free < arr) q_free = arr;
-          q_free += prefill * D.prefill_ns;
+          q_free += prefill * prefill_ns;
           const uint64_t v = q_free - arr;
-          if (lane == 0 && n_arr < D.n_turns) D.ttft[n_arr] = v;
+          if (lane == 0 && n_arr < n_turns) ttft_out[n_arr] = v;
           n_arr++;
           const unsigned long long lo2 = s_lo + v;
           s_hi += (lo2 < s_lo);
