@@ -386,6 +386,23 @@ def test_stale_snapshot_rejected(B):
         with pytest.raises(B.UnisonError) as ei:
             B.replay_batch(h, [q])
         assert ei.value.code == B.ERR_ARG, (pol, sy, m, online)
+    # more sessions than a stale-snapshot replay keeps in shared memory
+    big = synth.make_trace(5, np.full(40000, 2), 0.005, synth.GAP_MIX_GENERAL)
+    hb = [B.Trace(big).upload()]
+    with pytest.raises(B.UnisonError) as ei:
+        B.replay_batch(hb, [to_lib(base("spear_tide", 1 * GIB, 8 * GIB, 16384, stale="event"))])
+    assert ei.value.code == B.ERR_RANGE
+
+
+def test_stale_snapshot_with_a_signal_left_out(B):
+    """The two variants combine: snapshot keys without the hazard signal, and
+    without the gap signal, on the paper-scale coding trace."""
+    tr = synth.paper_scale_trace(2, "coding")
+    reps = [(0, base(pol, 2 * GIB, 16 * GIB, 131072, stale=sy, stale_m=8, no_gap=ng, no_hazard=not ng))
+            for pol in ONLINE_POLS for sy in ("arrivals", "gap_start") for ng in (False, True)]
+    res, _, _ = run_gpu(B, [tr], reps)
+    for i, (_, p) in enumerate(reps):
+        assert_same(res[i], oracle.replay(tr, to_oracle(p)), i)
 
 
 # ---- signal leave-one-out (Sec. V-D) ----------------------------------------------

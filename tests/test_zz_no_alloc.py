@@ -30,6 +30,10 @@ def _workload():
     for ti, (cs, ch, kvb) in enumerate([(512 * MIB, 8 * GIB, 28672), (2 * GIB, 32 * GIB, 131072)]):
         for pol in ("lru", "timeout", "spear", "spear_tide", "belady", "lru_tide"):
             reps.append((ti, base(pol, cs, ch, kvb)))
+        # the launch variants: online table, stale snapshot, a signal left out
+        reps.append((ti, base("spear_tide", cs, ch, kvb, online=True)))
+        reps.append((ti, base("spear", cs, ch, kvb, stale="arrivals", stale_m=4)))
+        reps.append((ti, base("spear_tide", cs, ch, kvb, no_hazard=True, stale="gap_start")))
     return trs, reps
 
 
