@@ -589,6 +589,18 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     sorted_insert<kLean>(st, st.S, v, lane, kTierS);
     return budget - rem;
   }
+  if (m == 1 && pairs == 1) {  // one pair (the next most common): swap it directly
+    uint4 v = st.H.e[0];
+    v.z |= kPromotedBit;
+    const uint4 d = st.S.e[st.S.n - 1];
+    __syncwarp();
+    shift_block(st.H.e, 1, st.H.n, -1, lane);
+    st.H.n -= 1;
+    st.S.n -= 1;
+    if (!sorted_insert<kLean>(st, st.S, v, lane, kTierS)) return budget - rem;
+    sorted_insert<kLean>(st, st.H, d, lane, kTierH);
+    return budget - rem;
+  }
   // stage the moved entries, then fix both arrays
   uint4 *pro = st.tmp, *dem = st.tmp + rcap_s;
   for (uint32_t i = lane; i < m; i += 32) {
