@@ -66,6 +66,9 @@ def parse():
     ap.add_argument("--no-online", action="store_true", help="skip the online hazard-table report")
     ap.add_argument("--no-stale", action="store_true", help="skip the stale-snapshot (dual design) report")
     ap.add_argument("--no-ablation", action="store_true", help="skip the component/signal/capacity ablations")
+    ap.add_argument("--table", action="store_true",
+                    help="per-config table instead of the bench line: GPU events/s, oracle 1-thread and all-core "
+                         "events/s, parity, rank GB/s per live-set size")
     return ap.parse_args()
 
 
@@ -465,6 +468,112 @@ def cpu_baseline_rank(rec, sigma, n: int = 1 << 22):
             "sample": f"{n} records of one 2^24 live set, k=1024, 64 GiB budget, single thread, {dt:.1f} s"}
 
 
+def _oracle_replay_job(job):
+    """One oracle replay in a worker process (the pool uses spawn)."""
+    import oracle
+    from cases import to_oracle
+    tr, p = job
+    return oracle.replay(tr, to_oracle(p))
+
+
+def _oracle_rank_job(job):
+    import oracle
+    import synth
+    rec, sigma, n = job
+    sub = synth.Records(*(a[:n].copy() for a in (rec.gap_q, rec.last_ret, rec.turn, rec.kv_tok, rec.tier,
+                                                 rec.flags)))
+    oracle.rank(sub, sigma, 500_000_000, 1024, 64 << 30, 131072, 0, 1 << 40, max_moves=1024)
+    return n
+
+
+def config_table(args):
+    """Configs 0-3 (replays) and 4 (ranking): device events/s of one batched
+    launch (CUDA events, warm), the oracle on one core and on all host cores
+    (a spawn pool, one replay per task) over a stated sample, and parity of
+    every replay the oracle ran (all counters and the decision hash)."""
+    import multiprocessing as mp
+    import torch
+    import synth
+    from cases import tiny_case, paper_scale_case, sweep_case, large_pool_params, to_lib, to_oracle
+    import oracle
+    from paper_2609_09643_gb300 import native
+    torch.cuda.set_device(0)
+    native.build()
+    from paper_2609_09643_gb300 import binding as B
+    cores = os.cpu_count() or 1
+    pool = mp.get_context("spawn").Pool(cores)
+    stream = torch.cuda.current_stream()
+    tr0, ps0 = tiny_case()
+    trs2, reps2 = sweep_case()
+    n_large = 16
+    cfgs = [("0 tiny", [tr0], [(0, p) for p in ps0], 50, "all 4"),
+            ("1 paper-scale", *paper_scale_case(), 10, "all 30"),
+            ("2 sweep", trs2, reps2, 5, "32 replays spread over the 1,024"),
+            (f"3 large pool ({n_large} of the 256 replays, seeds 100-{99 + n_large})",
+             [synth.large_pool_trace(100 + i) for i in range(n_large)],
+             [(i, large_pool_params()) for i in range(n_large)], 2, f"all {n_large}")]
+    fields = ["events", "req_warm", "hit_s", "hit_h", "miss", "evict", "demote", "promote", "tide_demote",
+              "tok_computed", "ttft_sum", "ttft_p50_ns", "decision_hash", "status"]
+    out = []
+    for name, trs, reps, steps, sample in cfgs:
+        handles = [B.Trace(t).upload(stream) for t in trs]
+        params = [to_lib(p, ti) for ti, p in reps]
+        ev = sum(2 * trs[ti].n_turns for ti, _ in reps)
+        res_dev = torch.zeros(B.result_nbytes(len(params)), dtype=torch.uint8, device="cuda")
+        B.replay_batch_async(handles, params, res_dev, stream=stream)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(steps):
+            B.replay_batch_async(handles, params, res_dev, stream=stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        gpu = ev * steps / (a.elapsed_time(b) / 1e3)
+        res = B.results_from_tensor(res_dev)
+        pick = list(range(len(reps))) if not name.startswith("2") else [int(i * 1024 / 32) for i in range(32)]
+        # one core: a bounded part of the sample, in this process
+        t0, ev1, n1 = time.perf_counter(), 0, 0
+        for i in pick:
+            ti, p = reps[i]
+            ev1 += oracle.replay(trs[ti], to_oracle(p))["events"]
+            n1 += 1
+            if time.perf_counter() - t0 > 10.0:
+                break
+        one = ev1 / (time.perf_counter() - t0)
+        # all cores: the whole sample
+        t0 = time.perf_counter()
+        ores = pool.map(_oracle_replay_job, [(trs[reps[i][0]], reps[i][1]) for i in pick], chunksize=1)
+        allc = sum(r["events"] for r in ores) / (time.perf_counter() - t0)
+        bad = [i for i, r in zip(pick, ores) if any(res[i][f] != r[f] for f in fields)]
+        out.append({"config": name, "replays": len(reps), "events_per_launch": ev, "gpu_events_per_s": gpu,
+                    "oracle_1core_events_per_s": one, "oracle_1core_sample": f"{n1} replays",
+                    "oracle_allcore_events_per_s": allc, "oracle_allcore_sample": sample, "cores": cores,
+                    "parity": f"{len(pick) - len(bad)}/{len(pick)} replays identical" + (f", differ: {bad[:5]}" if bad else "")})
+        del handles, res_dev
+    # config 4: the ranking at each live-set size (device), the oracle on 2^22 records
+    rec, tps = rank_workload()
+    tps_dev = torch.tensor(tps.astype("int32"), device="cuda")
+    sig_dev, _ = B.hazard_lut(tps_dev, 1)
+    sigma = sig_dev.cpu().numpy().astype("uint16")
+    host_rec = {k: v.pin_memory() for k, v in B.records_to_device(rec, device="cpu").items()}
+    B.profile_enable(True)
+    sizes = rank_size_sweep(B, host_rec, sigma, stream)
+    B.profile_enable(False)
+    one = cpu_baseline_rank(rec, sigma)
+    t0 = time.perf_counter()
+    n = sum(pool.map(_oracle_rank_job, [(rec, sigma, 1 << 22)] * cores, chunksize=1))
+    allc = n * RANK_BYTES_PER_RECORD / (time.perf_counter() - t0) / 1e9
+    pool.close()
+    pk = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))).get("hbm_gbs") or 6800.0
+    out.append({"config": "4 rank", "gpu": [{"n": e["n"], "sets": e["sets_per_call"], "call_gbs": e["call_gbs"],
+                                            "call_frac": e["call_gbs"] / pk, "filter_gbs": e["filter_gbs"],
+                                            "filter_frac": e["filter_gbs"] / pk if e["filter_gbs"] else None}
+                                           for e in sizes],
+                "oracle_1core_gbs": one["value"], "oracle_allcore_gbs": allc, "cores": cores,
+                "oracle_sample": "2^22 records of one 2^24 live set per core, k=1,024, full sort + fill"})
+    print(json.dumps({"table": out, "peak_hbm_gbs": pk}), flush=True)
+
+
 def run_reference(args):
     world, rank, _ = dist_env()
     if rank != 0:
@@ -505,6 +614,8 @@ def main():
     RANK_N = args.rank_n
     if args.impl == "reference":
         return run_reference(args)
+    if args.table:
+        return config_table(args)
     import torch
     world, rank, local = dist_env()
     if world > 1:
