@@ -25,6 +25,19 @@ constexpr uint32_t kLutN = 51u;
 constexpr uint64_t kKeyMax40 = (1ull << 40) - 1;
 constexpr uint32_t kIdMask = 0xFFFFFFu;
 
+// floor(x / s) for x < 2^43 and 2 <= s < 2^12 by one multiply-high
+// (Granlund and Montgomery, PLDI 1994, Thm 4.2 with N = 43): with
+// l = ceil(log2 s) and m = ceil(2^(43+l) / s), floor(x/s) = floor(x m / 2^(43+l));
+// storing m << (21 - l) turns that into the high word of a 64x64 product.
+__host__ __device__ inline uint64_t magic_for(uint32_t s) {
+  uint32_t l = 0;
+  while ((1u << l) < s) l++;
+  // m = ceil(2^(43+l) / s) fits 44 bits; compute without 128-bit division.
+  const uint64_t num = 1ull << (43 + l);  // 43 + l <= 55
+  const uint64_t m = (num + s - 1) / s;
+  return m << (21 - l);
+}
+
 __host__ __device__ __forceinline__ uint64_t pack_key(uint64_t key40, uint32_t id) {
   return (key40 << 24) | ((~id) & kIdMask);
 }

@@ -689,11 +689,13 @@ __device__ __forceinline__ bool has_tide(uint32_t policy) {
 struct OnlineTable {
   uint32_t n[kLutN], d[kLutN], sig[kLutN];
   unsigned long long t2[kLutN];
+  unsigned long long mg[kLutN];  // magic_for(sig): eq. (t1)'s division by a multiply-high
 };
 
+// g < 2^31 (gaps are clamped below 2^31 us), so g * Lambda < 2^43.
 __device__ __forceinline__ uint64_t online_key(const OnlineTable &ot, uint32_t g, uint32_t t, uint32_t s) {
   const uint32_t tt = t < kTMax ? t : kTMax;
-  return pack_key((uint64_t)g * kLambda / ot.sig[tt] + ot.t2[tt], s);
+  return pack_key(__umul64hi((uint64_t)g * kLambda, ot.mg[tt]) + ot.t2[tt], s);
 }
 
 // A session of `turns` turns has completed: add it to the counts and rebuild
@@ -732,6 +734,7 @@ __device__ bool online_add(OnlineTable &ot, uint32_t turns, uint32_t bucket, uin
   for (int q = 0; q < 2; q++) {
     const uint32_t t = lane + 32 * q;
     if (t < kLutN) {
+      if (ot.sig[t] != sg[q]) ot.mg[t] = magic_for(sg[q]);
       ot.sig[t] = sg[q];
       ot.t2[t] = t2[q];
     }
@@ -862,6 +865,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
         online_tab->n[t] = online_tab->d[t] = 0u;
         online_tab->sig[t] = kLambda;  // no session completed: zero hazard
         online_tab->t2[t] = 0ull;
+        online_tab->mg[t] = magic_for(kLambda);
       }
       __syncwarp();
     }
