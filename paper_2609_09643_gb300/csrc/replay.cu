@@ -798,6 +798,7 @@ __device__ void online_rerank(Sorted &T, const OnlineTable &ot, const uint32_t *
   }, lane);
 }
 
+constexpr uint32_t kDirtyCap = 32;  // sessions a stale-snapshot sync updates one by one
 constexpr int kKeyStream = 0;  // keys from the per-session key stream
 constexpr int kKeyOnline = 1;  // keys under the online hazard table
 constexpr int kKeyStale = 2;   // snapshot keys of a dual design
@@ -824,6 +825,17 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
   uint16_t *online_ks = nullptr;
   OnlineTable *online_tab = nullptr;
   uint64_t *stale_live = nullptr, *stale_snap = nullptr;
+  uint8_t *stale_dflag = nullptr;
+  uint32_t *stale_dlist = nullptr, stale_ndirty = 0;
+  // a session's live key changed: note it for the next sync (every lane
+  // stores the same values)
+  auto mark_dirty = [&](uint32_t s) {
+    if (!stale_dflag[s]) {
+      stale_dflag[s] = 1;
+      if (stale_ndirty < kDirtyCap) stale_dlist[stale_ndirty] = s;
+      stale_ndirty++;
+    }
+  };
   {
     uint4 *p = reinterpret_cast<uint4 *>(kGlobalLists ? reinterpret_cast<unsigned char *>(D.glist) : smem);
     // online and stale-snapshot replays keep power-of-two tiers (for re-sorts)
@@ -876,8 +888,15 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
                          2 * ((D.n_sessions + 7) & ~7u);
       stale_live = reinterpret_cast<uint64_t *>(q);
       stale_snap = stale_live + ((D.n_sessions + 1) & ~1u);
+      // then a flag per session changed since the last sync, and the list of
+      // the first kDirtyCap of them
+      stale_dflag = reinterpret_cast<uint8_t *>(stale_snap + ((D.n_sessions + 1) & ~1u));
+      stale_dlist = reinterpret_cast<uint32_t *>(stale_dflag + ((D.n_sessions + 15) & ~15u));
       const uint64_t k0 = D.t2[0];
-      for (uint32_t i = lane; i < D.n_sessions; i += 32) stale_live[i] = stale_snap[i] = pack_key(k0, i);
+      for (uint32_t i = lane; i < D.n_sessions; i += 32) {
+        stale_live[i] = stale_snap[i] = pack_key(k0, i);
+        stale_dflag[i] = 0;
+      }
       __syncwarp();
     }
     st.live = stale_live;
@@ -1067,6 +1086,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
         } else if (kStale) {
           pk = stale_snap[s];
           stale_live[s] = spk[bi][j];  // every lane stores the same key
+          mark_dirty(s);
         } else if (spear_keys)
           pk = spk[bi][j];
         else if (belady) {
@@ -1077,7 +1097,10 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
         if (!place<kStale, kLean>(st, hot, s, pk, out, lane)) break;
       } else {
         // completion: unpin (if resident) and rank the session with its new key
-        if (kStale) stale_live[s] = spk[bi][j];
+        if (kStale) {
+          stale_live[s] = spk[bi][j];
+          mark_dirty(s);
+        }
         uint32_t pi = kNoSlot;
         if (kLean || st.pslot) {
           pi = st.pslot[s];
@@ -1146,12 +1169,37 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
         bool sync = D.stale_sync == UNISON_SYNC_EVENT;
         if (arrival && D.stale_sync == UNISON_SYNC_ARRIVALS) sync = ++stale_arrivals % D.stale_m == 0;
         if (!arrival && D.stale_sync == UNISON_SYNC_GAP_START) sync = !edge;
-        if (sync) {
-          for (uint32_t i = lane; i < D.n_sessions; i += 32) stale_snap[i] = stale_live[i];
+        if (sync && stale_ndirty <= kDirtyCap) {
+          // few sessions changed: move just their resident entries
+          for (uint32_t k = 0; k < stale_ndirty; k++) {
+            const uint32_t d = stale_dlist[k];
+            const uint64_t nk = stale_live[d], ok = stale_snap[d];
+            stale_snap[d] = nk;
+            stale_dflag[d] = 0;
+            const uint32_t t = st.tmap[d];
+            if (t != kTierNone && nk != ok) {
+              Sorted &T = t == kTierS ? st.S : st.H;
+              const uint32_t pos = lower_bound(T, ok, lane);
+              uint4 v = T.e[pos];
+              __syncwarp();
+              v.x = (uint32_t)nk;
+              v.y = (uint32_t)(nk >> 32);
+              sorted_erase(T, pos, lane);
+              sorted_insert<kLean>(st, T, v, lane, t);
+            }
+          }
+          __syncwarp();
+          stale_ndirty = 0;
+        } else if (sync) {
+          for (uint32_t i = lane; i < D.n_sessions; i += 32) {
+            stale_snap[i] = stale_live[i];
+            stale_dflag[i] = 0;
+          }
           __syncwarp();
           const auto snap_key = [&](uint64_t k) { return stale_snap[packed_id(k)]; };
           rerank(st.S, snap_key, lane);
           rerank(st.H, snap_key, lane);
+          stale_ndirty = 0;
         }
       }
     }
@@ -1350,7 +1398,7 @@ size_t list_bytes(uint32_t cs, uint32_t ch) { return 16ull * (4ull * cs + 2ull *
 size_t stale_bytes(uint32_t cs, uint32_t ch, uint32_t n_sessions) {
   const size_t n = n_sessions;
   return 16ull * (ring_size(cs) + ring_size(ch) + 3ull * cs + ch) + align_up(n, 16) + 2 * align_up(n, 8) +
-         16 * align_up(n, 2);
+         16 * align_up(n, 2) + align_up(n, 16) + 4 * kDirtyCap;
 }
 
 size_t online_bytes(uint32_t cs, uint32_t ch, uint32_t n_sessions) {
