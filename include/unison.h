@@ -246,6 +246,12 @@ typedef struct {
  *    strictly more evictable, the pair fits the remaining budget and both
  *    tiers stay within capacity.  The DMA is then busy for
  *    ceil(moved / dma_bytes_per_us) us.
+ * Per-replay variants (definitions above): UNISON_HAZARD_ONLINE (the table
+ * grows as sessions complete), UNISON_SIGNAL_NO_GAP / _NO_HAZARD (the score
+ * without one signal), stale_sync (decisions on a register-file snapshot).
+ * Replays of one call may mix policies and variants; each runs in the
+ * launch for its kind, and a launch whose replays share the policy and
+ * simple settings runs a kernel specialised for them.
  *
  * traces[n_traces]: uploaded handles (host array of pointers).
  * params[n_replays]: host array.
