@@ -470,12 +470,16 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
   // 1. this thread's samples j = tid + 1024 q: run j / 8 of the CTA's share
   uint32_t f[kLists][Q];
   uint32_t m = 0;  // bit L * Q + q: sample q is eligible for list L
+  // the sampled records' indices first, then all their loads at once (they
+  // are independent random reads), then their keys
+  uint32_t rr[Q];
+  bool ok[Q];
 #pragma unroll
   for (int q = 0; q < Q; q++) {
-#pragma unroll
-    for (int L = 0; L < kLists; L++) f[L][q] = 0;
     const uint32_t jt = tid + kSampleThreads * q;
-    if (jt < per) {
+    ok[q] = jt < per;
+    rr[q] = 0;
+    if (ok[q]) {
       // stratum bounds floor(run n / nruns) with n = sq nruns + srem, in 32 bits
       const uint32_t nruns = S.nruns, run = c * (per / 8) + jt / 8, o = jt % 8;
       const uint32_t lo = run * S.sq + (run * S.srem) / nruns;
@@ -485,11 +489,27 @@ __global__ void __launch_bounds__(kSampleThreads) rank_sample_kernel(const RankS
       h *= 0x85EBCA6Bu;
       h ^= h >> 13;
       const uint32_t span = hi - lo - 8;  // strata hold at least 8 records
-      const uint32_t r = lo + (h % (span + 1)) + o;
-      const uint8_t fl = S.flags[r], tr = S.tier[r];
-      const uint32_t t = min((uint32_t)S.turn[r], kTMax);
-      const uint64_t ck = ck_of(score_of(S.gap[r], t, (fl & 2) != 0, t2s, mgs), r);
-      const uint32_t em = elig_mask(fl, tr) & act;
+      rr[q] = lo + (h % (span + 1)) + o;
+    }
+  }
+  uint8_t fl[Q], tr[Q];
+  uint16_t tu[Q];
+  uint32_t gg[Q];
+#pragma unroll
+  for (int q = 0; q < Q; q++) {  // index 0 for an unused slot: a valid record
+    fl[q] = S.flags[rr[q]];
+    tr[q] = S.tier[rr[q]];
+    tu[q] = S.turn[rr[q]];
+    gg[q] = S.gap[rr[q]];
+  }
+#pragma unroll
+  for (int q = 0; q < Q; q++) {
+#pragma unroll
+    for (int L = 0; L < kLists; L++) f[L][q] = 0;
+    if (ok[q]) {
+      const uint32_t t = min((uint32_t)tu[q], kTMax);
+      const uint64_t ck = ck_of(score_of(gg[q], t, (fl[q] & 2) != 0, t2s, mgs), rr[q]);
+      const uint32_t em = elig_mask(fl[q], tr[q]) & act;
 #pragma unroll
       for (int L = 0; L < kLists; L++) {
         f[L][q] = summary_of(list_val(ck, L));
