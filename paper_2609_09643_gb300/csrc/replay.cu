@@ -342,8 +342,11 @@ __device__ __forceinline__ bool sorted_insert(ReplayState &st, Sorted &T, uint4 
     st.status = UNISON_ERR_CAPACITY;
     return false;
   }
-  const uint32_t p = lower_bound(T, ekey(v), lane);
-  shift_block(T.e, p, T.n, 1, lane);
+  uint32_t p = T.n;  // past the last key: an append, no search or shift
+  if (T.n > 0 && ekey(v) < ekey(T.e[T.n - 1])) {
+    p = lower_bound(T, ekey(v), lane);
+    shift_block(T.e, p, T.n, 1, lane);
+  }
   if (lane == 0) T.e[p] = v;
   __syncwarp();
   T.n++;
