@@ -144,10 +144,9 @@ __global__ void hazard_lut_single_kernel(const uint32_t *tps, uint32_t n, uint32
 // Every thread loads the table before any may leave, so the barrier is uniform.
 __global__ void key_stream_kernel(const ComboDesc *combos) {
   const ComboDesc &c = combos[blockIdx.y];
-  __shared__ uint32_t sig[kLutN];
-  __shared__ unsigned long long t2[kLutN];
+  __shared__ unsigned long long mg[kLutN], t2[kLutN];
   for (uint32_t i = threadIdx.x; i < kLutN; i += blockDim.x) {
-    sig[i] = c.sigma[i];
+    mg[i] = magic_for(c.sigma[i]);  // eq. (t1)'s division by sigma as a multiply-high
     t2[i] = c.t2[i];
   }
   __syncthreads();
@@ -155,6 +154,10 @@ __global__ void key_stream_kernel(const ComboDesc *combos) {
   if (s >= c.n_sessions) return;
   const uint32_t b = c.turn_off[s], ts = c.tps[s];
   const uint64_t a_num = c.ema_num, a_rest = c.ema_den - c.ema_num, a_den = c.ema_den;
+  // eq. (ema-int)'s division by a_den: its numerator stays below a_den * 2^31,
+  // so below 2^43 when a_den < 2^12 -- then a multiply-high (a_den >= 2)
+  const bool den_magic = a_den >= 2 && a_den < 4096;
+  const uint64_t den_mg = den_magic ? magic_for((uint32_t)a_den) : 0;
   const bool no_gap = (c.signals & UNISON_SIGNAL_NO_GAP) != 0;
   uint64_t g = 0, prev_pk = 0;
   uint32_t prev_c = 0;
@@ -163,12 +166,14 @@ __global__ void key_stream_kernel(const ComboDesc *combos) {
     const uint32_t ta = c.turn_t[2 * ti], tc = c.turn_t[2 * ti + 1];
     if (k) {
       const uint64_t gap = (uint32_t)(ta - prev_c);
-      g = (a_num * gap + a_rest * g) / a_den;
+      const uint64_t num = a_num * gap + a_rest * g;
+      g = den_magic ? __umul64hi(num, den_mg) : num / a_den;
     }
     prev_c = tc;
     const uint32_t t = k < kTMax ? k : kTMax;
-    // without the gap signal (Sec. V-D) the score sees a zero gap average
-    const uint64_t key = ((no_gap ? 0 : g) * kLambda) / sig[t] + t2[t];
+    // without the gap signal (Sec. V-D) the score sees a zero gap average;
+    // g < 2^31 (gaps are clamped below 2^31 us), so g * Lambda < 2^43
+    const uint64_t key = __umul64hi((no_gap ? 0 : g) * kLambda, mg[t]) + t2[t];
     const uint64_t pk = pack_key(key, s);
     const uint32_t ea = c.turn_ev[2 * ti], ec = c.turn_ev[2 * ti + 1];
     c.pkey[ea] = pk;
