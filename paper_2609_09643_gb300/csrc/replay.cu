@@ -1277,7 +1277,7 @@ __global__ void __launch_bounds__(256) ttft_median_kernel(const ReplayDesc *desc
   const ReplayDesc &D = descs[blockIdx.x];
   __shared__ unsigned int hist[256];
   __shared__ unsigned long long red[8];
-  __shared__ unsigned int sel_digit;
+  __shared__ unsigned int sel_digit, sel_count;
   __shared__ unsigned long long sel_target;
   const uint64_t n = min((uint64_t)D.result->ttft_n, (uint64_t)D.n_turns);
   if (n == 0) {
@@ -1303,15 +1303,38 @@ __global__ void __launch_bounds__(256) ttft_median_kernel(const ReplayDesc *desc
       top = b;
       break;
     }
-  uint64_t target = (n - 1) / 2, prefix = 0, mask = 0;
+  // Once the values that share the selected prefix fit in shared memory, a
+  // global pass copies them there and the remaining passes read only those.
+  constexpr uint32_t kMedCap = 4096;
+  __shared__ unsigned long long cand[kMedCap];
+  __shared__ unsigned int ncand;
+  uint64_t target = (n - 1) / 2, prefix = 0, mask = 0, cnt = n;  // cnt: values matching the prefix
+  bool in_smem = false;
+  uint32_t m = 0;
   for (int b = top; b >= 0; b--) {
     for (uint32_t i = threadIdx.x; i < 256; i += blockDim.x) hist[i] = 0;
+    const bool copy = !in_smem && cnt <= kMedCap;
+    if (threadIdx.x == 0) ncand = 0;
     __syncthreads();
-    for (uint64_t i = threadIdx.x; i < n; i += blockDim.x) {
-      const uint64_t x = v[i];
-      if ((x & mask) == prefix) atomicAdd(&hist[(x >> (8 * b)) & 0xFF], 1u);
+    if (in_smem) {
+      for (uint32_t i = threadIdx.x; i < m; i += blockDim.x) {
+        const uint64_t x = cand[i];
+        if ((x & mask) == prefix) atomicAdd(&hist[(x >> (8 * b)) & 0xFF], 1u);
+      }
+    } else {
+      for (uint64_t i = threadIdx.x; i < n; i += blockDim.x) {
+        const uint64_t x = v[i];
+        if ((x & mask) == prefix) {
+          atomicAdd(&hist[(x >> (8 * b)) & 0xFF], 1u);
+          if (copy) cand[atomicAdd(&ncand, 1u)] = x;
+        }
+      }
     }
     __syncthreads();
+    if (copy) {
+      in_smem = true;
+      m = ncand;
+    }
     if (threadIdx.x == 0) {
       uint64_t cum = 0;
       uint32_t d = 0;
@@ -1321,11 +1344,13 @@ __global__ void __launch_bounds__(256) ttft_median_kernel(const ReplayDesc *desc
       }
       sel_digit = d < 256 ? d : 255;
       sel_target = target - cum;
+      sel_count = d < 256 ? hist[d] : 0;
     }
     __syncthreads();
     prefix |= (uint64_t)sel_digit << (8 * b);
     mask |= 0xFFull << (8 * b);
     target = sel_target;
+    cnt = sel_count;
     __syncthreads();
   }
   if (threadIdx.x == 0) D.result->ttft_p50_ns = prefix;
