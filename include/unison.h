@@ -358,6 +358,22 @@ int unison_attainment(const unison_trace *trace, const unison_decision *log_onli
                       const unison_decision *log_offline, uint64_t len_offline, const unison_decision *log_lru,
                       uint64_t len_lru, uint32_t n_points, unison_attainment_point *out);
 
+/* Device self-check of the division every score of eq. (t1) uses:
+ * floor(x / s) as the high word of x times a magic number (Granlund and
+ * Montgomery), for x < 2^43 and 2 <= s < 2^12.  Checks every divisor s in
+ * [2, 4095] at every x < 2^20 and at x = q*s - 1, q*s, q*s + s - 1 for 2^16
+ * quotients q per divisor spread up to the largest below 2^43, each against
+ * q*s <= x < (q+1)*s.  *mismatches (host) receives the number of failures;
+ * the call synchronises cuda_stream.  NULL mismatches: UNISON_ERR_ARG. */
+int unison_selftest_division(uint64_t *mismatches, void *cuda_stream);
+
+/* Fault injection for error-path tests (host side only): the next n device
+ * allocations the library makes -- a replay call's scratch, the ranking
+ * scratch when it grows, a trace's device block at its first upload -- fail
+ * as if the device were out of memory, and those calls return
+ * UNISON_ERR_OOM.  n <= 0 clears pending faults. */
+void unison_debug_fail_allocations(int n);
+
 /* ============================================================ hazard LUT */
 /* The survival table of eqs. (hazard), (hq), (survq) built on the device
  * from turns-per-session counts: n(t) = #{T_s >= t+1}, d(t) = #{T_s = t+1}

@@ -95,7 +95,8 @@ EXPORTS = ["unison_strerror", "unison_version", "unison_trace_create", "unison_t
            "unison_trace_upload", "unison_trace_free", "unison_trace_info", "unison_trace_device_bytes",
            "unison_replay_batch", "unison_stats", "unison_hazard_lut", "unison_rank_batch",
            "unison_profile_enable", "unison_profile_read", "unison_launch_count",
-           "unison_replay_batch_noalloc", "unison_ase", "unison_attainment"]
+           "unison_replay_batch_noalloc", "unison_ase", "unison_attainment", "unison_selftest_division",
+           "unison_debug_fail_allocations"]
 
 
 def lib_path() -> str:
@@ -135,6 +136,9 @@ def lib():
             L.unison_launch_count.restype = C.c_uint64
             L.unison_replay_batch_noalloc.argtypes = L.unison_replay_batch.argtypes
             L.unison_ase.argtypes = [C.POINTER(Stats), C.c_int, C.c_int, C.POINTER(C.c_double)]
+            L.unison_selftest_division.argtypes = [C.POINTER(C.c_uint64), C.c_void_p]
+            L.unison_debug_fail_allocations.argtypes = [C.c_int]
+            L.unison_debug_fail_allocations.restype = None
             L.unison_attainment.argtypes = [C.c_void_p, C.c_void_p, C.c_uint64, C.c_void_p, C.c_uint64,
                                             C.c_void_p, C.c_uint64, C.c_uint32, C.POINTER(AttainmentPoint)]
             _lib = L
@@ -323,6 +327,20 @@ def attainment(trace: Trace, logs, n_points: int) -> List[dict]:
         args += [a.ctypes.data, a.shape[0]]
     _check("unison_attainment", lib().unison_attainment(trace.handle, *args, n_points, out))
     return [{f: getattr(out[i], f) for f, _ in AttainmentPoint._fields_ if f != "reserved"} for i in range(n_points)]
+
+
+def selftest_division(stream=None) -> int:
+    """unison_selftest_division: mismatches of the scores' multiply-high
+    division against the quotient's definition (0 expected)."""
+    out = C.c_uint64()
+    _check("unison_selftest_division", lib().unison_selftest_division(C.byref(out), _stream_handle(stream)))
+    return int(out.value)
+
+
+def debug_fail_allocations(n: int) -> None:
+    """The next n device allocations of the library fail as out of memory
+    (fault injection for error-path tests; 0 clears)."""
+    lib().unison_debug_fail_allocations(int(n))
 
 
 def hazard_lut(turns_dev, bucket: int = 1, stream=None):

@@ -38,6 +38,10 @@ __host__ __device__ inline uint64_t magic_for(uint32_t s) {
   return m << (21 - l);
 }
 
+// Fault injection (unison_debug_fail_allocations): true, once per pending
+// fault, at a device allocation that should then fail as out of memory.
+bool unison_fault_alloc();
+
 __host__ __device__ __forceinline__ uint64_t pack_key(uint64_t key40, uint32_t id) {
   return (key40 << 24) | ((~id) & kIdMask);
 }

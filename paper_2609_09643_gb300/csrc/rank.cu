@@ -1512,7 +1512,7 @@ int scratch_acquire(cudaStream_t stream, size_t bytes, char **out) {
     e.first = nullptr;
     e.second = 0;
     char *p = nullptr;
-    if (cudaMallocAsync(reinterpret_cast<void **>(&p), bytes, stream) != cudaSuccess) {
+    if (unison_fault_alloc() || cudaMallocAsync(reinterpret_cast<void **>(&p), bytes, stream) != cudaSuccess) {
       cudaGetLastError();
       return UNISON_ERR_OOM;
     }

@@ -1702,7 +1702,7 @@ extern "C" int unison_replay_batch(const unison_trace *const *traces, int n_trac
   rc = plan_replays(traces, params, n_replays, smem_limit, results_dev == nullptr, P, off_res);
   if (rc != UNISON_OK) return rc;
   char *scratch = nullptr;
-  if (cudaMallocAsync(reinterpret_cast<void **>(&scratch), P.bytes, stream) != cudaSuccess) {
+  if (unison_fault_alloc() || cudaMallocAsync(reinterpret_cast<void **>(&scratch), P.bytes, stream) != cudaSuccess) {
     cudaGetLastError();
     return UNISON_ERR_OOM;
   }

@@ -253,7 +253,7 @@ extern "C" int unison_trace_upload(unison_trace *tr, void *cuda_stream) {
   if (cudaGetDevice(&dev) != cudaSuccess) return UNISON_ERR_CUDA;
   if (tr->d_block && tr->device != dev) return UNISON_ERR_ARG;
   if (!tr->d_block) {
-    if (cudaMalloc(&tr->d_block, tr->block_bytes) != cudaSuccess) {
+    if (unison_fault_alloc() || cudaMalloc(&tr->d_block, tr->block_bytes) != cudaSuccess) {
       cudaGetLastError();
       tr->d_block = nullptr;
       return UNISON_ERR_OOM;

@@ -450,3 +450,49 @@ def test_signal_flags_rejected(B):
         with pytest.raises(B.UnisonError) as ei:
             B.replay_batch(h, [q])
         assert ei.value.code == B.ERR_ARG, (pol, flags)
+
+
+# ---- library self-check and host-side fault injection -------------------------------
+
+def test_selftest_division(B):
+    """Every divisor 2..4095 at every x < 2^20 and at quotient boundaries up
+    to 2^43: the multiply-high division equals the quotient's definition."""
+    assert B.selftest_division() == 0
+
+
+def test_allocation_faults_return_oom(B):
+    """A failing device allocation (injected on the host) makes each call
+    return UNISON_ERR_OOM and leaves the library usable."""
+    import torch
+    tr, _ = tiny_case()
+    h = [B.Trace(tr).upload()]
+    params = [to_lib(base("spear_tide", 512 * MIB, 8 * GIB, 28672))]
+    ref, _ = B.replay_batch(h, params)
+    B.debug_fail_allocations(1)
+    with pytest.raises(B.UnisonError) as ei:
+        B.replay_batch(h, params)
+    assert ei.value.code == B.ERR_OOM
+    assert B.replay_batch(h, params)[0] == ref
+    # a trace's first upload
+    B.debug_fail_allocations(1)
+    t2 = B.Trace(tr)
+    with pytest.raises(B.UnisonError) as ei:
+        t2.upload()
+    assert ei.value.code == B.ERR_OOM
+    assert B.replay_batch([t2.upload()], params)[0] == ref
+    # the ranking scratch, when a new stream needs its own
+    _, sigma = oracle.hazard_lut(synth.geometric_turns(1, 1415, 23.7, 2, 200))
+    rec = synth.make_records(3, 5000)
+    p = dict(sigma_q=sigma, k=64, penalty_q=500_000_000, budget_bytes=4 << 30, kv_bytes_per_token=131072,
+             max_moves=64, free_fast_tok=0, free_hbm_tok=1 << 40)
+    dev = B.records_to_device(rec)
+    out = B.rank_outputs(rec.n, 64, 64)
+    s = torch.cuda.Stream()
+    B.debug_fail_allocations(1)
+    with pytest.raises(B.UnisonError) as ei:
+        B.rank_batch([dev], [p], [out], stream=s)
+    assert ei.value.code == B.ERR_OOM
+    B.rank_batch([dev], [p], [out], stream=s)
+    s.synchronize()
+    assert B.rank_result(out)["status"] == 0
+    B.debug_fail_allocations(0)
