@@ -496,3 +496,20 @@ def test_allocation_faults_return_oom(B):
     s.synchronize()
     assert B.rank_result(out)["status"] == 0
     B.debug_fail_allocations(0)
+
+
+def test_sweep_resume_on_device(B, tmp_path):
+    """A sweep interrupted after some rows and rerun equals one run straight
+    through, and its rows equal the oracle's results."""
+    from paper_2609_09643_gb300 import sweep
+    trs = {"tiny0": synth.tiny_trace(0), "tiny1": synth.tiny_trace(1)}
+    handles = {k: B.Trace(v).upload() for k, v in trs.items()}
+    ps = {pol: base(pol, 512 * MIB, 8 * GIB, 28672) for pol in ("lru", "spear", "spear_tide", "belady")}
+    jobs = [(k, to_lib(p)) for k in trs for p in ps.values()]
+    full = sweep.run_sweep(jobs, str(tmp_path / "full.jsonl"), sweep.replay_runner(handles), batch=8)
+    path = str(tmp_path / "rows.jsonl")
+    sweep.run_sweep(jobs[:3], path, sweep.replay_runner(handles), batch=2)
+    assert sweep.run_sweep(jobs, path, sweep.replay_runner(handles), batch=2) == full
+    for (k, q), r in zip(jobs, full):
+        pol = next(p for p in ps.values() if to_lib(p) == q)
+        assert r["decision_hash"] == oracle.replay(trs[k], to_oracle(pol))["decision_hash"]
