@@ -177,6 +177,16 @@ def test_global_list_path(B):
         assert_same(res[i], oracle.replay(tr, to_oracle(p)), i)
 
 
+def test_global_list_path_spear_tide_only(B):
+    """A global-memory launch whose replays are all SPEAR+TIDE runs the
+    kernel specialised for that policy."""
+    tr = synth.make_trace(3, np.full(6000, 4), 0.01, synth.GAP_MIX_CODING)
+    reps = [(0, base("spear_tide", cs, ch, 1024)) for cs, ch in ((1 << 60, 1 << 60), (400 * MIB, 4 * GIB))]
+    res, _, _ = run_gpu(B, [tr], reps)
+    for i, (_, p) in enumerate(reps):
+        assert_same(res[i], oracle.replay(tr, to_oracle(p)), i)
+
+
 def test_many_sessions_search_path(B):
     """More sessions than the shared-memory session map holds: residents are
     found by a warp-wide search."""
