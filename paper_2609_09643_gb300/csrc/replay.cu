@@ -35,6 +35,9 @@ namespace {
 
 constexpr uint32_t kFull = 0xFFFFFFFFu;
 constexpr uint32_t kTierNone = 0, kTierS = 1, kTierH = 2;
+// Per-session maps in shared memory beside the resident lists: none, the tier
+// byte and the pin slot, or the tier byte alone.
+constexpr uint32_t kMapNone = 0, kMapSlots = 1, kMapTier = 2;
 
 struct ComboDesc {
   const uint32_t *turn_ev;   // [2T]
@@ -70,7 +73,7 @@ struct ReplayDesc {
   uint32_t n_events, n_turns, n_sessions, policy;
   uint32_t max_sessions, kvb, ttl, load;
   uint32_t rcap_s, rcap_h;
-  uint32_t tmap;    // 1: a per-session tier byte follows the lists in shared memory
+  uint32_t tmap;    // kMapNone, kMapSlots (tier byte and pin slot per session) or kMapTier (tier byte)
   uint32_t bucket;  // hazard bucket width (online hazard replays)
   uint64_t penalty;  // P_Z in quantised units (online hazard replays)
   const uint64_t *t2;  // eq. (t2) per turn index of the offline table (stale-snapshot replays)
@@ -857,14 +860,16 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
     p += 2 * D.rcap_s;
     st.tmap = nullptr;
     st.pslot = nullptr;
-    if (!kGlobalLists && D.tmap) {
+    if (!kGlobalLists && D.tmap != kMapNone) {
       // tier map (1 B per session), then pin slots (2 B per session)
       st.tmap = reinterpret_cast<uint8_t *>(p);
       uint32_t *m32 = reinterpret_cast<uint32_t *>(p);
       for (uint32_t i = lane; i < (D.n_sessions + 3) / 4; i += 32) m32[i] = 0u;
-      st.pslot = reinterpret_cast<uint16_t *>(reinterpret_cast<unsigned char *>(p) + ((D.n_sessions + 15) & ~15u));
-      uint32_t *s32 = reinterpret_cast<uint32_t *>(st.pslot);
-      for (uint32_t i = lane; i < (D.n_sessions + 1) / 2; i += 32) s32[i] = 0xFFFFFFFFu;
+      if (kLean || D.tmap == kMapSlots) {
+        st.pslot = reinterpret_cast<uint16_t *>(reinterpret_cast<unsigned char *>(p) + ((D.n_sessions + 15) & ~15u));
+        uint32_t *s32 = reinterpret_cast<uint32_t *>(st.pslot);
+        for (uint32_t i = lane; i < (D.n_sessions + 1) / 2; i += 32) s32[i] = 0xFFFFFFFFu;
+      }
       __syncwarp();
     }
     if (kOnline) {
@@ -1419,8 +1424,10 @@ uint32_t list_cap(uint64_t cap_tok, const unison_trace *tr) {
 }
 
 // 16-byte entries: fast and HBM arrays, the pinned list (both tiers) and the
-// TIDE staging area (two fast-tier capacities).  A tier map of one byte per
-// session follows when the trace has at most kTierMapMax sessions.
+// TIDE staging area (two fast-tier capacities).  The tier map and pin slots
+// (3 B per session) follow when the trace has at most kTierMapMax sessions
+// and they fit; else the tier map alone (1 B per session) when the launch's
+// replays still run in as few waves of CTAs.
 constexpr uint32_t kTierMapMax = 32768;
 size_t list_bytes(uint32_t cs, uint32_t ch) { return 16ull * (4ull * cs + 2ull * ch); }
 
@@ -1439,6 +1446,49 @@ size_t online_bytes(uint32_t cs, uint32_t ch, uint32_t n_sessions) {
   return 16ull * (ring_size(cs) + ring_size(ch) + 3ull * cs + ch) + align_up(n, 16) + 2 * align_up(n, 8) +
          4 * align_up(n, 4) +
          2 * align_up(n, 8) + align_up(sizeof(OnlineTable), 16);
+}
+
+// The shared-memory replay kernel the plan launches, for a log or not.
+void (*smem_kernel(const ReplayPlan &P, bool logged))(const ReplayDesc *, const uint32_t *) {
+  return !P.smem_all_st              ? replay_kernel<false, kKeyStream, -1, false>
+         : (P.smem_lean && !logged) ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true>
+                                    : replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, false>;
+}
+
+// Waves of CTAs the shared-memory group needs with `dyn` bytes per CTA.
+uint64_t smem_waves(const ReplayPlan &P, size_t dyn) {
+  int dev = 0, sms = 0, nb = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const auto k = smem_kernel(P, true);
+  cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k, 32, dyn) != cudaSuccess || nb <= 0 || sms <= 0) {
+    cudaGetLastError();
+    return ~0ull;
+  }
+  const uint64_t slots = (uint64_t)nb * (uint64_t)sms;
+  return (P.in_smem.size() + slots - 1) / slots;
+}
+
+// Replays of the shared-memory group without a map take the tier map alone
+// (an arrival then searches only its own tier, and nothing on a miss) when it
+// fits and the group needs no more waves with it.
+void add_tier_maps(const unison_trace *const *traces, const unison_replay_params *params, size_t smem_limit,
+                   ReplayPlan &P) {
+  size_t with = P.max_smem;
+  std::vector<uint32_t> add;
+  for (uint32_t r : P.in_smem) {
+    if (P.tmap[r] != kMapNone) continue;
+    const unison_trace *tr = traces[params[r].trace_idx];
+    const size_t b = list_bytes(P.rcap_s[r], P.rcap_h[r]) + align_up(tr->n_sessions, 16);
+    if (b > smem_limit) continue;
+    add.push_back(r);
+    with = std::max(with, b);
+  }
+  if (add.empty()) return;
+  if (with > P.max_smem && smem_waves(P, with) > smem_waves(P, P.max_smem)) return;
+  for (uint32_t r : add) P.tmap[r] = kMapTier;
+  P.max_smem = with;
 }
 
 int plan_replays(const unison_trace *const *traces, const unison_replay_params *params, int n_replays,
@@ -1486,26 +1536,26 @@ int plan_replays(const unison_trace *const *traces, const unison_replay_params *
     const size_t lists = list_bytes(P.rcap_s[r], P.rcap_h[r]);
     // the tier map and pin slots (3 bytes per session) when they fit beside the lists
     const size_t map = align_up(tr->n_sessions, 16) + 2 * align_up(tr->n_sessions, 8);
-    P.tmap[r] = tr->n_sessions <= kTierMapMax && lists + map <= smem_limit;
+    P.tmap[r] = tr->n_sessions <= kTierMapMax && lists + map <= smem_limit ? kMapSlots : kMapNone;
     if (p.flags & UNISON_HAZARD_ONLINE) {
       // online hazard replays run from shared memory only
       const size_t ob = online_bytes(P.rcap_s[r], P.rcap_h[r], tr->n_sessions);
       if (tr->n_sessions > kTierMapMax || ob > smem_limit) return UNISON_ERR_RANGE;
-      P.tmap[r] = 1;
+      P.tmap[r] = kMapSlots;
       P.in_online.push_back((uint32_t)r);
       P.max_smem_online = std::max(P.max_smem_online, ob);
     } else if (p.stale_sync != UNISON_SYNC_LIVE) {
       // stale-snapshot replays too
       const size_t sb = stale_bytes(P.rcap_s[r], P.rcap_h[r], tr->n_sessions);
       if (tr->n_sessions > kTierMapMax || sb > smem_limit) return UNISON_ERR_RANGE;
-      P.tmap[r] = 1;
+      P.tmap[r] = kMapSlots;
       P.in_stale.push_back((uint32_t)r);
       P.max_smem_stale = std::max(P.max_smem_stale, sb);
     } else if (lists <= smem_limit) {
       P.in_smem.push_back((uint32_t)r);
-      P.max_smem = std::max<size_t>(P.max_smem, lists + (P.tmap[r] ? map : 0));
+      P.max_smem = std::max<size_t>(P.max_smem, lists + (P.tmap[r] == kMapSlots ? map : 0));
     } else {
-      P.tmap[r] = 0;
+      P.tmap[r] = kMapNone;
       P.in_global.push_back((uint32_t)r);
       P.off_glist[r] = off;
       off = align_up(off + lists, 256);
@@ -1513,10 +1563,9 @@ int plan_replays(const unison_trace *const *traces, const unison_replay_params *
     P.off_ttft[r] = off;
     off = align_up(off + 8 * (tr->n_turns + 1), 256);
   }
-  for (uint32_t r : P.in_smem) {
-    P.smem_all_st &= params[r].policy == UNISON_SPEAR_TIDE;
-    P.smem_lean &= P.tmap[r] && params[r].max_sessions == 0;
-  }
+  for (uint32_t r : P.in_smem) P.smem_all_st &= params[r].policy == UNISON_SPEAR_TIDE;
+  add_tier_maps(traces, params, smem_limit, P);
+  for (uint32_t r : P.in_smem) P.smem_lean &= P.tmap[r] == kMapSlots && params[r].max_sessions == 0;
   for (uint32_t r : P.in_global) P.global_all_st &= params[r].policy == UNISON_SPEAR_TIDE;
   off_res = 0;
   if (results_in_scratch) {
@@ -1627,9 +1676,7 @@ int launch_replays(const ReplayPlan &P, char *scratch, const std::vector<ComboDe
   {
     ProfSpan span(profile ? "replay" : "", stream);
     if (!P.in_smem.empty()) {
-      const auto k = !P.smem_all_st ? replay_kernel<false, kKeyStream, -1, false>
-                     : (P.smem_lean && !logged) ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true>
-                                                : replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, false>;
+      const auto k = smem_kernel(P, logged);
       ck(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P.max_smem));
       k<<<(unsigned)P.in_smem.size(), 32, P.max_smem, stream>>>(d_desc, d_order);
       count_launches(1);

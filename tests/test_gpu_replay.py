@@ -187,11 +187,15 @@ def test_global_list_path_spear_tide_only(B):
         assert_same(res[i], oracle.replay(tr, to_oracle(p)), i)
 
 
-def test_many_sessions_search_path(B):
-    """More sessions than the shared-memory session map holds: residents are
-    found by a warp-wide search."""
-    tr = synth.make_trace(4, np.full(20000, 3), 0.005, synth.GAP_MIX_GENERAL)
-    reps = [(0, base(pol, 2 * GIB, 16 * GIB, 16384)) for pol in ("spear_tide", "belady", "timeout")]
+@pytest.mark.parametrize("n_sessions", [20000, 40000, 240000])
+def test_many_sessions_paths(B, n_sessions):
+    """20,000 sessions: tier map and pin slots in shared memory.  40,000: the
+    tier map alone (completions scan the pinned list).  240,000: no map fits
+    beside the lists, so residents are found by a warp-wide search of both
+    tiers."""
+    tr = synth.make_trace(4, np.full(n_sessions, 3 if n_sessions < 100000 else 2), 0.005, synth.GAP_MIX_GENERAL)
+    pols = ("spear_tide", "belady", "timeout") if n_sessions < 100000 else ("spear_tide", "lru")
+    reps = [(0, base(pol, 2 * GIB, 16 * GIB, 16384)) for pol in pols]
     res, _, _ = run_gpu(B, [tr], reps)
     for i, (_, p) in enumerate(reps):
         assert_same(res[i], oracle.replay(tr, to_oracle(p)), p["policy"])
