@@ -69,6 +69,7 @@ def parse():
     ap.add_argument("--table", action="store_true",
                     help="per-config table instead of the bench line: GPU events/s, oracle 1-thread and all-core "
                          "events/s, parity, rank GB/s per live-set size")
+    ap.add_argument("--table-configs", default="01234", help="which configs the table covers (digits 0-4)")
     return ap.parse_args()
 
 
@@ -486,6 +487,74 @@ def _oracle_rank_job(job):
     return n
 
 
+def _large_trace_job(seed):
+    """One large-pool trace, generated in a worker process."""
+    import synth
+    return synth.large_pool_trace(seed)
+
+
+def _oracle_large_job(seed):
+    """One large-pool oracle replay in a worker (it generates its own trace)."""
+    import oracle
+    import synth
+    from cases import large_pool_params, to_oracle
+    return oracle.replay(synth.large_pool_trace(seed), to_oracle(large_pool_params()))
+
+
+def large_pool_table(B, pool, stream, fields, cores):
+    """Config 3 at full size: 256 replays (seeds 100-355) in one launch, each
+    on its own 65,536-session trace; every replay checked against the oracle.
+    Traces are generated in the worker pool and their handles built on host
+    threads, so the parent never holds more than the pinned upload copies."""
+    from concurrent.futures import ThreadPoolExecutor
+    import torch
+    from cases import large_pool_params, to_lib, to_oracle
+    import oracle
+    import synth
+    seeds = list(range(100, 356))
+    with ThreadPoolExecutor(cores) as ex:
+        futs = [ex.submit(lambda t: B.Trace(t), tr) for tr in pool.imap(_large_trace_job, seeds, chunksize=1)]
+        handles = [f.result() for f in futs]
+    for h in handles:
+        h.upload(stream)
+    ev = sum(2 * h.info()[1] for h in handles)
+    params = [to_lib(large_pool_params(), i) for i in range(len(seeds))]
+    res_dev = torch.zeros(B.result_nbytes(len(params)), dtype=torch.uint8, device="cuda")
+    B.replay_batch_async(handles, params, res_dev, stream=stream)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    steps = 2
+    a.record(stream)
+    for _ in range(steps):
+        B.replay_batch_async(handles, params, res_dev, stream=stream)
+    b.record(stream)
+    torch.cuda.synchronize()
+    gpu = ev * steps / (a.elapsed_time(b) / 1e3)
+    res = B.results_from_tensor(res_dev)
+    del handles, res_dev
+    spent, ev1, n1 = 0.0, 0, 0
+    for sd in seeds:
+        tr = synth.large_pool_trace(sd)
+        t0 = time.perf_counter()
+        ev1 += oracle.replay(tr, to_oracle(large_pool_params()))["events"]
+        spent += time.perf_counter() - t0
+        n1 += 1
+        if spent > 10.0:
+            break
+    one = ev1 / spent
+    t0 = time.perf_counter()
+    ores = pool.map(_oracle_large_job, seeds, chunksize=1)
+    allc = sum(r["events"] for r in ores) / (time.perf_counter() - t0)
+    bad = [sd for sd, r, g in zip(seeds, ores, res) if any(g[f] != r[f] for f in fields)]
+    return {"config": "3 large pool (256 replays, seeds 100-355)", "replays": len(seeds), "events_per_launch": ev,
+            "gpu_events_per_s": gpu, "oracle_1core_events_per_s": one,
+            "oracle_1core_sample": f"{n1} replays",
+            "oracle_allcore_events_per_s": allc,
+            "oracle_allcore_sample": "all 256 (each worker generates its trace inside the timed region)",
+            "cores": cores,
+            "parity": f"{len(seeds) - len(bad)}/{len(seeds)} replays identical" + (f", differ: {bad[:5]}" if bad else "")}
+
+
 def config_table(args):
     """Configs 0-3 (replays) and 4 (ranking): device events/s of one batched
     launch (CUDA events, warm), the oracle on one core and on all host cores
@@ -505,13 +574,10 @@ def config_table(args):
     stream = torch.cuda.current_stream()
     tr0, ps0 = tiny_case()
     trs2, reps2 = sweep_case()
-    n_large = 16
     cfgs = [("0 tiny", [tr0], [(0, p) for p in ps0], 50, "all 4"),
             ("1 paper-scale", *paper_scale_case(), 10, "all 30"),
-            ("2 sweep", trs2, reps2, 5, "32 replays spread over the 1,024"),
-            (f"3 large pool ({n_large} of the 256 replays, seeds 100-{99 + n_large})",
-             [synth.large_pool_trace(100 + i) for i in range(n_large)],
-             [(i, large_pool_params()) for i in range(n_large)], 2, f"all {n_large}")]
+            ("2 sweep", trs2, reps2, 5, "32 replays spread over the 1,024")]
+    cfgs = [c for c in cfgs if c[0][0] in args.table_configs]
     fields = ["events", "req_warm", "hit_s", "hit_h", "miss", "evict", "demote", "promote", "tide_demote",
               "tok_computed", "ttft_sum", "ttft_p50_ns", "decision_hash", "status"]
     out = []
@@ -550,6 +616,13 @@ def config_table(args):
                     "oracle_allcore_events_per_s": allc, "oracle_allcore_sample": sample, "cores": cores,
                     "parity": f"{len(pick) - len(bad)}/{len(pick)} replays identical" + (f", differ: {bad[:5]}" if bad else "")})
         del handles, res_dev
+    if "3" in args.table_configs:
+        out.append(large_pool_table(B, pool, stream, fields, cores))
+    pk = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))).get("hbm_gbs") or 6800.0
+    if "4" not in args.table_configs:
+        pool.close()
+        print(json.dumps({"table": out, "peak_hbm_gbs": pk}), flush=True)
+        return
     # config 4: the ranking at each live-set size (device), the oracle on 2^22 records
     rec, tps = rank_workload()
     tps_dev = torch.tensor(tps.astype("int32"), device="cuda")
@@ -564,7 +637,6 @@ def config_table(args):
     n = sum(pool.map(_oracle_rank_job, [(rec, sigma, 1 << 22)] * cores, chunksize=1))
     allc = n * RANK_BYTES_PER_RECORD / (time.perf_counter() - t0) / 1e9
     pool.close()
-    pk = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))).get("hbm_gbs") or 6800.0
     out.append({"config": "4 rank", "gpu": [{"n": e["n"], "sets": e["sets_per_call"], "call_gbs": e["call_gbs"],
                                             "call_frac": e["call_gbs"] / pk, "filter_gbs": e["filter_gbs"],
                                             "filter_frac": e["filter_gbs"] / pk if e["filter_gbs"] else None}
