@@ -251,7 +251,13 @@ typedef struct {
  * without one signal), stale_sync (decisions on a register-file snapshot).
  * Replays of one call may mix policies and variants; each runs in the
  * launch for its kind, and a launch whose replays share the policy and
- * simple settings runs a kernel specialised for them.
+ * simple settings runs a kernel specialised for them.  SPEAR+TIDE replays
+ * always run in their own launch.  The launches of one call are independent
+ * and run concurrently: the first on cuda_stream, the others on side
+ * streams the library owns (one set per device, made on the first call that
+ * needs them), forked from cuda_stream and joined back to it before the
+ * call's last kernel.  The call's work therefore stays ordered on
+ * cuda_stream, and a stream capture of cuda_stream captures all of it.
  *
  * traces[n_traces]: uploaded handles (host array of pointers).
  * params[n_replays]: host array.

@@ -1409,10 +1409,13 @@ struct ReplayPlan {
   std::vector<int> replay_combo;
   size_t off_desc = 0, off_order = 0, off_combo = 0, bytes = 0;
   std::vector<size_t> off_lut, off_stream, off_ttft, off_glist;
-  std::vector<uint32_t> rcap_s, rcap_h, in_smem, in_global, in_online, in_stale, tmap;
-  size_t max_smem = 0, max_smem_online = 0, max_smem_stale = 0;
-  bool smem_all_st = true, global_all_st = true;  // every replay of the group is SPEAR+TIDE
-  bool smem_lean = true;  // ... and has the tier map and no slot limit (the log is per call)
+  // Replay groups, one kernel launch each: lists in shared memory (SPEAR+TIDE,
+  // other policies), in global memory (the same split), online hazard table,
+  // stale snapshot.  The launches are independent and run concurrently.
+  std::vector<uint32_t> in_st, in_mix, in_gst, in_gmix, in_online, in_stale;
+  std::vector<uint32_t> rcap_s, rcap_h, tmap;
+  size_t max_smem_st = 0, max_smem_mix = 0, max_smem_online = 0, max_smem_stale = 0;
+  bool st_lean = true;  // every shared-memory SPEAR+TIDE replay has the map with pin slots and no slot limit
 };
 
 // Resident-list capacity of a tier: at most one entry per session and no more
@@ -1448,36 +1451,36 @@ size_t online_bytes(uint32_t cs, uint32_t ch, uint32_t n_sessions) {
          2 * align_up(n, 8) + align_up(sizeof(OnlineTable), 16);
 }
 
-// The shared-memory replay kernel the plan launches, for a log or not.
-void (*smem_kernel(const ReplayPlan &P, bool logged))(const ReplayDesc *, const uint32_t *) {
-  return !P.smem_all_st              ? replay_kernel<false, kKeyStream, -1, false>
-         : (P.smem_lean && !logged) ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true>
-                                    : replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, false>;
+using ReplayKernel = void (*)(const ReplayDesc *, const uint32_t *);
+
+// The kernel of the shared-memory SPEAR+TIDE group, for a log or not.
+ReplayKernel st_kernel(const ReplayPlan &P, bool logged) {
+  return P.st_lean && !logged ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true>
+                              : replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, false>;
 }
 
-// Waves of CTAs the shared-memory group needs with `dyn` bytes per CTA.
-uint64_t smem_waves(const ReplayPlan &P, size_t dyn) {
+// Waves of CTAs a group of n replays needs with `dyn` bytes per CTA.
+uint64_t smem_waves(ReplayKernel k, size_t n, size_t dyn) {
   int dev = 0, sms = 0, nb = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const auto k = smem_kernel(P, true);
   cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, k, 32, dyn) != cudaSuccess || nb <= 0 || sms <= 0) {
     cudaGetLastError();
     return ~0ull;
   }
   const uint64_t slots = (uint64_t)nb * (uint64_t)sms;
-  return (P.in_smem.size() + slots - 1) / slots;
+  return (n + slots - 1) / slots;
 }
 
-// Replays of the shared-memory group without a map take the tier map alone
-// (an arrival then searches only its own tier, and nothing on a miss) when it
+// Replays of a shared-memory group without a map take the tier map alone (an
+// arrival then searches only its own tier, and nothing on a miss) when it
 // fits and the group needs no more waves with it.
 void add_tier_maps(const unison_trace *const *traces, const unison_replay_params *params, size_t smem_limit,
-                   ReplayPlan &P) {
-  size_t with = P.max_smem;
+                   const std::vector<uint32_t> &group, ReplayKernel k, size_t &max_smem, ReplayPlan &P) {
+  size_t with = max_smem;
   std::vector<uint32_t> add;
-  for (uint32_t r : P.in_smem) {
+  for (uint32_t r : group) {
     if (P.tmap[r] != kMapNone) continue;
     const unison_trace *tr = traces[params[r].trace_idx];
     const size_t b = list_bytes(P.rcap_s[r], P.rcap_h[r]) + align_up(tr->n_sessions, 16);
@@ -1486,9 +1489,9 @@ void add_tier_maps(const unison_trace *const *traces, const unison_replay_params
     with = std::max(with, b);
   }
   if (add.empty()) return;
-  if (with > P.max_smem && smem_waves(P, with) > smem_waves(P, P.max_smem)) return;
+  if (with > max_smem && smem_waves(k, group.size(), with) > smem_waves(k, group.size(), max_smem)) return;
   for (uint32_t r : add) P.tmap[r] = kMapTier;
-  P.max_smem = with;
+  max_smem = with;
 }
 
 int plan_replays(const unison_trace *const *traces, const unison_replay_params *params, int n_replays,
@@ -1552,21 +1555,23 @@ int plan_replays(const unison_trace *const *traces, const unison_replay_params *
       P.in_stale.push_back((uint32_t)r);
       P.max_smem_stale = std::max(P.max_smem_stale, sb);
     } else if (lists <= smem_limit) {
-      P.in_smem.push_back((uint32_t)r);
-      P.max_smem = std::max<size_t>(P.max_smem, lists + (P.tmap[r] == kMapSlots ? map : 0));
+      const bool st = p.policy == UNISON_SPEAR_TIDE;
+      (st ? P.in_st : P.in_mix).push_back((uint32_t)r);
+      size_t &m = st ? P.max_smem_st : P.max_smem_mix;
+      m = std::max<size_t>(m, lists + (P.tmap[r] == kMapSlots ? map : 0));
     } else {
       P.tmap[r] = kMapNone;
-      P.in_global.push_back((uint32_t)r);
+      (p.policy == UNISON_SPEAR_TIDE ? P.in_gst : P.in_gmix).push_back((uint32_t)r);
       P.off_glist[r] = off;
       off = align_up(off + lists, 256);
     }
     P.off_ttft[r] = off;
     off = align_up(off + 8 * (tr->n_turns + 1), 256);
   }
-  for (uint32_t r : P.in_smem) P.smem_all_st &= params[r].policy == UNISON_SPEAR_TIDE;
-  add_tier_maps(traces, params, smem_limit, P);
-  for (uint32_t r : P.in_smem) P.smem_lean &= P.tmap[r] == kMapSlots && params[r].max_sessions == 0;
-  for (uint32_t r : P.in_global) P.global_all_st &= params[r].policy == UNISON_SPEAR_TIDE;
+  add_tier_maps(traces, params, smem_limit, P.in_st, st_kernel(P, true), P.max_smem_st, P);
+  add_tier_maps(traces, params, smem_limit, P.in_mix, replay_kernel<false, kKeyStream, -1, false>, P.max_smem_mix,
+                P);
+  for (uint32_t r : P.in_st) P.st_lean &= P.tmap[r] == kMapSlots && params[r].max_sessions == 0;
   off_res = 0;
   if (results_in_scratch) {
     off_res = off;
@@ -1641,10 +1646,42 @@ void fill_descs(const unison_trace *const *traces, const unison_replay_params *p
     d.stale_m = p.stale_m;
   }
   order.clear();
-  order.insert(order.end(), P.in_smem.begin(), P.in_smem.end());
-  order.insert(order.end(), P.in_global.begin(), P.in_global.end());
-  order.insert(order.end(), P.in_online.begin(), P.in_online.end());
-  order.insert(order.end(), P.in_stale.begin(), P.in_stale.end());
+  for (const auto *g : {&P.in_st, &P.in_mix, &P.in_gst, &P.in_gmix, &P.in_online, &P.in_stale})
+    order.insert(order.end(), g->begin(), g->end());
+}
+
+// Side streams for the replay groups of one call, one set per device, made
+// on first use.  The caller holds the lock while it forks and joins, so two
+// host threads never interleave their events.
+constexpr int kSideStreams = 5;
+struct SideStreams {
+  cudaStream_t s[kSideStreams] = {};
+  cudaEvent_t fork = nullptr, join[kSideStreams] = {};
+  bool ready = false;
+};
+std::mutex g_side_mu;
+SideStreams g_side[64];
+
+SideStreams *side_streams(std::unique_lock<std::mutex> &hold) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  hold = std::unique_lock<std::mutex>(g_side_mu);
+  SideStreams &g = g_side[dev];
+  if (!g.ready) {
+    bool ok = cudaEventCreateWithFlags(&g.fork, cudaEventDisableTiming) == cudaSuccess;
+    for (int i = 0; ok && i < kSideStreams; i++)
+      ok = cudaStreamCreateWithFlags(&g.s[i], cudaStreamNonBlocking) == cudaSuccess &&
+           cudaEventCreateWithFlags(&g.join[i], cudaEventDisableTiming) == cudaSuccess;
+    if (!ok) {
+      cudaGetLastError();
+      return nullptr;  // the handles made so far are kept for the next try
+    }
+    g.ready = true;
+  }
+  return &g;
 }
 
 // Queue the kernels of a planned batch on `stream`.
@@ -1675,35 +1712,48 @@ int launch_replays(const ReplayPlan &P, char *scratch, const std::vector<ComboDe
   }
   {
     ProfSpan span(profile ? "replay" : "", stream);
-    if (!P.in_smem.empty()) {
-      const auto k = smem_kernel(P, logged);
-      ck(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P.max_smem));
-      k<<<(unsigned)P.in_smem.size(), 32, P.max_smem, stream>>>(d_desc, d_order);
-      count_launches(1);
-      ck(cudaGetLastError());
+    // one launch per non-empty group, in the order of `order`
+    struct Launch {
+      ReplayKernel k;
+      size_t n, smem;
+    };
+    const Launch all[] = {
+        {st_kernel(P, logged), P.in_st.size(), P.max_smem_st},
+        {replay_kernel<false, kKeyStream, -1, false>, P.in_mix.size(), P.max_smem_mix},
+        {replay_kernel<true, kKeyStream, UNISON_SPEAR_TIDE, false>, P.in_gst.size(), 0},
+        {replay_kernel<true, kKeyStream, -1, false>, P.in_gmix.size(), 0},
+        {replay_kernel<false, kKeyOnline, -1, false>, P.in_online.size(), P.max_smem_online},
+        {replay_kernel<false, kKeyStale, -1, false>, P.in_stale.size(), P.max_smem_stale}};
+    std::vector<Launch> ls;
+    std::vector<size_t> first;
+    size_t off = 0;
+    for (const Launch &l : all) {
+      if (l.n) {
+        ls.push_back(l);
+        first.push_back(off);
+      }
+      off += l.n;
     }
-    if (!P.in_global.empty()) {
-      const auto k = P.global_all_st ? replay_kernel<true, kKeyStream, UNISON_SPEAR_TIDE, false>
-                                     : replay_kernel<true, kKeyStream, -1, false>;
-      k<<<(unsigned)P.in_global.size(), 32, 0, stream>>>(d_desc, d_order + P.in_smem.size());
-      count_launches(1);
-      ck(cudaGetLastError());
+    // the first group runs on the caller's stream, the others on side
+    // streams forked from it and joined back before the TTFT medians
+    std::unique_lock<std::mutex> hold;
+    SideStreams *side = nullptr;
+    if (ls.size() > 1) {
+      side = side_streams(hold);
+      if (!side) rc = UNISON_ERR_CUDA;
+      if (side) ck(cudaEventRecord(side->fork, stream));
     }
-    if (!P.in_online.empty()) {
-      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyOnline, -1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)P.max_smem_online));
-      replay_kernel<false, kKeyOnline, -1, false><<<(unsigned)P.in_online.size(), 32, P.max_smem_online, stream>>>(
-          d_desc, d_order + P.in_smem.size() + P.in_global.size());
+    for (size_t i = 0; i < ls.size() && rc == UNISON_OK; i++) {
+      cudaStream_t s = i == 0 ? stream : side->s[i - 1];
+      if (i > 0) ck(cudaStreamWaitEvent(s, side->fork, 0));
+      if (ls[i].smem) ck(cudaFuncSetAttribute(ls[i].k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ls[i].smem));
+      ls[i].k<<<(unsigned)ls[i].n, 32, ls[i].smem, s>>>(d_desc, d_order + first[i]);
       count_launches(1);
       ck(cudaGetLastError());
-    }
-    if (!P.in_stale.empty()) {
-      ck(cudaFuncSetAttribute(replay_kernel<false, kKeyStale, -1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              (int)P.max_smem_stale));
-      replay_kernel<false, kKeyStale, -1, false><<<(unsigned)P.in_stale.size(), 32, P.max_smem_stale, stream>>>(
-          d_desc, d_order + P.in_smem.size() + P.in_global.size() + P.in_online.size());
-      count_launches(1);
-      ck(cudaGetLastError());
+      if (i > 0) {
+        ck(cudaEventRecord(side->join[i - 1], s));
+        ck(cudaStreamWaitEvent(stream, side->join[i - 1], 0));
+      }
     }
   }
   {
