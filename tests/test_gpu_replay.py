@@ -187,6 +187,32 @@ def test_global_list_path_spear_tide_only(B):
         assert_same(res[i], oracle.replay(tr, to_oracle(p)), i)
 
 
+def test_all_six_launch_groups_in_one_call(B):
+    """One call with a replay in every launch group (SPEAR+TIDE and other
+    policies with lists in shared and in global memory, online table, stale
+    snapshot): the groups run concurrently on forked streams, and each replay
+    must still equal the oracle, with full decision logs."""
+    big = synth.make_trace(3, np.full(6000, 4), 0.01, synth.GAP_MIX_CODING)
+    small = synth.paper_scale_trace(2, "general")
+    reps = [(0, base("spear_tide", 1 << 60, 1 << 60, 1024)),            # global, SPEAR+TIDE
+            (0, base("lru", 1 << 60, 1 << 60, 1024)),                   # global, other
+            (1, base("spear_tide", 2 * GIB, 32 * GIB, 131072)),         # shared, SPEAR+TIDE
+            (1, base("belady", 2 * GIB, 32 * GIB, 131072)),             # shared, other
+            (1, base("spear_tide", 2 * GIB, 32 * GIB, 131072, online=True)),
+            (1, base("spear", 2 * GIB, 32 * GIB, 131072, stale="arrivals", stale_m=3))]
+    cap = 8 * max(big.n_events, small.n_events)
+    trs = [big, small]
+    res, log, _ = run_gpu(B, trs, reps, log_capacity=cap)
+    for i, (ti, p) in enumerate(reps):
+        o = oracle.replay(trs[ti], to_oracle(p), log=True)
+        assert_same(res[i], o, i)
+        assert_same_log(B, log[i], res[i], o, i)
+    # the same replays one per call give the same results
+    for i, (ti, p) in enumerate(reps):
+        one, _, _ = run_gpu(B, [trs[ti]], [(0, p)])
+        assert_same(one[0], res[i], i)
+
+
 @pytest.mark.parametrize("n_sessions", [20000, 40000, 240000])
 def test_many_sessions_paths(B, n_sessions):
     """20,000 sessions: tier map and pin slots in shared memory.  40,000: the
