@@ -1671,13 +1671,15 @@ SideStreams *side_streams(std::unique_lock<std::mutex> &hold) {
   hold = std::unique_lock<std::mutex>(g_side_mu);
   SideStreams &g = g_side[dev];
   if (!g.ready) {
-    bool ok = cudaEventCreateWithFlags(&g.fork, cudaEventDisableTiming) == cudaSuccess;
-    for (int i = 0; ok && i < kSideStreams; i++)
-      ok = cudaStreamCreateWithFlags(&g.s[i], cudaStreamNonBlocking) == cudaSuccess &&
-           cudaEventCreateWithFlags(&g.join[i], cudaEventDisableTiming) == cudaSuccess;
+    // handles made by an earlier, failed try are kept and not made again
+    bool ok = g.fork || cudaEventCreateWithFlags(&g.fork, cudaEventDisableTiming) == cudaSuccess;
+    for (int i = 0; ok && i < kSideStreams; i++) {
+      ok = g.s[i] || cudaStreamCreateWithFlags(&g.s[i], cudaStreamNonBlocking) == cudaSuccess;
+      ok = ok && (g.join[i] || cudaEventCreateWithFlags(&g.join[i], cudaEventDisableTiming) == cudaSuccess);
+    }
     if (!ok) {
       cudaGetLastError();
-      return nullptr;  // the handles made so far are kept for the next try
+      return nullptr;
     }
     g.ready = true;
   }

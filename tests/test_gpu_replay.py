@@ -213,6 +213,45 @@ def test_all_six_launch_groups_in_one_call(B):
         assert_same(one[0], res[i], i)
 
 
+def test_mixed_calls_from_two_host_threads(B):
+    """Two host threads issue mixed-policy calls (which fork onto the
+    library's side streams) on their own streams at the same time; every
+    call's results equal those of a call made alone."""
+    import threading
+    import torch
+    tr = synth.paper_scale_trace(6, "coding")
+    h = B.Trace(tr).upload()
+    reps = [base(pol, 2 * GIB, 32 * GIB, 131072) for pol in ("spear_tide", "lru", "belady", "spear")]
+    params = [to_lib(p) for p in reps]
+    ref, _ = B.replay_batch([h], params)
+    torch.cuda.synchronize()
+    got, errs = [[], []], []
+
+    def worker(k):
+        try:
+            s = torch.cuda.Stream()
+            for _ in range(4):
+                with torch.cuda.stream(s):  # the buffer is zeroed on s, before the call
+                    out = torch.zeros(B.result_nbytes(len(params)), dtype=torch.uint8, device="cuda")
+                B.replay_batch_async([h], params, out, stream=s)
+                s.synchronize()
+                got[k].append(B.results_from_tensor(out))
+        except Exception as e:  # reported on the main thread
+            errs.append(e)
+
+    ts = [threading.Thread(target=worker, args=(k,)) for k in range(2)]
+    for t in ts:
+        t.start()
+    for t in ts:
+        t.join()
+    assert not errs, errs
+    for k in range(2):
+        assert len(got[k]) == 4
+        for res in got[k]:
+            for i in range(len(params)):
+                assert_same(res[i], ref[i], (k, i))
+
+
 @pytest.mark.parametrize("n_sessions", [20000, 40000, 240000])
 def test_many_sessions_paths(B, n_sessions):
     """20,000 sessions: tier map and pin slots in shared memory.  40,000: the
