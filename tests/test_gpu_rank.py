@@ -228,3 +228,6 @@ def test_rank_rejects_bad_args(B, sigma):
     off = dict(d, gap_q=d["gap_q"][1:])  # misaligned
     with pytest.raises(B.UnisonError):
         B.rank_batch([off], [prm(sigma)], [B.rank_outputs(99, 1024, 1024)])
+    empty = {k: v[:0] for k, v in d.items()}  # a live set needs at least one record
+    with pytest.raises(B.UnisonError):
+        B.rank_batch([empty], [prm(sigma)], [B.rank_outputs(1, 1024, 1024)])

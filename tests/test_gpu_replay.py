@@ -266,6 +266,22 @@ def test_many_sessions_paths(B, n_sessions):
         assert_same(res[i], oracle.replay(tr, to_oracle(p)), p["policy"])
 
 
+def test_degenerate_traces(B):
+    """One session with one turn; one session with the most turns a session
+    may have (65,535, spanning 40 hours of 32-bit wrapping microseconds);
+    every policy at tight, unbounded and zero capacities; and a call with no
+    replays."""
+    trs = [synth.make_trace(21, np.array([1]), 0.01, synth.GAP_MIX_CODING),
+           synth.make_trace(22, np.array([65535]), 0.01, synth.GAP_MIX_CODING)]
+    reps = [(ti, base(pol, cs, ch, 28672)) for ti in range(2) for cs, ch in
+            ((512 * MIB, 8 * GIB), (1 << 60, 1 << 60), (0, 0)) for pol in POLS]
+    res, _, handles = run_gpu(B, trs, reps)
+    for i, (ti, p) in enumerate(reps):
+        assert_same(res[i], oracle.replay(trs[ti], to_oracle(p)), (ti, p["policy"], p["cap_s"]))
+    none, _ = B.replay_batch(handles, [])
+    assert none == []
+
+
 def test_log_overflow_reported(B):
     tr, _ = tiny_case()
     p = base("spear_tide", 512 * MIB, 8 * GIB, 28672)
