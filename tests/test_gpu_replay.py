@@ -282,6 +282,53 @@ def test_degenerate_traces(B):
     assert none == []
 
 
+def _random_replays(rng, n_traces, n):
+    """n replays with every parameter drawn at random within its valid range:
+    policy, capacities from zero to unbounded, KV size, DMA rate, TTL, TTFT
+    load, EMA weight, hazard bucket, P_Z, slot limit, and the variants (online
+    table, stale snapshot, a signal left out) where the policy allows them."""
+    reps = []
+    for _ in range(n):
+        pol = str(rng.choice(POLS))
+        kvb = int(rng.choice([1, 1024, 16384, 28672, 131072, 163840, 1 << 24]))
+        cap = lambda: int(rng.choice([0, 1, 64 * MIB, 512 * MIB, 2 * GIB, 16 * GIB, 1 << 60]))
+        den = int(rng.choice([1, 2, 5, 10, 33, 4095, 4096, 1 << 20]))
+        kw = dict(ema_num=int(rng.integers(0, den + 1)), ema_den=den, bucket=int(rng.choice([1, 2, 3, 8, 60])),
+                  penalty=int(rng.choice([0, 1, 500_000_000, (1 << 32) - 1])),
+                  ttl=int(rng.choice([0, 1, 2_000_000, (1 << 31) - 1, 0xFFFFFFFF])),
+                  dma=int(rng.choice([0, 1, 64_000, (1 << 32) - 1])), load=int(rng.choice([1, 4, 1000])),
+                  max_sessions=int(rng.choice([0, 0, 0, 1, 3, 40])))
+        if pol in ("spear", "spear_tide"):
+            v = int(rng.integers(0, 5))
+            if v == 1:
+                kw["online"] = True
+            elif v == 2:
+                kw["stale"] = str(rng.choice(["event", "arrivals", "gap_start"]))
+                kw["stale_m"] = int(rng.integers(1, 9))
+            elif v == 3:
+                kw["no_gap"] = True
+            elif v == 4:
+                kw["no_hazard"] = bool(rng.integers(0, 2))
+                kw["no_gap"] = not kw["no_hazard"]
+        reps.append((int(rng.integers(0, n_traces)), base(pol, cap(), cap(), kvb, **kw)))
+    return reps
+
+
+@pytest.mark.parametrize("seed", [20261202, 7, 99])
+def test_random_parameters_one_call(B, seed):
+    """240 replays with random parameters over four small traces of both gap
+    mixes, all in one call (every launch group at once): each replay equals
+    the oracle in every counter and its decision hash."""
+    rng = np.random.default_rng(seed)
+    shapes = ((40, synth.GAP_MIX_CODING), (150, synth.GAP_MIX_GENERAL), (400, synth.GAP_MIX_CODING),
+              (90, synth.GAP_MIX_GENERAL))
+    trs = [synth.make_trace(40 + i, rng.integers(1, 40, size=n), 0.5, mix) for i, (n, mix) in enumerate(shapes)]
+    reps = _random_replays(rng, len(trs), 240)
+    res, _, _ = run_gpu(B, trs, reps)
+    for i, (ti, p) in enumerate(reps):
+        assert_same(res[i], oracle.replay(trs[ti], to_oracle(p)), (i, ti, p))
+
+
 def test_log_overflow_reported(B):
     tr, _ = tiny_case()
     p = base("spear_tide", 512 * MIB, 8 * GIB, 28672)
