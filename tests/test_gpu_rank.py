@@ -231,3 +231,35 @@ def test_rank_rejects_bad_args(B, sigma):
     empty = {k: v[:0] for k, v in d.items()}  # a live set needs at least one record
     with pytest.raises(B.UnisonError):
         B.rank_batch([empty], [prm(sigma)], [B.rank_outputs(1, 1024, 1024)])
+
+
+@pytest.mark.parametrize("seed", [1, 2, 3])
+def test_random_sets_and_parameters(B, seed):
+    """Ten live sets per call with random sizes (1 to 2^20 records), random
+    shares of pinned, completed and fast-tier records, gap averages with many
+    ties, and random k, move limit, DMA budget, free space, P_Z, KV size and
+    hazard table: victims, fill and moved bytes equal the oracle's."""
+    rng = np.random.default_rng(1000 + seed)
+    recs, ps = [], []
+    for j in range(10):
+        n = int(rng.choice([1, 3, 100, 2047, 4097, 30000, 200000, 1 << 20]))
+        base = synth.make_records(100 * seed + j, n)
+        u = rng.random(n)
+        p_pin, p_done = rng.choice([0.0, 1 / 64, 0.3]), rng.choice([0.0, 0.05, 0.5])
+        flags = np.where(u < p_pin, 1, np.where(u < p_pin + p_done, 2, 0)).astype(np.uint8)
+        tier = np.where(rng.random(n) < rng.choice([0.0, 1 / 16, 0.5, 1.0]), 1, 2).astype(np.uint8)
+        tier[rng.random(n) < rng.choice([0.0, 0.1])] = 0
+        gap = base.gap_q.astype(np.int64)
+        if rng.random() < 0.5:  # coarse gaps: many equal keys, ties broken by index
+            gap = (gap // 1_000_000) * 1_000_000
+        gap = np.clip(gap, 0, (1 << 31) - 1).astype(np.uint32)
+        recs.append(synth.Records(gap, base.last_ret, base.turn, base.kv_tok, tier, flags))
+        sig = rng.integers(41, 4096, size=51).astype(np.uint16)
+        ps.append(dict(sigma_q=sig, k=int(rng.integers(0, 4097)), penalty_q=int(rng.integers(0, 1 << 32)),
+                       budget_bytes=int(rng.choice([0, 1 << 30, 1 << 36, 1 << 40, 1 << 44, (1 << 63) + 5])),
+                       kv_bytes_per_token=int(rng.choice([1, 1024, 28672, 131072, 1 << 24])),
+                       max_moves=int(rng.integers(0, 4097)),
+                       free_fast_tok=int(rng.choice([0, 1000, 1 << 20, (1 << 64) - 1])),
+                       free_hbm_tok=int(rng.choice([0, 5000, 1 << 40, (1 << 64) - 1]))))
+    for r, rec, p in zip(run(B, recs, ps), recs, ps):
+        check(r, rec, p)
