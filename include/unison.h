@@ -257,7 +257,8 @@ typedef struct {
  * streams the library owns (one set per device, made on the first call that
  * needs them), forked from cuda_stream and joined back to it before the
  * call's last kernel.  The call's work therefore stays ordered on
- * cuda_stream, and a stream capture of cuda_stream captures all of it.
+ * cuda_stream.  The call is not meant for stream capture: it copies its
+ * descriptors from host memory that it frees when it returns.
  *
  * traces[n_traces]: uploaded handles (host array of pointers).
  * params[n_replays]: host array.
