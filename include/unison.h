@@ -301,8 +301,8 @@ int unison_replay_batch(const unison_trace *const *traces, int n_traces,
  *    in shared memory) exceeds UNISON_NOALLOC_SCRATCH_BYTES is rejected with
  *    UNISON_ERR_RANGE before anything is queued.
  *  - The first call on a device looks up the array's device address on that
- *    device (cudaGetSymbolAddress, with that device current); make that
- *    first call before any stream capture.
+ *    device (cudaGetSymbolAddress, with that device current).  Like
+ *    unison_replay_batch, the call is not meant for stream capture.
  *  - All calls share the one array, which keeps what the last call left in
  *    it; each call writes every region it reads before reading it, so no
  *    region needs clearing.  Calls whose work overlaps on the GPU (on
