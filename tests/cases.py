@@ -8,6 +8,8 @@ TTFT under 4x load.
 """
 from __future__ import annotations
 
+import functools
+
 import synth
 
 GIB = 1 << 30
@@ -81,3 +83,16 @@ def sweep_case(n_seeds: int = 8):
 
 def large_pool_params():
     return base("spear_tide", 16 * GIB, 160 * GIB, 163840)
+
+
+@functools.lru_cache(maxsize=8)
+def _coding_trace(seed: int):
+    return synth.paper_scale_trace(seed, "coding")
+
+
+def oracle_sweep_job(job):
+    """One oracle replay of the sweep in a worker process: (trace seed,
+    params) -> counters.  The worker builds (and keeps) the seed's trace."""
+    import oracle
+    seed, p = job
+    return oracle.replay(_coding_trace(seed), to_oracle(p))

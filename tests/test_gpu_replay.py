@@ -81,16 +81,21 @@ def test_paper_scale_30_replays(B):
             assert_same_log(B, log[i], res[i], o, (ti, p["policy"], p["kvb"]))
 
 
-def test_sweep_1024_replays_sampled(B):
-    """The benchmark's launch configuration: one call over all 1,024 replays;
-    a spread of replays is checked against the oracle one by one."""
+def test_sweep_1024_replays_all(B):
+    """The benchmark's launch configuration: one call over all 1,024 replays,
+    every replay checked against the oracle (a spawn pool on the host cores;
+    spawned workers do not inherit this process's CUDA context)."""
+    import multiprocessing as mp
+    import os
+    from cases import oracle_sweep_job
     trs, reps = sweep_case()
     res, _, _ = run_gpu(B, trs, reps)
     assert len(res) == 1024
     assert all(r["status"] == 0 for r in res)
-    for i in list(range(0, 1024, 67)) + [1023]:
-        ti, p = reps[i]
-        assert_same(res[i], oracle.replay(trs[ti], to_oracle(p)), i)
+    with mp.get_context("spawn").Pool(min(os.cpu_count() or 1, 16)) as pool:
+        ores = pool.map(oracle_sweep_job, [(ti, p) for ti, p in reps], chunksize=32)
+    for i, o in enumerate(ores):
+        assert_same(res[i], o, i)
 
 
 @pytest.mark.parametrize("seed", [100, 101])
