@@ -96,3 +96,13 @@ def oracle_sweep_job(job):
     import oracle
     seed, p = job
     return oracle.replay(_coding_trace(seed), to_oracle(p))
+
+
+def oracle_rank_job(job):
+    """One oracle ranking in a worker process: (record seed, records, params)
+    -> victims, moves and moved bytes.  The worker builds the live set."""
+    import oracle
+    seed, n, p = job
+    rec = synth.make_records(seed, n)
+    return oracle.rank(rec, p["sigma_q"], p["penalty_q"], p["k"], p["budget_bytes"], p["kv_bytes_per_token"],
+                       p["free_fast_tok"], p["free_hbm_tok"], max_moves=max(p["max_moves"], 1))

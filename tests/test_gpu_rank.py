@@ -39,6 +39,10 @@ def run(B, recs, params, keys=False):
 def check(r, rec, p, keys=False):
     o = oracle.rank(rec, p["sigma_q"], p["penalty_q"], p["k"], p["budget_bytes"], p["kv_bytes_per_token"],
                     p["free_fast_tok"], p["free_hbm_tok"], keys=keys, max_moves=max(p["max_moves"], 1))
+    compare(r, o, p, keys)
+
+
+def compare(r, o, p, keys=False):
     if p["max_moves"] == 0:
         o["promote"] = o["promote"][:0]
         o["demote"] = o["demote"][:0]
@@ -82,6 +86,22 @@ def test_full_size_2p24(B, sigma):
     p = prm(sigma, k=1024, budget=64 * GIB)
     r = run(B, [rec], [p], keys=True)[0]
     check(r, rec, p, keys=True)
+
+
+def test_bench_launch_seven_sets(B, sigma):
+    """The benchmark's ranking launch: seven copies of one 2^24-record live
+    set with TIDE budgets 1..64 GiB and k = 1,024, in one call.  Every set's
+    victims, moves and moved bytes equal the oracle's (a spawn pool runs the
+    seven oracle rankings, each worker building the set itself)."""
+    import multiprocessing as mp
+    from cases import oracle_rank_job
+    rec = synth.make_records(4, 1 << 24)
+    ps = [prm(sigma, k=1024, budget=b * GIB) for b in (1, 2, 4, 8, 16, 32, 64)]
+    res = run(B, [rec] * len(ps), ps)
+    with mp.get_context("spawn").Pool(len(ps)) as pool:
+        ores = pool.map(oracle_rank_job, [(4, 1 << 24, p) for p in ps], chunksize=1)
+    for r, o, p in zip(res, ores, ps):
+        compare(r, o, p)
 
 
 def _sorted_records(n, ascending=True):
