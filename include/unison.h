@@ -94,7 +94,9 @@ typedef struct unison_trace unison_trace; /* opaque, library-owned */
 
 /* Validate and order a trace on the host (events, per-turn event indices,
  * next-arrival indices).  *out receives a new handle; free it with
- * unison_trace_free.  No device memory is touched. */
+ * unison_trace_free.  No device memory is touched; the host copy is
+ * page-locked (cudaMallocHost) when a CUDA driver is present, else ordinary
+ * memory. */
 int unison_trace_create(const unison_turns *turns, unison_trace **out);
 
 /* Read a .utr file (little endian: "UTR1", u32 n_sessions, u64 n_turns,
@@ -115,7 +117,8 @@ void unison_trace_free(unison_trace *tr);
 int unison_trace_info(const unison_trace *tr, uint32_t *n_sessions, uint64_t *n_turns,
                       uint64_t *n_events);
 
-/* Bytes the last upload copied host-to-device for this trace. */
+/* Bytes an upload copies host-to-device for this trace (the size of its
+ * device block, fixed when the trace is created). */
 uint64_t unison_trace_device_bytes(const unison_trace *tr);
 
 /* ================================================================ replay */
@@ -164,7 +167,9 @@ typedef struct {
  * decides exactly as the live replay.  SPEAR and SPEAR+TIDE only, not with
  * UNISON_HAZARD_ONLINE, stale_m >= 1 for UNISON_SYNC_ARRIVALS (else
  * UNISON_ERR_ARG); the same shared-memory and session limits as the online
- * table apply, with 16 bytes per session (else UNISON_ERR_RANGE). */
+ * table apply, with 20 bytes per session (tier, pin slot, live and snapshot
+ * keys, a changed flag) beside the power-of-two lists (else
+ * UNISON_ERR_RANGE). */
 #define UNISON_SYNC_LIVE 0u      /* no snapshot: the live ranking          */
 #define UNISON_SYNC_EVENT 1u     /* copy after every event                 */
 #define UNISON_SYNC_ARRIVALS 2u  /* copy after every stale_m-th arrival    */
@@ -176,8 +181,9 @@ typedef struct {
  * re-ranks every resident under the rebuilt table before the next event.
  * SPEAR and SPEAR+TIDE only (else UNISON_ERR_ARG); the trace must have at
  * most 32,768 sessions and the replay's resident lists, rounded up to powers
- * of two, plus 7 bytes per session must fit in shared memory (else
- * UNISON_ERR_RANGE).  A bit of `flags` not defined here is UNISON_ERR_ARG. */
+ * of two, plus 9 bytes per session (tier, pin slot, gap average, arrival
+ * count) and the table must fit in shared memory (else UNISON_ERR_RANGE).
+ * A bit of `flags` not defined here is UNISON_ERR_ARG. */
 #define UNISON_HAZARD_ONLINE 1u
 
 /* Signal leave-one-out (Sec. V-D, Fig. signal), SPEAR and SPEAR+TIDE only,
