@@ -399,7 +399,8 @@ int unison_hazard_lut(const uint32_t *turns_dev, uint64_t n_sessions, uint32_t b
 
 /* ================================================================ ranking */
 /* A live set of n session records, structure of arrays, device memory
- * (caller-owned).  gap_q: gap average in us (eq. gapq, < 2^31); last_ret:
+ * (caller-owned).  gap_q: gap average in us (eq. gapq, < 2^31: the device
+ * does not check it, and a larger value gives an unspecified key); last_ret:
  * last completion time (carried, not read by the score); turn: register turn
  * t; kv_tok: resident tokens; tier: 1 fast, 2 HBM, other = not resident;
  * flags: bit0 pinned (mid-turn), bit1 done (completed session).  1 <= n <= 2^24
