@@ -1702,14 +1702,19 @@ int launch_replays(const ReplayPlan &P, char *scratch, const std::vector<ComboDe
   if (!P.combos.empty()) {
     ck(cudaMemcpyAsync(d_combo, hc.data(), sizeof(ComboDesc) * P.combos.size(), cudaMemcpyHostToDevice, stream));
     hazard_lut_kernel<<<(unsigned)P.combos.size(), 256, 0, stream>>>(d_combo);
+    count_launches(1);
     uint32_t max_s = 0;
     for (auto &c : hc) max_s = std::max(max_s, c.n_sessions);
-    dim3 g((max_s + 127) / 128, (unsigned)P.combos.size());
     {
       ProfSpan span(profile ? "key_stream" : "", stream);
-      key_stream_kernel<<<g, 128, 0, stream>>>(d_combo);
+      // one grid row per combination; a grid has at most 65,535 rows
+      constexpr size_t kRows = 65535;
+      for (size_t c0 = 0; c0 < P.combos.size(); c0 += kRows) {
+        const unsigned rows = (unsigned)std::min(kRows, P.combos.size() - c0);
+        key_stream_kernel<<<dim3((max_s + 127) / 128, rows), 128, 0, stream>>>(d_combo + c0);
+        count_launches(1);
+      }
     }
-    count_launches(2);
     ck(cudaGetLastError());
   }
   {

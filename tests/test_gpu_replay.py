@@ -334,6 +334,21 @@ def test_random_parameters_one_call(B, seed):
         assert_same(res[i], oracle.replay(trs[ti], to_oracle(p)), (i, ti, p))
 
 
+def test_more_key_streams_than_grid_rows(B):
+    """65,600 SPEAR replays with distinct P_Z need 65,600 key streams, more
+    than one launch's 65,535 grid rows: the streams are built in two
+    launches.  The replays past the boundary use another gap-average weight,
+    which changes their decisions, so a second launch reading the first
+    launch's streams would fail; replays on both sides equal the oracle."""
+    tr, _ = tiny_case()
+    reps = [(0, base("spear", 512 * MIB, 8 * GIB, 28672, penalty=7000 * i,
+                     ema_num=3 if i < 65535 else 1, ema_den=10 if i < 65535 else 1 << 20)) for i in range(65600)]
+    res, _, _ = run_gpu(B, [tr], reps)
+    assert all(r["status"] == 0 for r in res)
+    for i in list(range(0, 65600, 4099)) + [65533, 65534, 65535, 65536, 65599]:
+        assert_same(res[i], oracle.replay(tr, to_oracle(reps[i][1])), i)
+
+
 def test_log_overflow_reported(B):
     tr, _ = tiny_case()
     p = base("spear_tide", 512 * MIB, 8 * GIB, 28672)
