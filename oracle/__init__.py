@@ -88,32 +88,55 @@ def build(force: bool = False) -> str:
     return _LIB
 
 
+def _bind(L):
+    """Declare the argument and result types of the oracle's entry points."""
+    L.or_replay.argtypes = [C.POINTER(_Trace), C.POINTER(_Params), C.POINTER(_Result),
+                            C.c_void_p, C.c_uint64, C.c_void_p]
+    L.or_replay.restype = C.c_int
+    L.or_hazard_lut.argtypes = [C.c_void_p, C.c_uint64, C.c_uint32, C.c_void_p, C.c_void_p]
+    L.or_hazard_lut.restype = C.c_int
+    L.or_spear_score.argtypes = [C.c_uint64, C.c_uint32, C.c_uint64, C.c_int]
+    L.or_spear_score.restype = C.c_uint64
+    L.or_ema.argtypes = [C.c_uint64, C.c_uint64, C.c_uint32, C.c_uint32]
+    L.or_ema.restype = C.c_uint64
+    L.or_rank.argtypes = ([C.POINTER(_Records), C.c_void_p, C.c_uint64, C.c_uint32,
+                           C.c_uint64, C.c_uint32, C.c_uint64, C.c_uint64]
+                          + [C.c_void_p] * 8 + [C.c_uint32])
+    L.or_rank.restype = C.c_int
+    L.or_kendall_brute.argtypes = [C.c_void_p, C.c_void_p, C.c_uint64]
+    L.or_kendall_brute.restype = C.c_double
+    L.or_ase.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_void_p]
+    L.or_ase.restype = None
+    L.or_attainment.argtypes = [C.POINTER(_Trace), C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p]
+    L.or_attainment.restype = C.c_int
+    return L
+
+
 def lib():
     global _lib
     with _lock:
         if _lib is None:
-            L = C.CDLL(build())
-            L.or_replay.argtypes = [C.POINTER(_Trace), C.POINTER(_Params), C.POINTER(_Result),
-                                    C.c_void_p, C.c_uint64, C.c_void_p]
-            L.or_replay.restype = C.c_int
-            L.or_hazard_lut.argtypes = [C.c_void_p, C.c_uint64, C.c_uint32, C.c_void_p, C.c_void_p]
-            L.or_hazard_lut.restype = C.c_int
-            L.or_spear_score.argtypes = [C.c_uint64, C.c_uint32, C.c_uint64, C.c_int]
-            L.or_spear_score.restype = C.c_uint64
-            L.or_ema.argtypes = [C.c_uint64, C.c_uint64, C.c_uint32, C.c_uint32]
-            L.or_ema.restype = C.c_uint64
-            L.or_rank.argtypes = ([C.POINTER(_Records), C.c_void_p, C.c_uint64, C.c_uint32,
-                                   C.c_uint64, C.c_uint32, C.c_uint64, C.c_uint64]
-                                  + [C.c_void_p] * 8 + [C.c_uint32])
-            L.or_rank.restype = C.c_int
-            L.or_kendall_brute.argtypes = [C.c_void_p, C.c_void_p, C.c_uint64]
-            L.or_kendall_brute.restype = C.c_double
-            L.or_ase.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_int, C.c_int, C.c_void_p]
-            L.or_ase.restype = None
-            L.or_attainment.argtypes = [C.POINTER(_Trace), C.c_void_p, C.c_void_p, C.c_uint32, C.c_void_p]
-            L.or_attainment.restype = C.c_int
-            _lib = L
+            _lib = _bind(C.CDLL(build()))
     return _lib
+
+
+def build_variant(source: str, out_dir: str):
+    """Compile a modified copy of the oracle's C source (a test plants one
+    mistake in it to show that a pin catches that mistake) and load it.  The
+    result is passed as ``lib_`` to ``replay``."""
+    src = os.path.join(out_dir, "variant.c")
+    so = os.path.join(out_dir, "libvariant.so")
+    with open(src, "w") as f:
+        f.write(source)
+    subprocess.check_call(["gcc", "-O1", "-std=gnu11", "-ffp-contract=off", "-fPIC", "-shared", "-o", so, src,
+                           "-lm"])
+    return _bind(C.CDLL(so))
+
+
+def source() -> str:
+    """The oracle's C source text."""
+    with open(_SRC) as f:
+        return f.read()
 
 
 def _ptr(a: np.ndarray) -> int:
@@ -142,11 +165,12 @@ def _params_struct(p: dict, debug: bool):
 
 
 def replay(tr, params: dict, log: bool = False, ttft: bool = False, debug: bool = False,
-           log_capacity: int | None = None) -> dict:
+           log_capacity: int | None = None, lib_=None) -> dict:
     """Replay one trace under one policy; returns the counters (and, on
     request, the decision log as (event, kind, session) arrays and the
-    per-request TTFT values in ns)."""
-    L = lib()
+    per-request TTFT values in ns).  ``lib_``: a library from
+    ``build_variant`` instead of the oracle itself."""
+    L = lib_ if lib_ is not None else lib()
     ts, keep = _trace_struct(tr)
     ps = _params_struct(params, debug)
     res = _Result()

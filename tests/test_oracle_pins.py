@@ -175,6 +175,51 @@ def test_hand_replay_spear():
         assert r[k] == v, k
 
 
+HAND_TIDE_PARAMS = dict(policy="spear_tide", kv_bytes_per_token=1, cap_s_bytes=100, cap_h_bytes=1000,
+                        dma_bytes_per_us=4, t_p_ps_per_tok=20_000_000, ttft_load=4)
+
+
+def test_hand_replay_spear_tide():
+    """Sec. III-C inside a replay, worked by hand: a phase-1 promotion beside
+    pinned fast-tier sessions, a phase-2 stop on the order test and one on
+    the budget, a gap_start inside the DMA-busy window and one exactly at its
+    end, and prefetch accuracy over a promoted session that hits the fast
+    tier and one that was demoted before its next request."""
+    tr, log, counts = _hand_trace("replay_hand_tide.txt")
+    r = oracle.replay(tr, HAND_TIDE_PARAMS, log=True, debug=True)
+    assert r["status"] == 0
+    got = list(zip(*(map(int, a) for a in r["log"])))
+    assert got == log
+    for k, v in counts.items():
+        assert r[k] == v, k
+
+
+def test_tide_unaffordable_budget_equals_spear():
+    """Closed form of eq. (budget): if g_q * B is below the cost of the
+    smallest possible move (its tokens x kvB) at every gap_start, TIDE runs
+    and moves nothing, so SPEAR+TIDE decides exactly as SPEAR.  The gap
+    average is a convex combination of observed gaps (eq. ema-int), so the
+    largest gap of the trace bounds it."""
+    tr = synth.paper_scale_trace(1, "coding")
+    kvb = 1 << 24
+    max_gap = int(max(np.max(tr.arrival_us[i + 1:j] - tr.completion_us[i:j - 1]) if j - i > 1 else 0
+                      for i, j in zip(tr.turn_off[:-1], tr.turn_off[1:])))
+    min_cost = int(np.min(tr.out_tok)) * kvb
+    rate = (min_cost - 1) // max_gap
+    assert rate >= 1
+    p = dict(kv_bytes_per_token=kvb, cap_s_bytes=4 << 40, cap_h_bytes=64 << 40, dma_bytes_per_us=rate)
+    a = oracle.replay(tr, dict(p, policy="spear_tide"), log=True)
+    b = oracle.replay(tr, dict(p, policy="spear"), log=True)
+    assert a["status"] == b["status"] == 0
+    assert a["tide_calls"] > 1000 and a["promote"] == a["tide_demote"] == a["dma_bytes"] == 0
+    assert a["decision_hash"] == b["decision_hash"]
+    for x, y in zip(a["log"], b["log"]):
+        assert np.array_equal(x, y)
+    # at 64 times that rate some move becomes affordable: the bound is not vacuous
+    c = oracle.replay(tr, dict(p, policy="spear_tide", dma_bytes_per_us=64 * rate))
+    assert c["promote"] > 0
+
+
 # ------------------------------------------------------ capacity extremes ----
 
 POLICIES = ["lru", "timeout", "spear", "spear_tide", "belady", "lru_tide"]
