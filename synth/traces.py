@@ -199,12 +199,13 @@ def tiny_trace(seed: int = 0) -> Trace:
     return make_trace(seed, np.full(64, 12), 2.0, GAP_MIX_CONFIG0)
 
 
-def paper_scale_trace(seed: int = 1, mix: str = "coding") -> Trace:
+def paper_scale_trace(seed: int = 1, mix: str = "coding", gap_persist: float = GAP_PERSIST) -> Trace:
     """1,415 sessions / 33,596 turns, T_s ~ Geometric(mean 23.7) on [2, 200]
-    adjusted to the exact total, starts Poisson with mean 2 s."""
+    adjusted to the exact total, starts Poisson with mean 2 s.  gap_persist 0
+    draws every gap's component and value independently."""
     gm = {"coding": GAP_MIX_CODING, "general": GAP_MIX_GENERAL}[mix]
     t = geometric_turns(seed, 1415, 23.7, 2, 200, total=33596)
-    return make_trace(seed, t, 2.0, gm)
+    return make_trace(seed, t, 2.0, gm, gap_persist=gap_persist)
 
 
 def large_pool_trace(seed: int, n_sessions: int = 65536) -> Trace:
