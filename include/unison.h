@@ -295,9 +295,18 @@ int unison_replay_batch(const unison_trace *const *traces, int n_traces,
  * allocation can fail in the middle of a run).  This entry point replays
  * exactly like unison_replay_batch (same arguments, same results) but takes
  * its scratch from one fixed device array compiled into the library,
- * UNISON_NOALLOC_SCRATCH_BYTES long, which every GPU that loads the library
- * holds until the process exits.  It calls no cudaMalloc, cudaFree or other
- * allocating routine.
+ * UNISON_NOALLOC_SCRATCH_BYTES long.  It calls no cudaMalloc, cudaFree or
+ * other allocating routine.
+ *  - When the array and other set-up come into being: CUDA loads a library's
+ *    device code lazily by default, so the array is created on a device when
+ *    the library first launches a kernel or looks up the array there (this
+ *    entry point's first call on the device at the latest), and that device
+ *    holds it until the process exits.  The first call on a device whose
+ *    batch needs more than one launch group (policies other than SPEAR+TIDE
+ *    beside it, online-table or stale-snapshot replays) also creates the
+ *    library's side streams and their events there.  A caller whose memory
+ *    manager will later own the whole device should therefore make its first
+ *    call, with the kinds of replays it will run, during start-up.
  *  - results_dev is required (the caller provides the output buffer);
  *    results_host, log_dev and the traces are as in unison_replay_batch.
  *    The traces must already be uploaded (unison_trace_upload allocates, so
@@ -448,25 +457,63 @@ typedef struct {
  * score_q (eq. scoreq); order as in replay (larger key, then smaller index,
  * is more evictable).  Results are exact: candidate thresholds come from a
  * sample, and a set whose candidates fall short is re-selected exactly on
- * the device.  sets, params, outs: host arrays [n_sets].  Asynchronous.
- * Memory: the call's device scratch (about 2.2 MB per set) is kept per
+ * the device.  sets, params, outs: host arrays [n_sets].  Asynchronous: the
+ * call queues one upload of its descriptors and one cooperative kernel on
+ * cuda_stream (every CTA of the grid resident at once; each set is ranked
+ * by a group of CTAs, or, with more sets than resident CTAs, each CTA takes
+ * whole sets in turn).  Any n_sets >= 0 that fits in memory is accepted.
+ * Memory: the call's device scratch (about 1.7 MB per set) is kept per
  * (device, stream) and grown when a call needs more, and the per-call
  * descriptors go up from a small pinned host ring; both are held for the
  * life of the process.  Calls on one stream run in order and share that
- * stream's scratch; calls on different streams use different scratch.
+ * stream's scratch; calls on different streams use different scratch.  The
+ * scratch is found by the stream's handle, so a stream must outlive the
+ * ranking calls queued on it.
  * Errors: UNISON_ERR_ARG (null or misaligned arrays), UNISON_ERR_RANGE
  * (limits above), UNISON_ERR_OOM (scratch or staging), UNISON_ERR_CUDA
- * (launch); a bounded device wait that gives up sets counts[3] of its set to
- * UNISON_ERR_TIMEOUT.
+ * (launch; a device without cooperative launch); a bounded device wait that
+ * gives up sets counts[3] of its set to UNISON_ERR_TIMEOUT.
  */
 int unison_rank_batch(const unison_records *sets, const unison_rank_params *params,
                       const unison_rank_out *outs, int n_sets, void *cuda_stream);
 
+/* One live set: the ranking of Sec. IV-D and the TIDE fill of Sec. III-C
+ * (eqs. scoreq, pipe/scan, promote, demote, budget) for a single set, with
+ * the same arguments, outputs, limits and errors as unison_rank_batch with
+ * n_sets = 1 (records, params and out point to one element each). */
+int unison_rank(const unison_records *records, const unison_rank_params *params,
+                const unison_rank_out *out, void *cuda_stream);
+
+/* Record-sharded ranking of one live set over several GPUs (Sec. IV-D's
+ * scan and Sec. III-C's selections, eqs. promote/demote, split by records).
+ * Each GPU ranks its slice -- records [index_offset, index_offset + n) of
+ * the whole set, 16-byte-aligned device arrays as for unison_rank -- and
+ * writes its candidate lists to cands_dev: its k most evictable unpinned
+ * records (V), its max_moves most evictable unpinned fast-tier records (D)
+ * and its max_moves least evictable unpinned HBM records (P), each in
+ * ranking order with its KV size, keyed by its index in the whole set.  The
+ * global top-k of V, and the first max_moves of D and of P, lie in the union
+ * of the slices' lists, so after one all-gather of the fixed-size buffers
+ * (n_shards x unison_rank_cands_bytes(k, max_moves), in any order) every GPU
+ * runs unison_rank_merge, which selects the global lists and runs the TIDE
+ * fill exactly as unison_rank does for the whole set: the outputs are equal.
+ * params must be the same on every GPU (budget and free tier capacities are
+ * the whole set's).  index_offset + n <= 2^24 (the index is packed into 24
+ * bits of the ranking key), else UNISON_ERR_RANGE.  cands_dev: device,
+ * caller-owned, 256-byte aligned, at least unison_rank_cands_bytes(k,
+ * max_moves) bytes; gathered_dev: n_shards such buffers back to back.
+ * Errors as for unison_rank_batch; asynchronous on cuda_stream. */
+uint64_t unison_rank_cands_bytes(uint32_t k, uint32_t max_moves);
+int unison_rank_shard(const unison_records *slice, uint64_t index_offset, const unison_rank_params *params,
+                      void *cands_dev, void *cuda_stream);
+int unison_rank_merge(const void *gathered_dev, int n_shards, const unison_rank_params *params,
+                      const unison_rank_out *out, void *cuda_stream);
+
 /* ============================================================ measurement */
 /* While enabled (on != 0), every replay and ranking call records a pair of
  * CUDA events on its own stream around each launch of its main kernels
- * ("replay" = the event loop, "key_stream", "ttft_median", "rank_sample",
- * "rank_filter", "rank_finish").  Not thread-safe; meant for benchmarks. */
+ * ("replay" = the event loop, "key_stream", "ttft_median", "rank" = the
+ * whole ranking kernel).  Not thread-safe; meant for benchmarks. */
 int unison_profile_enable(int on);
 
 /* Synchronise the recorded events of one kernel name and return the summed

@@ -13,7 +13,7 @@ from typing import Iterable, List, Sequence
 
 import numpy as np
 
-from .native import LIB
+from .native import LIB, LIB_DEBUG
 
 POLICY = {"lru": 0, "timeout": 1, "spear": 2, "spear_tide": 3, "belady": 4, "lru_tide": 5}
 FLAG_HAZARD_ONLINE = 1  # unison_replay_params.flags bit 0
@@ -91,9 +91,12 @@ _lock = threading.Lock()
 _lib = None
 
 # Every symbol include/unison.h declares (checked by the ABI tests).
+# the test library of native.build_debug() (include/unison_debug.h) adds these
+DEBUG_EXPORTS = ["unison_debug_rank_wait_hooks"]
 EXPORTS = ["unison_strerror", "unison_version", "unison_trace_create", "unison_trace_load",
            "unison_trace_upload", "unison_trace_free", "unison_trace_info", "unison_trace_device_bytes",
-           "unison_replay_batch", "unison_stats", "unison_hazard_lut", "unison_rank_batch",
+           "unison_replay_batch", "unison_stats", "unison_hazard_lut", "unison_rank_batch", "unison_rank",
+           "unison_rank_cands_bytes", "unison_rank_shard", "unison_rank_merge",
            "unison_profile_enable", "unison_profile_read", "unison_launch_count",
            "unison_replay_batch_noalloc", "unison_ase", "unison_attainment", "unison_selftest_division",
            "unison_debug_fail_allocations"]
@@ -101,6 +104,35 @@ EXPORTS = ["unison_strerror", "unison_version", "unison_trace_create", "unison_t
 
 def lib_path() -> str:
     return LIB
+
+
+def _bind_rank(L):
+    L.unison_rank_batch.argtypes = [C.POINTER(Records), C.POINTER(RankParams), C.POINTER(RankOut), C.c_int,
+                                    C.c_void_p]
+    L.unison_rank.argtypes = [C.POINTER(Records), C.POINTER(RankParams), C.POINTER(RankOut), C.c_void_p]
+    L.unison_rank_cands_bytes.argtypes = [C.c_uint32, C.c_uint32]
+    L.unison_rank_cands_bytes.restype = C.c_uint64
+    L.unison_rank_shard.argtypes = [C.POINTER(Records), C.c_uint64, C.POINTER(RankParams), C.c_void_p, C.c_void_p]
+    L.unison_rank_merge.argtypes = [C.c_void_p, C.c_int, C.POINTER(RankParams), C.POINTER(RankOut), C.c_void_p]
+    return L
+
+
+_debug_lib = None
+
+
+def debug_lib():
+    """Load the ranking test library with its wait hooks (built by
+    paper_2609_09643_gb300.native.build_debug()); pass it as ``lib_`` to
+    RankCall."""
+    global _debug_lib
+    with _lock:
+        if _debug_lib is None:
+            if not os.path.exists(LIB_DEBUG):
+                raise RuntimeError(f"{LIB_DEBUG} is missing: run native.build_debug() first")
+            L = _bind_rank(C.CDLL(LIB_DEBUG))
+            L.unison_debug_rank_wait_hooks.argtypes = [C.c_int, C.c_int]
+            _debug_lib = L
+    return _debug_lib
 
 
 def lib():
@@ -129,8 +161,7 @@ def lib():
             L.unison_stats.argtypes = [C.POINTER(ReplayResult), C.POINTER(ReplayParams), C.POINTER(Stats)]
             L.unison_hazard_lut.argtypes = [C.c_void_p, C.c_uint64, C.c_uint32, C.c_void_p, C.c_void_p,
                                             C.c_void_p]
-            L.unison_rank_batch.argtypes = [C.POINTER(Records), C.POINTER(RankParams), C.POINTER(RankOut), C.c_int,
-                                            C.c_void_p]
+            _bind_rank(L)
             L.unison_profile_enable.argtypes = [C.c_int]
             L.unison_profile_read.argtypes = [C.c_char_p, C.POINTER(C.c_double), C.POINTER(C.c_uint64), C.c_int]
             L.unison_launch_count.restype = C.c_uint64
@@ -410,36 +441,38 @@ class RankCall:
     """The marshalled arguments of one unison_rank_batch call (ctypes arrays
     over the tensors' device pointers), reusable while those tensors live."""
 
-    def __init__(self, sets: Sequence[dict], params: Sequence[dict], outs: Sequence[dict]):
+    def __init__(self, sets: Sequence[dict], params: Sequence[dict], outs: Sequence[dict], lib_=None):
         n = len(sets)
         self.n = n
+        self._lib = lib_
         self.rs = (Records * n)()
         self.ps = (RankParams * n)()
         self.os = (RankOut * n)()
         self._keep = (list(sets), list(outs))  # the pointers stay valid while these live
         for i, (r, p, o) in enumerate(zip(sets, params, outs)):
-            self.rs[i] = Records(r["gap_q"].data_ptr(), r["last_ret"].data_ptr(), r["turn"].data_ptr(),
-                                 r["kv_tok"].data_ptr(), r["tier"].data_ptr(), r["flags"].data_ptr(),
-                                 r["gap_q"].numel())
-            sig = np.ascontiguousarray(np.asarray(p["sigma_q"], dtype=np.uint16))
-            if sig.shape != (51,):
-                raise ValueError("sigma_q must have 51 entries")
-            self.ps[i] = RankParams((C.c_uint16 * 51).from_buffer_copy(sig.tobytes()), 0, p.get("k", 0),
-                                    p.get("penalty_q", 500_000_000), p.get("budget_bytes", 0),
-                                    p.get("kv_bytes_per_token", 131072), p.get("max_moves", 0),
-                                    p.get("free_fast_tok", 0), p.get("free_hbm_tok", 0))
-            self.os[i] = RankOut(o["victims"].data_ptr(), o["promote"].data_ptr(), o["demote"].data_ptr(),
-                                 o["counts"].data_ptr(), o["moved"].data_ptr(),
-                                 None if o.get("keys") is None else o["keys"].data_ptr())
+            self.rs[i] = _records(r)
+            self.ps[i] = _rank_params(p)
+            self.os[i] = _rank_out(o)
 
     def run(self, stream=None) -> None:
-        _check("unison_rank_batch", lib().unison_rank_batch(self.rs, self.ps, self.os, self.n,
-                                                            _stream_handle(stream)))
+        L = self._lib if self._lib is not None else lib()
+        _check("unison_rank_batch", L.unison_rank_batch(self.rs, self.ps, self.os, self.n, _stream_handle(stream)))
+
+    def run_single(self, stream=None) -> None:
+        """unison_rank on the one set this call holds."""
+        assert self.n == 1
+        L = self._lib if self._lib is not None else lib()
+        _check("unison_rank", L.unison_rank(self.rs, self.ps, self.os, _stream_handle(stream)))
 
 
 def rank_prepare(sets: Sequence[dict], params: Sequence[dict], outs: Sequence[dict]) -> RankCall:
     """Marshal a rank call once (see RankCall) for repeated launches."""
     return RankCall(sets, params, outs)
+
+
+def rank(rec: dict, params: dict, out: dict, stream=None) -> None:
+    """unison_rank: one device record set, one params dict, one output dict."""
+    RankCall([rec], [params], [out]).run_single(stream)
 
 
 def rank_batch(sets: Sequence[dict], params: Sequence[dict], outs: Sequence[dict], stream=None) -> None:
@@ -449,13 +482,63 @@ def rank_batch(sets: Sequence[dict], params: Sequence[dict], outs: Sequence[dict
     RankCall(sets, params, outs).run(stream)
 
 
+def _rank_params(p: dict) -> RankParams:
+    sig = np.ascontiguousarray(np.asarray(p["sigma_q"], dtype=np.uint16))
+    if sig.shape != (51,):
+        raise ValueError("sigma_q must have 51 entries")
+    return RankParams((C.c_uint16 * 51).from_buffer_copy(sig.tobytes()), 0, p.get("k", 0),
+                      p.get("penalty_q", 500_000_000), p.get("budget_bytes", 0),
+                      p.get("kv_bytes_per_token", 131072), p.get("max_moves", 0),
+                      p.get("free_fast_tok", 0), p.get("free_hbm_tok", 0))
+
+
+def _rank_out(o: dict) -> RankOut:
+    return RankOut(o["victims"].data_ptr(), o["promote"].data_ptr(), o["demote"].data_ptr(),
+                   o["counts"].data_ptr(), o["moved"].data_ptr(),
+                   None if o.get("keys") is None else o["keys"].data_ptr())
+
+
+def _records(r: dict) -> Records:
+    return Records(r["gap_q"].data_ptr(), r["last_ret"].data_ptr(), r["turn"].data_ptr(), r["kv_tok"].data_ptr(),
+                   r["tier"].data_ptr(), r["flags"].data_ptr(), r["gap_q"].numel())
+
+
+def rank_cands_bytes(k: int, max_moves: int) -> int:
+    """Bytes of one shard's candidate buffer (unison_rank_cands_bytes)."""
+    return int(lib().unison_rank_cands_bytes(k, max_moves))
+
+
+def rank_cands(k: int, max_moves: int, n_shards: int = 1, device="cuda"):
+    """A uint8 device buffer for n_shards candidate buffers, back to back."""
+    import torch
+    return torch.zeros(n_shards * rank_cands_bytes(k, max_moves), dtype=torch.uint8, device=device)
+
+
+def rank_shard(rec_slice: dict, index_offset: int, params: dict, cands, stream=None) -> None:
+    """unison_rank_shard: rank records [index_offset, index_offset + n) of a
+    live set (rec_slice: device arrays of the slice) into the uint8 device
+    tensor cands (rank_cands_bytes(k, max_moves) bytes, 256-byte aligned)."""
+    r, p = _records(rec_slice), _rank_params(params)
+    _check("unison_rank_shard", lib().unison_rank_shard(C.byref(r), index_offset, C.byref(p), cands.data_ptr(),
+                                                        _stream_handle(stream)))
+
+
+def rank_merge(gathered, n_shards: int, params: dict, out: dict, stream=None) -> None:
+    """unison_rank_merge over n_shards candidate buffers back to back in the
+    uint8 device tensor gathered; writes out as unison_rank does."""
+    p, o = _rank_params(params), _rank_out(out)
+    _check("unison_rank_merge", lib().unison_rank_merge(gathered.data_ptr(), n_shards, C.byref(p), C.byref(o),
+                                                        _stream_handle(stream)))
+
+
 def rank_result(o: dict) -> dict:
     """Host copy of one set's outputs."""
     c = o["counts"].cpu().numpy().astype(np.uint32)
     res = dict(victims=o["victims"].cpu().numpy().astype(np.uint32)[: c[0]],
                promote=o["promote"].cpu().numpy().astype(np.uint32)[: c[1]],
                demote=o["demote"].cpu().numpy().astype(np.uint32)[: c[2]],
-               moved_bytes=int(o["moved"].cpu().numpy().astype(np.uint64)[0]), status=int(c[3]))
+               moved_bytes=int(o["moved"].cpu().numpy().astype(np.uint64)[0]),
+               status=int(c[3:4].view(np.int32)[0]))  # a status word: 0 or a negative UNISON_ERR_* code
     if o.get("keys") is not None:
         res["keys"] = o["keys"].cpu().numpy().view(np.uint64)
     return res

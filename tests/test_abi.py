@@ -21,8 +21,8 @@ def B():
     return binding
 
 
-def declared_symbols():
-    src = open(os.path.join(ROOT, "include", "unison.h")).read()
+def declared_symbols(header="unison.h"):
+    src = open(os.path.join(ROOT, "include", header)).read()
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
     return sorted(set(re.findall(r"\b(unison_[a-z0-9_]+)\s*\(", src)))
 
@@ -34,6 +34,22 @@ def test_every_declared_symbol_is_exported(B):
     for name in decl:
         assert hasattr(lib, name), name
     assert sorted(B.EXPORTS) == decl
+
+
+def test_debug_library_exports_its_hooks(B):
+    """The ranking test library (include/unison_debug.h) builds for sm_103a
+    and exports its hooks beside the ranking calls; the default library does
+    not contain them."""
+    from paper_2609_09643_gb300 import native
+    path = native.build_debug()
+    dbg = C.CDLL(path)
+    decl = declared_symbols("unison_debug.h")
+    assert decl == sorted(B.DEBUG_EXPORTS)
+    for name in decl + ["unison_rank_batch", "unison_rank", "unison_strerror"]:
+        assert hasattr(dbg, name), name
+    lib = C.CDLL(B.lib_path())
+    for name in decl:
+        assert not hasattr(lib, name), name
 
 
 def test_strerror_and_version(B):

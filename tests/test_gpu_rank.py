@@ -61,6 +61,27 @@ def prm(sig, k=1024, budget=16 * GIB, max_moves=1024, free_s=0, free_h=1 << 40):
                 free_fast_tok=free_s, free_hbm_tok=free_h)
 
 
+def test_sigma_from_device_table(B):
+    """The chain the library offers end to end: the survival table built on
+    the device from turn counts (unison_hazard_lut, eqs. hazard/hq/survq)
+    feeds the ranking call, and the victims and fill equal the oracle's with
+    the oracle's own table."""
+    import torch
+    tps = synth.geometric_turns(2, 5000, 23.7, 2, 200)
+    turns = torch.from_numpy(np.asarray(tps, dtype=np.int32)).to("cuda")
+    sig_dev, _ = B.hazard_lut(turns)
+    sig = sig_dev.cpu().numpy().view(np.uint16)
+    _, sig_oracle = oracle.hazard_lut(tps)
+    assert np.array_equal(sig, sig_oracle)
+    rec = synth.make_records(21, 300_000)
+    ps = [prm(sig, k=k, budget=b, free_s=fs) for k, b, fs in [(1024, 8 * GIB, 0), (64, 64 * GIB, 50_000)]]
+    res = run(B, [rec] * len(ps), ps)
+    for r, p in zip(res, ps):
+        o = oracle.rank(rec, sig_oracle, p["penalty_q"], p["k"], p["budget_bytes"], p["kv_bytes_per_token"],
+                        p["free_fast_tok"], p["free_hbm_tok"], max_moves=p["max_moves"])
+        compare(r, o, p)
+
+
 @pytest.mark.parametrize("n", [1, 7, 1000, 2047, 2049, 4096, 16384])
 def test_small_sets_all_candidates(B, sigma, n):
     rec = synth.make_records(n, n)
@@ -283,3 +304,80 @@ def test_random_sets_and_parameters(B, seed):
                        free_hbm_tok=int(rng.choice([0, 5000, 1 << 40, (1 << 64) - 1]))))
     for r, rec, p in zip(run(B, recs, ps), recs, ps):
         check(r, rec, p)
+
+
+def test_single_set_entry_point(B, sigma):
+    """unison_rank, the one-set form, against the oracle and against the batch
+    call on the same set."""
+    import torch
+    rec = synth.make_records(31, 1 << 20)
+    dev = B.records_to_device(rec)
+    for p in (prm(sigma), prm(sigma, k=3, budget=2 * GIB, max_moves=64, free_s=20_000)):
+        out = B.rank_outputs(rec.n, p["k"], p["max_moves"])
+        B.rank(dev, p, out)
+        torch.cuda.synchronize()
+        r = B.rank_result(out)
+        check(r, rec, p)
+        (rb,) = run(B, [rec], [p])
+        for key in ("victims", "promote", "demote"):
+            assert np.array_equal(r[key], rb[key]), key
+
+
+def test_bounded_waits_report_timeout_and_recover(B, sigma):
+    """The test library's short waits: a threshold wait on a flag that nothing
+    sets and a tile wait on a barrier that nothing arrives at each run out,
+    record UNISON_ERR_TIMEOUT in their set's counts[3] and let the kernel
+    finish (the other outputs are still exact).  The next ordinary call on
+    the same stream then ranks every set exactly, with status OK."""
+    import torch
+    from paper_2609_09643_gb300 import native
+    native.build_debug()
+    D = B.debug_lib()
+    recs = [synth.make_records(41 + i, 300_000) for i in range(3)]
+    ps = [prm(sigma, k=256, budget=4 * GIB, max_moves=128) for _ in recs]
+    devs = [B.records_to_device(r) for r in recs]
+    outs = [B.rank_outputs(r.n, p["k"], p["max_moves"]) for r, p in zip(recs, ps)]
+    call = B.RankCall(devs, ps, outs, lib_=D)
+    stream = torch.cuda.current_stream()
+    try:
+        assert D.unison_debug_rank_wait_hooks(0, 2) == B.OK
+        call.run(stream)
+        torch.cuda.synchronize()
+        res = [B.rank_result(o) for o in outs]
+        assert [r["status"] for r in res] == [B.ERR_TIMEOUT, 0, B.ERR_TIMEOUT]
+        for r, rec, p in zip(res, recs, ps):
+            r["status"] = 0
+            check(r, rec, p)
+    finally:
+        assert D.unison_debug_rank_wait_hooks(-1, -1) == B.OK
+    for o in outs:
+        o["counts"].zero_()
+    call.run(stream)
+    torch.cuda.synchronize()
+    for o, rec, p in zip(outs, recs, ps):
+        check(B.rank_result(o), rec, p)
+
+
+@pytest.mark.parametrize("world", [2, 4])
+def test_record_sharded_ranking_equals_whole_set(B, sigma, world):
+    """Sec. IV-D's scan split by records: each slice ranked into its candidate
+    lists (global indices), the lists gathered (here: concatenated on one
+    GPU, as the all-gather lays them out) and merged; the victims, moves and
+    moved bytes equal the oracle's for the whole set."""
+    import torch
+    from paper_2609_09643_gb300 import shard
+    n = 1 << 22
+    rec = synth.make_records(51, n)
+    dev = B.records_to_device(rec)
+    for p in (prm(sigma, k=1024, budget=16 * GIB, max_moves=1024),
+              prm(sigma, k=37, budget=3 * GIB, max_moves=300, free_s=40_000)):
+        parts = []
+        for r in range(world):
+            off, cnt = shard.record_slice(n, r, world)
+            c = B.rank_cands(p["k"], p["max_moves"])
+            B.rank_shard({k: v[off:off + cnt] for k, v in dev.items()}, off, p, c)
+            parts.append(c)
+        out = B.rank_outputs(n, p["k"], p["max_moves"])
+        B.rank_merge(torch.cat(parts), world, p, out)
+        torch.cuda.synchronize()
+        check(B.rank_result(out), rec, p)

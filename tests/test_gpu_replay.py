@@ -70,6 +70,23 @@ def test_hand_trace_on_device(B):
         assert r[k] == v, k
 
 
+def test_hand_tide_trace_on_device(B):
+    """The hand-worked SPEAR+TIDE replay (phase-1 promotion beside pinned
+    sessions, order and budget stops of the pair loop, the DMA-busy window
+    and its exact end, prefetch accuracy) decided the same way on the
+    device."""
+    from test_oracle_pins import _hand_trace
+    tr, log, counts = _hand_trace("replay_hand_tide.txt")
+    p = base("spear_tide", 100, 1000, 1, t_p=20_000_000, dma=4)
+    res, lg, _ = run_gpu(B, [tr], [(0, p)], log_capacity=64)
+    r = res[0]
+    got = list(zip(*(map(int, a) for a in B.decode_log(lg[0], r["log_len"]))))
+    assert got == log
+    for k, v in counts.items():
+        assert r[k] == v, k
+    assert_same(r, oracle.replay(tr, to_oracle(p)), "hand tide")
+
+
 def test_paper_scale_30_replays(B):
     trs, reps = paper_scale_case()
     cap = 4 * trs[0].n_events
@@ -104,6 +121,24 @@ def test_large_pool_replay(B, seed):
     p = large_pool_params()
     res, _, _ = run_gpu(B, [tr], [(0, p)])
     assert_same(res[0], oracle.replay(tr, to_oracle(p)), seed)
+
+
+def test_large_pool_16_replays_one_call(B):
+    """The large-pool launch as the benchmark table runs it: many replays, each
+    on its own 65,536-session trace, in one call (the tier map without pin
+    slots, two CTAs per SM); every replay checked against the oracle in a
+    spawn pool."""
+    import multiprocessing as mp
+    import os
+    from cases import oracle_large_pool_job
+    seeds = list(range(100, 116))
+    trs = [synth.large_pool_trace(s) for s in seeds]
+    p = large_pool_params()
+    res, _, _ = run_gpu(B, trs, [(i, p) for i in range(len(seeds))])
+    with mp.get_context("spawn").Pool(min(os.cpu_count() or 1, 16)) as pool:
+        ores = pool.map(oracle_large_pool_job, seeds, chunksize=1)
+    for i, o in enumerate(ores):
+        assert_same(res[i], o, seeds[i])
 
 
 POLS = ["lru", "timeout", "spear", "spear_tide", "belady", "lru_tide"]

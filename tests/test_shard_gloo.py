@@ -2,7 +2,9 @@
 
 Replays shard with no data-path collective (each rank replays its own trace
 seeds); the job's time is the maximum over ranks and its rate counts every
-rank's units.  These tests run that logic in real processes over gloo."""
+rank's units.  A record-sharded ranking exchanges each rank's fixed-size
+candidate buffer in one all-gather.  These tests run that logic in real
+processes over gloo."""
 import os
 import socket
 
@@ -60,3 +62,49 @@ def test_single_process_is_identity():
         shard.job_rate([1], 1, 0.0)
     with pytest.raises(ValueError):
         shard.rank_seeds(-1)
+
+
+def _cands_worker(rank: int, world: int, port: int, out):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+    from paper_2609_09643_gb300 import binding as B
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        nbytes = B.rank_cands_bytes(1024, 512)
+        mine = torch.from_numpy(np.random.default_rng(100 + rank).integers(0, 256, nbytes, dtype=np.uint8))
+        got = shard.gather_cands(mine)
+        out.put((rank, nbytes, mine.numpy().tobytes(), got.numpy().tobytes()))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_gather_candidate_buffers():
+    """Every rank ends with the same merge input: the ranks' buffers back to
+    back in rank order, each of the size the library states."""
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_cands_worker, args=(r, 2, port, q)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = sorted(q.get(timeout=120) for _ in procs)
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    (_, nb, b0, g0), (_, _, b1, g1) = res
+    assert nb == 64 + 16 * (1024 + 2 * 512)
+    assert g0 == g1 == b0 + b1
+
+
+def test_record_slices_partition_the_set():
+    for n, world in ((10, 1), (10, 3), (1 << 22, 4), (7, 7)):
+        spans = [shard.record_slice(n, r, world) for r in range(world)]
+        assert spans[0][0] == 0 and all(c > 0 for _, c in spans)
+        assert all(spans[i][0] + spans[i][1] == spans[i + 1][0] for i in range(world - 1))
+        assert spans[-1][0] + spans[-1][1] == n
+        assert max(c for _, c in spans) - min(c for _, c in spans) <= 1
+    with pytest.raises(ValueError):
+        shard.record_slice(3, 0, 4)
