@@ -25,27 +25,24 @@ import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
-sys.path.insert(0, os.path.join(ROOT, "tests"))
 
 METRIC = "replay events/s (SPEAR+TIDE batched)"
 
 
-def filter_traffic(records_per_launch: int):
-    """DRAM bytes (read + write) per rank_filter launch from the ncu capture
-    summarised in profiles/rank_filter_2p24_ncu.md, scaled from one 2^24 set
-    to the launch's records; None when rank.cu has changed since the capture
-    (its hash no longer matches the recorded one) or the record is missing."""
+def rank_traffic(records_per_launch: int):
+    """DRAM bytes (read + write) of one rank_kernel launch from the ncu record
+    profiles/rank_kernel_traffic.json (one capture, per record), scaled to the
+    launch's records; None when rank.cu has changed since the capture (its
+    hash no longer matches the recorded one) or the record is missing."""
     import hashlib
     try:
-        text = open(os.path.join(ROOT, "profiles", "rank_filter_2p24_ncu.md")).read()
-        line = next(l for l in text.splitlines() if l.startswith("traffic-record:"))
-        rec = dict(kv.split("=") for kv in line.split()[1:])
+        rec = json.load(open(os.path.join(ROOT, "profiles", "rank_kernel_traffic.json")))
         src = open(os.path.join(ROOT, "paper_2609_09643_gb300", "csrc", "rank.cu"), "rb").read()
-        if hashlib.sha256(src).hexdigest()[:16] != rec["rank.cu-sha256-16"]:
+        if hashlib.sha256(src).hexdigest()[:16] != rec["rank_cu_sha256_16"]:
             return None
-        per_set = int(rec["dram_read_bytes_per_set"]) + int(rec["dram_write_bytes_per_set"])
-        return per_set * records_per_launch / int(rec["records_per_set"])
-    except (OSError, StopIteration, KeyError, ValueError):
+        per = (rec["dram_read_bytes"] + rec["dram_write_bytes"]) / rec["records"]
+        return per * records_per_launch
+    except (OSError, KeyError, ValueError, ZeroDivisionError):
         return None
 
 
@@ -63,9 +60,12 @@ def parse():
     ap.add_argument("--rank-n", type=int, default=1 << 24, help="records per live set")
     ap.add_argument("--rank-sets", type=int, default=7, help="live sets per call (<= 7)")
     ap.add_argument("--no-rank-sizes", action="store_true", help="skip the live-set size sweep")
-    ap.add_argument("--no-online", action="store_true", help="skip the online hazard-table report")
-    ap.add_argument("--no-stale", action="store_true", help="skip the stale-snapshot (dual design) report")
-    ap.add_argument("--no-ablation", action="store_true", help="skip the component/signal/capacity ablations")
+    ap.add_argument("--no-iid", action="store_true", help="skip the sweep on traces with independent gaps")
+    ap.add_argument("--online", action="store_true", help="add the online hazard-table report (Sec. V-F)")
+    ap.add_argument("--stale", action="store_true", help="add the stale-snapshot (dual design) report")
+    ap.add_argument("--ablation", action="store_true", help="add the component/signal/capacity ablations")
+    ap.add_argument("--ase", action="store_true", help="add eq. (ase) over the sweep's settings")
+    ap.add_argument("--reports", action="store_true", help="all of --online --stale --ablation --ase")
     ap.add_argument("--table", action="store_true",
                     help="per-config table instead of the bench line: GPU events/s, oracle 1-thread and all-core "
                          "events/s, parity, rank GB/s per live-set size")
@@ -133,7 +133,7 @@ class ClockSampler:
 def sweep_workload(rank: int):
     """The 1,024-replay sweep; under torchrun each rank replays it on its own
     trace seeds (rank 0: seeds 0-7, the single-GPU workload)."""
-    from cases import sweep_case, to_lib
+    from synth.workloads import sweep_case, to_lib
     import synth
     from paper_2609_09643_gb300 import shard
     trs, reps = sweep_case()
@@ -167,12 +167,15 @@ RANK_SIZES = (1 << 10, 1 << 14, 1 << 18, 1 << 20, 1 << 22, 1 << 24)
 RANK_KS = (1, 2, 4, 8, 16, 32, 64, 128, 256, 512, 1024)
 
 
-def rank_size_sweep(B, host_rec, sigma, stream, steps: int = 10, warmup: int = 3):
+def rank_size_sweep(B, host_rec, sigma, stream, peak: float, steps: int = 10, warmup: int = 3):
     """The live-set sizes of the ranking microbenchmark.  At each size one call
     ranks enough distinct sets (slices of the 2^24-record set, at most 64) to
     stream at least 2x the 129 MB L2, so no set is re-read from L2 between
     calls; k cycles through 1..1,024 and the budget through 1..64 GiB.
-    Call time = CUDA events around the call on its stream."""
+    call_us = CUDA events around `steps` back-to-back calls on their stream,
+    per call (the whole API call: descriptor upload and the kernel); host_us =
+    the host's time to issue one call.  frac = GB/s at 8 B/record over the
+    measured HBM peak; frac_12B at the plan's 12 B/record."""
     import torch
     out = []
     full = {k: v.to("cuda", non_blocking=True) for k, v in host_rec.items()}
@@ -196,27 +199,39 @@ def rank_size_sweep(B, host_rec, sigma, stream, steps: int = 10, warmup: int = 3
             call.run(stream)
         torch.cuda.synchronize()
         assert all(B.rank_result(o)["status"] == 0 for o in outs), "rank status"
-        for kname in ("rank_sample", "rank_filter", "rank_finish"):
-            B.profile_read(kname, reset=True)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
+        t0 = time.perf_counter()
         for _ in range(steps):
             call.run(stream)
+        host_us = 1e6 * (time.perf_counter() - t0) / steps
         e1.record(stream)
         torch.cuda.synchronize()
         call_us = 1e3 * e0.elapsed_time(e1) / steps
-        f_ms, f_n = B.profile_read("rank_filter", reset=True)
-        sm_ms, sm_n = B.profile_read("rank_sample", reset=True)
-        fi_ms, fi_n = B.profile_read("rank_finish", reset=True)
         recs = n * n_sets
         gbs = recs * RANK_BYTES_PER_RECORD / (call_us / 1e6) / 1e9
-        filter_us = 1e3 * f_ms / max(f_n, 1) if f_n else None
-        out.append({"n": n, "sets_per_call": n_sets, "call_us": call_us, "filter_us": filter_us,
-                    "sample_us": 1e3 * sm_ms / max(sm_n, 1), "finish_us": 1e3 * fi_ms / max(fi_n, 1), "call_gbs": gbs,
-                    "filter_gbs": recs * RANK_BYTES_PER_RECORD / (filter_us / 1e6) / 1e9 if filter_us else None,
-                    "l2_resident": recs * RANK_BYTES_PER_RECORD < (2 * 129 << 20)})
+        out.append({"n": n, "sets": n_sets, "call_us": round(call_us, 2), "host_us": round(host_us, 1),
+                    "gbs": round(gbs, 1), "frac": round(gbs / peak, 4), "frac_12B": round(1.5 * gbs / peak, 4)})
         del call, sets, outs
-    return out
+    # one set of 2^20 records: the latency of a single call (idle stream)
+    n = 1 << 20
+    one = [{k: v[:n] for k, v in full.items()}]
+    p1 = [dict(sigma_q=sigma, k=1024, penalty_q=500_000_000, budget_bytes=8 << 30, kv_bytes_per_token=131072,
+               max_moves=1024, free_fast_tok=0, free_hbm_tok=1 << 40)]
+    o1 = [B.rank_outputs(n, 1024, 1024)]
+    call = B.rank_prepare(one, p1, o1)
+    lat = []
+    for i in range(steps + warmup):
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        call.run(stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        if i >= warmup:
+            lat.append(1e3 * a.elapsed_time(b))
+    single = {"n": n, "sets": 1, "call_us_median": round(statistics.median(lat), 2)}
+    return out, single
 
 
 def kendall_fp32_vs_fixed(B, host_rec, sigma, stream, n: int = 1 << 20):
@@ -246,8 +261,7 @@ def kendall_fp32_vs_fixed(B, host_rec, sigma, stream, n: int = 1 << 20):
     done = (host_rec["flags"][:n].numpy() & 2) != 0
     f32 = np.where(done, np.float32(np.inf), f32).astype(np.float32)
     tau = kendalltau(fixed.astype(np.float64), f32.astype(np.float64))[0]
-    return {"tau_b": float(tau), "records": n, "fixed": "rank kernel keys (eq. scoreq)",
-            "float": "float32 g*Lambda/sigma_q + (Lambda-sigma_q)*P_Z/Lambda"}
+    return {"tau_b": float(tau), "records": n}
 
 
 def sweep_ase(B, results, reps, lib_params):
@@ -274,7 +288,7 @@ def online_hazard_report(B, stream, steps: int = 3, points: int = 8):
     import math
     import torch
     import synth
-    from cases import GIB, KVB_PAPER, base, to_lib
+    from synth.workloads import GIB, KVB_PAPER, base, to_lib
     mixes = ("coding", "general")
     trs = [synth.paper_scale_trace(1, m) for m in mixes]
     handles = [B.Trace(t).upload(stream) for t in trs]
@@ -328,7 +342,7 @@ def stale_snapshot_report(B, stream, steps: int = 3):
     rate, fast-tier hit share, prefill reduction (points) and AMAT (percent)."""
     import torch
     import synth
-    from cases import GIB, base, to_lib
+    from synth.workloads import GIB, base, to_lib
     mixes = ("coding", "general")
     trs = [synth.paper_scale_trace(1, m) for m in mixes]
     handles = [B.Trace(t).upload(stream) for t in trs]
@@ -383,7 +397,7 @@ def ablation_report(B, stream):
       fast 32K tokens, the fast tier swept at HBM 512K tokens, and the fast
       share of a 256K-token total swept: mean gains over the two traces."""
     import synth
-    from cases import base, to_lib
+    from synth.workloads import base, to_lib
     kvb, tok = 131072, lambda n: n * 131072
     mixes = ("coding", "general")
     trs = [synth.paper_scale_trace(1, m) for m in mixes]
@@ -441,7 +455,7 @@ def cpu_baseline_replay(trs, reps, budget_s: float = 12.0):
     """The oracle as it stands, single-threaded, on a bounded sample of the
     sweep's replays (spread over the batch) until budget_s of CPU work."""
     import oracle
-    from cases import to_oracle
+    from synth.workloads import to_oracle
     order = list(range(0, len(reps), 37)) + list(range(1, len(reps), 37))
     ev, n, t0 = 0, 0, time.perf_counter()
     for i in order:
@@ -472,7 +486,7 @@ def cpu_baseline_rank(rec, sigma, n: int = 1 << 22):
 def _oracle_replay_job(job):
     """One oracle replay in a worker process (the pool uses spawn)."""
     import oracle
-    from cases import to_oracle
+    from synth.workloads import to_oracle
     tr, p = job
     return oracle.replay(tr, to_oracle(p))
 
@@ -497,7 +511,7 @@ def _oracle_large_job(seed):
     """One large-pool oracle replay in a worker (it generates its own trace)."""
     import oracle
     import synth
-    from cases import large_pool_params, to_oracle
+    from synth.workloads import large_pool_params, to_oracle
     return oracle.replay(synth.large_pool_trace(seed), to_oracle(large_pool_params()))
 
 
@@ -508,7 +522,7 @@ def large_pool_table(B, pool, stream, fields, cores):
     threads, so the parent never holds more than the pinned upload copies."""
     from concurrent.futures import ThreadPoolExecutor
     import torch
-    from cases import large_pool_params, to_lib, to_oracle
+    from synth.workloads import large_pool_params, to_lib, to_oracle
     import oracle
     import synth
     seeds = list(range(100, 356))
@@ -563,7 +577,7 @@ def config_table(args):
     import multiprocessing as mp
     import torch
     import synth
-    from cases import tiny_case, paper_scale_case, sweep_case, large_pool_params, to_lib, to_oracle
+    from synth.workloads import tiny_case, paper_scale_case, sweep_case, large_pool_params, to_lib, to_oracle
     import oracle
     from paper_2609_09643_gb300 import native
     torch.cuda.set_device(0)
@@ -629,18 +643,13 @@ def config_table(args):
     sig_dev, _ = B.hazard_lut(tps_dev, 1)
     sigma = sig_dev.cpu().numpy().astype("uint16")
     host_rec = {k: v.pin_memory() for k, v in B.records_to_device(rec, device="cpu").items()}
-    B.profile_enable(True)
-    sizes = rank_size_sweep(B, host_rec, sigma, stream)
-    B.profile_enable(False)
+    sizes, single = rank_size_sweep(B, host_rec, sigma, stream, pk)
     one = cpu_baseline_rank(rec, sigma)
     t0 = time.perf_counter()
     n = sum(pool.map(_oracle_rank_job, [(rec, sigma, 1 << 22)] * cores, chunksize=1))
     allc = n * RANK_BYTES_PER_RECORD / (time.perf_counter() - t0) / 1e9
     pool.close()
-    out.append({"config": "4 rank", "gpu": [{"n": e["n"], "sets": e["sets_per_call"], "call_gbs": e["call_gbs"],
-                                            "call_frac": e["call_gbs"] / pk, "filter_gbs": e["filter_gbs"],
-                                            "filter_frac": e["filter_gbs"] / pk if e["filter_gbs"] else None}
-                                           for e in sizes],
+    out.append({"config": "4 rank", "gpu": sizes, "gpu_single_set": single,
                 "oracle_1core_gbs": one["value"], "oracle_allcore_gbs": allc, "cores": cores,
                 "oracle_sample": "2^22 records of one 2^24 live set per core, k=1,024, full sort + fill"})
     print(json.dumps({"table": out, "peak_hbm_gbs": pk}), flush=True)
@@ -651,7 +660,7 @@ def run_reference(args):
     if rank != 0:
         return
     import oracle
-    from cases import to_oracle
+    from synth.workloads import to_oracle
     trs, reps, _ = sweep_workload(0)
     per_step = 8
     order = list(range(0, len(reps), 127))
@@ -672,7 +681,8 @@ def run_reference(args):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
             "data": "synthetic",
             "config": {"workload": "sweep-1024 (8 seeds x 8 capacity pairs x 16 window/bucket settings, "
-                                   "paper-scale coding trace, 131072 B/token, SPEAR+TIDE)",
+                                   "paper-scale coding trace, gap persistence rho = 0.7, 131072 B/token, "
+                                   "SPEAR+TIDE)",
                        "sample_per_step": f"{per_step} replays", "l2": "n/a (CPU)"},
             "cpu_baseline": {"kind": "oracle", "cores": 1, "value": v, "unit": "events/s",
                              "sample": f"{per_step} sweep replays per step, single-threaded C oracle"},
@@ -748,7 +758,7 @@ def main():
     if not args.rank_only:
         res = B.results_from_tensor(res_dev)
         assert all(r["status"] == 0 for r in res), "replay status"
-        if len(res) == 1024:
+        if len(res) == 1024 and (args.ase or args.reports):
             ase = sweep_ase(B, res, reps, lib_params)
     if not args.replay_only:
         assert all(B.rank_result(o)["status"] == 0 for o in rank_outs), "rank status"
@@ -761,7 +771,7 @@ def main():
     torch.cuda.synchronize()
     clk = ClockSampler(dev)
     B.profile_enable(True)
-    for kname in ("replay", "key_stream", "ttft_median", "rank_sample", "rank_filter", "rank_finish"):
+    for kname in ("replay", "key_stream", "ttft_median", "rank"):
         B.profile_read(kname, reset=True)
     launches0 = B.launch_count()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -776,37 +786,64 @@ def main():
     rep_ms, rep_n = B.profile_read("replay", reset=True)
     ks_ms, ks_n = B.profile_read("key_stream", reset=True)
     md_ms, md_n = B.profile_read("ttft_median", reset=True)
-    rs_ms, rs_n = B.profile_read("rank_sample", reset=True)
-    rf_ms, rf_n = B.profile_read("rank_filter", reset=True)
-    rn_ms, rn_n = B.profile_read("rank_finish", reset=True)
+    rk_ms, rk_n = B.profile_read("rank", reset=True)
     B.profile_enable(False)
     clocks = clk.stop()
     from paper_2609_09643_gb300 import shard
     ms = shard.max_over_ranks(ms, device="cuda")
     units = shard.units_over_ranks(events_per_step, device="cuda")
     value = shard.job_rate(units, args.steps, ms) if not args.rank_only else None
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        pass
+    hbm_peak = peaks.get("hbm_gbs") or 6800.0
 
-    sizes = None
+    sizes = single = None
     tau = None
     if not args.replay_only:
         tau = kendall_fp32_vs_fixed(B, host_rec, sigma, stream)
     if not args.replay_only and not args.no_rank_sizes:
-        B.profile_enable(True)
-        sizes = rank_size_sweep(B, host_rec, sigma, stream)
-        B.profile_enable(False)
-        pk = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json"))).get("hbm_gbs") or 6800.0
-        for e in sizes:
-            e["call_frac_of_peak"] = e["call_gbs"] / pk
-            e["filter_frac_of_peak"] = e["filter_gbs"] / pk if e["filter_gbs"] else None
+        sizes, single = rank_size_sweep(B, host_rec, sigma, stream, hbm_peak)
 
+    # the sweep on traces whose gaps are drawn independently (no per-session
+    # persistence): the survey's gap model, timed like the main leg
+    iid = None
+    if not (args.no_iid or args.rank_only or world > 1):
+        from synth.workloads import sweep_case, to_lib
+        trs0, reps0 = sweep_case(gap_persist=0.0)
+        h0 = [B.Trace(t).upload(stream) for t in trs0]
+        p0 = [to_lib(p, ti) for ti, p in reps0]
+        ev0 = sum(2 * trs0[ti].n_turns for ti, _ in reps0)
+        r0 = torch.zeros(B.result_nbytes(len(p0)), dtype=torch.uint8, device="cuda")
+        for _ in range(2):
+            B.replay_batch_async(h0, p0, r0, stream=stream)
+        torch.cuda.synchronize()
+        assert all(r["status"] == 0 for r in B.results_from_tensor(r0)), "replay status"
+        n_iid = max(3, args.steps // 2)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n_iid):
+            flush.zero_()
+            B.replay_batch_async(h0, p0, r0, stream=stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        iid = {"gap_persistence": 0.0, "events_per_step": ev0, "steps": n_iid,
+               "ms_per_step": round(a.elapsed_time(b) / n_iid, 3),
+               "events_per_s": ev0 * n_iid / (a.elapsed_time(b) / 1e3)}
+        for h in h0:
+            h.close()
+
+    rep_all = args.reports
     online = None
-    if not (args.no_online or args.rank_only or args.replay_only) and rank == 0:
+    if (args.online or rep_all) and not (args.rank_only or args.replay_only) and rank == 0:
         online = online_hazard_report(B, stream)
     stale = None
-    if not (args.no_stale or args.rank_only or args.replay_only) and rank == 0:
+    if (args.stale or rep_all) and not (args.rank_only or args.replay_only) and rank == 0:
         stale = stale_snapshot_report(B, stream)
     ablation = None
-    if not (args.no_ablation or args.rank_only or args.replay_only) and rank == 0:
+    if (args.ablation or rep_all) and not (args.rank_only or args.replay_only) and rank == 0:
         ablation = ablation_report(B, stream)
 
     # end to end through the public API, every step: the step's traces and live
@@ -881,32 +918,26 @@ def main():
                    "hbm_gbs": alg_bytes / (avg_rep_ms / 1e3) / 1e9, "launches_timed": rep_n,
                    "share_of_step": avg_rep_ms * args.steps / ms if ms else None,
                    "key_stream_avg_ms": ks_ms / max(ks_n, 1), "ttft_median_avg_ms": md_ms / max(md_n, 1)}
-    peaks = {}
-    try:
-        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
-    except Exception:
-        pass
-    hbm_peak = peaks.get("hbm_gbs") or 6800.0
-    avg_rf = rf_ms / max(rf_n, 1) if rf_n else float("nan")
-    achieved = rank_bytes / (avg_rf / 1e3) / 1e9 if rf_n else float("nan")
-    roofline = {"bound": "hbm", "kernel": "rank_filter_kernel", "achieved": achieved, "peak": hbm_peak,
+    avg_rk = rk_ms / max(rk_n, 1) if rk_n else float("nan")
+    achieved = rank_bytes / (avg_rk / 1e3) / 1e9 if rk_n else float("nan")
+    n_rec = len(r_params) * RANK_N
+    # the whole ranking call is one kernel: sample, filter and finish of every set
+    roofline = {"bound": "hbm", "kernel": "rank_kernel", "achieved": achieved, "peak": hbm_peak,
                 "unit": "GB/s", "frac": achieved / hbm_peak,
                 "peak_source": "measured (MEASURED_PEAKS.json hbm_gbs, burst copy)" if peaks.get("hbm_gbs")
-                else "fallback 6.8 TB/s", "traffic": filter_traffic(len(r_params) * RANK_N),
-                "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum of one 2^24 set, scaled by records",
-                "avg_ms": avg_rf, "launches_timed": rf_n,
-                "algorithmic_bytes_per_launch": rank_bytes,
-                "bytes_per_record": RANK_BYTES_PER_RECORD, "records_per_launch": len(r_params) * RANK_N}
-    call_ms = (rs_ms + rf_ms + rn_ms) / max(rf_n, 1) if rf_n else float("nan")
-    rank_leg = {"metric": "rank-kernel HBM GB/s", "sets_per_call": len(r_params), "records_per_set": RANK_N,
-                "k": 1024, "budgets_gib": list(RANK_BUDGETS_GIB),
-                "call_ms": call_ms, "call_gbs": rank_bytes / (call_ms / 1e3) / 1e9,
+                else "fallback 6.8 TB/s", "traffic": rank_traffic(n_rec),
+                "traffic_source": "profiles/rank_kernel_traffic.json (ncu dram bytes per record, scaled)",
+                "avg_ms": avg_rk, "launches_timed": rk_n, "algorithmic_bytes_per_launch": rank_bytes,
+                "bytes_per_record": RANK_BYTES_PER_RECORD, "records_per_launch": n_rec,
+                "at_12B_per_record": {"achieved": 1.5 * achieved, "frac": 1.5 * achieved / hbm_peak},
+                "bytes_reading": "8 B/record streamed (gap 4, turn 2, flags 1, tier 1); sizes are gathered "
+                                 "only for the <= 4,096 movable records per list, so kv_tok is not streamed"}
+    call_ms = (sum(a.elapsed_time(b) for a, b in rank_marks) / len(rank_marks)) if rank_marks else float("nan")
+    rank_leg = {"sets_per_call": len(r_params), "records_per_set": RANK_N, "k": 1024,
+                "call_ms": call_ms, "kernel_ms": avg_rk,
+                "call_gbs": rank_bytes / (call_ms / 1e3) / 1e9,
                 "call_frac_of_peak": rank_bytes / (call_ms / 1e3) / 1e9 / hbm_peak,
-                "records_per_s": len(r_params) * RANK_N / (call_ms / 1e3),
-                "sample_ms": rs_ms / max(rs_n, 1), "filter_ms": avg_rf, "finish_ms": rn_ms / max(rn_n, 1),
-                # the whole API call on its stream: kernels plus the upload and launch gaps
-                "call_ms_events": (sum(a.elapsed_time(b) for a, b in rank_marks) / len(rank_marks)
-                                   if rank_marks else None)}
+                "call_frac_of_peak_12B": 1.5 * rank_bytes / (call_ms / 1e3) / 1e9 / hbm_peak}
     if rank != 0:
         return
     cpu = None if (args.no_cpu_baseline or world > 1) else cpu_baseline_replay(trs, reps)
@@ -914,12 +945,17 @@ def main():
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int64", "data": "synthetic",
             "config": {"workload": "sweep-1024 (8 seeds x 8 capacity pairs x 16 window/bucket settings, "
-                                   "paper-scale coding trace, 131072 B/token, SPEAR+TIDE)",
+                                   "paper-scale coding trace, gap persistence rho = 0.7, 131072 B/token, "
+                                   "SPEAR+TIDE)",
                        "replays": n_rep, "events_per_step": events_per_step,
                        "l2": "flushed before every step (256 MiB write, inside the timed region)"},
-            "roofline": roofline, "rank": rank_leg, "rank_sizes": sizes, "rank_kendall": tau, "sweep_ase": ase, "online_hazard": online, "stale_snapshot": stale, "ablation": ablation, "replay_roofline": replay_roof, "cpu_baseline": cpu, "e2e": e2e,
-            "gpu_launches": launches, "clocks": clocks,
-            "peaks": {"hbm_gbs": peaks.get("hbm_gbs"), "source": "MEASURED_PEAKS.json"}}
+            "roofline": roofline, "rank": rank_leg, "rank_sizes": sizes, "rank_single_set": single,
+            "rank_kendall": tau, "sweep_iid_gaps": iid, "replay_roofline": replay_roof, "cpu_baseline": cpu,
+            "e2e": e2e, "gpu_launches": launches, "clocks": clocks}
+    for key, val in (("sweep_ase", ase), ("online_hazard", online), ("stale_snapshot", stale),
+                     ("ablation", ablation)):
+        if val is not None:
+            line[key] = val
     if cpu is not None:
         cpu["rank"] = cpu_baseline_rank(rec, sigma)
     print(json.dumps(line), flush=True)
