@@ -12,27 +12,31 @@
 // One cooperative, persistent kernel does a whole call.  Each set owns a
 // group of CTAs (in proportion to its records; with more sets than CTAs,
 // each CTA takes whole sets in turn).  Per set, inside the group:
-//   sample   up to 16 CTAs gather a jittered stratified sample and count it
-//            into a 4,096-bin histogram per list (bins monotone in the list
-//            value); the last of them cuts each histogram at the list's
-//            sample rank, which gives per-list thresholds and per-turn
-//            thresholds on the gap average (the score is monotone in the gap
-//            for a fixed turn, so the streaming test needs no division), and
-//            publishes them with a flag.  Meanwhile every CTA's producer warp
-//            already streams its first tiles into shared memory.
+//   sample   up to 16 CTAs gather a jittered stratified sample, count it in
+//            shared memory and add it to a 4,096-bin histogram per list (bins
+//            monotone in the list value).  Once every sampling CTA's counts
+//            are in, each CTA of the group cuts the histograms at the lists'
+//            sample ranks itself: per-list thresholds and per-turn thresholds
+//            on the gap average (the score is monotone in the gap for a fixed
+//            turn, so the streaming test needs no division).  Meanwhile every
+//            CTA's producer warp already streams its first tiles into shared
+//            memory.
 //   filter   the group's CTAs take the set's tiles from a shared counter;
 //            every record is read once (8 B: gap average, turn, flags, tier)
 //            by TMA bulk copies and tested against the thresholds, and the
-//            exact values of the records that pass are appended per list and
-//            counted into a candidate histogram per list.
+//            exact values of the records that pass are appended per list to
+//            the CTA's own region, which moves into the set's list when the
+//            CTA is done.
 //   finish   the last three CTAs of the group to finish streaming take one
-//            list each: the candidate histogram gives a bin cut, the
-//            candidates at or above it are sorted (bitonic network) and the
-//            first M kept; a list whose cut holds too many or too few values
-//            falls back to a radix select, and one whose candidates
-//            overflowed or fell short is re-selected exactly by streaming the
-//            set.  The last list's CTA runs the fill as block scans and
-//            writes the outputs.
+//            list each: a 256-bucket cut below the candidates' common prefix
+//            keeps the bucket holding the rank-M value and those above it,
+//            which are bucket-sorted and the first M kept; a list whose cut
+//            holds too many values falls back to a radix select, and one
+//            whose candidates overflowed or fell short is re-selected exactly
+//            by streaming the set.  The last list's CTA runs the fill, 256
+//            items at a time, and writes the outputs.
+// The work words and sample histograms of a call are held twice: calls on a
+// stream alternate between the two, and each call zeroes the other.
 // Every wait on another CTA or on a copy is bounded: a wait that gives up
 // records UNISON_ERR_TIMEOUT in the set's status word and the CTA carries on
 // to the end of the kernel.  A cooperative launch keeps every CTA of the grid
@@ -120,12 +124,11 @@ struct alignas(128) RankWork {
   unsigned int cand[kLists];    // candidates emitted per list
   unsigned int next_tile;       // the group's tile counter
   unsigned int pad0[28];
-  // the sample
+  // the sample's reads done (polled by the producers)
   unsigned int gathered;        // sampling CTAs whose sample has arrived
-  unsigned int sample_ticket;   // sampling CTAs finished
-  unsigned int pad1[30];
-  // thresholds published (polled by every CTA of the group)
-  unsigned int ready;
+  unsigned int pad1[31];
+  // the sample's counts in the histogram (polled by every CTA of the group)
+  unsigned int sample_ticket;   // sampling CTAs whose counts have landed
   unsigned int pad2[31];
   // the finish
   unsigned int done_ctas;       // CTAs of the group done streaming
@@ -496,9 +499,6 @@ __device__ void hist_cut3(unsigned int *hist, const uint32_t (&need)[kLists], in
   }
 #pragma unroll
   for (int L = 0; L < kLists; L++) {
-    uint4 *h4 = reinterpret_cast<uint4 *>(hist + L * kBins + lo);
-#pragma unroll
-    for (int q = 0; q < 4; q++) h4[q] = make_uint4(0u, 0u, 0u, 0u);
     tot[L] = 0;
 #pragma unroll
     for (int q = 0; q < 16; q++) tot[L] += c[L][q];
@@ -835,14 +835,11 @@ void plan_sample(RankSet &s) {
 // Sampling CTA r of set S (consumer threads): samples j = r * per + jt of
 // the CTA's share, run j / 8 covering stratum j / 8 (records [run n / nruns,
 // (run+1) n / nruns)), 8 consecutive records at a hashed offset in it; each
-// eligible sample is counted into its lists' histograms.  The last sampling
-// CTA cuts each list's histogram at r_L: its threshold is the smallest list
-// value in the bin holding the rank-r_L sample (at least r_L samples reach
-// it), plus, per turn index, the smallest gap whose key reaches the
-// threshold's key (gA) or exceeds it (gB).  It publishes them (ready = 1).
+// eligible sample is counted into its lists' histograms (first in shared
+// memory, then the non-zero bins into the set's), and the CTA's ticket says
+// its counts are in.
 __device__ __noinline__ void sample_share(const RankSet &S, uint32_t r, const uint64_t *t2s, const uint64_t *mgs,
-                                         const uint32_t *sgs, unsigned int *lh, uint64_t *sfree) {
-  __shared__ unsigned int is_last;
+                                         unsigned int *lh, uint64_t *sfree) {
   const uint32_t tid = threadIdx.x;
   const uint32_t nct = S.sctas, act = S.act;
   const uint32_t per = S.ns / nct;  // samples of this CTA (<= 1024, a multiple of 8)
@@ -906,59 +903,57 @@ __device__ __noinline__ void sample_share(const RankSet &S, uint32_t r, const ui
   __threadfence();
   consumers_sync();
   if (tid == 0) {
-    mbar_arrive(sfree);  // the stage area is the producer's again
-    is_last = (atomicAdd(&S.work->sample_ticket, 1u) == nct - 1);
+    mbar_arrive(sfree);                      // the stage area is the producer's again
+    atomicAdd(&S.work->sample_ticket, 1u);  // this CTA's counts are in the histogram
   }
-  consumers_sync();
-  if (!is_last) return;
-  __threadfence();
-  const uint32_t need[kLists] = {S.rL[0], S.rL[1], S.rL[2]};
-  int cut[kLists];
-  hist_cut3(S.shist, need, cut);
-#pragma unroll 1
-  for (int L = 0; L < kLists; L++) {
-    // 0 (fewer than r_L eligible samples, or none taken): accept every eligible record
-    const uint64_t thrv = cut[L] >= 0 ? summary_floor(bin_floor((uint32_t)cut[L])) : 0ull;
-    if (tid == 0) {
-      S.thr[L] = thrv;
-      S.thr[kLists + L] = (act >> L) & 1;
-    }
-    if (tid < kLutN) {
-      const uint64_t thr_ck = (L == 2) ? ~thrv : thrv;
-      const uint64_t K = thr_ck >> 24;
-      S.gthr[L * kLutN + tid] = make_uint2(g_at_least(K, sgs[tid], t2s[tid]), g_at_least(K + 1, sgs[tid], t2s[tid]));
-    }
-  }
-  __threadfence();
-  consumers_sync();
-  if (tid == 0) atomicExch(&S.work->ready, 1u);
 }
 
 // ------------------------------------------------------------- filter ----
 struct SetConst {
+  uint64_t thr[kLists];        // threshold per list, in list-value space (0: every eligible record)
   uint32_t loV, loD, loP;      // index thresholds of the tie on the threshold key
   uint32_t dV, dD;             // completed records pass V / D iff lo >= dV / dD
   int32_t dP;                  // completed records pass P iff lo <= dP
   uint32_t act;                // active lists (bit L)
 };
 
-// Thresholds of one set into shared memory (consumer threads).  Per turn
-// index: vd = (gA_V, gB_V, gA_D, gB_D), pp = (gA_P, gB_P); an inactive list
-// gets bounds no gap passes.
-__device__ void load_set(const RankSet &S, uint4 *vd, uint2 *pp, SetConst &c) {
-  const bool aV = __ldcg(&S.thr[kLists + 0]) != 0, aD = __ldcg(&S.thr[kLists + 1]) != 0,
-             aP = __ldcg(&S.thr[kLists + 2]) != 0;
+// Thresholds of one set into shared memory (consumer threads), computed by
+// every CTA of the group alike once the sample's counts are all in the
+// histogram: each list's histogram is cut at its sample rank r_L, the
+// threshold is the smallest list value of the cut's bin (0, every eligible
+// record, when the sample holds fewer than r_L), and per turn index t the
+// bounds are the smallest gap whose key reaches the threshold's key (gA) or
+// exceeds it (gB): vd = (gA_V, gB_V, gA_D, gB_D), pp = (gA_P, gB_P).  An
+// inactive list gets bounds no gap passes.
+__device__ void thresholds(const RankSet &S, const uint64_t *t2s, const uint32_t *sgs, uint4 *vd, uint2 *pp,
+                           SetConst &c) {
+  __shared__ uint64_t sthr[kLists];
+  int cut[kLists] = {-1, -1, -1};
+  if (S.ns) {
+    const uint32_t need[kLists] = {S.rL[0], S.rL[1], S.rL[2]};
+    hist_cut3(S.shist, need, cut);
+  }
+  if (threadIdx.x < kLists) sthr[threadIdx.x] = cut[threadIdx.x] >= 0 ? summary_floor(bin_floor((uint32_t)cut[threadIdx.x])) : 0ull;
+  consumers_sync();
+  const bool aV = S.act & 1, aD = (S.act >> 1) & 1, aP = (S.act >> 2) & 1;
   if (threadIdx.x < kLutN) {
     const uint32_t t = threadIdx.x;
-    const uint2 a0 = __ldcg(&S.gthr[t]), a1 = __ldcg(&S.gthr[kLutN + t]), a2 = __ldcg(&S.gthr[2 * kLutN + t]);
-    vd[t] = make_uint4(aV ? a0.x : kFull, aV ? a0.y : kFull, aD ? a1.x : kFull, aD ? a1.y : kFull);
-    pp[t] = aP ? a2 : make_uint2(0u, 0u);
+    uint2 g[kLists];
+#pragma unroll
+    for (int L = 0; L < kLists; L++) {
+      const uint64_t thr_ck = (L == 2) ? ~sthr[L] : sthr[L];
+      const uint64_t K = thr_ck >> 24;
+      g[L] = make_uint2(g_at_least(K, sgs[t], t2s[t]), g_at_least(K + 1, sgs[t], t2s[t]));
+    }
+    vd[t] = make_uint4(aV ? g[0].x : kFull, aV ? g[0].y : kFull, aD ? g[1].x : kFull, aD ? g[1].y : kFull);
+    pp[t] = aP ? g[2] : make_uint2(0u, 0u);
   }
   if (threadIdx.x == 32) {
     uint32_t lo[kLists], dok[kLists];
 #pragma unroll
     for (int L = 0; L < kLists; L++) {
-      const uint64_t thrv = __ldcg(&S.thr[L]);
+      const uint64_t thrv = sthr[L];
+      c.thr[L] = thrv;
       const uint64_t thr_ck = (L == 2) ? ~thrv : thrv;
       const uint64_t K = thr_ck >> 24;
       lo[L] = (uint32_t)(thr_ck & kIdMask);
@@ -972,7 +967,7 @@ __device__ void load_set(const RankSet &S, uint4 *vd, uint2 *pp, SetConst &c) {
     c.dV = !aV ? 0x1000000u : (dok[0] == 2 ? 0u : (dok[0] == 1 ? lo[0] : 0x1000000u));
     c.dD = !aD ? 0x1000000u : (dok[1] == 2 ? 0u : (dok[1] == 1 ? lo[1] : 0x1000000u));
     c.dP = (aP && dok[2] == 1) ? (int32_t)lo[2] : -1;
-    c.act = (aV ? 1u : 0u) | (aD ? 2u : 0u) | (aP ? 4u : 0u);
+    c.act = S.act;
   }
   consumers_sync();
 }
@@ -1030,7 +1025,7 @@ __device__ __noinline__ uint32_t stream_topM(const RankSet &S, int L, uint32_t M
 // records' sizes; victims are written out directly.  fin: the 64 KB dynamic
 // area (the stages are idle).  Returns true when this was the set's last list.
 __device__ __noinline__ bool finish_list(const RankSet &S, int L, uint64_t *fin, const uint64_t *t2s, const uint64_t *mgs,
-                                         SelectScratch &ss) {
+                                         SelectScratch &ss, const SetConst &cs) {
   __shared__ __align__(8) uint64_t cbar;
   __shared__ unsigned int last, sh_emitted, sh_flags, nsurv;
   uint64_t *buf = fin;               // [kSmemCand] candidates
@@ -1040,7 +1035,7 @@ __device__ __noinline__ bool finish_list(const RankSet &S, int L, uint64_t *fin,
   // takes the same path through the barriers below
   if (tid == 0) {
     sh_emitted = __ldcg(&S.work->cand[L]);
-    sh_flags = (__ldcg(&S.thr[kLists + L]) != 0 ? 1u : 0u) | (__ldcg(&S.thr[L]) == 0 ? 2u : 0u);
+    sh_flags = ((cs.act >> L) & 1u) | (cs.thr[L] == 0 ? 2u : 0u);
   }
   consumers_sync();
   const bool active = sh_flags & 1;
@@ -1245,7 +1240,7 @@ __device__ __noinline__ void fill(const RankSet &S, uint64_t *fin) {
   const uint32_t tid = threadIdx.x;
   if (tid == 0) {  // read once and shared: one path through the barriers
     for (int L = 0; L < kLists; L++) sh_got[L] = min(__ldcg(&S.work->got[L]), kMaxSel);
-    sh_act = (__ldcg(&S.thr[kLists + 1]) != 0 ? 2u : 0u) | (__ldcg(&S.thr[kLists + 2]) != 0 ? 4u : 0u);
+    sh_act = S.act & 6u;
     sh_st = *(volatile unsigned int *)&S.work->status;
   }
   consumers_sync();
@@ -1380,8 +1375,11 @@ __device__ __noinline__ void fill(const RankSet &S, uint64_t *fin) {
 // set's counter and announces each stage's tile in stile[]; a partial last
 // tile (read directly from global memory by the consumers) and the end of
 // the set (kEndTile) are announced with a plain arrival.
+// zero_a / zero_b (n_a, n_b 16-byte words): the other parity's work words
+// and sample histograms, zeroed here for the next call on the stream.
 __global__ void __launch_bounds__(kCtaThreads, 3)
-    rank_kernel(const RankSet *sets, int n_sets, int sequential) {
+    rank_kernel(const RankSet *sets, int n_sets, int sequential, uint4 *zero_a, uint32_t n_a, uint4 *zero_b,
+                uint32_t n_b) {
   extern __shared__ __align__(128) unsigned char dsm[];
   FilterStage *stage = reinterpret_cast<FilterStage *>(dsm);
   uint64_t *fin = reinterpret_cast<uint64_t *>(dsm);
@@ -1401,6 +1399,11 @@ __global__ void __launch_bounds__(kCtaThreads, 3)
   __shared__ __align__(8) uint64_t dummy_bar;
 #endif
 
+  {  // every CTA takes its share, before any returns
+    const uint32_t g = blockIdx.x * blockDim.x + threadIdx.x, gs = gridDim.x * blockDim.x;
+    for (uint32_t w = g; w < n_a; w += gs) zero_a[w] = make_uint4(0u, 0u, 0u, 0u);
+    for (uint32_t w = g; w < n_b; w += gs) zero_b[w] = make_uint4(0u, 0u, 0u, 0u);
+  }
   int s0, sstep;
   if (sequential) {
     s0 = blockIdx.x;
@@ -1540,14 +1543,14 @@ __global__ void __launch_bounds__(kCtaThreads, 3)
       sgs[ct] = S.tab->sigma[ct];
     }
     consumers_sync();
-    // 1. thresholds: the sampling CTAs sample, the last of them publishes
-    if (r < S.sctas) sample_share(S, r, t2s, mgs, sgs, reinterpret_cast<unsigned int *>(dsm), &sfree);
+    // 1. thresholds: the sampling CTAs sample; every CTA cuts the histograms
+    if (r < S.sctas) sample_share(S, r, t2s, mgs, reinterpret_cast<unsigned int *>(dsm), &sfree);
 #ifdef UNISON_DEBUG_HOOKS
     if (s == g_hook_flag_set) wait_word(S, &S.work->dummy, 1u);  // nothing sets it: runs out
 #endif
-    wait_word(S, &S.work->ready, 1u);
-    if (ct < kLists) ccnt_s[ct] = 0;  // published by load_set's barrier
-    load_set(S, vd, pp, c);
+    wait_word(S, &S.work->sample_ticket, S.sctas);
+    if (ct < kLists) ccnt_s[ct] = 0;  // published by the barriers below
+    thresholds(S, t2s, sgs, vd, pp, c);
     const uint32_t s_n = S.n;
     const bool s_keys = S.keys != nullptr;
     // Segment: a run of tiles over which every index condition of the set has
@@ -1858,7 +1861,7 @@ __global__ void __launch_bounds__(kCtaThreads, 3)
       bool last = false;
 #pragma unroll 1
       for (int L = 0; L < kLists; L++)
-        if ((mine >> L) & 1) last = finish_list(S, L, fin, t2s, mgs, u.s);
+        if ((mine >> L) & 1) last = finish_list(S, L, fin, t2s, mgs, u.s, c);
       if (last && !S.cands) fill(S, fin);
       if (last && S.cands && ct == 0) {  // a shard: the header closes its lists
         CandHeader *h = reinterpret_cast<CandHeader *>(S.cands);
@@ -2132,15 +2135,19 @@ namespace {
 // candidate lists going to cands instead of outputs.
 // The last ranking call's plan per (device, stream): a call whose arguments
 // are byte for byte those of the previous call on its stream finds its
-// descriptors, tables and scratch layout already on the device, so it only
-// zeroes the work words and launches.  Any other use of the stream's
-// scratch (a merge, a different call, a reallocation) replaces or drops it.
+// descriptors, tables and scratch layout already on the device and only
+// launches.  The per-call state (work words, sample histograms) is held
+// twice; calls alternate between the two, and each launch zeroes the
+// other's for the next call.  Any other use of the stream's scratch (a
+// merge, a different call, a reallocation) replaces or drops the plan.
 struct RankPlan {
   std::vector<unsigned char> key;
-  size_t bytes = 0, hist_bytes = 0, work_off = 0;
+  size_t bytes = 0, hist_bytes = 0;
+  size_t desc_b = 0, work_off = 0, work_b = 0, hist_b = 0;  // per parity: descriptors, work words, histograms
   char *scratch = nullptr, *hists = nullptr;
   uint32_t grid = 0;
   int sequential = 0;
+  int parity = 0;  // the parity the next call uses (its state is zero)
 };
 std::mutex g_plan_mu;
 std::map<std::pair<int, cudaStream_t>, RankPlan> g_plan;
@@ -2170,7 +2177,8 @@ void plan_drop(cudaStream_t stream) {
   g_plan.erase(std::make_pair(dev, stream));
 }
 
-cudaError_t launch_rank_kernel(uint32_t grid, const RankSet *d_sets, int n_sets, int sequential, cudaStream_t stream) {
+cudaError_t launch_rank_kernel(uint32_t grid, const RankSet *d_sets, int n_sets, int sequential, char *zero_a,
+                               size_t bytes_a, char *zero_b, size_t bytes_b, cudaStream_t stream) {
   ProfSpan span("rank", stream);
   cudaLaunchAttribute coop[1];
   coop[0].id = cudaLaunchAttributeCooperative;
@@ -2182,7 +2190,8 @@ cudaError_t launch_rank_kernel(uint32_t grid, const RankSet *d_sets, int n_sets,
   lc.stream = stream;
   lc.attrs = coop;
   lc.numAttrs = 1;
-  return cudaLaunchKernelEx(&lc, rank_kernel, d_sets, n_sets, sequential);
+  return cudaLaunchKernelEx(&lc, rank_kernel, d_sets, n_sets, sequential, reinterpret_cast<uint4 *>(zero_a),
+                            (uint32_t)(bytes_a / 16), reinterpret_cast<uint4 *>(zero_b), (uint32_t)(bytes_b / 16));
 }
 
 int rank_launch(const unison_records *sets, const unison_rank_params *params, const unison_rank_out *outs,
@@ -2198,17 +2207,20 @@ int rank_launch(const unison_records *sets, const unison_rank_params *params, co
     std::lock_guard<std::mutex> lock(g_plan_mu);
     auto it = g_plan.find(std::make_pair(dev, stream));
     if (it != g_plan.end() && it->second.key == key) {
-      const RankPlan &pl = it->second;
+      RankPlan &pl = it->second;
       char *scratch = nullptr, *hists = nullptr;
       if (scratch_acquire(stream, pl.bytes, pl.hist_bytes, &scratch, &hists) == UNISON_OK && scratch == pl.scratch &&
           hists == pl.hists) {
+        const int pa = pl.parity, pb = 1 - pa;
         int rc = UNISON_OK;
-        if (cudaMemsetAsync(scratch + pl.work_off, 0, sizeof(RankWork) * n_sets, stream) != cudaSuccess ||
-            launch_rank_kernel(pl.grid, reinterpret_cast<const RankSet *>(scratch), n_sets, pl.sequential, stream) !=
-                cudaSuccess)
+        if (launch_rank_kernel(pl.grid, reinterpret_cast<const RankSet *>(scratch + pa * pl.desc_b), n_sets,
+                               pl.sequential, scratch + pl.work_off + pb * pl.work_b, pl.work_b, hists + pb * pl.hist_b,
+                               pl.hist_b, stream) != cudaSuccess)
           rc = UNISON_ERR_CUDA;
         count_launches(1);
         if (cudaGetLastError() != cudaSuccess) rc = UNISON_ERR_CUDA;
+        if (rc == UNISON_OK) pl.parity = pb;
+        else g_plan.erase(it);
         return rc;
       }
       g_plan.erase(it);
@@ -2324,7 +2336,7 @@ int rank_launch(const unison_records *sets, const unison_rank_params *params, co
                            align_up(sizeof(uint64_t) * kLists * kMaxSel, 256) +
                            align_up(sizeof(uint32_t) * kLists * kMaxSel, 256);
   const size_t hist_set = sizeof(unsigned int) * kLists * kBins;
-  size_t sets_b = 0;
+  size_t sets_b = 0, hist_b = 0;  // hist_b: one parity's histograms (sampled sets only)
   for (int i = 0; i < n_sets; i++) {
     RankSet &s = hs[i];
     // without a sample every eligible record is a candidate: at most n
@@ -2334,6 +2346,7 @@ int rank_launch(const unison_records *sets, const unison_rank_params *params, co
     s.cr = std::max<uint32_t>(s.ccap / s.nctas, std::min<uint32_t>(s.ccap, 1024u));
     sets_b += fixed_set + align_up(sizeof(uint64_t) * kLists * s.ccap, 256) +
               align_up(sizeof(uint64_t) * kLists * s.nctas * s.cr, 256);
+    if (s.ns) hist_b += hist_set;
   }
   const size_t desc_b = align_up(sizeof(RankSet) * n_sets, 256);
   const size_t tab_b = align_up(sizeof(RankTab) * tabs.size(), 256);
@@ -2341,17 +2354,23 @@ int rank_launch(const unison_records *sets, const unison_rank_params *params, co
   char *scratch = nullptr, *hists = nullptr;
   {
     plan_drop(stream);  // the scratch is rewritten below; the plan returns only if the launch succeeds
-    const int ar = scratch_acquire(stream, desc_b + tab_b + work_b + sets_b, hist_set * n_sets, &scratch, &hists);
+    const int ar =
+        scratch_acquire(stream, 2 * desc_b + tab_b + 2 * work_b + sets_b, std::max<size_t>(2 * hist_b, 256), &scratch, &hists);
     if (ar != UNISON_OK) return ar;
   }
-  RankTab *d_tabs = reinterpret_cast<RankTab *>(scratch + desc_b);
-  RankWork *works = reinterpret_cast<RankWork *>(scratch + desc_b + tab_b);
-  char *p = scratch + desc_b + tab_b + work_b;
+  // image: descriptors of parity 0 and 1, tables, work words of parity 0 and
+  // 1, then the per-set areas; histograms of parity 0 then 1
+  RankTab *d_tabs = reinterpret_cast<RankTab *>(scratch + 2 * desc_b);
+  const size_t work_off = 2 * desc_b + tab_b;
+  RankWork *works = reinterpret_cast<RankWork *>(scratch + work_off);
+  char *p = scratch + work_off + 2 * work_b;
+  size_t hoff = 0;
   for (int i = 0; i < n_sets; i++) {
     RankSet &s = hs[i];
     s.tab = d_tabs + tab_of[i];
     s.work = works + i;
-    s.shist = reinterpret_cast<unsigned int *>(hists + hist_set * i);
+    s.shist = s.ns ? reinterpret_cast<unsigned int *>(hists + hoff) : nullptr;
+    if (s.ns) hoff += hist_set;
     s.thr = reinterpret_cast<uint64_t *>(p);
     p += align_up(sizeof(uint64_t) * 2 * kLists, 256);
     s.gthr = reinterpret_cast<uint2 *>(p);
@@ -2370,30 +2389,43 @@ int rank_launch(const unison_records *sets, const unison_rank_params *params, co
     if (e != cudaSuccess && rc == UNISON_OK) rc = UNISON_ERR_CUDA;
   };
   RankSet *d_sets = reinterpret_cast<RankSet *>(scratch);
-  // descriptors, tables and zeroed work words: one copy from pinned staging
+  // descriptors of both parities, tables and both parities' zeroed work
+  // words: one copy from pinned staging; both parities' histograms zeroed
   {
-    const size_t up = desc_b + tab_b + sizeof(RankWork) * n_sets;
+    const size_t up = work_off + 2 * work_b;
     unsigned char *h = nullptr;
     cudaEvent_t done = nullptr;
     const int sr = staging_acquire(up, &h, &done);
     if (sr != UNISON_OK) return sr;
     std::memcpy(h, hs.data(), sizeof(RankSet) * n_sets);
-    std::memcpy(h + desc_b, tabs.data(), sizeof(RankTab) * tabs.size());
-    std::memset(h + desc_b + tab_b, 0, sizeof(RankWork) * n_sets);
+    for (int i = 0; i < n_sets; i++) {  // parity 1: the other work words and histograms
+      RankSet s1 = hs[i];
+      s1.work = reinterpret_cast<RankWork *>(reinterpret_cast<char *>(s1.work) + work_b);
+      if (s1.shist) s1.shist = reinterpret_cast<unsigned int *>(reinterpret_cast<char *>(s1.shist) + hist_b);
+      std::memcpy(h + desc_b + sizeof(RankSet) * i, &s1, sizeof(RankSet));
+    }
+    std::memcpy(h + 2 * desc_b, tabs.data(), sizeof(RankTab) * tabs.size());
+    std::memset(h + work_off, 0, 2 * work_b);
     ck(cudaMemcpyAsync(d_sets, h, up, cudaMemcpyHostToDevice, stream));
     ck(cudaEventRecord(done, stream));  // the buffer is reused after this copy
     staging_release();
+    if (hist_b) ck(cudaMemsetAsync(hists, 0, 2 * hist_b, stream));
   }
-  ck(launch_rank_kernel(grid, d_sets, n_sets, sequential, stream));
+  ck(launch_rank_kernel(grid, d_sets, n_sets, sequential, scratch + work_off + work_b, work_b, hists + hist_b,
+                        hist_b, stream));
   count_launches(1);
   ck(cudaGetLastError());
   if (rc == UNISON_OK) {
     std::lock_guard<std::mutex> lock(g_plan_mu);
     RankPlan &pl = g_plan[std::make_pair(dev, stream)];
     pl.key = key;
-    pl.bytes = desc_b + tab_b + work_b + sets_b;
-    pl.hist_bytes = hist_set * n_sets;
-    pl.work_off = desc_b + tab_b;
+    pl.bytes = 2 * desc_b + tab_b + 2 * work_b + sets_b;
+    pl.hist_bytes = std::max<size_t>(2 * hist_b, 256);
+    pl.desc_b = desc_b;
+    pl.work_off = work_off;
+    pl.work_b = work_b;
+    pl.hist_b = hist_b;
+    pl.parity = 1;
     pl.scratch = scratch;
     pl.hists = hists;
     pl.grid = grid;
