@@ -880,15 +880,18 @@ __device__ __noinline__ void sample_share(const RankSet &S, uint32_t r, const ui
     tu[q] = S.turn[rr[q]];
     gg[q] = S.gap[rr[q]];
   }
+  // near keys share bins: the lanes of a warp that hit one bin add to it once
 #pragma unroll
   for (int q = 0; q < (int)kSampleQ; q++) {
-    if (!ok[q]) continue;
     const uint32_t t = min((uint32_t)tu[q], kTMax);
     const uint64_t ck = ck_of(score_of(gg[q], t, (fl[q] & 2) != 0, t2s, mgs), S.off + rr[q]);
-    const uint32_t em = elig_mask(fl[q], tr[q]) & act;
+    const uint32_t em = ok[q] ? elig_mask(fl[q], tr[q]) & act : 0u;
 #pragma unroll
-    for (int L = 0; L < kLists; L++)
-      if ((em >> L) & 1) atomicAdd(&lh[L * kBins + bin_of(summary_of(list_val(ck, L)))], 1u);
+    for (int L = 0; L < kLists; L++) {
+      const uint32_t b = ((em >> L) & 1) ? L * kBins + bin_of(summary_of(list_val(ck, L))) : 0xFFFFFFFFu;
+      const unsigned grp = __match_any_sync(kFull, b);
+      if (b != 0xFFFFFFFFu && (__ffs(grp) - 1) == (int)(tid & 31)) atomicAdd(&lh[b], (unsigned)__popc(grp));
+    }
   }
   if (tid == 0) atomicAdd(&S.work->gathered, 1u);  // the group's copies may start now
   consumers_sync();
@@ -1377,9 +1380,11 @@ __device__ __noinline__ void fill(const RankSet &S, uint64_t *fin) {
 // the set (kEndTile) are announced with a plain arrival.
 // zero_a / zero_b (n_a, n_b 16-byte words): the other parity's work words
 // and sample histograms, zeroed here for the next call on the stream.
+// cmap (grouped launches): CTA b serves set cmap[b] & 0xFFFF, whose tables are
+// tabs[cmap[b] >> 16]; null for a sequential launch.
 __global__ void __launch_bounds__(kCtaThreads, 3)
-    rank_kernel(const RankSet *sets, int n_sets, int sequential, uint4 *zero_a, uint32_t n_a, uint4 *zero_b,
-                uint32_t n_b) {
+    rank_kernel(const RankSet *sets, int n_sets, int sequential, const uint32_t *cmap, const RankTab *tabs,
+                uint4 *zero_a, uint32_t n_a, uint4 *zero_b, uint32_t n_b) {
   extern __shared__ __align__(128) unsigned char dsm[];
   FilterStage *stage = reinterpret_cast<FilterStage *>(dsm);
   uint64_t *fin = reinterpret_cast<uint64_t *>(dsm);
@@ -1405,18 +1410,15 @@ __global__ void __launch_bounds__(kCtaThreads, 3)
     for (uint32_t w = g; w < n_b; w += gs) zero_b[w] = make_uint4(0u, 0u, 0u, 0u);
   }
   int s0, sstep;
+  const RankTab *tab0 = nullptr;  // the first set's tables, when the map names them
   if (sequential) {
     s0 = blockIdx.x;
     sstep = gridDim.x;
   } else {
-    int lo = 0, hi = n_sets - 1;
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (sets[mid].cta0 <= blockIdx.x) lo = mid; else hi = mid - 1;
-    }
-    s0 = lo;
+    const uint32_t e = __ldg(cmap + blockIdx.x);
+    s0 = (int)(e & 0xFFFFu);
+    tab0 = tabs + (e >> 16);
     sstep = n_sets;  // one set
-    if (blockIdx.x >= sets[s0].cta0 + sets[s0].nctas) return;  // an idle CTA
   }
   if (s0 >= n_sets) return;
   if (threadIdx.x == 0) {
@@ -1530,19 +1532,27 @@ __global__ void __launch_bounds__(kCtaThreads, 3)
   uint32_t i = 0;    // the CTA's running stage count (the producer's sequence)
   for (int s = s0; s < n_sets; s += sstep) {
     // the set's descriptor in shared memory: its fields are read throughout
-    // the set's phases, each read from global memory a round trip
+    // the set's phases, each read from global memory a round trip.  The
+    // tables come in the same round trip when the map names them.
     static_assert(sizeof(RankSet) % 8 == 0, "copied in 8-byte words");
     for (uint32_t w = ct; w < sizeof(RankSet) / 8; w += kConsumers)
       reinterpret_cast<uint64_t *>(&rset)[w] = reinterpret_cast<const uint64_t *>(sets + s)[w];
+    if (tab0 && ct < kLutN) {
+      t2s[ct] = tab0->t2v[ct];
+      mgs[ct] = tab0->mgv[ct];
+      sgs[ct] = tab0->sigma[ct];
+    }
     consumers_sync();
     const RankSet &S = rset;
     const uint32_t r = sequential ? 0u : blockIdx.x - S.cta0;
-    if (ct < kLutN) {
-      t2s[ct] = S.tab->t2v[ct];
-      mgs[ct] = S.tab->mgv[ct];
-      sgs[ct] = S.tab->sigma[ct];
+    if (!tab0) {
+      if (ct < kLutN) {
+        t2s[ct] = S.tab->t2v[ct];
+        mgs[ct] = S.tab->mgv[ct];
+        sgs[ct] = S.tab->sigma[ct];
+      }
+      consumers_sync();
     }
-    consumers_sync();
     // 1. thresholds: the sampling CTAs sample; every CTA cuts the histograms
     if (r < S.sctas) sample_share(S, r, t2s, mgs, reinterpret_cast<unsigned int *>(dsm), &sfree);
 #ifdef UNISON_DEBUG_HOOKS
@@ -2144,6 +2154,7 @@ struct RankPlan {
   std::vector<unsigned char> key;
   size_t bytes = 0, hist_bytes = 0;
   size_t desc_b = 0, work_off = 0, work_b = 0, hist_b = 0;  // per parity: descriptors, work words, histograms
+  size_t cmap_off = 0, tabs_off = 0;
   char *scratch = nullptr, *hists = nullptr;
   uint32_t grid = 0;
   int sequential = 0;
@@ -2177,8 +2188,9 @@ void plan_drop(cudaStream_t stream) {
   g_plan.erase(std::make_pair(dev, stream));
 }
 
-cudaError_t launch_rank_kernel(uint32_t grid, const RankSet *d_sets, int n_sets, int sequential, char *zero_a,
-                               size_t bytes_a, char *zero_b, size_t bytes_b, cudaStream_t stream) {
+cudaError_t launch_rank_kernel(uint32_t grid, const RankSet *d_sets, int n_sets, int sequential, const uint32_t *cmap,
+                               const RankTab *tabs, char *zero_a, size_t bytes_a, char *zero_b, size_t bytes_b,
+                               cudaStream_t stream) {
   ProfSpan span("rank", stream);
   cudaLaunchAttribute coop[1];
   coop[0].id = cudaLaunchAttributeCooperative;
@@ -2190,7 +2202,7 @@ cudaError_t launch_rank_kernel(uint32_t grid, const RankSet *d_sets, int n_sets,
   lc.stream = stream;
   lc.attrs = coop;
   lc.numAttrs = 1;
-  return cudaLaunchKernelEx(&lc, rank_kernel, d_sets, n_sets, sequential, reinterpret_cast<uint4 *>(zero_a),
+  return cudaLaunchKernelEx(&lc, rank_kernel, d_sets, n_sets, sequential, cmap, tabs, reinterpret_cast<uint4 *>(zero_a),
                             (uint32_t)(bytes_a / 16), reinterpret_cast<uint4 *>(zero_b), (uint32_t)(bytes_b / 16));
 }
 
@@ -2214,8 +2226,11 @@ int rank_launch(const unison_records *sets, const unison_rank_params *params, co
         const int pa = pl.parity, pb = 1 - pa;
         int rc = UNISON_OK;
         if (launch_rank_kernel(pl.grid, reinterpret_cast<const RankSet *>(scratch + pa * pl.desc_b), n_sets,
-                               pl.sequential, scratch + pl.work_off + pb * pl.work_b, pl.work_b, hists + pb * pl.hist_b,
-                               pl.hist_b, stream) != cudaSuccess)
+                               pl.sequential,
+                               pl.sequential ? nullptr : reinterpret_cast<const uint32_t *>(scratch + pl.cmap_off),
+                               reinterpret_cast<const RankTab *>(scratch + pl.tabs_off),
+                               scratch + pl.work_off + pb * pl.work_b, pl.work_b, hists + pb * pl.hist_b, pl.hist_b,
+                               stream) != cudaSuccess)
           rc = UNISON_ERR_CUDA;
         count_launches(1);
         if (cudaGetLastError() != cudaSuccess) rc = UNISON_ERR_CUDA;
@@ -2349,19 +2364,21 @@ int rank_launch(const unison_records *sets, const unison_rank_params *params, co
     if (s.ns) hist_b += hist_set;
   }
   const size_t desc_b = align_up(sizeof(RankSet) * n_sets, 256);
+  const size_t cmap_b = sequential ? 0 : align_up(sizeof(uint32_t) * grid, 256);
   const size_t tab_b = align_up(sizeof(RankTab) * tabs.size(), 256);
   const size_t work_b = align_up(sizeof(RankWork) * n_sets, 256);
   char *scratch = nullptr, *hists = nullptr;
   {
     plan_drop(stream);  // the scratch is rewritten below; the plan returns only if the launch succeeds
-    const int ar =
-        scratch_acquire(stream, 2 * desc_b + tab_b + 2 * work_b + sets_b, std::max<size_t>(2 * hist_b, 256), &scratch, &hists);
+    const int ar = scratch_acquire(stream, 2 * desc_b + cmap_b + tab_b + 2 * work_b + sets_b,
+                                   std::max<size_t>(2 * hist_b, 256), &scratch, &hists);
     if (ar != UNISON_OK) return ar;
   }
-  // image: descriptors of parity 0 and 1, tables, work words of parity 0 and
-  // 1, then the per-set areas; histograms of parity 0 then 1
-  RankTab *d_tabs = reinterpret_cast<RankTab *>(scratch + 2 * desc_b);
-  const size_t work_off = 2 * desc_b + tab_b;
+  // image: descriptors of parity 0 and 1, the CTA map, tables, work words of
+  // parity 0 and 1, then the per-set areas; histograms of parity 0 then 1
+  const size_t cmap_off = 2 * desc_b, tabs_off = cmap_off + cmap_b;
+  RankTab *d_tabs = reinterpret_cast<RankTab *>(scratch + tabs_off);
+  const size_t work_off = tabs_off + tab_b;
   RankWork *works = reinterpret_cast<RankWork *>(scratch + work_off);
   char *p = scratch + work_off + 2 * work_b;
   size_t hoff = 0;
@@ -2404,22 +2421,30 @@ int rank_launch(const unison_records *sets, const unison_rank_params *params, co
       if (s1.shist) s1.shist = reinterpret_cast<unsigned int *>(reinterpret_cast<char *>(s1.shist) + hist_b);
       std::memcpy(h + desc_b + sizeof(RankSet) * i, &s1, sizeof(RankSet));
     }
-    std::memcpy(h + 2 * desc_b, tabs.data(), sizeof(RankTab) * tabs.size());
+    if (!sequential) {
+      uint32_t *cm = reinterpret_cast<uint32_t *>(h + cmap_off);
+      for (int i = 0; i < n_sets; i++)
+        for (uint32_t b = hs[i].cta0; b < hs[i].cta0 + hs[i].nctas; b++) cm[b] = (uint32_t)i | ((uint32_t)tab_of[i] << 16);
+    }
+    std::memcpy(h + tabs_off, tabs.data(), sizeof(RankTab) * tabs.size());
     std::memset(h + work_off, 0, 2 * work_b);
     ck(cudaMemcpyAsync(d_sets, h, up, cudaMemcpyHostToDevice, stream));
     ck(cudaEventRecord(done, stream));  // the buffer is reused after this copy
     staging_release();
     if (hist_b) ck(cudaMemsetAsync(hists, 0, 2 * hist_b, stream));
   }
-  ck(launch_rank_kernel(grid, d_sets, n_sets, sequential, scratch + work_off + work_b, work_b, hists + hist_b,
-                        hist_b, stream));
+  ck(launch_rank_kernel(grid, d_sets, n_sets, sequential,
+                        sequential ? nullptr : reinterpret_cast<const uint32_t *>(scratch + cmap_off), d_tabs,
+                        scratch + work_off + work_b, work_b, hists + hist_b, hist_b, stream));
   count_launches(1);
   ck(cudaGetLastError());
   if (rc == UNISON_OK) {
     std::lock_guard<std::mutex> lock(g_plan_mu);
     RankPlan &pl = g_plan[std::make_pair(dev, stream)];
     pl.key = key;
-    pl.bytes = 2 * desc_b + tab_b + 2 * work_b + sets_b;
+    pl.bytes = 2 * desc_b + cmap_b + tab_b + 2 * work_b + sets_b;
+    pl.cmap_off = cmap_off;
+    pl.tabs_off = tabs_off;
     pl.hist_bytes = std::max<size_t>(2 * hist_b, 256);
     pl.desc_b = desc_b;
     pl.work_off = work_off;
