@@ -160,7 +160,8 @@ struct RankSet {
   const RankTab *tab;
   uint32_t ntiles;
   uint32_t cta0, nctas;          // the group: CTAs [cta0, cta0 + nctas)
-  uint32_t ns, nruns, sq, srem;  // sample size, its runs of 8, n = sq * nruns + srem
+  uint32_t ns, nruns;            // sample size, its runs of 8
+  uint64_t sstep;                // stratum width n / nruns in 16.16 fixed point
   uint32_t sctas;                // sampling CTAs (the group's first sctas)
   uint32_t act;                  // active lists (bit L)
   uint32_t rL[kLists];           // sample rank of each list's threshold
@@ -826,15 +827,15 @@ void plan_sample(RankSet &s) {
   ns -= ns % (8ull * s.sctas);  // whole runs, evenly split over the sampling CTAs
   s.ns = (uint32_t)ns;
   s.nruns = s.ns / 8;
-  s.sq = s.nruns ? s.n / s.nruns : 0;
-  s.srem = s.nruns ? s.n % s.nruns : 0;
+  s.sstep = s.nruns ? ((uint64_t)s.n << 16) / s.nruns : 0;
   for (int L = 0; L < kLists; L++)
     s.rL[L] = (s.ns && list_active(s, L)) ? (uint32_t)((list_target_of(s, L, wide) * s.ns + s.n - 1) / s.n) : 0u;
 }
 
 // Sampling CTA r of set S (consumer threads): samples j = r * per + jt of
-// the CTA's share, run j / 8 covering stratum j / 8 (records [run n / nruns,
-// (run+1) n / nruns)), 8 consecutive records at a hashed offset in it; each
+// the CTA's share, run j / 8 covering stratum j / 8 (records from about
+// run n / nruns to (run+1) n / nruns), 8 consecutive records at a hashed
+// offset in it; each
 // eligible sample is counted into its lists' histograms (first in shared
 // memory, then the non-zero bins into the set's), and the CTA's ticket says
 // its counts are in.
@@ -858,16 +859,16 @@ __device__ __noinline__ void sample_share(const RankSet &S, uint32_t r, const ui
     ok[q] = jt < per;
     rr[q] = 0;
     if (ok[q]) {
-      // stratum bounds floor(run n / nruns) with n = sq nruns + srem, in 32 bits
-      const uint32_t nruns = S.nruns, run = r * (per / 8) + jt / 8, o = jt % 8;
-      const uint32_t lo = run * S.sq + (run * S.srem) / nruns;
-      const uint32_t hi = (run + 1) * S.sq + ((run + 1) * S.srem) / nruns;
+      // stratum bounds about run n / nruns (16.16 fixed point: no division
+      // on the sample's path; any stratification samples correctly)
+      const uint32_t run = r * (per / 8) + jt / 8, o = jt % 8;
+      const uint32_t lo = (uint32_t)((run * S.sstep) >> 16), hi = (uint32_t)(((run + 1) * S.sstep) >> 16);
       uint32_t h = run * 0x9E3779B1u;
       h ^= h >> 16;
       h *= 0x85EBCA6Bu;
       h ^= h >> 13;
-      const uint32_t span = hi - lo - 8;  // strata hold at least 8 records
-      rr[q] = lo + (h % (span + 1)) + o;
+      const uint32_t span = hi - lo >= 8 ? hi - lo - 8 : 0u;  // strata hold at least 8 records
+      rr[q] = min(lo + __umulhi(h, span + 1) + o, S.n - 1);
     }
   }
   uint8_t fl[kSampleQ], tr[kSampleQ];
