@@ -918,6 +918,17 @@ def main():
                    "hbm_gbs": alg_bytes / (avg_rep_ms / 1e3) / 1e9, "launches_timed": rep_n,
                    "share_of_step": avg_rep_ms * args.steps / ms if ms else None,
                    "key_stream_avg_ms": ks_ms / max(ks_n, 1), "ttft_median_avg_ms": md_ms / max(md_n, 1)}
+    if replay_roof is not None:
+        # The launch ends with its slowest replay: its cycles per event, against
+        # the chain an event needs on sorted arrays in shared memory (about 17
+        # dependent accesses -- tier byte, two search rounds, the entry, a
+        # shift's load and store, the store of the new entry, pops, pin slot and
+        # pin entry, TIDE's two heads -- at about 30 cycles each).
+        mhz = (clocks or {}).get("sm_mhz") or 2070.0
+        replay_roof["cycles_per_event_slowest_replay"] = avg_rep_ms * 1e3 * mhz / (events_per_step / n_rep)
+        replay_roof["floor_cycles_per_event"] = 17 * 30
+        replay_roof["floor_basis"] = ("17 dependent shared-memory accesses per event x ~30 cycles "
+                                      "(search, shift, entry store, pops, pin slot, TIDE heads)")
     avg_rk = rk_ms / max(rk_n, 1) if rk_n else float("nan")
     achieved = rank_bytes / (avg_rk / 1e3) / 1e9 if rk_n else float("nan")
     n_rec = len(r_params) * RANK_N
@@ -941,6 +952,9 @@ def main():
     if rank != 0:
         return
     cpu = None if (args.no_cpu_baseline or world > 1) else cpu_baseline_replay(trs, reps)
+    # the whole ranking call's fraction per live-set size as flat keys (8 B/record)
+    flat = {"rank_call_frac_2p%d_x%d" % (z["n"].bit_length() - 1, z["sets"]): z["frac"]
+            for z in sizes or [] if z["n"] >= (1 << 20)}
     line = {"metric": METRIC, "value": value, "unit": "events/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int64", "data": "synthetic",
@@ -949,6 +963,7 @@ def main():
                                    "SPEAR+TIDE)",
                        "replays": n_rep, "events_per_step": events_per_step,
                        "l2": "flushed before every step (256 MiB write, inside the timed region)"},
+            "rank_call_frac_of_peak": rank_leg["call_frac_of_peak"], **flat,
             "roofline": roofline, "rank": rank_leg, "rank_sizes": sizes, "rank_single_set": single,
             "rank_kendall": tau, "sweep_iid_gaps": iid, "replay_roofline": replay_roof, "cpu_baseline": cpu,
             "e2e": e2e, "gpu_launches": launches, "clocks": clocks}

@@ -1648,6 +1648,15 @@ void fill_descs(const unison_trace *const *traces, const unison_replay_params *p
   order.clear();
   for (const auto *g : {&P.in_st, &P.in_mix, &P.in_gst, &P.in_gmix, &P.in_online, &P.in_stale})
     order.insert(order.end(), g->begin(), g->end());
+  // A launch lasts as long as its slowest replay, and CTAs start in index
+  // order: the SPEAR+TIDE launch takes its replays by predicted cost,
+  // largest first, so the long ones start early and the short ones fill in.
+  // The predictor is the product of the tiers' capacities (the larger both
+  // tiers, the more tier moves a replay makes); decisions do not depend on
+  // the order.
+  std::stable_sort(order.begin(), order.begin() + P.in_st.size(), [&](uint32_t a, uint32_t b) {
+    return (double)hd[a].cap_s * (double)hd[a].cap_h > (double)hd[b].cap_s * (double)hd[b].cap_h;
+  });
 }
 
 // Side streams for the replay groups of one call, one set per device, made

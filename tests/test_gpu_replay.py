@@ -115,6 +115,18 @@ def test_sweep_1024_replays_all(B):
         assert_same(res[i], o, i)
 
 
+def test_sweep_iid_gaps_subset(B):
+    """The sweep's settings on a trace with independent gaps (gap
+    persistence 0: every gap's mixture component and value drawn afresh),
+    the workload the bench's `sweep_iid_gaps` rate is measured on: one
+    seed's 128 replays in one call, every replay against the oracle."""
+    trs, reps = sweep_case(n_seeds=1, gap_persist=0.0)
+    res, _, _ = run_gpu(B, trs, reps)
+    assert len(res) == 128 and all(r["status"] == 0 for r in res)
+    for i, (ti, p) in enumerate(reps):
+        assert_same(res[i], oracle.replay(trs[ti], to_oracle(p)), i)
+
+
 @pytest.mark.parametrize("seed", [100, 101])
 def test_large_pool_replay(B, seed):
     tr = synth.large_pool_trace(seed)
