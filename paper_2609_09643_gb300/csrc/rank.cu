@@ -175,8 +175,6 @@ struct RankSet {
   uint32_t cr;       // region size
   uint64_t *sorted;  // [3][kMaxSel]
   uint32_t *ssz;     // [3][kMaxSel] KV tokens of the sorted entries (D and P)
-  uint2 *gthr;       // [3][51] (gA, gB)
-  uint64_t *thr;     // [3] threshold in list-value space; [3+L] = active flag
   unsigned int *shist;  // [3][kBins] sample histogram (zero between calls)
 };
 
@@ -2348,8 +2346,7 @@ int rank_launch(const unison_records *sets, const unison_rank_params *params, co
   // scratch: descriptors, tables, every set's work words (zeroed by the
   // upload), then per set: thresholds, tables, sorted lists and sizes,
   // candidates; and the per-set histograms in their own block
-  const size_t fixed_set = align_up(sizeof(uint64_t) * 2 * kLists, 256) + align_up(sizeof(uint2) * kLists * kLutN, 256) +
-                           align_up(sizeof(uint64_t) * kLists * kMaxSel, 256) +
+  const size_t fixed_set = align_up(sizeof(uint64_t) * kLists * kMaxSel, 256) +
                            align_up(sizeof(uint32_t) * kLists * kMaxSel, 256);
   const size_t hist_set = sizeof(unsigned int) * kLists * kBins;
   size_t sets_b = 0, hist_b = 0;  // hist_b: one parity's histograms (sampled sets only)
@@ -2389,10 +2386,6 @@ int rank_launch(const unison_records *sets, const unison_rank_params *params, co
     s.work = works + i;
     s.shist = s.ns ? reinterpret_cast<unsigned int *>(hists + hoff) : nullptr;
     if (s.ns) hoff += hist_set;
-    s.thr = reinterpret_cast<uint64_t *>(p);
-    p += align_up(sizeof(uint64_t) * 2 * kLists, 256);
-    s.gthr = reinterpret_cast<uint2 *>(p);
-    p += align_up(sizeof(uint2) * kLists * kLutN, 256);
     s.sorted = reinterpret_cast<uint64_t *>(p);
     p += align_up(sizeof(uint64_t) * kLists * kMaxSel, 256);
     s.ssz = reinterpret_cast<uint32_t *>(p);
@@ -2509,20 +2502,18 @@ extern "C" int unison_rank_merge(const void *gathered_dev, int n_shards, const u
   s.counts = o.counts;
   s.moved = o.moved_bytes;
   for (int L = 0; L < kLists; L++) s.act |= list_active(s, L) ? 1u << L : 0u;
-  // scratch: descriptor, work words and active flags (one upload), sorted lists
+  // scratch: descriptor and work words (one upload), sorted lists
   const size_t desc_b = align_up(sizeof(RankSet), 256), work_b = align_up(sizeof(RankWork), 256);
-  const size_t thr_b = align_up(sizeof(uint64_t) * 2 * kLists, 256);
   const size_t lists_b = align_up(sizeof(uint64_t) * kLists * kMaxSel, 256) + align_up(sizeof(uint32_t) * kLists * kMaxSel, 256);
   char *scratch = nullptr, *hists = nullptr;
   {
     plan_drop(stream);  // the descriptor area is rewritten below
-    const int ar = scratch_acquire(stream, desc_b + work_b + thr_b + lists_b, 0, &scratch, &hists);
+    const int ar = scratch_acquire(stream, desc_b + work_b + lists_b, 0, &scratch, &hists);
     if (ar != UNISON_OK) return ar;
   }
   s.work = reinterpret_cast<RankWork *>(scratch + desc_b);
-  s.thr = reinterpret_cast<uint64_t *>(scratch + desc_b + work_b);
-  s.sorted = reinterpret_cast<uint64_t *>(scratch + desc_b + work_b + thr_b);
-  s.ssz = reinterpret_cast<uint32_t *>(scratch + desc_b + work_b + thr_b + align_up(sizeof(uint64_t) * kLists * kMaxSel, 256));
+  s.sorted = reinterpret_cast<uint64_t *>(scratch + desc_b + work_b);
+  s.ssz = reinterpret_cast<uint32_t *>(scratch + desc_b + work_b + align_up(sizeof(uint64_t) * kLists * kMaxSel, 256));
   const LaunchCfg &cfg = launch_cfg();
   if (!cfg.ok) return UNISON_ERR_CUDA;
   int rc = UNISON_OK;
@@ -2530,15 +2521,13 @@ extern "C" int unison_rank_merge(const void *gathered_dev, int n_shards, const u
     if (e != cudaSuccess && rc == UNISON_OK) rc = UNISON_ERR_CUDA;
   };
   {
-    const size_t up = desc_b + work_b + thr_b;
+    const size_t up = desc_b + work_b;
     unsigned char *h = nullptr;
     cudaEvent_t done = nullptr;
     const int sr = staging_acquire(up, &h, &done);
     if (sr != UNISON_OK) return sr;
     std::memset(h, 0, up);
     std::memcpy(h, &s, sizeof(RankSet));
-    uint64_t *thr = reinterpret_cast<uint64_t *>(h + desc_b + work_b);
-    for (int L = 0; L < kLists; L++) thr[kLists + L] = (s.act >> L) & 1;
     ck(cudaMemcpyAsync(scratch, h, up, cudaMemcpyHostToDevice, stream));
     ck(cudaEventRecord(done, stream));
     staging_release();
