@@ -156,6 +156,21 @@ def test_massive_ties(B, sigma):
         check(r, rec, p, keys=True)
 
 
+def test_crowded_buckets(B, sigma):
+    """A few records whose keys sit far above thousands of equal ones: below
+    the candidates' common prefix every equal-key record falls in one bucket,
+    so the finish's bucket cut keeps them all (the radix select when they
+    exceed 4,096) and the bucket sort declines for the sorting network."""
+    n = 300000
+    base = synth.make_records(11, n)
+    gap = np.zeros(n, np.uint32)
+    gap[np.arange(0, n, n // 7)[:7]] = 1 << 30  # seven far larger gap averages
+    rec = synth.Records(gap, base.last_ret, np.zeros(n, np.uint16), base.kv_tok, base.tier, np.zeros(n, np.uint8))
+    ps = [prm(sigma, k=1024, budget=64 * GIB), prm(sigma, k=4096, budget=1 << 45, free_s=50000, max_moves=4096)]
+    for r, p in zip(run(B, [rec] * 2, ps), ps):
+        check(r, rec, p)
+
+
 def test_degenerate_sets(B, sigma):
     n = 50000
     base = synth.make_records(8, n)
