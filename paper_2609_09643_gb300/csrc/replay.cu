@@ -281,6 +281,35 @@ __device__ __noinline__ void shift_block(uint4 *e, uint32_t lo, uint32_t hi, int
   }
 }
 
+// The fast tier in registers (kRegS launches, every replay's fast tier at
+// most 32 entries): lane i holds entry i of the sorted array, so a search is
+// one ballot and an insert, an erase or a pop is a few shuffles, with no
+// shared-memory round trip.
+struct RegTier {
+  uint4 v;  // this lane's entry
+  uint32_t n;
+};
+__device__ __forceinline__ uint32_t reg_lower_bound(const RegTier &R, uint64_t k, int lane) {
+  return __popc(__ballot_sync(kFull, (uint32_t)lane < R.n && ekey(R.v) < k));
+}
+__device__ __forceinline__ uint4 reg_at(const RegTier &R, uint32_t i) {
+  return make_uint4(__shfl_sync(kFull, R.v.x, i), __shfl_sync(kFull, R.v.y, i), __shfl_sync(kFull, R.v.z, i),
+                    __shfl_sync(kFull, R.v.w, i));
+}
+__device__ __forceinline__ void reg_insert_at(RegTier &R, uint32_t p, uint4 e, int lane) {
+  const uint4 u = make_uint4(__shfl_up_sync(kFull, R.v.x, 1), __shfl_up_sync(kFull, R.v.y, 1),
+                             __shfl_up_sync(kFull, R.v.z, 1), __shfl_up_sync(kFull, R.v.w, 1));
+  if ((uint32_t)lane > p) R.v = u;
+  if ((uint32_t)lane == p) R.v = e;
+  R.n++;
+}
+__device__ __forceinline__ void reg_erase_at(RegTier &R, uint32_t p, int lane) {
+  const uint4 u = make_uint4(__shfl_down_sync(kFull, R.v.x, 1), __shfl_down_sync(kFull, R.v.y, 1),
+                             __shfl_down_sync(kFull, R.v.z, 1), __shfl_down_sync(kFull, R.v.w, 1));
+  if ((uint32_t)lane >= p) R.v = u;
+  R.n--;
+}
+
 // Descriptor fields the placement and fill read on every event, held in
 // registers (the descriptor itself sits in shared memory).
 struct Hot {
@@ -291,6 +320,7 @@ struct Hot {
 
 struct ReplayState {
   Sorted S, H;      // unpinned residents per tier
+  RegTier R;        // the fast tier's residents instead of S, in kRegS launches
   uint4 *pin;       // pinned residents
   uint32_t npin, pin_cap;
   uint4 *tmp;       // TIDE staging: [0, cap_s) promoted, [cap_s, 2 cap_s) demoted
@@ -372,6 +402,24 @@ __device__ __forceinline__ uint4 sorted_pop_back(ReplayState &st, Sorted &T) {
   const uint4 v = T.e[T.n - 1];
   __syncwarp();
   T.n--;
+  set_tier<kLean>(st, packed_id(ekey(v)), kTierNone);
+  return v;
+}
+
+template <bool kLean>
+__device__ __forceinline__ bool reg_sorted_insert(ReplayState &st, uint4 v, int lane) {
+  if (st.R.n >= st.S.cap) {
+    st.status = UNISON_ERR_CAPACITY;
+    return false;
+  }
+  reg_insert_at(st.R, reg_lower_bound(st.R, ekey(v), lane), v, lane);
+  set_tier<kLean>(st, packed_id(ekey(v)), kTierS);
+  return true;
+}
+template <bool kLean>
+__device__ __forceinline__ uint4 reg_pop_back(ReplayState &st) {
+  const uint4 v = reg_at(st.R, st.R.n - 1);
+  st.R.n--;
   set_tier<kLean>(st, packed_id(ekey(v)), kTierNone);
   return v;
 }
@@ -462,7 +510,7 @@ __device__ __forceinline__ bool pin_append(ReplayState &st, uint64_t pk, uint32_
 }
 
 // Placement of the arriving (pinned) session s with n tokens.
-template <bool kStale, bool kLean>
+template <bool kStale, bool kLean, bool kRegS = false>
 __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s, uint64_t pk, uint32_t n,
                                       int lane) {
   if (!kLean && D.max_sessions && st.npin >= D.max_sessions) {
@@ -472,12 +520,13 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
   }
   if (st.pinned_s <= D.cap_s && n <= D.cap_s - st.pinned_s) {
     while (st.used_s + n > D.cap_s) {
-      if (st.S.n == 0) {
+      if ((kRegS ? st.R.n : st.S.n) == 0) {
         st.status = UNISON_ERR_CAPACITY;
         return false;
       }
       if (kStale) count_victim(st, packed_id(ekey(st.S.e[st.S.n - 1])), live_max(st, st.S, 0, st.S.n, lane));
-      const uint4 d = sorted_pop_back<kLean>(st, st.S);  // most evictable unpinned fast-tier session
+      // most evictable unpinned fast-tier session
+      const uint4 d = kRegS ? reg_pop_back<kLean>(st) : sorted_pop_back<kLean>(st, st.S);
       st.used_s -= esize(d);
       if (!admit_demoted<kStale, kLean>(st, D, d, lane)) return false;
     }
@@ -536,9 +585,10 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
 // free fast-tier space; phase 2: pair the next least evictable HBM session
 // with the most evictable fast-tier one), which makes the same moves as the
 // pair loop of Algorithm 1, and are then applied in bulk.
-template <bool kStale, bool kLean>
+template <bool kStale, bool kLean, bool kRegS = false>
 __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t budget, uint32_t rcap_s,
                                          int lane) {
+  const uint32_t sn = kRegS ? st.R.n : st.S.n;  // fast-tier entries; the fast tier changes only at the end
   uint64_t rem = budget;
   const uint64_t kvb = D.kvb;
   uint32_t n1 = 0;
@@ -556,9 +606,9 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
   }
   uint32_t pairs = 0;
   for (;;) {
-    if (n1 + pairs >= st.H.n || pairs >= st.S.n) break;
+    if (n1 + pairs >= st.H.n || pairs >= sn) break;
     const uint4 p = st.H.e[n1 + pairs];
-    const uint4 d = st.S.e[st.S.n - 1 - pairs];
+    const uint4 d = kRegS ? reg_at(st.R, sn - 1 - pairs) : st.S.e[st.S.n - 1 - pairs];
     // the next most evictable of (fast tier + promoted) is a promoted session
     // when the largest promoted key beats d: then it cannot beat p, stop
     if (n1 > 0 && ekey(st.H.e[n1 - 1]) > ekey(d)) break;
@@ -597,18 +647,24 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     __syncwarp();
     shift_block(st.H.e, 1, st.H.n, -1, lane);
     st.H.n -= 1;
-    sorted_insert<kLean>(st, st.S, v, lane, kTierS);
+    if (kRegS) reg_sorted_insert<kLean>(st, v, lane);
+    else sorted_insert<kLean>(st, st.S, v, lane, kTierS);
     return budget - rem;
   }
   if (m == 1 && pairs == 1) {  // one pair (the next most common): swap it directly
     uint4 v = st.H.e[0];
     v.z |= kPromotedBit;
-    const uint4 d = st.S.e[st.S.n - 1];
+    const uint4 d = kRegS ? reg_at(st.R, sn - 1) : st.S.e[st.S.n - 1];
     __syncwarp();
     shift_block(st.H.e, 1, st.H.n, -1, lane);
     st.H.n -= 1;
-    st.S.n -= 1;
-    if (!sorted_insert<kLean>(st, st.S, v, lane, kTierS)) return budget - rem;
+    if (kRegS) {
+      st.R.n -= 1;
+      if (!reg_sorted_insert<kLean>(st, v, lane)) return budget - rem;
+    } else {
+      st.S.n -= 1;
+      if (!sorted_insert<kLean>(st, st.S, v, lane, kTierS)) return budget - rem;
+    }
     sorted_insert<kLean>(st, st.H, d, lane, kTierH);
     return budget - rem;
   }
@@ -619,13 +675,20 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     v.z |= kPromotedBit;
     pro[i] = v;
   }
-  for (uint32_t i = lane; i < pairs; i += 32) dem[i] = st.S.e[st.S.n - pairs + i];
+  if (kRegS) {  // pairs <= fast-tier entries <= 32: one entry a lane
+    const uint4 dv = reg_at(st.R, min(sn - pairs + (uint32_t)lane, 31u));
+    if ((uint32_t)lane < pairs) dem[lane] = dv;
+  } else {
+    for (uint32_t i = lane; i < pairs; i += 32) dem[i] = st.S.e[st.S.n - pairs + i];
+  }
   __syncwarp();
   shift_block(st.H.e, m, st.H.n, -(int32_t)m, lane);
   st.H.n -= m;
-  st.S.n -= pairs;
+  if (kRegS) st.R.n -= pairs;
+  else st.S.n -= pairs;
   for (uint32_t i = 0; i < m; i++)
-    if (!sorted_insert<kLean>(st, st.S, pro[i], lane, kTierS)) return budget - rem;
+    if (kRegS ? !reg_sorted_insert<kLean>(st, pro[i], lane) : !sorted_insert<kLean>(st, st.S, pro[i], lane, kTierS))
+      return budget - rem;
   for (uint32_t i = 0; i < pairs; i++)
     if (!sorted_insert<kLean>(st, st.H, dem[i], lane, kTierH)) return budget - rem;
   return budget - rem;
@@ -826,7 +889,7 @@ struct EventBufs {
 // One replay: Algorithm 1 over the trace's events.  kPol is the replay's
 // policy when the body is specialised for it (its policy tests then fold
 // away), or -1 for the body that reads the policy from the descriptor.
-template <bool kGlobalLists, int kKeys, int kPol, bool kLean>
+template <bool kGlobalLists, int kKeys, int kPol, bool kLean, bool kRegS = false>
 __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs, unsigned char *smem, int lane) {
   constexpr bool kOnline = kKeys == kKeyOnline, kStale = kKeys == kKeyStale;
   const Hot hot{D.cap_s, D.cap_h, D.kvb, D.dma, D.max_sessions};
@@ -915,6 +978,8 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
     st.live = stale_live;
     st.vict_n = st.vict_diff = st.prom_n = st.prom_diff = 0;
     st.S.n = st.H.n = 0;
+    st.R.n = 0;
+    st.R.v = make_uint4(0u, 0u, 0u, 0u);
     st.S.cap = D.rcap_s;
     st.H.cap = D.rcap_h;
     st.npin = 0;
@@ -1022,10 +1087,19 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
           // nothing for a session that is not resident)
           const uint32_t mt = (kLean || st.tmap) ? st.tmap[s] : (kTierS | kTierH);
           if (mt & kTierS) {
-            pos = lower_bound(st.S, pkb, lane);
-            if (pos < st.S.n && ekey(st.S.e[pos]) == pkb) {
-              tier = kTierS;
-              ent = st.S.e[pos];
+            if (kRegS) {
+              pos = reg_lower_bound(st.R, pkb, lane);
+              const uint4 cand = reg_at(st.R, min(pos, 31u));
+              if (pos < st.R.n && ekey(cand) == pkb) {
+                tier = kTierS;
+                ent = cand;
+              }
+            } else {
+              pos = lower_bound(st.S, pkb, lane);
+              if (pos < st.S.n && ekey(st.S.e[pos]) == pkb) {
+                tier = kTierS;
+                ent = st.S.e[pos];
+              }
             }
           }
           if (tier == kTierNone && (mt & kTierH)) {
@@ -1077,7 +1151,8 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
         }
         if (tier == kTierS) {
           st.used_s -= esize(ent);
-          sorted_erase(st.S, pos, lane);
+          if (kRegS) reg_erase_at(st.R, pos, lane);
+          else sorted_erase(st.S, pos, lane);
           set_tier<kLean>(st, s, kTierNone);
         } else if (tier == kTierH) {
           st.used_h -= esize(ent);
@@ -1107,7 +1182,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
           pk = pack_key(nr == kNoRef ? kKeyMax40 : (uint64_t)nr, s);
         } else
           pk = pack_key(0xFFFFFFFFull - e, s);
-        if (!place<kStale, kLean>(st, hot, s, pk, out, lane)) break;
+        if (!place<kStale, kLean, kRegS>(st, hot, s, pk, out, lane)) break;
       } else {
         // completion: unpin (if resident) and rank the session with its new key
         if (kStale) {
@@ -1149,7 +1224,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
           const uint4 v = make_uint4((uint32_t)pk, (uint32_t)(pk >> 32), sz, now);
           if (tier == kTierS) {
             st.pinned_s -= sz;
-            if (!sorted_insert<kLean>(st, st.S, v, lane, kTierS)) break;
+            if (kRegS ? !reg_sorted_insert<kLean>(st, v, lane) : !sorted_insert<kLean>(st, st.S, v, lane, kTierS)) break;
           } else {
             st.pinned_h -= sz;
             if (!sorted_insert<kLean>(st, st.H, v, lane, kTierH)) break;
@@ -1167,7 +1242,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
           const uint64_t g = sgq[bi][j];
           const uint64_t budget = g * D.dma;
           CNT(st, n_tide_calls, 1);
-          const uint64_t moved = tide<kStale, kLean>(st, hot, budget, D.rcap_s, lane);
+          const uint64_t moved = tide<kStale, kLean, kRegS>(st, hot, budget, D.rcap_s, lane);
           CNT(st, dma_bytes, moved);
           if (moved > 0 && D.dma > 0) {
             dma_busy = true;
@@ -1261,7 +1336,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
 // replay of the launch has that policy, and the kernel holds only its body
 // (and is sized for it alone); kLean: every replay of the launch is lean
 // (see log_dec).
-template <bool kGlobalLists, int kKeys, int kOnly, bool kLean>
+template <bool kGlobalLists, int kKeys, int kOnly, bool kLean, bool kRegS = false>
 __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, const uint32_t *order) {
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ ReplayDesc Dsh;
@@ -1270,7 +1345,7 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
   if (lane == 0) Dsh = descs[order[blockIdx.x]];
   __syncwarp();
   if (kOnly >= 0)
-    replay_body<kGlobalLists, kKeys, kOnly, kLean>(Dsh, bufs, smem, lane);
+    replay_body<kGlobalLists, kKeys, kOnly, kLean, kRegS>(Dsh, bufs, smem, lane);
   else if (kKeys == kKeyStream && Dsh.policy == UNISON_SPEAR_TIDE)
     replay_body<kGlobalLists, kKeys, UNISON_SPEAR_TIDE, false>(Dsh, bufs, smem, lane);
   else
@@ -1416,6 +1491,7 @@ struct ReplayPlan {
   std::vector<uint32_t> rcap_s, rcap_h, tmap;
   size_t max_smem_st = 0, max_smem_mix = 0, max_smem_online = 0, max_smem_stale = 0;
   bool st_lean = true;  // every shared-memory SPEAR+TIDE replay has the map with pin slots and no slot limit
+  bool st_reg = true;   // and a fast tier of at most 32 entries (held in the warp's registers)
 };
 
 // Resident-list capacity of a tier: at most one entry per session and no more
@@ -1455,8 +1531,10 @@ using ReplayKernel = void (*)(const ReplayDesc *, const uint32_t *);
 
 // The kernel of the shared-memory SPEAR+TIDE group, for a log or not.
 ReplayKernel st_kernel(const ReplayPlan &P, bool logged) {
-  return P.st_lean && !logged ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true>
-                              : replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, false>;
+  if (P.st_lean && !logged)
+    return P.st_reg ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true, true>
+                    : replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true>;
+  return replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, false>;
 }
 
 // Waves of CTAs a group of n replays needs with `dyn` bytes per CTA.
@@ -1572,6 +1650,7 @@ int plan_replays(const unison_trace *const *traces, const unison_replay_params *
   add_tier_maps(traces, params, smem_limit, P.in_mix, replay_kernel<false, kKeyStream, -1, false>, P.max_smem_mix,
                 P);
   for (uint32_t r : P.in_st) P.st_lean &= P.tmap[r] == kMapSlots && params[r].max_sessions == 0;
+  for (uint32_t r : P.in_st) P.st_reg &= P.rcap_s[r] <= 32;
   off_res = 0;
   if (results_in_scratch) {
     off_res = off;
