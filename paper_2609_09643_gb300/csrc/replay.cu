@@ -310,6 +310,107 @@ __device__ __forceinline__ void reg_erase_at(RegTier &R, uint32_t p, int lane) {
   R.n--;
 }
 
+// The HBM tier in registers (kRegH launches): lane l holds entries l, 32 + l,
+// 64 + l and 96 + l of the sorted array, three words each (key and size; an
+// entry's fourth word, its completion time, is read only by the timeout
+// policy, which these launches never run).  A search is four ballots, an
+// insert or an erase two shuffles per word and slot from the changed
+// position on.  A replay whose HBM tier would pass 128 entries writes it to
+// its shared-memory array once and continues there.
+constexpr uint32_t kHSlots = 4;
+constexpr uint32_t kHRegCap = 32 * kHSlots;
+struct RegTierH {
+  uint32_t x[kHSlots], y[kHSlots], z[kHSlots];  // key low, key high, size (and the promoted bit)
+};
+__device__ __forceinline__ uint64_t hkey(const RegTierH &G, int j) { return ((uint64_t)G.y[j] << 32) | G.x[j]; }
+// Entry i (warp-uniform, below 128; a larger i reads a slot-0 entry).
+__device__ __forceinline__ uint4 hreg_at(const RegTierH &G, uint32_t i) {
+  const uint32_t sl = i >> 5, ln = i & 31;
+  uint32_t a = G.x[0], b = G.y[0], c = G.z[0];
+#pragma unroll
+  for (int j = 1; j < (int)kHSlots; j++)
+    if (sl == (uint32_t)j) {
+      a = G.x[j];
+      b = G.y[j];
+      c = G.z[j];
+    }
+  return make_uint4(__shfl_sync(kFull, a, ln), __shfl_sync(kFull, b, ln), __shfl_sync(kFull, c, ln), 0u);
+}
+// Entries with key < k among the first n.
+__device__ __forceinline__ uint32_t hreg_lower_bound(const RegTierH &G, uint32_t n, uint64_t k, int lane) {
+  uint32_t cnt = 0;
+#pragma unroll
+  for (int j = 0; j < (int)kHSlots; j++) cnt += __popc(__ballot_sync(kFull, 32u * j + lane < n && hkey(G, j) < k));
+  return cnt;
+}
+// Insert e at position p of n < 128 entries: entries p.. move up one place
+// (slots from the top down, each taking lane 31 of the slot below).
+__device__ __forceinline__ void hreg_insert_at(RegTierH &G, uint32_t n, uint32_t p, uint4 e, int lane) {
+#pragma unroll
+  for (int j = (int)kHSlots - 1; j >= 0; j--) {
+    if (32u * j > n || 32u * j + 31 < p) continue;  // no position of [p, n] in slot j
+    const uint32_t ux = __shfl_up_sync(kFull, G.x[j], 1), uy = __shfl_up_sync(kFull, G.y[j], 1),
+                   uz = __shfl_up_sync(kFull, G.z[j], 1);
+    uint32_t cx = 0, cy = 0, cz = 0;
+    if (j > 0) {
+      cx = __shfl_sync(kFull, G.x[j - 1], 31);
+      cy = __shfl_sync(kFull, G.y[j - 1], 31);
+      cz = __shfl_sync(kFull, G.z[j - 1], 31);
+    }
+    const uint32_t idx = 32u * j + lane;
+    if (idx > p) {
+      G.x[j] = lane ? ux : cx;
+      G.y[j] = lane ? uy : cy;
+      G.z[j] = lane ? uz : cz;
+    } else if (idx == p) {
+      G.x[j] = e.x;
+      G.y[j] = e.y;
+      G.z[j] = e.z;
+    }
+  }
+}
+// Erase position p of n entries: entries p + 1.. move down one place (slots
+// from the bottom up, each taking lane 0 of the slot above).
+__device__ __forceinline__ void hreg_erase_at(RegTierH &G, uint32_t n, uint32_t p, int lane) {
+#pragma unroll
+  for (int j = 0; j < (int)kHSlots; j++) {
+    if (32u * j >= n || 32u * j + 31 < p) continue;  // no position of [p, n) in slot j
+    const uint32_t dx = __shfl_down_sync(kFull, G.x[j], 1), dy = __shfl_down_sync(kFull, G.y[j], 1),
+                   dz = __shfl_down_sync(kFull, G.z[j], 1);
+    uint32_t cx = 0, cy = 0, cz = 0;
+    if (j + 1 < (int)kHSlots) {
+      cx = __shfl_sync(kFull, G.x[j + 1], 0);
+      cy = __shfl_sync(kFull, G.y[j + 1], 0);
+      cz = __shfl_sync(kFull, G.z[j + 1], 0);
+    }
+    if (32u * j + lane >= p) {
+      G.x[j] = lane == 31 ? cx : dx;
+      G.y[j] = lane == 31 ? cy : dy;
+      G.z[j] = lane == 31 ? cz : dz;
+    }
+  }
+}
+// Drop the first m (1..32) of n >= m entries: entry i takes entry i + m.
+__device__ __forceinline__ void hreg_drop_front(RegTierH &G, uint32_t n, uint32_t m, int lane) {
+  const uint32_t src = (lane + m) & 31;
+  const bool above = lane + m >= 32;  // the source is in the next slot
+#pragma unroll
+  for (int j = 0; j < (int)kHSlots; j++) {
+    if (32u * j + m >= n) continue;  // nothing moves into slot j
+    const uint32_t ax = __shfl_sync(kFull, G.x[j], src), ay = __shfl_sync(kFull, G.y[j], src),
+                   az = __shfl_sync(kFull, G.z[j], src);
+    uint32_t bx = 0, by = 0, bz = 0;
+    if (j + 1 < (int)kHSlots) {
+      bx = __shfl_sync(kFull, G.x[j + 1], src);
+      by = __shfl_sync(kFull, G.y[j + 1], src);
+      bz = __shfl_sync(kFull, G.z[j + 1], src);
+    }
+    G.x[j] = above ? bx : ax;
+    G.y[j] = above ? by : ay;
+    G.z[j] = above ? bz : az;
+  }
+}
+
 // Descriptor fields the placement and fill read on every event, held in
 // registers (the descriptor itself sits in shared memory).
 struct Hot {
@@ -321,6 +422,8 @@ struct Hot {
 struct ReplayState {
   Sorted S, H;      // unpinned residents per tier
   RegTier R;        // the fast tier's residents instead of S, in kRegS launches
+  RegTierH G;       // the HBM tier's residents while hreg (kRegH launches); the count is H.n
+  bool hreg;
   uint4 *pin;       // pinned residents
   uint32_t npin, pin_cap;
   uint4 *tmp;       // TIDE staging: [0, cap_s) promoted, [cap_s, 2 cap_s) demoted
@@ -424,6 +527,61 @@ __device__ __forceinline__ uint4 reg_pop_back(ReplayState &st) {
   return v;
 }
 
+// HBM-tier operations on the registers while st.hreg, else on the array.
+template <bool kRegH>
+__device__ __forceinline__ uint4 h_at(const ReplayState &st, uint32_t i) {
+  if (kRegH && st.hreg) return hreg_at(st.G, i);
+  return st.H.e[i];
+}
+template <bool kRegH>
+__device__ __forceinline__ void h_erase_at(ReplayState &st, uint32_t p, int lane) {
+  if (kRegH && st.hreg) {
+    hreg_erase_at(st.G, st.H.n, p, lane);
+    st.H.n--;
+  } else {
+    sorted_erase(st.H, p, lane);
+  }
+}
+template <bool kLean, bool kRegH>
+__device__ __forceinline__ uint4 h_pop_back(ReplayState &st) {
+  if (kRegH && st.hreg) {
+    const uint4 v = hreg_at(st.G, st.H.n - 1);
+    st.H.n--;
+    set_tier<kLean>(st, packed_id(ekey(v)), kTierNone);
+    return v;
+  }
+  return sorted_pop_back<kLean>(st, st.H);
+}
+// Drop the first m entries (m <= 32 while st.hreg).
+template <bool kRegH>
+__device__ __forceinline__ void h_drop_front(ReplayState &st, uint32_t m, int lane) {
+  if (kRegH && st.hreg) hreg_drop_front(st.G, st.H.n, m, lane);
+  else shift_block(st.H.e, m, st.H.n, -(int32_t)m, lane);
+  st.H.n -= m;
+}
+template <bool kLean, bool kRegH>
+__device__ __forceinline__ bool h_insert(ReplayState &st, uint4 v, int lane) {
+  if (kRegH && st.hreg) {
+    if (st.H.n >= st.H.cap) {
+      st.status = UNISON_ERR_CAPACITY;
+      return false;
+    }
+    if (st.H.n < kHRegCap) {
+      hreg_insert_at(st.G, st.H.n, hreg_lower_bound(st.G, st.H.n, ekey(v), lane), v, lane);
+      st.H.n++;
+      set_tier<kLean>(st, packed_id(ekey(v)), kTierH);
+      return true;
+    }
+    // the 129th entry: the tier moves to its array for the rest of the replay
+#pragma unroll
+    for (int j = 0; j < (int)kHSlots; j++)
+      st.H.e[32u * j + lane] = make_uint4(st.G.x[j], st.G.y[j], st.G.z[j], 0u);
+    __syncwarp();
+    st.hreg = false;
+  }
+  return sorted_insert<kLean>(st, st.H, v, lane, kTierH);
+}
+
 __device__ __forceinline__ uint32_t esize(uint4 v) { return v.z & kSizeMask; }
 
 // Stale-snapshot replays (eq. stale): the arrays are ordered by snapshot
@@ -464,8 +622,9 @@ __device__ __forceinline__ void count_promotion(ReplayState &st, uint32_t chosen
 // A session demoted out of the fast tier enters HBM, displacing the most
 // evictable unpinned HBM sessions, or is dropped when it is itself the most
 // evictable of (unpinned HBM) + {itself}.
-template <bool kStale, bool kLean>
+template <bool kStale, bool kLean, bool kRegH = false>
 __device__ __forceinline__ bool admit_demoted(ReplayState &st, const Hot &D, uint4 d, int lane) {
+  static_assert(!(kRegH && kStale), "the register HBM tier serves live-key replays only");
   const uint32_t id = packed_id(ekey(d));
   const uint32_t size = esize(d);
   if (st.pinned_h > D.cap_h || size > D.cap_h - st.pinned_h) {
@@ -479,17 +638,17 @@ __device__ __forceinline__ bool admit_demoted(ReplayState &st, const Hot &D, uin
       count_victim(st, drop ? id : packed_id(ekey(st.H.e[st.H.n - 1])),
                    max(live_max(st, st.H, 0, st.H.n, lane), st.live[id]));
     }
-    if (st.H.n == 0 || ekey(d) > ekey(st.H.e[st.H.n - 1])) {
+    if (st.H.n == 0 || ekey(d) > ekey(h_at<kRegH>(st, st.H.n - 1))) {
       log_dec<kLean>(st, UNISON_KIND_EVICT, id, lane);
       CNT(st, n_evict, 1);
       return true;
     }
-    const uint4 v = sorted_pop_back<kLean>(st, st.H);
+    const uint4 v = h_pop_back<kLean, kRegH>(st);
     st.used_h -= esize(v);
     log_dec<kLean>(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
     CNT(st, n_evict, 1);
   }
-  if (!sorted_insert<kLean>(st, st.H, d, lane, kTierH)) return false;
+  if (!h_insert<kLean, kRegH>(st, d, lane)) return false;
   st.used_h += size;
   log_dec<kLean>(st, UNISON_KIND_DEMOTE, id, lane);
   CNT(st, n_demote, 1);
@@ -510,7 +669,7 @@ __device__ __forceinline__ bool pin_append(ReplayState &st, uint64_t pk, uint32_
 }
 
 // Placement of the arriving (pinned) session s with n tokens.
-template <bool kStale, bool kLean, bool kRegS = false>
+template <bool kStale, bool kLean, bool kRegS = false, bool kRegH = false>
 __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s, uint64_t pk, uint32_t n,
                                       int lane) {
   if (!kLean && D.max_sessions && st.npin >= D.max_sessions) {
@@ -528,7 +687,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
       // most evictable unpinned fast-tier session
       const uint4 d = kRegS ? reg_pop_back<kLean>(st) : sorted_pop_back<kLean>(st, st.S);
       st.used_s -= esize(d);
-      if (!admit_demoted<kStale, kLean>(st, D, d, lane)) return false;
+      if (!admit_demoted<kStale, kLean, kRegH>(st, D, d, lane)) return false;
     }
     if (!pin_append(st, pk, n, s, kTierS, lane)) return false;
     st.used_s += n;
@@ -542,7 +701,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
         return false;
       }
       if (kStale) count_victim(st, packed_id(ekey(st.H.e[st.H.n - 1])), live_max(st, st.H, 0, st.H.n, lane));
-      const uint4 v = sorted_pop_back<kLean>(st, st.H);
+      const uint4 v = h_pop_back<kLean, kRegH>(st);
       st.used_h -= esize(v);
       log_dec<kLean>(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
       CNT(st, n_evict, 1);
@@ -585,7 +744,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
 // free fast-tier space; phase 2: pair the next least evictable HBM session
 // with the most evictable fast-tier one), which makes the same moves as the
 // pair loop of Algorithm 1, and are then applied in bulk.
-template <bool kStale, bool kLean, bool kRegS = false>
+template <bool kStale, bool kLean, bool kRegS = false, bool kRegH = false>
 __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t budget, uint32_t rcap_s,
                                          int lane) {
   const uint32_t sn = kRegS ? st.R.n : st.S.n;  // fast-tier entries; the fast tier changes only at the end
@@ -593,7 +752,7 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
   const uint64_t kvb = D.kvb;
   uint32_t n1 = 0;
   while (n1 < st.H.n) {
-    const uint4 p = st.H.e[n1];
+    const uint4 p = h_at<kRegH>(st, n1);
     const uint64_t sz = esize(p), by = sz * kvb;
     if (by > rem || st.used_s + sz > D.cap_s) break;
     // (the loop form's candidates: HBM less the sessions promoted so far)
@@ -607,11 +766,11 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
   uint32_t pairs = 0;
   for (;;) {
     if (n1 + pairs >= st.H.n || pairs >= sn) break;
-    const uint4 p = st.H.e[n1 + pairs];
+    const uint4 p = h_at<kRegH>(st, n1 + pairs);
     const uint4 d = kRegS ? reg_at(st.R, sn - 1 - pairs) : st.S.e[st.S.n - 1 - pairs];
     // the next most evictable of (fast tier + promoted) is a promoted session
     // when the largest promoted key beats d: then it cannot beat p, stop
-    if (n1 > 0 && ekey(st.H.e[n1 - 1]) > ekey(d)) break;
+    if (n1 > 0 && ekey(h_at<kRegH>(st, n1 - 1)) > ekey(d)) break;
     if (!(ekey(d) > ekey(p))) break;
     const uint64_t sp = esize(p), sd = esize(d), by = (sp + sd) * kvb;
     if (by > rem) break;
@@ -642,22 +801,20 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     return budget - rem;
   }
   if (m == 1 && pairs == 0) {  // one promotion (the common case): move it directly
-    uint4 v = st.H.e[0];
+    uint4 v = h_at<kRegH>(st, 0);
     v.z |= kPromotedBit;
     __syncwarp();
-    shift_block(st.H.e, 1, st.H.n, -1, lane);
-    st.H.n -= 1;
+    h_drop_front<kRegH>(st, 1, lane);
     if (kRegS) reg_sorted_insert<kLean>(st, v, lane);
     else sorted_insert<kLean>(st, st.S, v, lane, kTierS);
     return budget - rem;
   }
   if (m == 1 && pairs == 1) {  // one pair (the next most common): swap it directly
-    uint4 v = st.H.e[0];
+    uint4 v = h_at<kRegH>(st, 0);
     v.z |= kPromotedBit;
     const uint4 d = kRegS ? reg_at(st.R, sn - 1) : st.S.e[st.S.n - 1];
     __syncwarp();
-    shift_block(st.H.e, 1, st.H.n, -1, lane);
-    st.H.n -= 1;
+    h_drop_front<kRegH>(st, 1, lane);
     if (kRegS) {
       st.R.n -= 1;
       if (!reg_sorted_insert<kLean>(st, v, lane)) return budget - rem;
@@ -665,15 +822,19 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
       st.S.n -= 1;
       if (!sorted_insert<kLean>(st, st.S, v, lane, kTierS)) return budget - rem;
     }
-    sorted_insert<kLean>(st, st.H, d, lane, kTierH);
+    h_insert<kLean, kRegH>(st, d, lane);
     return budget - rem;
   }
   // stage the moved entries, then fix both arrays
   uint4 *pro = st.tmp, *dem = st.tmp + rcap_s;
-  for (uint32_t i = lane; i < m; i += 32) {
-    uint4 v = st.H.e[i];
-    v.z |= kPromotedBit;
-    pro[i] = v;
+  if (kRegH && st.hreg) {  // m <= 32: the first m entries are slot 0's
+    if ((uint32_t)lane < m) pro[lane] = make_uint4(st.G.x[0], st.G.y[0], st.G.z[0] | kPromotedBit, 0u);
+  } else {
+    for (uint32_t i = lane; i < m; i += 32) {
+      uint4 v = st.H.e[i];
+      v.z |= kPromotedBit;
+      pro[i] = v;
+    }
   }
   if (kRegS) {  // pairs <= fast-tier entries <= 32: one entry a lane
     const uint4 dv = reg_at(st.R, min(sn - pairs + (uint32_t)lane, 31u));
@@ -682,15 +843,14 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     for (uint32_t i = lane; i < pairs; i += 32) dem[i] = st.S.e[st.S.n - pairs + i];
   }
   __syncwarp();
-  shift_block(st.H.e, m, st.H.n, -(int32_t)m, lane);
-  st.H.n -= m;
+  h_drop_front<kRegH>(st, m, lane);
   if (kRegS) st.R.n -= pairs;
   else st.S.n -= pairs;
   for (uint32_t i = 0; i < m; i++)
     if (kRegS ? !reg_sorted_insert<kLean>(st, pro[i], lane) : !sorted_insert<kLean>(st, st.S, pro[i], lane, kTierS))
       return budget - rem;
   for (uint32_t i = 0; i < pairs; i++)
-    if (!sorted_insert<kLean>(st, st.H, dem[i], lane, kTierH)) return budget - rem;
+    if (!h_insert<kLean, kRegH>(st, dem[i], lane)) return budget - rem;
   return budget - rem;
 }
 
@@ -889,9 +1049,13 @@ struct EventBufs {
 // One replay: Algorithm 1 over the trace's events.  kPol is the replay's
 // policy when the body is specialised for it (its policy tests then fold
 // away), or -1 for the body that reads the policy from the descriptor.
-template <bool kGlobalLists, int kKeys, int kPol, bool kLean, bool kRegS = false>
+template <bool kGlobalLists, int kKeys, int kPol, bool kLean, bool kRegS = false, bool kRegH = false>
 __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs, unsigned char *smem, int lane) {
   constexpr bool kOnline = kKeys == kKeyOnline, kStale = kKeys == kKeyStale;
+  // the register HBM tier drops the entries' completion times (timeout only)
+  // and drop_front's m <= 32 rests on the fast tier's 32-entry bound
+  static_assert(!kRegH || (kRegS && kLean && kPol == UNISON_SPEAR_TIDE && !kOnline && !kStale),
+                "register HBM tier: lean SPEAR+TIDE launches with the register fast tier");
   const Hot hot{D.cap_s, D.cap_h, D.kvb, D.dma, D.max_sessions};
 
   ReplayState st;
@@ -980,6 +1144,9 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
     st.S.n = st.H.n = 0;
     st.R.n = 0;
     st.R.v = make_uint4(0u, 0u, 0u, 0u);
+    st.hreg = kRegH;
+#pragma unroll
+    for (int j = 0; j < (int)kHSlots; j++) st.G.x[j] = st.G.y[j] = st.G.z[j] = 0u;
     st.S.cap = D.rcap_s;
     st.H.cap = D.rcap_h;
     st.npin = 0;
@@ -1103,10 +1270,19 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
             }
           }
           if (tier == kTierNone && (mt & kTierH)) {
-            pos = lower_bound(st.H, pkb, lane);
-            if (pos < st.H.n && ekey(st.H.e[pos]) == pkb) {
-              tier = kTierH;
-              ent = st.H.e[pos];
+            if (kRegH && st.hreg) {
+              pos = hreg_lower_bound(st.G, st.H.n, pkb, lane);
+              const uint4 cand = hreg_at(st.G, pos);  // (pos 128 reads a slot-0 entry; not taken)
+              if (pos < st.H.n && ekey(cand) == pkb) {
+                tier = kTierH;
+                ent = cand;
+              }
+            } else {
+              pos = lower_bound(st.H, pkb, lane);
+              if (pos < st.H.n && ekey(st.H.e[pos]) == pkb) {
+                tier = kTierH;
+                ent = st.H.e[pos];
+              }
             }
           }
           __syncwarp();
@@ -1156,7 +1332,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
           set_tier<kLean>(st, s, kTierNone);
         } else if (tier == kTierH) {
           st.used_h -= esize(ent);
-          sorted_erase(st.H, pos, lane);
+          h_erase_at<kRegH>(st, pos, lane);
           set_tier<kLean>(st, s, kTierNone);
         }
         uint64_t pk;
@@ -1182,7 +1358,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
           pk = pack_key(nr == kNoRef ? kKeyMax40 : (uint64_t)nr, s);
         } else
           pk = pack_key(0xFFFFFFFFull - e, s);
-        if (!place<kStale, kLean, kRegS>(st, hot, s, pk, out, lane)) break;
+        if (!place<kStale, kLean, kRegS, kRegH>(st, hot, s, pk, out, lane)) break;
       } else {
         // completion: unpin (if resident) and rank the session with its new key
         if (kStale) {
@@ -1227,7 +1403,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
             if (kRegS ? !reg_sorted_insert<kLean>(st, v, lane) : !sorted_insert<kLean>(st, st.S, v, lane, kTierS)) break;
           } else {
             st.pinned_h -= sz;
-            if (!sorted_insert<kLean>(st, st.H, v, lane, kTierH)) break;
+            if (!h_insert<kLean, kRegH>(st, v, lane)) break;
           }
         }
         if (kOnline && edge) {
@@ -1242,7 +1418,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
           const uint64_t g = sgq[bi][j];
           const uint64_t budget = g * D.dma;
           CNT(st, n_tide_calls, 1);
-          const uint64_t moved = tide<kStale, kLean, kRegS>(st, hot, budget, D.rcap_s, lane);
+          const uint64_t moved = tide<kStale, kLean, kRegS, kRegH>(st, hot, budget, D.rcap_s, lane);
           CNT(st, dma_bytes, moved);
           if (moved > 0 && D.dma > 0) {
             dma_busy = true;
@@ -1336,7 +1512,7 @@ __device__ __forceinline__ void replay_body(const ReplayDesc &D, EventBufs &bufs
 // replay of the launch has that policy, and the kernel holds only its body
 // (and is sized for it alone); kLean: every replay of the launch is lean
 // (see log_dec).
-template <bool kGlobalLists, int kKeys, int kOnly, bool kLean, bool kRegS = false>
+template <bool kGlobalLists, int kKeys, int kOnly, bool kLean, bool kRegS = false, bool kRegH = false>
 __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, const uint32_t *order) {
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ ReplayDesc Dsh;
@@ -1345,7 +1521,7 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
   if (lane == 0) Dsh = descs[order[blockIdx.x]];
   __syncwarp();
   if (kOnly >= 0)
-    replay_body<kGlobalLists, kKeys, kOnly, kLean, kRegS>(Dsh, bufs, smem, lane);
+    replay_body<kGlobalLists, kKeys, kOnly, kLean, kRegS, kRegH>(Dsh, bufs, smem, lane);
   else if (kKeys == kKeyStream && Dsh.policy == UNISON_SPEAR_TIDE)
     replay_body<kGlobalLists, kKeys, UNISON_SPEAR_TIDE, false>(Dsh, bufs, smem, lane);
   else
@@ -1532,7 +1708,7 @@ using ReplayKernel = void (*)(const ReplayDesc *, const uint32_t *);
 // The kernel of the shared-memory SPEAR+TIDE group, for a log or not.
 ReplayKernel st_kernel(const ReplayPlan &P, bool logged) {
   if (P.st_lean && !logged)
-    return P.st_reg ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true, true>
+    return P.st_reg ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true, true, true>
                     : replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true>;
   return replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, false>;
 }

@@ -127,6 +127,23 @@ def test_sweep_iid_gaps_subset(B):
         assert_same(res[i], oracle.replay(trs[ti], to_oracle(p)), i)
 
 
+def test_hbm_tier_past_register_capacity(B):
+    """SPEAR+TIDE replays whose HBM tier outgrows the 128 entries the lean
+    launch holds in registers: with a fast tier of at most 32 entries every
+    replay of the call takes the register tiers, and the HBM tier of the
+    first two configurations reaches about 200 unpinned sessions (the oracle
+    counts 210 and 192 on seed 0), so it moves to shared memory mid-replay;
+    the last stays just under the bound (126).  Every counter and the decision
+    hash against the oracle."""
+    trs = [synth.paper_scale_trace(s, "coding") for s in (0, 1)]
+    cfgs = [(28_672, 1 * GIB, 64 * GIB), (131_072, 1 * GIB, 256 * GIB), (28_672, 512 * MIB, 32 * GIB)]
+    reps = [(ti, base("spear_tide", cs, ch, kvb)) for ti in range(len(trs)) for kvb, cs, ch in cfgs]
+    res, _, _ = run_gpu(B, trs, reps)
+    for i, (ti, p) in enumerate(reps):
+        assert res[i]["status"] == 0
+        assert_same(res[i], oracle.replay(trs[ti], to_oracle(p)), (ti, p["kvb"], p["cap_s"], p["cap_h"]))
+
+
 @pytest.mark.parametrize("seed", [100, 101])
 def test_large_pool_replay(B, seed):
     tr = synth.large_pool_trace(seed)
