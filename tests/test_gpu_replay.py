@@ -132,9 +132,10 @@ def test_hbm_tier_past_register_capacity(B):
     launch holds in registers: with a fast tier of at most 32 entries every
     replay of the call takes the register tiers, and the HBM tier of the
     first two configurations reaches about 200 unpinned sessions (the oracle
-    counts 210 and 192 on seed 0), so it moves to shared memory mid-replay;
-    the last stays just under the bound (126).  Every counter and the decision
-    hash against the oracle."""
+    counts 210 and 192 on seed 0), so those replays stop at the 129th entry
+    and run again from their start with the tier in shared memory; the last
+    stays just under the bound (126).  Every counter and the decision hash
+    against the oracle."""
     trs = [synth.paper_scale_trace(s, "coding") for s in (0, 1)]
     cfgs = [(28_672, 1 * GIB, 64 * GIB), (131_072, 1 * GIB, 256 * GIB), (28_672, 512 * MIB, 32 * GIB)]
     reps = [(ti, base("spear_tide", cs, ch, kvb)) for ti in range(len(trs)) for kvb, cs, ch in cfgs]
