@@ -1170,7 +1170,7 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
   unsigned long long s_lo = 0, s_hi = 0;
   uint32_t stale_arrivals = 0;
   bool dma_busy = false;
-  uint32_t busy_until = 0;
+  uint64_t busy_from = 0, busy_bytes = 0;  // the DMA's last batch: start (rel_us) and bytes
 
   auto &sev = bufs.sev;
   auto &sprev = bufs.sprev, &spev = bufs.spev, &snref = bufs.snref, &sgq = bufs.sgq;
@@ -1219,7 +1219,13 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
       rel_us += (uint32_t)(now - prev_now);
       prev_now = now;
       if (timeout) expire_idle<kLean>(st, now, D.ttl, lane);
-      if (dma_busy && (int32_t)(now - busy_until) >= 0) dma_busy = false;
+      // the DMA is free again from start + ceil(bytes / rate) us on, i.e. once
+      // the elapsed us times the rate cover the bytes (no division; the high
+      // word of the product catches a product past 2^64)
+      if (dma_busy) {
+        const uint64_t el = rel_us - busy_from;
+        if (__umul64hi(el, hot.dma) != 0 || el * hot.dma >= busy_bytes) dma_busy = false;
+      }
 
       if (arrival) {
         const uint32_t in = ev.z;
@@ -1413,7 +1419,8 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
           CNT(st, dma_bytes, moved);
           if (moved > 0 && D.dma > 0) {
             dma_busy = true;
-            busy_until = now + (uint32_t)((moved + D.dma - 1) / D.dma);
+            busy_from = rel_us;
+            busy_bytes = moved;
           }
           if (st.status == UNISON_ERR_CAPACITY || st.status == kRegFull) break;
         }
