@@ -1249,7 +1249,27 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
             pkb = pack_key(0xFFFFFFFFull - spev[bi][j], s);
           // with the tier map only the session's own tier is searched (and
           // nothing for a session that is not resident)
-          const uint32_t mt = (kLean || st.tmap) ? st.tmap[s] : (kTierS | kTierH);
+          if (kRegH) {
+            // both tiers in registers: one equality ballot per slot finds the
+            // key (unique: it carries the session id) without the tier map
+            const unsigned fs = __ballot_sync(kFull, (uint32_t)lane < st.R.n && ekey(st.R.v) == pkb);
+            unsigned fh[kHSlots];
+#pragma unroll
+            for (int j = 0; j < (int)kHSlots; j++)
+              fh[j] = __ballot_sync(kFull, 32u * j + lane < st.H.n && hkey(st.G, j) == pkb);
+            uint32_t ph = 0;
+#pragma unroll
+            for (int j = (int)kHSlots - 1; j >= 0; j--)
+              if (fh[j]) ph = 32u * j + __ffs(fh[j]) - 1;
+            const uint32_t ps = fs ? __ffs(fs) - 1 : 0u;
+            const uint4 es = reg_at(st.R, ps), eh = hreg_at(st.G, ph);
+            const bool inh = (fh[0] | fh[1] | fh[2] | fh[3]) != 0;
+            static_assert(kHSlots == 4, "the found test names the four slots");
+            tier = fs ? kTierS : (inh ? kTierH : kTierNone);
+            pos = fs ? ps : ph;
+            ent = fs ? es : eh;
+          }
+          const uint32_t mt = kRegH ? 0u : ((kLean || st.tmap) ? st.tmap[s] : (kTierS | kTierH));
           if (mt & kTierS) {
             if (kRegS) {
               pos = reg_lower_bound(st.R, pkb, lane);
