@@ -310,29 +310,37 @@ __device__ __forceinline__ void reg_erase_at(RegTier &R, uint32_t p, int lane) {
   R.n--;
 }
 
-// The HBM tier in registers (kRegH launches): lane l holds entries l, 32 + l,
-// 64 + l and 96 + l of the sorted array, three words each (key and size; an
+// The HBM tier in registers (kHK > 0 slots a lane): lane l holds entries l,
+// 32 + l, 64 + l, ... of the sorted array, three words each (key and size; an
 // entry's fourth word, its completion time, is read only by the timeout
-// policy, which these launches never run).  A search is four ballots; an
+// policy, which these launches never run).  A search is kHK ballots; an
 // insert, an erase or a drop of the first entries one shuffle per word and
-// slot.  A replay whose HBM tier would pass 128 entries stops (kRegFull) and
-// is replayed from its start with the tier in shared memory: a replay is
+// slot.  A replay whose HBM tier would pass 32 kHK entries stops (kRegFull)
+// and is replayed from its start with the tier in shared memory: a replay is
 // deterministic, so its results are the same, and the register body needs no
 // test of where the tier is (measured: the sweep runs 6% faster than with a
 // one-way move of the tier to shared memory tested at every operation).
-constexpr uint32_t kHSlots = 4;
-constexpr uint32_t kHRegCap = 32 * kHSlots;
+// The restart is kept for the rare replay: while warps of one SM run
+// different bodies the launch slows down far beyond the repeated work
+// (measured: independent-gap sweep, 128 GiB replays restarting with 6
+// slots: 121 ms, against 70 ms with 6 slots from the start).  Five slots hold
+// both sweeps' HBM tiers (at most about 125 entries with per-session gap
+// recurrence, about 140 with independent gaps); four run the recurrent-gap
+// sweep 7% faster but send the other's 128 GiB replays to shared memory.
+constexpr int kHSlots = 5;
 constexpr int kRegFull = -1000;  // internal status: never reported
 struct RegTierH {
-  uint32_t x[kHSlots], y[kHSlots], z[kHSlots];  // key low, key high, size (and the promoted bit)
+  // key low, key high, size (and the promoted bit)
+  uint32_t x[kHSlots], y[kHSlots], z[kHSlots];
 };
 __device__ __forceinline__ uint64_t hkey(const RegTierH &G, int j) { return ((uint64_t)G.y[j] << 32) | G.x[j]; }
-// Entry i (warp-uniform, below 128; a larger i reads a slot-0 entry).
+// Entry i (warp-uniform, below 32 K; a larger i reads a slot-0 entry).
+template <int K>
 __device__ __forceinline__ uint4 hreg_at(const RegTierH &G, uint32_t i) {
   const uint32_t sl = i >> 5, ln = i & 31;
   uint32_t a = G.x[0], b = G.y[0], c = G.z[0];
 #pragma unroll
-  for (int j = 1; j < (int)kHSlots; j++)
+  for (int j = 1; j < K; j++)
     if (sl == (uint32_t)j) {
       a = G.x[j];
       b = G.y[j];
@@ -341,23 +349,25 @@ __device__ __forceinline__ uint4 hreg_at(const RegTierH &G, uint32_t i) {
   return make_uint4(__shfl_sync(kFull, a, ln), __shfl_sync(kFull, b, ln), __shfl_sync(kFull, c, ln), 0u);
 }
 // Entries with key < k among the first n.
+template <int K>
 __device__ __forceinline__ uint32_t hreg_lower_bound(const RegTierH &G, uint32_t n, uint64_t k, int lane) {
   uint32_t cnt = 0;
 #pragma unroll
-  for (int j = 0; j < (int)kHSlots; j++) cnt += __popc(__ballot_sync(kFull, 32u * j + lane < n && hkey(G, j) < k));
+  for (int j = 0; j < K; j++) cnt += __popc(__ballot_sync(kFull, 32u * j + lane < n && hkey(G, j) < k));
   return cnt;
 }
-// Insert e at position p (fewer than 128 entries): entries p.. move up one
+// Insert e at position p (fewer than 32 K entries): entries p.. move up one
 // place.  Lane l of a slot takes lane l - 1's entry, lane 0 the slot below's
 // lane 31: the providing lane picks the slot, so a word moves in one shuffle
 // (slots from the top down, each reading the slot below before it changes).
 // Here and below every slot moves whatever the count and position: entries
 // past the count may hold anything, and the shuffles cost less than branches
 // that would skip the unchanged slots (measured: the sweep runs 8% faster).
+template <int K>
 __device__ __forceinline__ void hreg_insert_at(RegTierH &G, uint32_t p, uint4 e, int lane) {
   const uint32_t from = (lane - 1) & 31;
 #pragma unroll
-  for (int j = (int)kHSlots - 1; j >= 0; j--) {
+  for (int j = K - 1; j >= 0; j--) {
     const bool low = j > 0 && lane == 31;  // lane 31 provides the slot below's entry
     const uint32_t ux = __shfl_sync(kFull, low ? G.x[j > 0 ? j - 1 : 0] : G.x[j], from),
                    uy = __shfl_sync(kFull, low ? G.y[j > 0 ? j - 1 : 0] : G.y[j], from),
@@ -377,11 +387,12 @@ __device__ __forceinline__ void hreg_insert_at(RegTierH &G, uint32_t p, uint4 e,
 // Erase position p: entries p + 1.. move down one place.  Lane l
 // takes lane l + 1's entry, lane 31 the slot above's lane 0 (slots from the
 // bottom up, each reading the slot above before it changes).
+template <int K>
 __device__ __forceinline__ void hreg_erase_at(RegTierH &G, uint32_t p, int lane) {
   const uint32_t from = (lane + 1) & 31;
 #pragma unroll
-  for (int j = 0; j < (int)kHSlots; j++) {
-    constexpr int kTop = (int)kHSlots - 1;
+  for (int j = 0; j < K; j++) {
+    constexpr int kTop = K - 1;
     const bool high = j < kTop && lane == 0;  // lane 0 provides the slot above's entry
     const uint32_t dx = __shfl_sync(kFull, high ? G.x[j < kTop ? j + 1 : kTop] : G.x[j], from),
                    dy = __shfl_sync(kFull, high ? G.y[j < kTop ? j + 1 : kTop] : G.y[j], from),
@@ -396,12 +407,13 @@ __device__ __forceinline__ void hreg_erase_at(RegTierH &G, uint32_t p, int lane)
 // Drop the first m (1..32) entries: entry i takes entry i + m, from
 // lane (l + m) mod 32 of the same slot, or of the next one where l + m >= 32;
 // the providing lanes below m give the next slot's entry.
+template <int K>
 __device__ __forceinline__ void hreg_drop_front(RegTierH &G, uint32_t m, int lane) {
   const uint32_t from = (lane + m) & 31;
   const bool next = (uint32_t)lane < m;
 #pragma unroll
-  for (int j = 0; j < (int)kHSlots; j++) {
-    constexpr int kTop = (int)kHSlots - 1;
+  for (int j = 0; j < K; j++) {
+    constexpr int kTop = K - 1;
     const bool up = j < kTop && next;
     G.x[j] = __shfl_sync(kFull, up ? G.x[j < kTop ? j + 1 : kTop] : G.x[j], from);
     G.y[j] = __shfl_sync(kFull, up ? G.y[j < kTop ? j + 1 : kTop] : G.y[j], from);
@@ -420,7 +432,7 @@ struct Hot {
 struct ReplayState {
   Sorted S, H;      // unpinned residents per tier
   RegTier R;        // the fast tier's residents instead of S, in kRegS launches
-  RegTierH G;       // the HBM tier's residents instead of H.e, in kRegH launches; the count is H.n
+  RegTierH G;       // the HBM tier's residents instead of H.e, in kHK > 0 bodies; the count is H.n
   uint4 *pin;       // pinned residents
   uint32_t npin, pin_cap;
   uint4 *tmp;       // TIDE staging: [0, cap_s) promoted, [cap_s, 2 cap_s) demoted
@@ -524,47 +536,47 @@ __device__ __forceinline__ uint4 reg_pop_back(ReplayState &st) {
   return v;
 }
 
-// HBM-tier operations on the registers (kRegH) or on the array.
-template <bool kRegH>
+// HBM-tier operations on kHK register slots a lane, or on the array (kHK 0).
+template <int kHK>
 __device__ __forceinline__ uint4 h_at(const ReplayState &st, uint32_t i) {
-  if (kRegH) return hreg_at(st.G, i);
+  if constexpr (kHK > 0) return hreg_at<kHK>(st.G, i);
   return st.H.e[i];
 }
-template <bool kRegH>
+template <int kHK>
 __device__ __forceinline__ void h_erase_at(ReplayState &st, uint32_t p, int lane) {
-  if (kRegH) {
-    hreg_erase_at(st.G, p, lane);
+  if constexpr (kHK > 0) {
+    hreg_erase_at<kHK>(st.G, p, lane);
     st.H.n--;
   } else {
     sorted_erase(st.H, p, lane);
   }
 }
-template <bool kLean, bool kRegH>
+template <bool kLean, int kHK>
 __device__ __forceinline__ uint4 h_pop_back(ReplayState &st) {
-  if (kRegH) {
-    const uint4 v = hreg_at(st.G, st.H.n - 1);
+  if constexpr (kHK > 0) {
+    const uint4 v = hreg_at<kHK>(st.G, st.H.n - 1);
     st.H.n--;
     set_tier<kLean>(st, packed_id(ekey(v)), kTierNone);
     return v;
   }
   return sorted_pop_back<kLean>(st, st.H);
 }
-// Drop the first m entries (m <= 32 in kRegH launches).
-template <bool kRegH>
+// Drop the first m entries (m <= 32 in register bodies).
+template <int kHK>
 __device__ __forceinline__ void h_drop_front(ReplayState &st, uint32_t m, int lane) {
-  if (kRegH) hreg_drop_front(st.G, m, lane);
+  if constexpr (kHK > 0) hreg_drop_front<kHK>(st.G, m, lane);
   else shift_block(st.H.e, m, st.H.n, -(int32_t)m, lane);
   st.H.n -= m;
 }
-template <bool kLean, bool kRegH>
+template <bool kLean, int kHK>
 __device__ __forceinline__ bool h_insert(ReplayState &st, uint4 v, int lane) {
-  if (kRegH) {
-    if (st.H.n >= st.H.cap || st.H.n >= kHRegCap) {
-      // the list bound, or the registers' 128 entries (the replay starts over)
+  if constexpr (kHK > 0) {
+    if (st.H.n >= st.H.cap || st.H.n >= 32u * kHK) {
+      // the list bound, or the registers' 32 kHK entries (the replay starts over)
       st.status = st.H.n >= st.H.cap ? UNISON_ERR_CAPACITY : kRegFull;
       return false;
     }
-    hreg_insert_at(st.G, hreg_lower_bound(st.G, st.H.n, ekey(v), lane), v, lane);
+    hreg_insert_at<kHK>(st.G, hreg_lower_bound<kHK>(st.G, st.H.n, ekey(v), lane), v, lane);
     st.H.n++;
     set_tier<kLean>(st, packed_id(ekey(v)), kTierH);
     return true;
@@ -612,9 +624,9 @@ __device__ __forceinline__ void count_promotion(ReplayState &st, uint32_t chosen
 // A session demoted out of the fast tier enters HBM, displacing the most
 // evictable unpinned HBM sessions, or is dropped when it is itself the most
 // evictable of (unpinned HBM) + {itself}.
-template <bool kStale, bool kLean, bool kRegH = false>
+template <bool kStale, bool kLean, int kHK = 0>
 __device__ __forceinline__ bool admit_demoted(ReplayState &st, const Hot &D, uint4 d, int lane) {
-  static_assert(!(kRegH && kStale), "the register HBM tier serves live-key replays only");
+  static_assert(!(kHK > 0 && kStale), "the register HBM tier serves live-key replays only");
   const uint32_t id = packed_id(ekey(d));
   const uint32_t size = esize(d);
   if (st.pinned_h > D.cap_h || size > D.cap_h - st.pinned_h) {
@@ -628,17 +640,17 @@ __device__ __forceinline__ bool admit_demoted(ReplayState &st, const Hot &D, uin
       count_victim(st, drop ? id : packed_id(ekey(st.H.e[st.H.n - 1])),
                    max(live_max(st, st.H, 0, st.H.n, lane), st.live[id]));
     }
-    if (st.H.n == 0 || ekey(d) > ekey(h_at<kRegH>(st, st.H.n - 1))) {
+    if (st.H.n == 0 || ekey(d) > ekey(h_at<kHK>(st, st.H.n - 1))) {
       log_dec<kLean>(st, UNISON_KIND_EVICT, id, lane);
       CNT(st, n_evict, 1);
       return true;
     }
-    const uint4 v = h_pop_back<kLean, kRegH>(st);
+    const uint4 v = h_pop_back<kLean, kHK>(st);
     st.used_h -= esize(v);
     log_dec<kLean>(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
     CNT(st, n_evict, 1);
   }
-  if (!h_insert<kLean, kRegH>(st, d, lane)) return false;
+  if (!h_insert<kLean, kHK>(st, d, lane)) return false;
   st.used_h += size;
   log_dec<kLean>(st, UNISON_KIND_DEMOTE, id, lane);
   CNT(st, n_demote, 1);
@@ -659,7 +671,7 @@ __device__ __forceinline__ bool pin_append(ReplayState &st, uint64_t pk, uint32_
 }
 
 // Placement of the arriving (pinned) session s with n tokens.
-template <bool kStale, bool kLean, bool kRegS = false, bool kRegH = false>
+template <bool kStale, bool kLean, bool kRegS = false, int kHK = 0>
 __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s, uint64_t pk, uint32_t n,
                                       int lane) {
   if (!kLean && D.max_sessions && st.npin >= D.max_sessions) {
@@ -677,7 +689,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
       // most evictable unpinned fast-tier session
       const uint4 d = kRegS ? reg_pop_back<kLean>(st) : sorted_pop_back<kLean>(st, st.S);
       st.used_s -= esize(d);
-      if (!admit_demoted<kStale, kLean, kRegH>(st, D, d, lane)) return false;
+      if (!admit_demoted<kStale, kLean, kHK>(st, D, d, lane)) return false;
     }
     if (!pin_append(st, pk, n, s, kTierS, lane)) return false;
     st.used_s += n;
@@ -691,7 +703,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
         return false;
       }
       if (kStale) count_victim(st, packed_id(ekey(st.H.e[st.H.n - 1])), live_max(st, st.H, 0, st.H.n, lane));
-      const uint4 v = h_pop_back<kLean, kRegH>(st);
+      const uint4 v = h_pop_back<kLean, kHK>(st);
       st.used_h -= esize(v);
       log_dec<kLean>(st, UNISON_KIND_EVICT, packed_id(ekey(v)), lane);
       CNT(st, n_evict, 1);
@@ -734,7 +746,7 @@ __device__ __forceinline__ bool place(ReplayState &st, const Hot &D, uint32_t s,
 // free fast-tier space; phase 2: pair the next least evictable HBM session
 // with the most evictable fast-tier one), which makes the same moves as the
 // pair loop of Algorithm 1, and are then applied in bulk.
-template <bool kStale, bool kLean, bool kRegS = false, bool kRegH = false>
+template <bool kStale, bool kLean, bool kRegS = false, int kHK = 0>
 __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t budget, uint32_t rcap_s,
                                          int lane) {
   const uint32_t sn = kRegS ? st.R.n : st.S.n;  // fast-tier entries; the fast tier changes only at the end
@@ -742,7 +754,7 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
   const uint64_t kvb = D.kvb;
   uint32_t n1 = 0;
   while (n1 < st.H.n) {
-    const uint4 p = h_at<kRegH>(st, n1);
+    const uint4 p = h_at<kHK>(st, n1);
     const uint64_t sz = esize(p), by = sz * kvb;
     if (by > rem || st.used_s + sz > D.cap_s) break;
     // (the loop form's candidates: HBM less the sessions promoted so far)
@@ -756,11 +768,11 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
   uint32_t pairs = 0;
   for (;;) {
     if (n1 + pairs >= st.H.n || pairs >= sn) break;
-    const uint4 p = h_at<kRegH>(st, n1 + pairs);
+    const uint4 p = h_at<kHK>(st, n1 + pairs);
     const uint4 d = kRegS ? reg_at(st.R, sn - 1 - pairs) : st.S.e[st.S.n - 1 - pairs];
     // the next most evictable of (fast tier + promoted) is a promoted session
     // when the largest promoted key beats d: then it cannot beat p, stop
-    if (n1 > 0 && ekey(h_at<kRegH>(st, n1 - 1)) > ekey(d)) break;
+    if (n1 > 0 && ekey(h_at<kHK>(st, n1 - 1)) > ekey(d)) break;
     if (!(ekey(d) > ekey(p))) break;
     const uint64_t sp = esize(p), sd = esize(d), by = (sp + sd) * kvb;
     if (by > rem) break;
@@ -791,20 +803,20 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     return budget - rem;
   }
   if (m == 1 && pairs == 0) {  // one promotion (the common case): move it directly
-    uint4 v = h_at<kRegH>(st, 0);
+    uint4 v = h_at<kHK>(st, 0);
     v.z |= kPromotedBit;
     __syncwarp();
-    h_drop_front<kRegH>(st, 1, lane);
+    h_drop_front<kHK>(st, 1, lane);
     if (kRegS) reg_sorted_insert<kLean>(st, v, lane);
     else sorted_insert<kLean>(st, st.S, v, lane, kTierS);
     return budget - rem;
   }
   if (m == 1 && pairs == 1) {  // one pair (the next most common): swap it directly
-    uint4 v = h_at<kRegH>(st, 0);
+    uint4 v = h_at<kHK>(st, 0);
     v.z |= kPromotedBit;
     const uint4 d = kRegS ? reg_at(st.R, sn - 1) : st.S.e[st.S.n - 1];
     __syncwarp();
-    h_drop_front<kRegH>(st, 1, lane);
+    h_drop_front<kHK>(st, 1, lane);
     if (kRegS) {
       st.R.n -= 1;
       if (!reg_sorted_insert<kLean>(st, v, lane)) return budget - rem;
@@ -812,12 +824,12 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
       st.S.n -= 1;
       if (!sorted_insert<kLean>(st, st.S, v, lane, kTierS)) return budget - rem;
     }
-    h_insert<kLean, kRegH>(st, d, lane);
+    h_insert<kLean, kHK>(st, d, lane);
     return budget - rem;
   }
   // stage the moved entries, then fix both arrays
   uint4 *pro = st.tmp, *dem = st.tmp + rcap_s;
-  if (kRegH) {  // m <= 32: the first m entries are slot 0's
+  if constexpr (kHK > 0) {  // m <= 32: the first m entries are slot 0's
     if ((uint32_t)lane < m) pro[lane] = make_uint4(st.G.x[0], st.G.y[0], st.G.z[0] | kPromotedBit, 0u);
   } else {
     for (uint32_t i = lane; i < m; i += 32) {
@@ -833,14 +845,14 @@ __device__ __forceinline__ uint64_t tide(ReplayState &st, const Hot &D, uint64_t
     for (uint32_t i = lane; i < pairs; i += 32) dem[i] = st.S.e[st.S.n - pairs + i];
   }
   __syncwarp();
-  h_drop_front<kRegH>(st, m, lane);
+  h_drop_front<kHK>(st, m, lane);
   if (kRegS) st.R.n -= pairs;
   else st.S.n -= pairs;
   for (uint32_t i = 0; i < m; i++)
     if (kRegS ? !reg_sorted_insert<kLean>(st, pro[i], lane) : !sorted_insert<kLean>(st, st.S, pro[i], lane, kTierS))
       return budget - rem;
   for (uint32_t i = 0; i < pairs; i++)
-    if (!h_insert<kLean, kRegH>(st, dem[i], lane)) return budget - rem;
+    if (!h_insert<kLean, kHK>(st, dem[i], lane)) return budget - rem;
   return budget - rem;
 }
 
@@ -1039,14 +1051,15 @@ struct EventBufs {
 // One replay: Algorithm 1 over the trace's events.  kPol is the replay's
 // policy when the body is specialised for it (its policy tests then fold
 // away), or -1 for the body that reads the policy from the descriptor.
-// False when a kRegH replay stopped at its HBM tier's register bound (no
-// result written): the caller replays it again without kRegH.
-template <bool kGlobalLists, int kKeys, int kPol, bool kLean, bool kRegS = false, bool kRegH = false>
+// False when a register body (kHK > 0) stopped at its HBM tier's register
+// bound (no result written): the caller replays it again with more slots or
+// none.
+template <bool kGlobalLists, int kKeys, int kPol, bool kLean, bool kRegS = false, int kHK = 0>
 __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs, unsigned char *smem, int lane) {
   constexpr bool kOnline = kKeys == kKeyOnline, kStale = kKeys == kKeyStale;
   // the register HBM tier drops the entries' completion times (timeout only)
   // and drop_front's m <= 32 rests on the fast tier's 32-entry bound
-  static_assert(!kRegH || (kRegS && kLean && kPol == UNISON_SPEAR_TIDE && !kOnline && !kStale),
+  static_assert(kHK == 0 || (kHK <= kHSlots && kRegS && kLean && kPol == UNISON_SPEAR_TIDE && !kOnline && !kStale),
                 "register HBM tier: lean SPEAR+TIDE launches with the register fast tier");
   const Hot hot{D.cap_s, D.cap_h, D.kvb, D.dma, D.max_sessions};
 
@@ -1137,7 +1150,7 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
     st.R.n = 0;
     st.R.v = make_uint4(0u, 0u, 0u, 0u);
 #pragma unroll
-    for (int j = 0; j < (int)kHSlots; j++) st.G.x[j] = st.G.y[j] = st.G.z[j] = 0u;
+    for (int j = 0; j < kHK; j++) st.G.x[j] = st.G.y[j] = st.G.z[j] = 0u;
     st.S.cap = D.rcap_s;
     st.H.cap = D.rcap_h;
     st.npin = 0;
@@ -1249,27 +1262,28 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
             pkb = pack_key(0xFFFFFFFFull - spev[bi][j], s);
           // with the tier map only the session's own tier is searched (and
           // nothing for a session that is not resident)
-          if (kRegH) {
+          if constexpr (kHK > 0) {
             // both tiers in registers: one equality ballot per slot finds the
             // key (unique: it carries the session id) without the tier map
             const unsigned fs = __ballot_sync(kFull, (uint32_t)lane < st.R.n && ekey(st.R.v) == pkb);
-            unsigned fh[kHSlots];
+            unsigned fh[kHK];
 #pragma unroll
-            for (int j = 0; j < (int)kHSlots; j++)
+            for (int j = 0; j < kHK; j++)
               fh[j] = __ballot_sync(kFull, 32u * j + lane < st.H.n && hkey(st.G, j) == pkb);
             uint32_t ph = 0;
+            unsigned inh = 0;
 #pragma unroll
-            for (int j = (int)kHSlots - 1; j >= 0; j--)
+            for (int j = kHK - 1; j >= 0; j--) {
               if (fh[j]) ph = 32u * j + __ffs(fh[j]) - 1;
+              inh |= fh[j];
+            }
             const uint32_t ps = fs ? __ffs(fs) - 1 : 0u;
-            const uint4 es = reg_at(st.R, ps), eh = hreg_at(st.G, ph);
-            const bool inh = (fh[0] | fh[1] | fh[2] | fh[3]) != 0;
-            static_assert(kHSlots == 4, "the found test names the four slots");
+            const uint4 es = reg_at(st.R, ps), eh = hreg_at<kHK>(st.G, ph);
             tier = fs ? kTierS : (inh ? kTierH : kTierNone);
             pos = fs ? ps : ph;
             ent = fs ? es : eh;
           }
-          const uint32_t mt = kRegH ? 0u : ((kLean || st.tmap) ? st.tmap[s] : (kTierS | kTierH));
+          const uint32_t mt = kHK > 0 ? 0u : ((kLean || st.tmap) ? st.tmap[s] : (kTierS | kTierH));
           if (mt & kTierS) {
             if (kRegS) {
               pos = reg_lower_bound(st.R, pkb, lane);
@@ -1287,19 +1301,10 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
             }
           }
           if (tier == kTierNone && (mt & kTierH)) {
-            if (kRegH) {
-              pos = hreg_lower_bound(st.G, st.H.n, pkb, lane);
-              const uint4 cand = hreg_at(st.G, pos);  // (pos 128 reads a slot-0 entry; not taken)
-              if (pos < st.H.n && ekey(cand) == pkb) {
-                tier = kTierH;
-                ent = cand;
-              }
-            } else {
-              pos = lower_bound(st.H, pkb, lane);
-              if (pos < st.H.n && ekey(st.H.e[pos]) == pkb) {
-                tier = kTierH;
-                ent = st.H.e[pos];
-              }
+            pos = lower_bound(st.H, pkb, lane);
+            if (pos < st.H.n && ekey(st.H.e[pos]) == pkb) {
+              tier = kTierH;
+              ent = st.H.e[pos];
             }
           }
           __syncwarp();
@@ -1349,7 +1354,7 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
           set_tier<kLean>(st, s, kTierNone);
         } else if (tier == kTierH) {
           st.used_h -= esize(ent);
-          h_erase_at<kRegH>(st, pos, lane);
+          h_erase_at<kHK>(st, pos, lane);
           set_tier<kLean>(st, s, kTierNone);
         }
         uint64_t pk;
@@ -1375,7 +1380,7 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
           pk = pack_key(nr == kNoRef ? kKeyMax40 : (uint64_t)nr, s);
         } else
           pk = pack_key(0xFFFFFFFFull - e, s);
-        if (!place<kStale, kLean, kRegS, kRegH>(st, hot, s, pk, out, lane)) break;
+        if (!place<kStale, kLean, kRegS, kHK>(st, hot, s, pk, out, lane)) break;
       } else {
         // completion: unpin (if resident) and rank the session with its new key
         if (kStale) {
@@ -1420,7 +1425,7 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
             if (kRegS ? !reg_sorted_insert<kLean>(st, v, lane) : !sorted_insert<kLean>(st, st.S, v, lane, kTierS)) break;
           } else {
             st.pinned_h -= sz;
-            if (!h_insert<kLean, kRegH>(st, v, lane)) break;
+            if (!h_insert<kLean, kHK>(st, v, lane)) break;
           }
         }
         if (kOnline && edge) {
@@ -1435,7 +1440,7 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
           const uint64_t g = sgq[bi][j];
           const uint64_t budget = g * D.dma;
           CNT(st, n_tide_calls, 1);
-          const uint64_t moved = tide<kStale, kLean, kRegS, kRegH>(st, hot, budget, D.rcap_s, lane);
+          const uint64_t moved = tide<kStale, kLean, kRegS, kHK>(st, hot, budget, D.rcap_s, lane);
           CNT(st, dma_bytes, moved);
           if (moved > 0 && D.dma > 0) {
             dma_busy = true;
@@ -1486,7 +1491,7 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
       }
     }
   }
-  if (kRegH && st.status == kRegFull) {
+  if (kHK > 0 && st.status == kRegFull) {
     cp_async_wait_all();  // the next batch's copies land before the replay starts over
     __syncwarp();
     return false;
@@ -1536,7 +1541,7 @@ __device__ __forceinline__ bool replay_body(const ReplayDesc &D, EventBufs &bufs
 // replay of the launch has that policy, and the kernel holds only its body
 // (and is sized for it alone); kLean: every replay of the launch is lean
 // (see log_dec).
-template <bool kGlobalLists, int kKeys, int kOnly, bool kLean, bool kRegS = false, bool kRegH = false>
+template <bool kGlobalLists, int kKeys, int kOnly, bool kLean, bool kRegS = false, int kHK = 0>
 __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, const uint32_t *order) {
   extern __shared__ __align__(16) unsigned char smem[];
   __shared__ ReplayDesc Dsh;
@@ -1545,8 +1550,14 @@ __global__ void __launch_bounds__(32) replay_kernel(const ReplayDesc *descs, con
   if (lane == 0) Dsh = descs[order[blockIdx.x]];
   __syncwarp();
   if (kOnly >= 0) {
-    if (!replay_body<kGlobalLists, kKeys, kOnly, kLean, kRegS, kRegH>(Dsh, bufs, smem, lane))
-      replay_body<kGlobalLists, kKeys, kOnly, kLean, kRegS, false>(Dsh, bufs, smem, lane);
+    if constexpr (kHK > 0) {
+      // a replay whose HBM tier outgrows kHK slots starts over with the tier
+      // in shared memory
+      if (!replay_body<kGlobalLists, kKeys, kOnly, kLean, kRegS, kHK>(Dsh, bufs, smem, lane))
+        replay_body<kGlobalLists, kKeys, kOnly, kLean, kRegS, 0>(Dsh, bufs, smem, lane);
+    } else {
+      replay_body<kGlobalLists, kKeys, kOnly, kLean, kRegS, 0>(Dsh, bufs, smem, lane);
+    }
   } else if (kKeys == kKeyStream && Dsh.policy == UNISON_SPEAR_TIDE)
     replay_body<kGlobalLists, kKeys, UNISON_SPEAR_TIDE, false>(Dsh, bufs, smem, lane);
   else
@@ -1733,7 +1744,7 @@ using ReplayKernel = void (*)(const ReplayDesc *, const uint32_t *);
 // The kernel of the shared-memory SPEAR+TIDE group, for a log or not.
 ReplayKernel st_kernel(const ReplayPlan &P, bool logged) {
   if (P.st_lean && !logged)
-    return P.st_reg ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true, true, true>
+    return P.st_reg ? replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true, true, kHSlots>
                     : replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, true>;
   return replay_kernel<false, kKeyStream, UNISON_SPEAR_TIDE, false>;
 }

@@ -128,17 +128,18 @@ def test_sweep_iid_gaps_subset(B):
 
 
 def test_hbm_tier_past_register_capacity(B):
-    """SPEAR+TIDE replays whose HBM tier outgrows the 128 entries the lean
-    launch holds in registers: with a fast tier of at most 32 entries every
-    replay of the call takes the register tiers, and the HBM tier of the
-    first two configurations reaches about 200 unpinned sessions (the oracle
-    counts 210 and 192 on seed 0), so those replays stop at the 129th entry
-    and run again from their start with the tier in shared memory; the last
-    stays just under the bound (126).  Every counter and the decision hash
-    against the oracle."""
-    trs = [synth.paper_scale_trace(s, "coding") for s in (0, 1)]
+    """SPEAR+TIDE replays around the 160 entries (five a lane) the lean launch
+    holds its HBM tier in: with a fast tier of at most 32 entries every replay
+    of the call takes the register tiers.  On seed 0 the oracle counts at most
+    210 and 192 unpinned HBM sessions for the first two configurations, so
+    those replays stop at the 161st entry and run again from their start with
+    the tier in shared memory; 126 for the third; and 142 on the trace with
+    independent gaps (its fifth slot in use).  Every counter and the decision
+    hash against the oracle."""
+    trs = [synth.paper_scale_trace(s, "coding") for s in (0, 1)] + [synth.paper_scale_trace(0, "coding", gap_persist=0.0)]
     cfgs = [(28_672, 1 * GIB, 64 * GIB), (131_072, 1 * GIB, 256 * GIB), (28_672, 512 * MIB, 32 * GIB)]
-    reps = [(ti, base("spear_tide", cs, ch, kvb)) for ti in range(len(trs)) for kvb, cs, ch in cfgs]
+    reps = [(ti, base("spear_tide", cs, ch, kvb)) for ti in range(2) for kvb, cs, ch in cfgs]
+    reps += [(2, base("spear_tide", cs, 128 * GIB, 131_072)) for cs in (1 * GIB, 4 * GIB)]
     res, _, _ = run_gpu(B, trs, reps)
     for i, (ti, p) in enumerate(reps):
         assert res[i]["status"] == 0
