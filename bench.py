@@ -920,15 +920,18 @@ def main():
                    "key_stream_avg_ms": ks_ms / max(ks_n, 1), "ttft_median_avg_ms": md_ms / max(md_n, 1)}
     if replay_roof is not None:
         # The launch ends with its slowest replay: its cycles per event, against
-        # the chain an event needs on sorted arrays in shared memory (about 17
-        # dependent accesses -- tier byte, two search rounds, the entry, a
-        # shift's load and store, the store of the new entry, pops, pin slot and
-        # pin entry, TIDE's two heads -- at about 30 cycles each).
+        # the chain an event needs with both tiers in the warp's registers and
+        # the pin list in shared memory (about 17 dependent steps of about 30
+        # cycles each: the event's and its key's loads, the lookup ballot and
+        # entry shuffle, the erase shuffle, pin slot, pin entry and its store,
+        # a demotion's pop, the HBM search ballot and insert shuffle, TIDE's
+        # two heads and its insert's ballot and shuffle).
         mhz = (clocks or {}).get("sm_mhz") or 2070.0
         replay_roof["cycles_per_event_slowest_replay"] = avg_rep_ms * 1e3 * mhz / (events_per_step / n_rep)
         replay_roof["floor_cycles_per_event"] = 17 * 30
-        replay_roof["floor_basis"] = ("17 dependent shared-memory accesses per event x ~30 cycles "
-                                      "(search, shift, entry store, pops, pin slot, TIDE heads)")
+        replay_roof["floor_basis"] = ("17 dependent steps per event x ~30 cycles: shared-memory loads (event, key, "
+                                      "pin slot and entry) and the register tiers' ballots and shuffles (lookup, "
+                                      "erase, demotion, HBM insert, TIDE heads and insert)")
     avg_rk = rk_ms / max(rk_n, 1) if rk_n else float("nan")
     achieved = rank_bytes / (avg_rk / 1e3) / 1e9 if rk_n else float("nan")
     n_rec = len(r_params) * RANK_N
