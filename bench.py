@@ -808,7 +808,8 @@ def main():
         sizes, single = rank_size_sweep(B, host_rec, sigma, stream, hbm_peak)
 
     # the sweep on traces whose gaps are drawn independently (no per-session
-    # persistence): the survey's gap model, timed like the main leg
+    # persistence: every gap's mixture component and value drawn afresh),
+    # timed like the main leg
     iid = None
     if not (args.no_iid or args.rank_only or world > 1):
         from synth.workloads import sweep_case, to_lib
